@@ -1,0 +1,511 @@
+"""Benchmark of the EAT MoE-layer hot path on GB300 (one JSON line on rank 0).
+
+Default workload: a Mixtral-8x7B-shaped layer (d=4096, 8 SwiGLU experts, d_ff=14336, K=2, bf16
+weights, fp32 accumulate) in decode: one step = one layer call at each of batch 1, 16 and 64 tokens
+(three handles sharing the weights, each with its own evolving expert accounts; 81 tokens/step).
+Inputs are resident in HBM before the timed region; the 2.8 GB of expert weights are larger than
+L2, so no flush is needed between steps.  Other workloads (--workload) are the prefill/decode
+configurations of the OLMoE-, Qwen-MoE- and DeepSeek-V2-Lite-shaped layers.
+
+--impl reference times the fp64 CPU oracle (the reference arm of this benchmark) on the host cores
+on a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+_CORES = os.cpu_count() or 1
+for _v in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
+    os.environ.setdefault(_v, str(_CORES))
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = ("MoE-layer tokens/s at 1 GB300 (decode & prefill); % HBM/tensor roofline; "
+          "experts/token")
+FALLBACK_HBM_GBS = 6800.0
+FALLBACK_BF16_TFLOPS = 1900.0
+
+
+# ------------------------------------------------------------------------------- workloads
+def workload_spec(name):
+    from paper_2609_33614_gb300 import workloads as W
+    specs = {
+        "mixtral-decode": dict(shape=W.MIXTRAL, batches=[1, 16, 64], layers=1,
+                               desc="mixtral-8x7b-shaped MoE layer, decode, batch 1+16+64 per step"),
+        "olmoe-prefill": dict(shape=W.OLMOE, batches=[4096], layers=1,
+                              desc="olmoe-shaped MoE layer, prefill 4096 tokens per step"),
+        "olmoe-decode": dict(shape=W.OLMOE, batches=[32], layers=1,
+                             desc="olmoe-shaped MoE layer, decode batch 32 per step"),
+        "qwen-prefill": dict(shape=W.QWEN, batches=[8192], layers=1,
+                             desc="qwen1.5-moe-shaped layer (60 routed + 4 shared), prefill 8192"),
+        "dsv2l-prefill": dict(shape=W.DSV2L, batches=[16384], layers=26,
+                              desc="deepseek-v2-lite-shaped 26-layer MoE stack, prefill 16384"),
+        "dsv2l-decode": dict(shape=W.DSV2L, batches=[128], layers=26,
+                             desc="deepseek-v2-lite-shaped 26-layer MoE stack, decode batch 128"),
+    }
+    return specs[name]
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as fh:
+            pk = json.load(fh)
+        return float(pk["hbm_gbs"]), float(pk["bf16_tflops"]), \
+            float(pk.get("bf16_tflops_sustained", pk["bf16_tflops"])), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS, 1700.0, "fallback"
+
+
+# ------------------------------------------------------------------------------- clocks
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons during the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *a):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        sm, mx, reasons = [], [], set()
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------------------------------- distributed
+def dist_setup(n_gpus):
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if torch.cuda.is_available():
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend)
+    elif torch.cuda.is_available():
+        torch.cuda.set_device(0)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(value, world):
+    """Max of a float over all ranks (the slowest replica sets the job time)."""
+    if world == 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([value], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def sum_over_ranks(value, world):
+    if world == 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([value], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+# ------------------------------------------------------------------------------- roofline
+def kernel_bytes(kind, shape, union, acts, T):
+    """Algorithmic HBM bytes of one launch: weights of the activated experts plus the
+    activation rows the kernel must read and write (bf16 = 2 B, fp32 partials = 4 B)."""
+    d, F = shape.d_model, shape.d_ff
+    if kind == "ffn_up":
+        return union * 2 * F * d * 2 + acts * d * 2 + acts * F * 2
+    if kind == "ffn_down":
+        return union * d * F * 2 + acts * F * 2 + acts * d * 4
+    if kind == "shared_up":
+        return shape.n_shared * 2 * shape.d_ff_shared * d * 2 + T * d * 2 + \
+            shape.n_shared * T * shape.d_ff_shared * 2
+    if kind == "shared_down":
+        return shape.n_shared * d * shape.d_ff_shared * 2 + \
+            shape.n_shared * T * (shape.d_ff_shared * 2 + d * 4)
+    raise KeyError(kind)
+
+
+def kernel_flops(kind, shape, acts, T):
+    d, F = shape.d_model, shape.d_ff
+    if kind == "ffn_up":
+        return acts * 2 * 2 * d * F
+    if kind == "ffn_down":
+        return acts * 2 * d * F
+    if kind == "shared_up":
+        return shape.n_shared * T * 2 * 2 * d * shape.d_ff_shared
+    if kind == "shared_down":
+        return shape.n_shared * T * 2 * d * shape.d_ff_shared
+    raise KeyError(kind)
+
+
+def traffic_for(kind, workload):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken on the current
+    kernel sources (its source hash matches); else None."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        from paper_2609_33614_gb300 import build
+        with open(path) as fh:
+            tr = json.load(fh)
+        ent = tr.get(workload, {}).get(kind)
+        if ent and ent.get("source_hash") == build._stamp():
+            return ent["dram_bytes_per_launch"]
+    except Exception:
+        pass
+    return None
+
+
+# ------------------------------------------------------------------------------- our arm
+def run_ours(args, world, rank, local):
+    import torch
+    from paper_2609_33614_gb300 import eat, workloads as W
+
+    spec = workload_spec(args.workload)
+    shape = spec["shape"]
+    batches = spec["batches"]
+    n_layers = spec["layers"]
+    dev = torch.device("cuda", torch.cuda.current_device())
+    stream = torch.cuda.current_stream()
+    n_steps_total = args.warmup + args.steps
+
+    # layers (weights drawn on the GPU generator) and one handle per (layer, batch)
+    layer_w = [W.make_layer(shape, l, device="cuda") for l in range(n_layers)]
+    handles = []  # [layer][batch]
+    for lw in layer_w:
+        row = []
+        for B in batches:
+            row.append(eat.EatLayer.from_workload(lw, B))
+        handles.append(row)
+    # inputs resident in HBM before the timed region
+    xs = {B: [W.make_tokens(shape, B, step=s, device="cuda") for s in range(min(n_steps_total, 64))]
+          for B in batches}
+    ys = {B: torch.empty(B, shape.d_model, dtype=shape.xdtype, device=dev) for B in batches}
+    tokens_per_step = sum(batches)
+
+    # residual stream buffers for stacks: x_{l+1} = x_l + y_l (the transformer block's residual
+    # add, outside the MoE layer)
+    xr = {B: [torch.empty(B, shape.d_model, dtype=shape.xdtype, device=dev) for _ in range(2)]
+          for B in batches}
+
+    def layers_fwd(bi, B, x):
+        for l in range(n_layers):
+            eat.eat_moe_forward(handles[l][bi].h, x, B, 0, ys[B])
+            if l + 1 < n_layers:
+                nxt = xr[B][l % 2]
+                torch.add(x, ys[B], out=nxt)
+                x = nxt
+        return ys[B]
+
+    def step(s):
+        for bi, B in enumerate(batches):
+            layers_fwd(bi, B, xs[B][s % len(xs[B])])
+
+    def reset_all():
+        for row in handles:
+            for h in row:
+                h.reset()
+
+    def timed(fn, profile=False):
+        reset_all()
+        for s in range(args.warmup):
+            fn(s)
+        if profile:
+            for row in handles:
+                for h in row:
+                    eat.eat_profile_begin(h.h, 16 * n_steps_total + 64)
+        before = [[eat.eat_get_counters(h.h) for h in row] for row in handles]
+        barrier(world)
+        torch.cuda.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for s in range(args.warmup, n_steps_total):
+            fn(s)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        barrier(world)
+        ms = e0.elapsed_time(e1)
+        after = [[eat.eat_get_counters(h.h) for h in row] for row in handles]
+        prof = None
+        if profile:
+            prof = [[eat.eat_profile_end(h.h) for h in row] for row in handles]
+        return ms, before, after, prof
+
+    with ClockSampler(local) as clk:
+        ms, c0, c1, _ = timed(step)
+    clocks = clk.summary()
+    job_ms = max_over_ranks(ms, world)
+    total_tokens = sum_over_ranks(tokens_per_step * args.steps, world)
+    value = total_tokens / (job_ms / 1e3)
+
+    launches = sum(c1[l][b]["launches"] - c0[l][b]["launches"]
+                   for l in range(n_layers) for b in range(len(batches)))
+    calls = sum(c1[l][b]["calls"] - c0[l][b]["calls"]
+                for l in range(n_layers) for b in range(len(batches)))
+    acts = sum(c1[l][b]["activations"] - c0[l][b]["activations"]
+               for l in range(n_layers) for b in range(len(batches)))
+    unions = {B: (sum(c1[l][bi]["union_sum"] - c0[l][bi]["union_sum"] for l in range(n_layers)) /
+                  max(1, sum(c1[l][bi]["calls"] - c0[l][bi]["calls"] for l in range(n_layers))))
+              for bi, B in enumerate(batches)}
+
+    # second pass with per-kernel CUDA events (roofline of the dominant kernel)
+    ms_p, p0, p1, prof = timed(step, profile=True)
+    kinds = {}
+    for l in range(n_layers):
+        for bi, B in enumerate(batches):
+            dU = p1[l][bi]["union_sum"] - p0[l][bi]["union_sum"]
+            dA = p1[l][bi]["activations"] - p0[l][bi]["activations"]
+            dC = p1[l][bi]["calls"] - p0[l][bi]["calls"]
+            for kind, (kms, n) in prof[l][bi].items():
+                k = kinds.setdefault(kind, {"ms": 0.0, "launches": 0, "bytes": 0.0, "flops": 0.0})
+                k["ms"] += kms
+                k["launches"] += n
+                if kind in ("ffn_up", "ffn_down", "shared_up", "shared_down") and n:
+                    # per-launch average union / activations of this handle
+                    k["bytes"] += n * kernel_bytes(kind, shape, dU / max(1, dC), dA / max(1, dC), B)
+                    k["flops"] += n * kernel_flops(kind, shape, dA / max(1, dC), B)
+    total_kernel_ms = sum(k["ms"] for k in kinds.values())
+    dom = max((k for k in kinds if k.startswith("ffn") or k.startswith("shared")),
+              key=lambda k: kinds[k]["ms"])
+    hbm, bf16_burst, bf16_sus, peak_src = load_peaks()
+    dk = kinds[dom]
+    avg_launch_s = dk["ms"] / 1e3 / max(1, dk["launches"])
+    decode = max(batches) <= 256
+    if decode:
+        achieved = dk["bytes"] / max(1, dk["launches"]) / avg_launch_s / 1e9
+        roof = {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
+                "frac": achieved / hbm, "peak_source": peak_src,
+                "traffic": traffic_for(dom, args.workload)}
+    else:
+        achieved = dk["flops"] / max(1, dk["launches"]) / avg_launch_s / 1e12
+        roof = {"bound": "tensor", "achieved": achieved, "peak": bf16_sus, "unit": "TFLOP/s",
+                "frac": achieved / bf16_sus, "peak_source": peak_src + " sustained",
+                "traffic": traffic_for(dom, args.workload)}
+    roof.update({"kernel": dom, "kernel_share": dk["ms"] / total_kernel_ms,
+                 "avg_launch_us": avg_launch_s * 1e6,
+                 "algorithmic_bytes_per_launch": dk["bytes"] / max(1, dk["launches"])})
+
+    # end to end through the public host-buffer entry point (copies inside the timed region)
+    xh = {B: [x.cpu().pin_memory() for x in xs[B]] for B in batches}
+    yh = {B: torch.empty(B, shape.d_model, dtype=shape.xdtype).pin_memory() for B in batches}
+
+    xd = {B: torch.empty(B, shape.d_model, dtype=shape.xdtype, device=dev) for B in batches}
+
+    def step_host(s):
+        for bi, B in enumerate(batches):
+            if n_layers == 1:
+                eat.eat_moe_forward_host(handles[0][bi].h, xh[B][s % len(xh[B])], B, 0, yh[B])
+            else:
+                xd[B].copy_(xh[B][s % len(xh[B])], non_blocking=True)
+                yh[B].copy_(layers_fwd(bi, B, xd[B]), non_blocking=True)
+                torch.cuda.current_stream().synchronize()
+
+    e2e_ms, _, _, _ = timed(step_host)
+    e2e_ms = max_over_ranks(e2e_ms, world)
+    elt = 2 if shape.xdtype == torch.bfloat16 else 4
+    e2e = {"value": sum_over_ranks(tokens_per_step * args.steps, world) / (e2e_ms / 1e3),
+           "unit": "tokens/s",
+           "h2d_bytes_per_step": tokens_per_step * shape.d_model * elt,
+           "d2h_bytes_per_step": tokens_per_step * shape.d_model * elt}
+
+    result = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": job_ms / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) hidden states, N(0,0.02^2) weights)",
+        "config": {"workload": spec["desc"], "d_model": shape.d_model,
+                   "n_experts": shape.n_experts, "d_ff": shape.d_ff, "n_shared": shape.n_shared,
+                   "max_k": shape.max_k, "layers": n_layers, "batches": batches,
+                   "l2": "inputs larger than L2 (expert weights > 129 MB), no flush"},
+        "roofline": roof,
+        "experts_per_token": acts / max(1, sum(B * args.steps for B in batches) * n_layers),
+        "union_per_call": unions,
+        "kernels_ms_per_step": {k: v["ms"] / args.steps for k, v in kinds.items()},
+        "gpu_launches": launches,
+        "clocks": clocks,
+        "e2e": e2e,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        result["cpu_baseline"] = oracle_sample(args.workload, layer_w[0], handles[0][0],
+                                               min_seconds=10.0)
+    for row in handles:
+        for h in row:
+            h.close()
+    return result
+
+
+# ------------------------------------------------------------------------------- oracle arm
+def _oracle_layer(lw):
+    import torch
+    import oracle.eat_oracle as orc
+    f = lambda t: None if t is None else t.detach().to("cpu").to(torch.float64).numpy()
+    return orc.Layer(f(lw.w_router), f(lw.b_router), f(lw.w_gate), f(lw.w_up), f(lw.w_down),
+                     f(lw.ws_gate), f(lw.ws_up), f(lw.ws_down))
+
+
+def oracle_sample(workload, lw, handle=None, min_seconds=10.0, max_steps=None, batches=None):
+    """Time the fp64 oracle, as it stands, on a bounded sample of the workload: successive layer
+    calls cycling through the workload's batch sizes (prefill workloads: the first 256 tokens of
+    the prefill batch), from the GPU handle's current accounts if given, until min_seconds of CPU
+    time have run (or max_steps calls)."""
+    import numpy as np
+    import torch
+    import oracle.eat_oracle as orc
+    from paper_2609_33614_gb300 import workloads as W
+
+    spec = workload_spec(workload)
+    shape = spec["shape"]
+    bs = batches or [min(B, 256) for B in spec["batches"]]
+    L = _oracle_layer(lw)
+    prm = orc.Params(max_k=shape.max_k, temperature=shape.temperature)
+    if handle is not None:
+        N, P, C = handle.accounts()
+        acc = orc.Accounts(N.cpu().numpy(), P.cpu().numpy(), C.cpu().numpy())
+    else:
+        acc = orc.Accounts.zeros(shape.n_experts)
+    toks, calls, el = 0, 0, 0.0
+    while el < min_seconds and (max_steps is None or calls < max_steps):
+        B = bs[calls % len(bs)]
+        x = W.make_tokens(shape, B, step=calls).to(torch.float64).numpy()
+        t0 = time.perf_counter()
+        res = orc.moe_forward(x, L, acc, prm, 0)
+        el += time.perf_counter() - t0
+        acc = res.accounts_after
+        toks += B
+        calls += 1
+    return {"value": toks / el, "unit": "tokens/s", "cores": int(os.environ["OPENBLAS_NUM_THREADS"]),
+            "kind": "oracle",
+            "sample": f"{calls} oracle layer calls cycling batches {bs} ({toks} tokens, "
+                      f"{el:.1f} s), fp64 numpy, weights widened to fp64 before timing"}
+
+
+def run_reference(args, world, rank):
+    """The reference arm: the fp64 oracle on the host cores, rank 0 only."""
+    if rank != 0:
+        return None
+    import torch
+    from paper_2609_33614_gb300 import workloads as W
+    spec = workload_spec(args.workload)
+    shape = spec["shape"]
+    lw = W.make_layer(shape, 0, device="cuda" if torch.cuda.is_available() else "cpu")
+    # each step: one oracle layer call at batch 1 (bounded so K steps end in minutes)
+    bs = [1] if spec["batches"][0] <= 256 else [64]
+    import oracle.eat_oracle as orc
+    L = _oracle_layer(lw)
+    del lw
+    prm = orc.Params(max_k=shape.max_k, temperature=shape.temperature)
+    acc = orc.Accounts.zeros(shape.n_experts)
+    toks, el = 0, 0.0
+    for s in range(args.warmup + args.steps):
+        B = bs[s % len(bs)]
+        x = W.make_tokens(shape, B, step=s).to(torch.float64).numpy()
+        t0 = time.perf_counter()
+        res = orc.moe_forward(x, L, acc, prm, 0)
+        dt = time.perf_counter() - t0
+        acc = res.accounts_after
+        if s >= args.warmup:
+            el += dt
+            toks += B
+    value = toks / el
+    cores = int(os.environ["OPENBLAS_NUM_THREADS"])
+    return {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": el * 1e3 / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "impl": "reference",
+            "config": {"workload": spec["desc"], "sample": f"batch {bs} per step"},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores,
+                             "kind": "oracle",
+                             "sample": f"{args.steps} timed oracle layer calls at batch {bs}"},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=64)
+    ap.add_argument("--warmup", type=int, default=8)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="mixtral-decode")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    world, rank, local = dist_setup(args.gpus)
+    if args.impl == "reference":
+        res = run_reference(args, world, rank)
+    else:
+        from paper_2609_33614_gb300 import build
+        if rank == 0:
+            build.build()
+        barrier(world)
+        res = run_ours(args, world, rank, local)
+    if rank == 0 and res is not None:
+        print(json.dumps(res))
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,168 @@
+/*
+ * eat.h -- C ABI of the GB300 (sm_103a) EAT MoE-layer hot path.
+ *
+ * EAT ("Expert Account Tracker", arxiv 2609.33614) replaces fixed Top-K routing in a
+ * Mixture-of-Experts layer by a history-aware importance score and an adaptive per-token
+ * threshold that activates a variable number of experts (§3.2-§3.4).  This library runs one MoE
+ * layer forward pass under that rule on one GPU:
+ *   router GEMM + softmax (§3.1-§3.2) -> history score S_h (Eq. 1) -> importance I (Eq. 2)
+ *   -> threshold tau (Eq. 3-5, PPL adjustment, boundedness, smoothing; §3.3)
+ *   -> variable-k selection and renormalisation (Eq. 6-8) -> permute by expert
+ *   -> SwiGLU expert FFNs over the activated experts -> weighted combine / unpermute
+ *   -> account update (N, P_total, C_s of §3.2).
+ *
+ * Conventions shared by every entry point:
+ *  - Array pointers are DEVICE pointers unless the name ends in _host.  Row-major, no padding.
+ *  - Weights are NOT owned: the caller keeps them alive and unchanged until eat_destroy.
+ *  - The handle owns the expert accounts and a workspace sized for desc.max_tokens at
+ *    eat_create; no entry point allocates afterwards.  One handle = one layer.
+ *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).  Calls are
+ *    asynchronous on that stream unless stated; arguments are validated on the host before any
+ *    launch, and an invalid call returns an error without touching the device.
+ *  - A handle is not thread-safe: calls on one handle must be serialised by the caller, and
+ *    calls that may overlap on the GPU (different streams) must not share a handle.
+ *  - Nothing throws across the ABI.  Every call returns an eat_status; eat_last_error gives a
+ *    one-line description of the last failure on that handle.
+ */
+#ifndef EAT_H_
+#define EAT_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum eat_status {
+  EAT_OK = 0,
+  EAT_ERR_INVALID_ARG = 1,  /* null pointer, size out of range, bad enum value */
+  EAT_ERR_UNSUPPORTED = 2,  /* valid request outside what this build implements */
+  EAT_ERR_OOM = 3,          /* device allocation failed in eat_create */
+  EAT_ERR_CUDA = 4,         /* a CUDA runtime call or kernel launch failed */
+  EAT_ERR_STATE = 5         /* handle not usable (e.g. device-side status word set) */
+} eat_status;
+
+typedef enum eat_dtype { EAT_F32 = 0, EAT_BF16 = 1 } eat_dtype;
+
+/* How the EMA contribution C_s enters Eq. 1 (§3.2).  EAT_C_SUM: as the share C_i / sum_j C_j,
+ * on the same [0, 1] scale as the other two terms (default).  EAT_C_RAW: the literal C_i. */
+typedef enum eat_c_mode { EAT_C_SUM = 0, EAT_C_RAW = 1 } eat_c_mode;
+
+/* Hyper-parameters of §3.2-§3.4; defaults (eat_default_params) are Table 1, the 1.2 / 0.9 factors
+ * and 10% / 90% bounds of §3.3, and eps of Eq. 7. */
+typedef struct eat_params {
+  double alpha;        /* EMA factor of C_s (0.95): C <- (1 - alpha) C + alpha ||o||_2 */
+  double w1, w2, w3;   /* Eq. 1 weights (0.3, 0.3, 0.4) */
+  double beta;         /* Eq. 2 balance (0.6): I = (1 - beta) p + beta S_h */
+  double alpha1;       /* Eq. 5 (0.5): tau = max(alpha1 mu, mu - alpha2 sigma) */
+  double alpha2;       /* Eq. 5 (1.0) */
+  double kappa1;       /* smoothing (0.7): tau_final = kappa1 tau_PPL + kappa2 tau */
+  double kappa2;       /* smoothing (0.3) */
+  double ppl_up;       /* factor when PPL rose (1.2) */
+  double ppl_down;     /* factor otherwise (0.9) */
+  double q_lo, q_hi;   /* boundedness: tau_final clamped to these quantiles of p (0.1, 0.9) */
+  double eps;          /* Eq. 7 (1e-8) */
+  double temperature;  /* router logits are divided by it before the softmax (1.0) */
+  int32_t max_k;       /* K of Eq. 6: at most K experts per token, 1 <= K <= min(E, 16) */
+  int32_t clamp_enabled; /* 1: apply the [q_lo, q_hi] bounds; 0: skip them */
+  int32_t c_mode;      /* eat_c_mode */
+} eat_params;
+
+/* Fill *p with the defaults above and max_k = 2.  Returns EAT_ERR_INVALID_ARG if p is NULL. */
+eat_status eat_default_params(eat_params* p);
+
+/* One MoE layer.  Shapes use nn.Linear layout (out_features x in_features), row-major:
+ *   w_router [E, d] fp32, b_router [E] fp32 or NULL;
+ *   w_gate, w_up [E, F, d], w_down [E, d, F] in wdtype;
+ *   ws_gate, ws_up [S, Fs, d], ws_down [S, d, Fs] in wdtype, all NULL when n_shared == 0
+ *   (always-on shared experts, added with weight 1, not routed, no account).
+ * Supported: 1 <= E <= 256; d, F, Fs multiples of 64; (wdtype, xdtype) both EAT_F32 or both
+ * EAT_BF16; 1 <= max_tokens <= 65536.  All weight pointers 16-byte aligned. */
+typedef struct eat_layer_desc {
+  int32_t d_model, n_experts, d_ff, n_shared, d_ff_shared, max_tokens;
+  int32_t wdtype, xdtype;
+  const float* w_router;
+  const float* b_router;
+  const void* w_gate;
+  const void* w_up;
+  const void* w_down;
+  const void* ws_gate;
+  const void* ws_up;
+  const void* ws_down;
+} eat_layer_desc;
+
+typedef struct eat_handle eat_handle;
+
+/* Validate desc/params, allocate the accounts (zeroed: the empty history of §3.2) and the
+ * workspace for max_tokens, and build the weight descriptors.  Synchronous.  On success *out
+ * receives the handle; on failure *out is set to NULL and nothing stays allocated. */
+eat_status eat_create(const eat_layer_desc* desc, const eat_params* params, eat_handle** out);
+
+/* Zero the accounts N, P_total, C_s (§3.2: an expert with no history) and the counters. */
+eat_status eat_reset_accounts(eat_handle* h, void* stream);
+
+/* Routing only (§3.2-§3.4, Eq. 1-8) for T tokens x [T, d] (xdtype), 1 <= T <= max_tokens,
+ * reading the current accounts and never changing them.  ppl_sign is the sign of
+ * PPL_curr - PPL_prev (§3.3): +1 -> factor ppl_up, -1 -> ppl_down, 0 -> no signal (factor 1).
+ * Outputs: idx [T, K] int32 selected experts in ascending index order, -1 after the k-th;
+ * w [T, K] fp32 renormalised gates g_norm (Eq. 7), 0 after the k-th; k [T] int32 count. */
+eat_status eat_route(eat_handle* h, const void* x, int32_t T, int32_t ppl_sign,
+                     int32_t* idx, float* w, int32_t* k, void* stream);
+
+/* One layer call = one EMA timestep of §3.2: routing as eat_route from the pre-call accounts,
+ * y [T, d] (xdtype) = sum over selected e of g_norm,e * E_e(x_t) + sum of shared experts, then
+ * the account update: N_e += n_e, P_total,e += sum of p over e's activations,
+ * C_e <- (1 - alpha) C_e + alpha * mean ||E_e(x_t)||_2 when n_e > 0.
+ * idx_opt / w_opt / k_opt may be NULL; when given they receive the routing as in eat_route.
+ * y must not alias x. */
+eat_status eat_moe_forward(eat_handle* h, const void* x, int32_t T, int32_t ppl_sign, void* y,
+                           int32_t* idx_opt, float* w_opt, int32_t* k_opt, void* stream);
+
+/* eat_moe_forward with HOST buffers: copies x_host [T, d] to the device, runs the layer, copies
+ * y back into y_host [T, d] and synchronises the stream before returning.  Pinned host memory
+ * gives asynchronous copies; pageable memory works but is staged by the driver. */
+eat_status eat_moe_forward_host(eat_handle* h, const void* x_host, int32_t T, int32_t ppl_sign,
+                                void* y_host, void* stream);
+
+/* Free everything the handle owns.  Synchronises the device first.  NULL is accepted. */
+eat_status eat_destroy(eat_handle* h);
+
+/* Snapshot / restore of the accounts (device pointers, [E] each): N int64, P_total fp64,
+ * C_s fp64.  Stream-ordered copies. */
+eat_status eat_get_accounts(eat_handle* h, int64_t* N, double* P, double* C, void* stream);
+eat_status eat_set_accounts(eat_handle* h, const int64_t* N, const double* P, const double* C,
+                            void* stream);
+
+/* Per-expert statistics of the last eat_moe_forward (device pointers, [E] each): activation
+ * count n_e, sum of p over the activations, sum of ||E_e(x_t)||_2 over the activations.  Any
+ * pointer may be NULL.  Stream-ordered copies. */
+eat_status eat_get_call_stats(eat_handle* h, int32_t* n_e, double* sum_p, double* sum_norm,
+                              void* stream);
+
+/* Counters since eat_create or the last eat_reset_accounts, into host array out[n]
+ * (synchronises the device):
+ *   out[0] forward calls, out[1] sum over calls of the number of distinct activated experts,
+ *   out[2] sum over calls of the activations (sum_t k_t), out[3] kernel launches issued by this
+ *   handle (all entry points). */
+eat_status eat_get_counters(eat_handle* h, int64_t* out, int32_t n);
+
+/* Per-kernel device timing.  eat_profile_begin(h, capacity) makes every later launch of this
+ * handle record a CUDA event pair (capacity = max launches recorded); eat_profile_end
+ * synchronises, writes for each kernel kind i < n the summed milliseconds ms[i] and the launch
+ * count launches[i], and stops recording.  Kernel kinds: 0 route, 1 permute, 2 routed
+ * gate/up FFN, 3 routed down FFN, 4 shared gate/up, 5 shared down, 6 combine, 7 account. */
+eat_status eat_profile_begin(eat_handle* h, int32_t capacity);
+eat_status eat_profile_end(eat_handle* h, double* ms, int64_t* launches, int32_t n);
+
+/* Which expert-FFN kernels this handle uses: 0 = CUDA-core (fp32 layers), 1 = tcgen05/TMA
+ * tensor-core kernels (bf16 layers).  -1 on a NULL handle. */
+int32_t eat_ffn_backend(const eat_handle* h);
+
+/* Last error on the handle (never NULL), or a generic text for a NULL handle. */
+const char* eat_last_error(const eat_handle* h);
+const char* eat_status_string(eat_status s);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* EAT_H_ */

@@ -1,0 +1,541 @@
+// extern "C" boundary of libeat.so (declared in include/eat.h): handle, argument validation,
+// workspace, and the stream-ordered launch sequence of one EAT MoE layer call.
+#include "eat_internal.cuh"
+#include "ffn_tc.cuh"
+
+#include <algorithm>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+using namespace eat;
+
+struct eat_handle {
+  eat_layer_desc desc;
+  eat_params prm;
+  int E = 0, d = 0, F = 0, S = 0, Fs = 0, Tmax = 0, K = 0;
+  bool bf16 = false;
+  int backend = 0;  // 0 CUDA-core kernels (fp32 layers), 1 tcgen05 kernels (bf16 layers)
+  size_t elt = 4;
+
+  void* mem = nullptr;
+  int64_t* N = nullptr;
+  double* P = nullptr;
+  double* C = nullptr;
+  int32_t* st_n = nullptr;
+  double* st_p = nullptr;
+  double* st_norm = nullptr;
+  long long* counters = nullptr;  // [4] on the device: calls, sum |union|, sum k, spare
+  float* logit_part = nullptr;
+  int32_t* idx = nullptr;
+  float* w = nullptr;
+  int32_t* k = nullptr;
+  float* psel = nullptr;
+  PermuteOut perm{};
+  void* act = nullptr;    // [Tmax*K, F]
+  float* opart = nullptr; // [splits][Tmax*K, d]
+  float* onorm = nullptr; // [Tmax*K]
+  void* sact = nullptr;   // [S*Tmax, Fs]
+  float* sout = nullptr;  // [S*Tmax, d]
+  void* xstage = nullptr; // [Tmax, d]
+  void* ystage = nullptr; // [Tmax, d]
+  int max_split = 1;      // split-K slices of the routed down projection held in opart
+
+  TcLayer tc{};
+
+  long long launches = 0;
+  std::string err;
+
+  bool prof = false;
+  int prof_cap = 0;
+  std::vector<cudaEvent_t> ev;  // 2 per recorded launch
+  std::vector<int> ev_kind;
+  int prof_n = 0;
+};
+
+namespace {
+
+thread_local std::string g_err;
+
+eat_status fail(eat_handle* h, eat_status s, const std::string& msg) {
+  if (h) h->err = msg;
+  else g_err = msg;
+  return s;
+}
+
+eat_status cuda_fail(eat_handle* h, cudaError_t e, const char* what) {
+  return fail(h, EAT_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
+}
+
+enum Kind { kRoute = 0, kPermute, kUp, kDown, kSUp, kSDown, kCombine, kAccount, kKinds };
+
+// Run one launch, optionally bracketed by CUDA events for the per-kernel profile.
+template <typename Fn>
+eat_status launch(eat_handle* h, int kind, cudaStream_t st, const char* what, Fn&& fn) {
+  const bool rec = h->prof && h->prof_n < h->prof_cap;
+  if (rec) cudaEventRecord(h->ev[2 * h->prof_n], st);
+  const cudaError_t e = fn();
+  ++h->launches;
+  if (rec) {
+    cudaEventRecord(h->ev[2 * h->prof_n + 1], st);
+    h->ev_kind[h->prof_n] = kind;
+    ++h->prof_n;
+  }
+  if (e != cudaSuccess) return cuda_fail(h, e, what);
+  return EAT_OK;
+}
+
+#define EAT_TRY(x)                    \
+  do {                                \
+    eat_status s__ = (x);             \
+    if (s__ != EAT_OK) return s__;    \
+  } while (0)
+
+RouteParams route_params(const eat_params& p, int ppl_sign) {
+  RouteParams r;
+  r.w1 = (float)p.w1;
+  r.w2 = (float)p.w2;
+  r.w3 = (float)p.w3;
+  r.beta = (float)p.beta;
+  r.alpha1 = (float)p.alpha1;
+  r.alpha2 = (float)p.alpha2;
+  r.kappa1 = (float)p.kappa1;
+  r.kappa2 = (float)p.kappa2;
+  r.ppl_factor = ppl_sign > 0 ? (float)p.ppl_up : (ppl_sign < 0 ? (float)p.ppl_down : 1.0f);
+  r.q_lo = (float)p.q_lo;
+  r.q_hi = (float)p.q_hi;
+  r.eps = (float)p.eps;
+  r.temperature = (float)p.temperature;
+  r.clamp = p.clamp_enabled;
+  r.c_mode = p.c_mode;
+  return r;
+}
+
+size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+eat_status check_call(eat_handle* h, const void* x, int32_t T, int32_t ppl_sign) {
+  if (!h) return fail(nullptr, EAT_ERR_INVALID_ARG, "null handle");
+  if (!x) return fail(h, EAT_ERR_INVALID_ARG, "x is NULL");
+  if (T < 1 || T > h->Tmax)
+    return fail(h, EAT_ERR_INVALID_ARG,
+                "T=" + std::to_string(T) + " outside [1, max_tokens=" + std::to_string(h->Tmax) +
+                    "]");
+  if (ppl_sign < -1 || ppl_sign > 1)
+    return fail(h, EAT_ERR_INVALID_ARG, "ppl_sign must be -1, 0 or +1");
+  return EAT_OK;
+}
+
+// Router + selection into (idx, w, k, psel).
+eat_status run_route(eat_handle* h, const void* x, int T, int ppl_sign, int32_t* idx, float* w,
+                     int32_t* k, float* psel, cudaStream_t st) {
+  const int split = router_split(T, h->d, h->E);
+  EAT_TRY(launch(h, kRoute, st, "router logits", [&] {
+    return launch_router_logits(x, h->bf16, h->desc.w_router, T, h->d, h->E, split,
+                                h->logit_part, st);
+  }));
+  const RouteParams rp = route_params(h->prm, ppl_sign);
+  EAT_TRY(launch(h, kRoute, st, "route select", [&] {
+    return launch_route_select(h->logit_part, split, h->desc.b_router, T, h->E, h->K, h->N, h->P,
+                               h->C, rp, idx, w, k, psel, st);
+  }));
+  return EAT_OK;
+}
+
+eat_status run_forward(eat_handle* h, const void* x, int T, int ppl_sign, void* y,
+                       int32_t* idx_opt, float* w_opt, int32_t* k_opt, cudaStream_t st) {
+  EAT_TRY(run_route(h, x, T, ppl_sign, h->idx, h->w, h->k, h->psel, st));
+  const int tile_rows = h->backend == 1 ? tc_tile_rows(h->tc, T) : kSimtTileRows;
+  EAT_TRY(launch(h, kPermute, st, "permute", [&] {
+    return launch_permute(h->idx, h->k, h->psel, T, h->K, h->E, tile_rows, h->perm, st);
+  }));
+  const int rows = T * h->K;
+  int n_split = 1;
+  if (h->backend == 1) {
+    TcCall c;
+    c.x = x;
+    c.T = T;
+    c.tile_rows = tile_rows;
+    c.offs = h->perm.offs;
+    c.tile_offs = h->perm.tile_offs;
+    c.perm_tok = h->perm.perm_tok;
+    c.act = h->act;
+    c.opart = h->opart;
+    c.sact = h->sact;
+    c.sout = h->sout;
+    c.max_split = h->max_split;
+    n_split = tc_down_split(h->tc, T);
+    EAT_TRY(launch(h, kUp, st, "tc gate/up", [&] { return tc_launch_up(h->tc, c, false, st); }));
+    EAT_TRY(launch(h, kDown, st, "tc down",
+                   [&] { return tc_launch_down(h->tc, c, false, n_split, st); }));
+    if (h->S > 0) {
+      EAT_TRY(launch(h, kSUp, st, "tc shared gate/up",
+                     [&] { return tc_launch_up(h->tc, c, true, st); }));
+      EAT_TRY(launch(h, kSDown, st, "tc shared down",
+                     [&] { return tc_launch_down(h->tc, c, true, 1, st); }));
+    }
+  } else {
+    GroupMap gm{h->perm.offs, h->perm.tile_offs, h->perm.perm_tok, kRowGather, h->E, 0,
+                (rows + kSimtTileRows - 1) / kSimtTileRows + h->E};
+    EAT_TRY(launch(h, kUp, st, "ffn gate/up", [&] {
+      return launch_ffn_gateup_simt(h->bf16, x, h->desc.w_gate, h->desc.w_up, h->F, h->d, gm,
+                                    h->act, st);
+    }));
+    EAT_TRY(launch(h, kDown, st, "ffn down", [&] {
+      return launch_ffn_down_simt(h->bf16, h->act, h->desc.w_down, h->d, h->F, gm, h->opart, st);
+    }));
+    if (h->S > 0) {
+      const int tpg = (T + kSimtTileRows - 1) / kSimtTileRows;
+      GroupMap gs{nullptr, nullptr, nullptr, kRowIdentity, h->S, T, tpg * h->S};
+      EAT_TRY(launch(h, kSUp, st, "shared gate/up", [&] {
+        return launch_ffn_gateup_simt(h->bf16, x, h->desc.ws_gate, h->desc.ws_up, h->Fs, h->d,
+                                      gs, h->sact, st);
+      }));
+      EAT_TRY(launch(h, kSDown, st, "shared down", [&] {
+        return launch_ffn_down_simt(h->bf16, h->sact, h->desc.ws_down, h->d, h->Fs, gs, h->sout,
+                                    st);
+      }));
+    }
+  }
+  EAT_TRY(launch(h, kCombine, st, "combine", [&] {
+    return launch_combine(h->bf16, h->opart, n_split, h->Tmax * h->K, h->perm.slot_of, h->w,
+                          h->k, h->sout, h->S, T, h->K, h->d, y, h->onorm, st);
+  }));
+  EAT_TRY(launch(h, kAccount, st, "account update", [&] {
+    return launch_account(h->perm.offs, h->perm.perm_p, h->onorm, h->E, h->prm.alpha, h->N, h->P,
+                          h->C, h->st_n, h->st_p, h->st_norm, h->counters, st);
+  }));
+  if (idx_opt || w_opt || k_opt) {
+    cudaError_t e = cudaSuccess;
+    if (idx_opt && e == cudaSuccess)
+      e = cudaMemcpyAsync(idx_opt, h->idx, sizeof(int32_t) * rows, cudaMemcpyDeviceToDevice, st);
+    if (w_opt && e == cudaSuccess)
+      e = cudaMemcpyAsync(w_opt, h->w, sizeof(float) * rows, cudaMemcpyDeviceToDevice, st);
+    if (k_opt && e == cudaSuccess)
+      e = cudaMemcpyAsync(k_opt, h->k, sizeof(int32_t) * T, cudaMemcpyDeviceToDevice, st);
+    if (e != cudaSuccess) return cuda_fail(h, e, "routing copy-out");
+  }
+  return EAT_OK;
+}
+
+void free_handle(eat_handle* h) {
+  if (!h) return;
+  for (cudaEvent_t e : h->ev) cudaEventDestroy(e);
+  tc_destroy(h->tc);
+  if (h->mem) cudaFree(h->mem);
+  delete h;
+}
+
+}  // namespace
+
+extern "C" {
+
+eat_status eat_default_params(eat_params* p) {
+  if (!p) return fail(nullptr, EAT_ERR_INVALID_ARG, "params is NULL");
+  p->alpha = 0.95;
+  p->w1 = 0.3;
+  p->w2 = 0.3;
+  p->w3 = 0.4;
+  p->beta = 0.6;
+  p->alpha1 = 0.5;
+  p->alpha2 = 1.0;
+  p->kappa1 = 0.7;
+  p->kappa2 = 0.3;
+  p->ppl_up = 1.2;
+  p->ppl_down = 0.9;
+  p->q_lo = 0.10;
+  p->q_hi = 0.90;
+  p->eps = 1e-8;
+  p->temperature = 1.0;
+  p->max_k = 2;
+  p->clamp_enabled = 1;
+  p->c_mode = EAT_C_SUM;
+  return EAT_OK;
+}
+
+eat_status eat_create(const eat_layer_desc* desc, const eat_params* params, eat_handle** out) {
+  if (!out) return fail(nullptr, EAT_ERR_INVALID_ARG, "out is NULL");
+  *out = nullptr;
+  if (!desc || !params) return fail(nullptr, EAT_ERR_INVALID_ARG, "desc or params is NULL");
+  const eat_layer_desc& D = *desc;
+  const eat_params& Pm = *params;
+  if (D.n_experts < 1 || D.n_experts > kMaxExperts)
+    return fail(nullptr, EAT_ERR_UNSUPPORTED, "n_experts must be in [1, 256]");
+  if (D.d_model < 64 || D.d_model % 64 || D.d_ff < 64 || D.d_ff % 64)
+    return fail(nullptr, EAT_ERR_UNSUPPORTED, "d_model and d_ff must be positive multiples of 64");
+  if (D.n_shared < 0 || (D.n_shared > 0 && (D.d_ff_shared < 64 || D.d_ff_shared % 64)))
+    return fail(nullptr, EAT_ERR_UNSUPPORTED, "d_ff_shared must be a positive multiple of 64");
+  if (D.max_tokens < 1 || D.max_tokens > 65536)
+    return fail(nullptr, EAT_ERR_INVALID_ARG, "max_tokens must be in [1, 65536]");
+  if (!((D.wdtype == EAT_F32 && D.xdtype == EAT_F32) ||
+        (D.wdtype == EAT_BF16 && D.xdtype == EAT_BF16)))
+    return fail(nullptr, EAT_ERR_UNSUPPORTED, "wdtype and xdtype must both be F32 or both BF16");
+  if (!D.w_router || !D.w_gate || !D.w_up || !D.w_down)
+    return fail(nullptr, EAT_ERR_INVALID_ARG, "router or expert weight pointer is NULL");
+  if (D.n_shared > 0 && (!D.ws_gate || !D.ws_up || !D.ws_down))
+    return fail(nullptr, EAT_ERR_INVALID_ARG, "shared expert weight pointer is NULL");
+  const uintptr_t al = (uintptr_t)D.w_gate | (uintptr_t)D.w_up | (uintptr_t)D.w_down |
+                       (uintptr_t)(D.n_shared > 0 ? ((uintptr_t)D.ws_gate | (uintptr_t)D.ws_up |
+                                                     (uintptr_t)D.ws_down)
+                                                  : 0);
+  if (al & 15) return fail(nullptr, EAT_ERR_INVALID_ARG, "weights must be 16-byte aligned");
+  if (Pm.max_k < 1 || Pm.max_k > kMaxK || Pm.max_k > D.n_experts)
+    return fail(nullptr, EAT_ERR_INVALID_ARG, "max_k must be in [1, min(E, 16)]");
+  if (!(Pm.temperature > 0.0)) return fail(nullptr, EAT_ERR_INVALID_ARG, "temperature <= 0");
+  if (!(Pm.alpha >= 0.0 && Pm.alpha <= 1.0))
+    return fail(nullptr, EAT_ERR_INVALID_ARG, "alpha outside [0, 1]");
+  if (!(Pm.q_lo >= 0.0 && Pm.q_lo <= Pm.q_hi && Pm.q_hi <= 1.0))
+    return fail(nullptr, EAT_ERR_INVALID_ARG, "need 0 <= q_lo <= q_hi <= 1");
+  if (Pm.c_mode != EAT_C_SUM && Pm.c_mode != EAT_C_RAW)
+    return fail(nullptr, EAT_ERR_INVALID_ARG, "bad c_mode");
+
+  eat_handle* h = new (std::nothrow) eat_handle();
+  if (!h) return fail(nullptr, EAT_ERR_OOM, "host allocation failed");
+  h->desc = D;
+  h->prm = Pm;
+  h->E = D.n_experts;
+  h->d = D.d_model;
+  h->F = D.d_ff;
+  h->S = D.n_shared;
+  h->Fs = D.n_shared > 0 ? D.d_ff_shared : 0;
+  h->Tmax = D.max_tokens;
+  h->K = Pm.max_k;
+  h->bf16 = D.wdtype == EAT_BF16;
+  h->elt = h->bf16 ? 2 : 4;
+  h->backend = 0;
+
+  if (h->backend == 1) {
+    const char* msg = nullptr;
+    if (tc_init(h->tc, D, h->K, h->Tmax, &msg) != 0) {
+      std::string m = msg ? msg : "tensor-core setup failed";
+      free_handle(h);
+      return fail(nullptr, EAT_ERR_CUDA, m);
+    }
+    h->max_split = tc_max_split(h->tc);
+  }
+
+  int max_lsplit = 0;
+  for (int T = 1; T <= h->Tmax; ++T)
+    max_lsplit = std::max(max_lsplit, router_split(T, h->d, h->E) * T);
+
+  const size_t rows = (size_t)h->Tmax * h->K;
+  struct Part { void** p; size_t bytes; };
+  std::vector<Part> parts;
+  auto add = [&](void* pp, size_t bytes) { parts.push_back({(void**)pp, bytes}); };
+  add(&h->N, sizeof(int64_t) * h->E);
+  add(&h->P, sizeof(double) * h->E);
+  add(&h->C, sizeof(double) * h->E);
+  add(&h->st_n, sizeof(int32_t) * h->E);
+  add(&h->st_p, sizeof(double) * h->E);
+  add(&h->st_norm, sizeof(double) * h->E);
+  add(&h->counters, sizeof(long long) * 4);
+  add(&h->logit_part, sizeof(float) * (size_t)max_lsplit * h->E);
+  add(&h->idx, sizeof(int32_t) * rows);
+  add(&h->w, sizeof(float) * rows);
+  add(&h->k, sizeof(int32_t) * h->Tmax);
+  add(&h->psel, sizeof(float) * rows);
+  add(&h->perm.n_e, sizeof(int32_t) * h->E);
+  add(&h->perm.offs, sizeof(int32_t) * (h->E + 1));
+  add(&h->perm.tile_offs, sizeof(int32_t) * (h->E + 1));
+  add(&h->perm.perm_tok, sizeof(int32_t) * rows);
+  add(&h->perm.slot_of, sizeof(int32_t) * rows);
+  add(&h->perm.perm_p, sizeof(float) * rows);
+  add(&h->perm.active, sizeof(int32_t) * (h->E + 1));
+  add(&h->act, h->elt * rows * h->F);
+  add(&h->opart, sizeof(float) * (size_t)h->max_split * rows * h->d);
+  add(&h->onorm, sizeof(float) * rows);
+  if (h->S > 0) {
+    add(&h->sact, h->elt * (size_t)h->S * h->Tmax * h->Fs);
+    add(&h->sout, sizeof(float) * (size_t)h->S * h->Tmax * h->d);
+  }
+  add(&h->xstage, h->elt * (size_t)h->Tmax * h->d);
+  add(&h->ystage, h->elt * (size_t)h->Tmax * h->d);
+  size_t total = 0;
+  for (auto& p : parts) total = align_up(total, 256) + align_up(p.bytes, 256);
+  cudaError_t e = cudaMalloc(&h->mem, total);
+  if (e != cudaSuccess) {
+    free_handle(h);
+    return fail(nullptr, EAT_ERR_OOM,
+                "cudaMalloc of " + std::to_string(total) + " bytes failed: " +
+                    cudaGetErrorString(e));
+  }
+  size_t off = 0;
+  for (auto& p : parts) {
+    off = align_up(off, 256);
+    *p.p = (char*)h->mem + off;
+    off += align_up(p.bytes, 256);
+  }
+  e = cudaMemset(h->mem, 0, total);
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) {
+    free_handle(h);
+    return fail(nullptr, EAT_ERR_CUDA, std::string("workspace init: ") + cudaGetErrorString(e));
+  }
+  *out = h;
+  return EAT_OK;
+}
+
+eat_status eat_reset_accounts(eat_handle* h, void* stream) {
+  if (!h) return fail(nullptr, EAT_ERR_INVALID_ARG, "null handle");
+  cudaStream_t st = (cudaStream_t)stream;
+  cudaError_t e = cudaMemsetAsync(h->N, 0, sizeof(int64_t) * h->E, st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(h->P, 0, sizeof(double) * h->E, st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(h->C, 0, sizeof(double) * h->E, st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(h->counters, 0, sizeof(long long) * 4, st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "reset accounts");
+  h->launches = 0;
+  return EAT_OK;
+}
+
+eat_status eat_route(eat_handle* h, const void* x, int32_t T, int32_t ppl_sign, int32_t* idx,
+                     float* w, int32_t* k, void* stream) {
+  EAT_TRY(check_call(h, x, T, ppl_sign));
+  if (!idx || !w || !k) return fail(h, EAT_ERR_INVALID_ARG, "idx, w and k must be non-NULL");
+  return run_route(h, x, T, ppl_sign, idx, w, k, nullptr, (cudaStream_t)stream);
+}
+
+eat_status eat_moe_forward(eat_handle* h, const void* x, int32_t T, int32_t ppl_sign, void* y,
+                           int32_t* idx_opt, float* w_opt, int32_t* k_opt, void* stream) {
+  EAT_TRY(check_call(h, x, T, ppl_sign));
+  if (!y) return fail(h, EAT_ERR_INVALID_ARG, "y is NULL");
+  if (y == x) return fail(h, EAT_ERR_INVALID_ARG, "y must not alias x");
+  return run_forward(h, x, T, ppl_sign, y, idx_opt, w_opt, k_opt, (cudaStream_t)stream);
+}
+
+eat_status eat_moe_forward_host(eat_handle* h, const void* x_host, int32_t T, int32_t ppl_sign,
+                                void* y_host, void* stream) {
+  EAT_TRY(check_call(h, x_host, T, ppl_sign));
+  if (!y_host) return fail(h, EAT_ERR_INVALID_ARG, "y_host is NULL");
+  cudaStream_t st = (cudaStream_t)stream;
+  const size_t bytes = h->elt * (size_t)T * h->d;
+  cudaError_t e = cudaMemcpyAsync(h->xstage, x_host, bytes, cudaMemcpyHostToDevice, st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "x host-to-device copy");
+  EAT_TRY(run_forward(h, h->xstage, T, ppl_sign, h->ystage, nullptr, nullptr, nullptr, st));
+  e = cudaMemcpyAsync(y_host, h->ystage, bytes, cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "y device-to-host copy");
+  return EAT_OK;
+}
+
+eat_status eat_destroy(eat_handle* h) {
+  if (!h) return EAT_OK;
+  cudaDeviceSynchronize();
+  free_handle(h);
+  return EAT_OK;
+}
+
+eat_status eat_get_accounts(eat_handle* h, int64_t* N, double* P, double* C, void* stream) {
+  if (!h) return fail(nullptr, EAT_ERR_INVALID_ARG, "null handle");
+  if (!N || !P || !C) return fail(h, EAT_ERR_INVALID_ARG, "N, P and C must be non-NULL");
+  cudaStream_t st = (cudaStream_t)stream;
+  cudaError_t e = cudaMemcpyAsync(N, h->N, sizeof(int64_t) * h->E, cudaMemcpyDeviceToDevice, st);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(P, h->P, sizeof(double) * h->E, cudaMemcpyDeviceToDevice, st);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(C, h->C, sizeof(double) * h->E, cudaMemcpyDeviceToDevice, st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "get accounts");
+  return EAT_OK;
+}
+
+eat_status eat_set_accounts(eat_handle* h, const int64_t* N, const double* P, const double* C,
+                            void* stream) {
+  if (!h) return fail(nullptr, EAT_ERR_INVALID_ARG, "null handle");
+  if (!N || !P || !C) return fail(h, EAT_ERR_INVALID_ARG, "N, P and C must be non-NULL");
+  cudaStream_t st = (cudaStream_t)stream;
+  cudaError_t e = cudaMemcpyAsync(h->N, N, sizeof(int64_t) * h->E, cudaMemcpyDeviceToDevice, st);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(h->P, P, sizeof(double) * h->E, cudaMemcpyDeviceToDevice, st);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(h->C, C, sizeof(double) * h->E, cudaMemcpyDeviceToDevice, st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "set accounts");
+  return EAT_OK;
+}
+
+eat_status eat_get_call_stats(eat_handle* h, int32_t* n_e, double* sum_p, double* sum_norm,
+                              void* stream) {
+  if (!h) return fail(nullptr, EAT_ERR_INVALID_ARG, "null handle");
+  cudaStream_t st = (cudaStream_t)stream;
+  cudaError_t e = cudaSuccess;
+  if (n_e) e = cudaMemcpyAsync(n_e, h->st_n, sizeof(int32_t) * h->E, cudaMemcpyDeviceToDevice, st);
+  if (sum_p && e == cudaSuccess)
+    e = cudaMemcpyAsync(sum_p, h->st_p, sizeof(double) * h->E, cudaMemcpyDeviceToDevice, st);
+  if (sum_norm && e == cudaSuccess)
+    e = cudaMemcpyAsync(sum_norm, h->st_norm, sizeof(double) * h->E, cudaMemcpyDeviceToDevice,
+                        st);
+  if (e != cudaSuccess) return cuda_fail(h, e, "get call stats");
+  return EAT_OK;
+}
+
+eat_status eat_get_counters(eat_handle* h, int64_t* out, int32_t n) {
+  if (!h) return fail(nullptr, EAT_ERR_INVALID_ARG, "null handle");
+  if (!out || n < 0) return fail(h, EAT_ERR_INVALID_ARG, "out is NULL or n < 0");
+  long long dev[4] = {0, 0, 0, 0};
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e == cudaSuccess) e = cudaMemcpy(dev, h->counters, sizeof(dev), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(h, e, "get counters");
+  const long long vals[4] = {dev[0], dev[1], dev[2], h->launches};
+  for (int i = 0; i < n && i < 4; ++i) out[i] = vals[i];
+  return EAT_OK;
+}
+
+eat_status eat_profile_begin(eat_handle* h, int32_t capacity) {
+  if (!h) return fail(nullptr, EAT_ERR_INVALID_ARG, "null handle");
+  if (capacity < 1) return fail(h, EAT_ERR_INVALID_ARG, "capacity < 1");
+  while ((int)h->ev.size() < 2 * capacity) {
+    cudaEvent_t e;
+    const cudaError_t r = cudaEventCreate(&e);
+    if (r != cudaSuccess) return cuda_fail(h, r, "event create");
+    h->ev.push_back(e);
+  }
+  h->ev_kind.assign(capacity, 0);
+  h->prof_cap = capacity;
+  h->prof_n = 0;
+  h->prof = true;
+  return EAT_OK;
+}
+
+eat_status eat_profile_end(eat_handle* h, double* ms, int64_t* launches, int32_t n) {
+  if (!h) return fail(nullptr, EAT_ERR_INVALID_ARG, "null handle");
+  if (!h->prof) return fail(h, EAT_ERR_STATE, "profiling was not started");
+  h->prof = false;
+  std::vector<double> acc(kKinds, 0.0);
+  std::vector<long long> cnt(kKinds, 0);
+  if (h->prof_n > 0) {
+    const cudaError_t r = cudaEventSynchronize(h->ev[2 * h->prof_n - 1]);
+    if (r != cudaSuccess) return cuda_fail(h, r, "event synchronize");
+  }
+  for (int i = 0; i < h->prof_n; ++i) {
+    float m = 0.f;
+    cudaEventElapsedTime(&m, h->ev[2 * i], h->ev[2 * i + 1]);
+    acc[h->ev_kind[i]] += m;
+    cnt[h->ev_kind[i]] += 1;
+  }
+  for (int i = 0; i < n && i < kKinds; ++i) {
+    if (ms) ms[i] = acc[i];
+    if (launches) launches[i] = cnt[i];
+  }
+  h->prof_n = 0;
+  return EAT_OK;
+}
+
+int32_t eat_ffn_backend(const eat_handle* h) { return h ? h->backend : -1; }
+
+const char* eat_last_error(const eat_handle* h) {
+  if (!h) return g_err.empty() ? "no error recorded" : g_err.c_str();
+  return h->err.empty() ? "no error recorded" : h->err.c_str();
+}
+
+const char* eat_status_string(eat_status s) {
+  switch (s) {
+    case EAT_OK: return "EAT_OK";
+    case EAT_ERR_INVALID_ARG: return "EAT_ERR_INVALID_ARG";
+    case EAT_ERR_UNSUPPORTED: return "EAT_ERR_UNSUPPORTED";
+    case EAT_ERR_OOM: return "EAT_ERR_OOM";
+    case EAT_ERR_CUDA: return "EAT_ERR_CUDA";
+    case EAT_ERR_STATE: return "EAT_ERR_STATE";
+  }
+  return "EAT_UNKNOWN_STATUS";
+}
+
+}  // extern "C"

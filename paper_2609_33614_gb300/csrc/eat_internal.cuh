@@ -1,0 +1,87 @@
+// Internal declarations shared by the translation units of libeat.so.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "../../include/eat.h"
+
+namespace eat {
+
+constexpr int kMaxExperts = 256;
+constexpr int kMaxK = 16;
+
+// ---------------------------------------------------------------------------------------------
+// Router (§3.1-§3.4)
+// ---------------------------------------------------------------------------------------------
+struct RouteParams {
+  float w1, w2, w3, beta, alpha1, alpha2, kappa1, kappa2, ppl_factor, q_lo, q_hi, eps,
+      temperature;
+  int clamp, c_mode;
+};
+
+// Partial router logits: part[s][t][e] = sum over the s-th slice of d of x[t, j] * Wr[e, j].
+cudaError_t launch_router_logits(const void* x, int x_bf16, const float* w_router, int T, int d,
+                                 int E, int n_split, float* part, cudaStream_t st);
+// Warp-per-token softmax + history score + threshold + selection + renormalisation.
+cudaError_t launch_route_select(const float* part, int n_split, const float* b_router, int T,
+                                int E, int K, const int64_t* accN, const double* accP,
+                                const double* accC, RouteParams rp, int32_t* idx, float* w,
+                                int32_t* k, float* psel, cudaStream_t st);
+int router_split(int T, int d, int E);
+
+// ---------------------------------------------------------------------------------------------
+// Permute by expert
+// ---------------------------------------------------------------------------------------------
+struct PermuteOut {
+  int32_t* n_e;        // [E]
+  int32_t* offs;       // [E+1] slot offsets per expert
+  int32_t* tile_offs;  // [E+1] prefix of ceil(n_e / tile_rows)
+  int32_t* perm_tok;   // [T*K] token of each slot
+  int32_t* slot_of;    // [T*K] slot of (t, j), -1 for j >= k_t
+  float* perm_p;       // [T*K] p of each slot
+  int32_t* active;     // [E+1] ascending active experts, active[E] = count
+};
+cudaError_t launch_permute(const int32_t* idx, const int32_t* k, const float* psel, int T, int K,
+                           int E, int tile_rows, PermuteOut o, cudaStream_t st);
+
+// ---------------------------------------------------------------------------------------------
+// Expert FFNs
+// ---------------------------------------------------------------------------------------------
+// Rows ("slots") of group g are row_offs[g] .. row_offs[g+1]-1, or g*uniform_rows ..
+// (g+1)*uniform_rows-1 when row_offs == nullptr.  Which input row feeds slot s:
+//   kRowGather:   in[row_tok[s]]            (routed experts: gather the token's hidden state)
+//   kRowSlot:     in[s]                     (down projection: act rows are in slot order)
+//   kRowIdentity: in[s - g*uniform_rows]    (shared experts: every token in order)
+enum RowMode { kRowGather = 0, kRowSlot = 1, kRowIdentity = 2 };
+struct GroupMap {
+  const int32_t* row_offs;   // [G+1] or nullptr (uniform)
+  const int32_t* tile_offs;  // [G+1] prefix of row tiles, or nullptr (uniform)
+  const int32_t* row_tok;    // [rows] gather index (kRowGather)
+  int row_mode;
+  int n_groups;
+  int uniform_rows;          // rows per group when row_offs == nullptr
+  int max_tiles;             // upper bound of the total number of row tiles (grid size)
+};
+
+// act[slot, f] = silu(sum_j in[row, j] Wg[g, f, j]) * (sum_j in[row, j] Wu[g, f, j])
+cudaError_t launch_ffn_gateup_simt(int dtype_bf16, const void* in, const void* wg, const void* wu,
+                                   int Fout, int Kdim, GroupMap gm, void* act, cudaStream_t st);
+// out[slot, c] = sum_f act[slot, f] Wd[g, c, f]   (fp32 output)
+cudaError_t launch_ffn_down_simt(int dtype_bf16, const void* act, const void* wd, int Dout,
+                                 int Kdim, GroupMap gm, float* out, cudaStream_t st);
+constexpr int kSimtTileRows = 32;
+
+// ---------------------------------------------------------------------------------------------
+// Combine / unpermute and account update
+// ---------------------------------------------------------------------------------------------
+cudaError_t launch_combine(int y_bf16, const float* opart, int n_split, int split_stride_rows,
+                           const int32_t* slot_of, const float* w, const int32_t* k,
+                           const float* sout, int S, int T, int K, int d, void* y, float* onorm,
+                           cudaStream_t st);
+cudaError_t launch_account(const int32_t* offs, const float* perm_p, const float* onorm, int E,
+                           double alpha, int64_t* N, double* P, double* C, int32_t* st_n,
+                           double* st_p, double* st_norm, long long* counters, cudaStream_t st);
+
+}  // namespace eat

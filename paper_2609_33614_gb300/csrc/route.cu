@@ -1,0 +1,376 @@
+// Router and EAT selection (§3.1-§3.4 of the EAT paper, Eq. 1-8).
+//
+//  router_logits_kernel: partial router scores x . w_r over slices of d, fp32 FMA in a fixed
+//      order (a [T, E] GEMM too small and too precision-sensitive for the bf16 tensor path:
+//      the selection compares I against tau at 1e-5).
+//  route_select_kernel: one warp per token.  Each lane owns experts lane, lane+32, ...; the warp
+//      does the softmax (§3.2), importance (Eq. 2), mean / population std (Eq. 3-4), tau (Eq. 5),
+//      PPL factor and smoothing (§3.3), the clamp to the type-7 q_lo / q_hi quantiles of p
+//      (order statistics by in-warp rank counting, no sort), the candidate set and K cap
+//      (Eq. 6, ties to the lower index) and the renormalised gates (Eq. 7-8), with shuffles only.
+//      The history score S_h (Eq. 1) is computed once per block in fp64 from the accounts.
+#include "eat_internal.cuh"
+
+#include <math.h>
+
+namespace eat {
+
+namespace {
+
+constexpr int kChunk = 32;
+constexpr int kLogitThreads = 256;
+constexpr int kMaxOut = 8;  // outputs per thread in the logits kernel
+
+__device__ __forceinline__ float load_x(const float* p, size_t i) { return p[i]; }
+__device__ __forceinline__ float load_x(const __nv_bfloat16* p, size_t i) {
+  return __bfloat162float(p[i]);
+}
+
+int logits_tile_tokens(int E) {
+  int tt = (kLogitThreads * kMaxOut) / E;
+  if (tt > 32) tt = 32;
+  if (tt < 1) tt = 1;
+  return tt;
+}
+
+template <typename TX>
+__global__ void __launch_bounds__(kLogitThreads)
+router_logits_kernel(const TX* __restrict__ x, const float* __restrict__ wr, int T, int d, int E,
+                     int TT, int d_per_split, float* __restrict__ part) {
+  extern __shared__ float sm[];
+  float* xs = sm;                        // [TT][kChunk + 1]
+  float* ws = sm + TT * (kChunk + 1);    // [E][kChunk + 1]
+  const int tid = threadIdx.x;
+  const int t0 = blockIdx.x * TT;
+  const int dbeg = blockIdx.y * d_per_split;
+  const int dend = min(d, dbeg + d_per_split);
+  const int n_out = TT * E;
+  float acc[kMaxOut];
+#pragma unroll
+  for (int q = 0; q < kMaxOut; ++q) acc[q] = 0.f;
+
+  for (int j0 = dbeg; j0 < dend; j0 += kChunk) {
+    for (int i = tid; i < TT * kChunk; i += kLogitThreads) {
+      const int tt = i / kChunk, jj = i % kChunk;
+      const int t = t0 + tt, j = j0 + jj;
+      xs[tt * (kChunk + 1) + jj] = (t < T && j < dend) ? load_x(x, (size_t)t * d + j) : 0.f;
+    }
+    for (int i = tid; i < E * kChunk; i += kLogitThreads) {
+      const int e = i / kChunk, jj = i % kChunk;
+      const int j = j0 + jj;
+      ws[e * (kChunk + 1) + jj] = (j < dend) ? wr[(size_t)e * d + j] : 0.f;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int q = 0; q < kMaxOut; ++q) {
+      const int o = tid + q * kLogitThreads;
+      if (o < n_out) {
+        const int tt = o / E, e = o % E;
+        const float* xr = xs + tt * (kChunk + 1);
+        const float* wrow = ws + e * (kChunk + 1);
+        float a = acc[q];
+#pragma unroll
+        for (int jj = 0; jj < kChunk; ++jj) a = fmaf(xr[jj], wrow[jj], a);
+        acc[q] = a;
+      }
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int q = 0; q < kMaxOut; ++q) {
+    const int o = tid + q * kLogitThreads;
+    if (o < n_out) {
+      const int tt = o / E, e = o % E;
+      const int t = t0 + tt;
+      if (t < T) part[((size_t)blockIdx.y * T + t) * E + e] = acc[q];
+    }
+  }
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+constexpr int kSelectThreads = 256;
+
+// S_h (Eq. 1) for all experts into smem, fp64 arithmetic, readings: empty-history terms are 0;
+// c_mode 0 uses C_i / sum C, c_mode 1 the raw C_i.
+__device__ void history_score_block(const int64_t* accN, const double* accP, const double* accC,
+                                    int E, const RouteParams& rp, float* s_h) {
+  __shared__ long long red_n[kSelectThreads / 32];
+  __shared__ double red_c[kSelectThreads / 32];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  long long n_sum = 0;
+  double c_sum = 0.0;
+  for (int e = tid; e < E; e += blockDim.x) {
+    n_sum += (long long)accN[e];
+    c_sum += accC[e];
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    n_sum += __shfl_xor_sync(0xffffffffu, n_sum, o);
+    c_sum += __shfl_xor_sync(0xffffffffu, c_sum, o);
+  }
+  if (lane == 0) { red_n[warp] = n_sum; red_c[warp] = c_sum; }
+  __syncthreads();
+  if (tid == 0) {
+    long long a = 0;
+    double b = 0.0;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) { a += red_n[w]; b += red_c[w]; }
+    red_n[0] = a;
+    red_c[0] = b;
+  }
+  __syncthreads();
+  const double total_n = (double)red_n[0];
+  const double total_c = red_c[0];
+  for (int e = tid; e < E; e += blockDim.x) {
+    const double n = (double)accN[e];
+    const double a = total_n > 0.0 ? n / total_n : 0.0;
+    const double b = n > 0.0 ? accP[e] / n : 0.0;
+    double c;
+    if (rp.c_mode == EAT_C_RAW) c = accC[e];
+    else c = total_c > 0.0 ? accC[e] / total_c : 0.0;
+    s_h[e] = (float)((double)rp.w1 * a + (double)rp.w2 * b + (double)rp.w3 * c);
+  }
+  __syncthreads();
+}
+
+// Value of rank r (0-based ascending, ties by index) among the token's probabilities.
+template <int EPL>
+__device__ __forceinline__ float order_stat(const float (&p)[EPL], const int (&rank)[EPL],
+                                            const bool (&valid)[EPL], int r) {
+  float v = 0.f;
+#pragma unroll
+  for (int i = 0; i < EPL; ++i) v += (valid[i] && rank[i] == r) ? p[i] : 0.f;
+  return warp_sum(v);  // exactly one lane-element matches: the sum is that value
+}
+
+template <int EPL>
+__global__ void __launch_bounds__(kSelectThreads)
+route_select_kernel(const float* __restrict__ part, int n_split, const float* __restrict__ bias,
+                    int T, int E, int K, const int64_t* __restrict__ accN,
+                    const double* __restrict__ accP, const double* __restrict__ accC,
+                    RouteParams rp, int32_t* __restrict__ out_idx, float* __restrict__ out_w,
+                    int32_t* __restrict__ out_k, float* __restrict__ out_p) {
+  __shared__ float s_h[kMaxExperts];
+  history_score_block(accN, accP, accC, E, rp, s_h);
+
+  const int lane = threadIdx.x & 31;
+  const int warps = blockDim.x >> 5;
+  const int t = blockIdx.x * warps + (threadIdx.x >> 5);
+  if (t >= T) return;
+  const unsigned full = 0xffffffffu;
+  const float inv_e = 1.0f / (float)E;
+
+  float p[EPL], I[EPL];
+  bool valid[EPL];
+  float lmax = -INFINITY;
+#pragma unroll
+  for (int i = 0; i < EPL; ++i) {
+    const int e = lane + 32 * i;
+    valid[i] = e < E;
+    float z = -INFINITY;
+    if (valid[i]) {
+      float s = 0.f;
+      for (int sp = 0; sp < n_split; ++sp) s += part[((size_t)sp * T + t) * E + e];
+      if (bias) s += bias[e];
+      z = s / rp.temperature;
+    }
+    p[i] = z;
+    lmax = fmaxf(lmax, z);
+  }
+  // softmax (§3.2): p = exp(z - max) / sum
+  const float m = warp_max(lmax);
+  float ssum = 0.f;
+#pragma unroll
+  for (int i = 0; i < EPL; ++i) {
+    p[i] = valid[i] ? expf(p[i] - m) : 0.f;
+    ssum += p[i];
+  }
+  ssum = warp_sum(ssum);
+  float psum = 0.f;
+#pragma unroll
+  for (int i = 0; i < EPL; ++i) {
+    p[i] = valid[i] ? p[i] / ssum : 0.f;
+    psum += p[i];
+  }
+  // Eq. 3-4: mean and population standard deviation of g = p
+  const float mu = warp_sum(psum) * inv_e;
+  float dev = 0.f;
+#pragma unroll
+  for (int i = 0; i < EPL; ++i) {
+    const float dlt = valid[i] ? p[i] - mu : 0.f;
+    dev += dlt * dlt;
+  }
+  const float sigma = sqrtf(warp_sum(dev) * inv_e);
+  // Eq. 5, PPL adjustment and smoothing (§3.3)
+  const float tau = fmaxf(rp.alpha1 * mu, mu - rp.alpha2 * sigma);
+  float tau_f = rp.kappa1 * (rp.ppl_factor * tau) + rp.kappa2 * tau;
+
+  int rank[EPL];
+#pragma unroll
+  for (int i = 0; i < EPL; ++i) rank[i] = 0;
+  if (rp.clamp) {
+    // rank of each p among all E (ascending, ties by index): sort-free order statistics
+#pragma unroll
+    for (int jb = 0; jb < EPL; ++jb) {
+      for (int jl = 0; jl < 32; ++jl) {
+        const int ej = jb * 32 + jl;
+        const float pj = __shfl_sync(full, p[jb], jl);
+        if (ej < E) {
+#pragma unroll
+          for (int i = 0; i < EPL; ++i) {
+            const int ei = lane + 32 * i;
+            rank[i] += (pj < p[i] || (pj == p[i] && ej < ei)) ? 1 : 0;
+          }
+        }
+      }
+    }
+    const float h_lo = (float)(E - 1) * rp.q_lo;
+    const float h_hi = (float)(E - 1) * rp.q_hi;
+    const int lo0 = (int)floorf(h_lo), hi0 = (int)floorf(h_hi);
+    const int lo1 = min(lo0 + 1, E - 1), hi1 = min(hi0 + 1, E - 1);
+    const float v_lo0 = order_stat<EPL>(p, rank, valid, lo0);
+    const float v_lo1 = order_stat<EPL>(p, rank, valid, lo1);
+    const float v_hi0 = order_stat<EPL>(p, rank, valid, hi0);
+    const float v_hi1 = order_stat<EPL>(p, rank, valid, hi1);
+    const float q_lo = v_lo0 + (h_lo - (float)lo0) * (v_lo1 - v_lo0);
+    const float q_hi = v_hi0 + (h_hi - (float)hi0) * (v_hi1 - v_hi0);
+    tau_f = fminf(fmaxf(tau_f, q_lo), q_hi);
+  }
+
+  // Eq. 2 importance and Eq. 6 candidate set
+  bool cand[EPL];
+  int ncand = 0;
+#pragma unroll
+  for (int i = 0; i < EPL; ++i) {
+    const int e = lane + 32 * i;
+    I[i] = valid[i] ? (1.f - rp.beta) * p[i] + rp.beta * s_h[e] : -INFINITY;
+    cand[i] = valid[i] && I[i] > tau_f;
+    ncand += __popc(__ballot_sync(full, cand[i]));
+  }
+  bool sel[EPL];
+  if (ncand == 0) {
+    // argmax I, lowest index on ties
+    float bv = -INFINITY;
+    int be = 0x7fffffff;
+#pragma unroll
+    for (int i = 0; i < EPL; ++i) {
+      const int e = lane + 32 * i;
+      if (valid[i] && (I[i] > bv || (I[i] == bv && e < be))) { bv = I[i]; be = e; }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float ov = __shfl_xor_sync(full, bv, o);
+      const int oe = __shfl_xor_sync(full, be, o);
+      if (ov > bv || (ov == bv && oe < be)) { bv = ov; be = oe; }
+    }
+#pragma unroll
+    for (int i = 0; i < EPL; ++i) sel[i] = (lane + 32 * i) == be;
+  } else if (ncand <= K) {
+#pragma unroll
+    for (int i = 0; i < EPL; ++i) sel[i] = cand[i];
+  } else {
+    // keep the K largest candidates by (I desc, index asc)
+    int r[EPL];
+#pragma unroll
+    for (int i = 0; i < EPL; ++i) r[i] = 0;
+#pragma unroll
+    for (int jb = 0; jb < EPL; ++jb) {
+      for (int jl = 0; jl < 32; ++jl) {
+        const int ej = jb * 32 + jl;
+        const float Ij = __shfl_sync(full, I[jb], jl);
+        const bool cj = __shfl_sync(full, cand[jb] ? 1 : 0, jl) != 0;
+        if (cj) {
+#pragma unroll
+          for (int i = 0; i < EPL; ++i) {
+            const int ei = lane + 32 * i;
+            r[i] += (Ij > I[i] || (Ij == I[i] && ej < ei)) ? 1 : 0;
+          }
+        }
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < EPL; ++i) sel[i] = cand[i] && r[i] < K;
+  }
+
+  // Eq. 7-8: renormalised gates over the selected experts, g = p
+  float gs = 0.f;
+#pragma unroll
+  for (int i = 0; i < EPL; ++i) gs += sel[i] ? p[i] : 0.f;
+  const float denom = warp_sum(gs) + rp.eps;
+  const unsigned lt = (1u << lane) - 1u;
+  int base = 0;
+  const size_t row = (size_t)t * K;
+#pragma unroll
+  for (int i = 0; i < EPL; ++i) {
+    const unsigned b = __ballot_sync(full, sel[i]);
+    if (sel[i]) {
+      const int pos = base + __popc(b & lt);
+      out_idx[row + pos] = lane + 32 * i;
+      out_w[row + pos] = p[i] / denom;
+      if (out_p) out_p[row + pos] = p[i];
+    }
+    base += __popc(b);
+  }
+  if (lane >= base && lane < K) {
+    out_idx[row + lane] = -1;
+    out_w[row + lane] = 0.f;
+    if (out_p) out_p[row + lane] = 0.f;
+  }
+  if (lane == 0) out_k[t] = base;
+}
+
+}  // namespace
+
+int router_split(int T, int d, int E) {
+  // Enough blocks to cover the SMs when T is small; each slice at least 256 of d.
+  const int tt = logits_tile_tokens(E);
+  const int tblocks = (T + tt - 1) / tt;
+  int split = 1;
+  while (tblocks * split < 2 * 152 && d / (split * 2) >= 256 && split < 64) split *= 2;
+  return split;
+}
+
+cudaError_t launch_router_logits(const void* x, int x_bf16, const float* w_router, int T, int d,
+                                 int E, int n_split, float* part, cudaStream_t st) {
+  const int TT = logits_tile_tokens(E);
+  int per = (d + n_split - 1) / n_split;
+  per = (per + kChunk - 1) / kChunk * kChunk;
+  dim3 grid((T + TT - 1) / TT, n_split);
+  const size_t smem = (size_t)(TT + E) * (kChunk + 1) * sizeof(float);
+  if (x_bf16)
+    router_logits_kernel<__nv_bfloat16><<<grid, kLogitThreads, smem, st>>>(
+        (const __nv_bfloat16*)x, w_router, T, d, E, TT, per, part);
+  else
+    router_logits_kernel<float><<<grid, kLogitThreads, smem, st>>>((const float*)x, w_router, T,
+                                                                    d, E, TT, per, part);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_route_select(const float* part, int n_split, const float* b_router, int T,
+                                int E, int K, const int64_t* accN, const double* accP,
+                                const double* accC, RouteParams rp, int32_t* idx, float* w,
+                                int32_t* k, float* psel, cudaStream_t st) {
+  const int warps = kSelectThreads / 32;
+  dim3 grid((T + warps - 1) / warps);
+#define EAT_SELECT(EPL)                                                                         \
+  route_select_kernel<EPL><<<grid, kSelectThreads, 0, st>>>(part, n_split, b_router, T, E, K,  \
+                                                            accN, accP, accC, rp, idx, w, k,   \
+                                                            psel)
+  if (E <= 32) EAT_SELECT(1);
+  else if (E <= 64) EAT_SELECT(2);
+  else if (E <= 128) EAT_SELECT(4);
+  else EAT_SELECT(8);
+#undef EAT_SELECT
+  return cudaGetLastError();
+}
+
+}  // namespace eat

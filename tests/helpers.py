@@ -28,3 +28,25 @@ def oracle_layer(lw, experts=None):
 
 def oracle_params(shape, **kw):
     return orc.Params(max_k=shape.max_k, temperature=shape.temperature, **kw)
+
+
+class LazyExperts:
+    """Per-expert float64 view of a (possibly device-resident) weight tensor, converted on first
+    use, so sampled oracle checks of large layers only widen the experts they touch."""
+
+    def __init__(self, t):
+        self.t = t
+        self.shape = tuple(t.shape)
+        self.cache = {}
+
+    def __getitem__(self, e):
+        e = int(e)
+        if e not in self.cache:
+            self.cache[e] = np64(self.t[e])
+        return self.cache[e]
+
+
+def oracle_layer_lazy(lw):
+    lz = lambda t: None if t is None else LazyExperts(t)
+    return orc.Layer(np64(lw.w_router), np64(lw.b_router), lz(lw.w_gate), lz(lw.w_up),
+                     lz(lw.w_down), lz(lw.ws_gate), lz(lw.ws_up), lz(lw.ws_down))

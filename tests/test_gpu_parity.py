@@ -1,0 +1,276 @@
+"""GPU-vs-oracle parity of the EAT MoE layer through the C ABI (needs a GB300).
+
+Every case draws seeded inputs (paper_2609_33614_gb300.workloads), runs steps through libeat.so and
+checks each step against the fp64 oracle from the GPU's own pre-step accounts (teacher forcing):
+selections and k bit-exact on non-ambiguous tokens, gates within 1e-5, n_e and N exact, P_total
+and the C_s update rule within 1e-6 relative, C_s against the oracle's norms within 1e-6 (fp32)
+or 2e-2 (bf16), layer outputs within 1e-5 (fp32) or 2e-2 (bf16) max relative error per token.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle.eat_oracle as orc
+from paper_2609_33614_gb300 import eat, workloads as W
+from tests import parity as par
+from tests.helpers import np64, oracle_layer, oracle_layer_lazy
+
+pytestmark = pytest.mark.gpu
+
+Y_TOL = {torch.float32: 1e-5, torch.bfloat16: 2e-2}
+C_TOL = {torch.float32: 1e-6, torch.bfloat16: 2e-2}
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2609_33614_gb300 import build
+    build.build()
+    torch.cuda.set_device(0)
+
+
+def oracle_params(shape, **kw):
+    return orc.Params(max_k=shape.max_k, temperature=shape.temperature, **kw)
+
+
+def gpu_params(shape, **kw):
+    return eat.eat_default_params(shape.max_k, temperature=shape.temperature, **kw)
+
+
+def _acc(layer):
+    N, P, C = layer.accounts()
+    return orc.Accounts(N.cpu().numpy(), P.cpu().numpy(), C.cpu().numpy())
+
+
+def run_parity(shape, lw, Ts, signs=None, prm_kw=None, layer=None, L=None, sample=None,
+               x_device="cpu", max_tokens=None, inputs=None):
+    """Run len(Ts) steps and check each one.  sample: number of tokens whose outputs are checked
+    (None: all).  inputs: optional list of x tensors replacing the seeded draws.  Returns the
+    list of GPU outputs."""
+    prm_kw = prm_kw or {}
+    own = layer is None
+    if own:
+        layer = eat.EatLayer.from_workload(lw, max(Ts) if max_tokens is None else max_tokens,
+                                           gpu_params(shape, **prm_kw))
+    if L is None:
+        L = oracle_layer(lw)
+    prm = oracle_params(shape, **prm_kw)
+    outs = []
+    rng = np.random.default_rng(99)
+    for step, T in enumerate(Ts):
+        sign = 0 if signs is None else signs[step]
+        x = inputs[step] if inputs is not None else W.make_tokens(shape, T, step=step,
+                                                                  device=x_device)
+        acc0 = _acc(layer)
+        y, idx, w, k = layer.forward(x.cuda(), sign, with_routing=True)
+        torch.cuda.synchronize()
+        n_e, s_p, s_n = (t.cpu().numpy() for t in layer.call_stats())
+        N1, P1, C1 = (t.cpu().numpy() for t in layer.accounts())
+        x64 = np64(x)
+        routing = orc.route(x64, L, acc0, prm, sign)
+        sel_gpu = par.gpu_selection(idx, k)
+        amb, _ = par.check_routing(routing, sel_gpu, w.cpu().numpy(), shape.max_k)
+        sel = par.substituted(routing, sel_gpu, amb, prm.eps)
+        y_gpu = np64(y)
+        if sample is None:
+            y_ref, norms = par.oracle_outputs_batched(x64, L, routing, sel, prm.eps)
+            toks = [t for t in range(T) if t not in amb]
+            err = par.rel_err_rows(y_gpu[toks], y_ref[toks])
+            norms_ref = norms
+        else:
+            toks = sorted(set(rng.choice(T, size=min(sample, T), replace=False).tolist()) -
+                          set(amb))
+            yd, _ = par.oracle_outputs(x64, L, routing, sel, prm.eps, toks)
+            err = par.rel_err_rows(y_gpu[toks], np.stack([yd[t] for t in toks]))
+            norms_ref = None
+        assert err.max() <= Y_TOL[shape.xdtype], \
+            f"step {step}: output rel err {err.max():.3g} (token {toks[int(err.argmax())]})"
+        par.check_accounts(acc0, (N1, P1, C1), (n_e, s_p, s_n), routing, sel, norms_ref,
+                           prm.alpha, C_TOL[shape.xdtype])
+        outs.append(y)
+    if own:
+        layer.close()
+    return outs
+
+
+# ------------------------------------------------------------------ toy (fp32), the full config
+def test_toy_16_steps():
+    lw = W.make_layer(W.TOY)
+    run_parity(W.TOY, lw, [64] * 16)
+
+
+def test_toy_ppl_signs():
+    lw = W.make_layer(W.TOY)
+    run_parity(W.TOY, lw, [64] * 16, signs=W.ppl_signs(16))
+
+
+def test_toy_c_mode_raw_and_no_clamp():
+    lw = W.make_layer(W.TOY)
+    run_parity(W.TOY, lw, [64] * 6, prm_kw={"c_mode": eat.EAT_C_RAW})
+    run_parity(W.TOY, lw, [64] * 6, prm_kw={"clamp_enabled": 0})
+
+
+# ------------------------------------------------------------------ reduced bf16 layers
+MIX_S = W.scaled(W.MIXTRAL, "mixtral-s", d_model=512, d_ff=704)
+OLMOE_S = W.scaled(W.OLMOE, "olmoe-s", d_model=256, d_ff=192)
+QWEN_S = W.scaled(W.QWEN, "qwen-s", d_model=256, d_ff=128, d_ff_shared=192)
+DSV2L_S = W.scaled(W.DSV2L, "dsv2l-s", d_model=256, d_ff=192, n_layers=3)
+
+
+def test_mixtral_shaped_ragged():
+    lw = W.make_layer(MIX_S)
+    run_parity(MIX_S, lw, [1, 37, 200, 64, 5], signs=[0, 1, -1, 0, 1])
+
+
+def test_olmoe_shaped_k8_temperature():
+    lw = W.make_layer(OLMOE_S)
+    run_parity(OLMOE_S, lw, [333, 32, 32, 32])
+
+
+def test_qwen_shaped_shared_experts():
+    lw = W.make_layer(QWEN_S)
+    run_parity(QWEN_S, lw, [300, 17, 1])
+
+
+def test_dsv2l_shaped_residual_chain():
+    """Three layers, independent accounts, x_{l+1} = bf16(x_l + y_l) with the GPU's x_l."""
+    T = 96
+    layers = [W.make_layer(DSV2L_S, l) for l in range(3)]
+    x = W.make_tokens(DSV2L_S, T)
+    for l, lw in enumerate(layers):
+        outs = run_parity(DSV2L_S, lw, [T], inputs=[x])
+        x = (x.cuda().float() + outs[0].float()).to(torch.bfloat16).cpu()
+
+
+# ------------------------------------------------------------------ edge and degenerate cases
+def test_single_expert_layer():
+    sh = W.scaled(W.TOY, "one-expert", d_model=64, n_experts=1, d_ff=64, max_k=1)
+    lw = W.make_layer(sh)
+    run_parity(sh, lw, [1, 9, 33])
+
+
+def test_k_equals_e():
+    sh = W.scaled(W.TOY, "k-eq-e", d_model=128, n_experts=4, d_ff=128, max_k=4)
+    lw = W.make_layer(sh)
+    run_parity(sh, lw, [50, 50, 50])
+
+
+def test_degenerate_fixed_topk_on_gpu():
+    """beta = 0, alpha1 = 0, alpha2 huge, no clamp: vanilla Top-K by p (index tie-break)."""
+    kw = {"beta": 0.0, "alpha1": 0.0, "alpha2": 1e30, "clamp_enabled": 0}
+    lw = W.make_layer(MIX_S)
+    layer = eat.EatLayer.from_workload(lw, 128, gpu_params(MIX_S, **kw))
+    x = W.make_tokens(MIX_S, 128).cuda()
+    idx, w, k = layer.route(x)
+    L = oracle_layer(lw)
+    r = orc.route(np64(x), L, orc.Accounts.zeros(8), oracle_params(MIX_S, **kw))
+    for t in range(128):
+        order = np.lexsort((np.arange(8), -r.p[t]))
+        assert sorted(idx[t, :k[t]].tolist()) == sorted(order[:2].tolist())
+    assert (k.cpu() == 2).all()
+    layer.close()
+    run_parity(MIX_S, lw, [128, 128], prm_kw=kw)
+
+
+def test_all_tokens_one_expert():
+    """Router bias forces one expert for every token: a single group of n_e = T rows."""
+    lw = W.make_layer(OLMOE_S)
+    lw.b_router = torch.full_like(lw.b_router, -30.0)
+    lw.b_router[5] = 30.0
+    run_parity(OLMOE_S, lw, [257, 1])
+
+
+def test_set_accounts_restore_and_route_is_pure():
+    lw = W.make_layer(QWEN_S)
+    layer = eat.EatLayer.from_workload(lw, 64, gpu_params(QWEN_S))
+    g = torch.Generator().manual_seed(3)
+    N = torch.randint(0, 100, (60,), generator=g).to(torch.int64)
+    P = torch.rand(60, generator=g, dtype=torch.float64) * N
+    C = torch.rand(60, generator=g, dtype=torch.float64) * 5
+    layer.set_accounts(N.cuda(), P.cuda(), C.cuda())
+    x = W.make_tokens(QWEN_S, 64).cuda()
+    a = layer.route(x, 1)
+    b = layer.route(x, 1)
+    for u, v in zip(a, b):
+        assert torch.equal(u, v)
+    N1, P1, C1 = layer.accounts()
+    assert torch.equal(N1.cpu(), N) and torch.equal(P1.cpu(), P) and torch.equal(C1.cpu(), C)
+    _, idx, w, k = layer.forward(x, 1, with_routing=True)
+    assert torch.equal(idx, a[0]) and torch.equal(w, a[1]) and torch.equal(k, a[2])
+    layer.set_accounts(N.cuda(), P.cuda(), C.cuda())
+    run_parity(QWEN_S, lw, [64, 64], layer=layer, signs=[1, -1])
+    layer.reset()
+    N2, P2, C2 = layer.accounts()
+    assert int(N2.abs().sum()) == 0 and float(P2.abs().sum()) == 0 and float(C2.abs().sum()) == 0
+    layer.close()
+
+
+def test_max_tokens_bound_and_host_path():
+    lw = W.make_layer(MIX_S)
+    layer = eat.EatLayer.from_workload(lw, 40, gpu_params(MIX_S))
+    x = W.make_tokens(MIX_S, 41).cuda()
+    y = torch.empty_like(x)
+    with pytest.raises(eat.EatError) as ei:
+        eat.eat_moe_forward(layer.h, x, 41, 0, y)
+    assert ei.value.status == eat.EAT_ERR_INVALID_ARG
+    acc = layer.accounts()
+    y_dev = layer.forward(x[:40].contiguous(), 0)
+    layer.set_accounts(*acc)
+    xh = x[:40].cpu().pin_memory()
+    yh = torch.empty_like(xh).pin_memory()
+    eat.eat_moe_forward_host(layer.h, xh, 40, 0, yh)
+    assert torch.equal(yh, y_dev.cpu())
+    layer.close()
+
+
+def test_deterministic_repeat():
+    lw = W.make_layer(OLMOE_S)
+    outs = []
+    for _ in range(2):
+        layer = eat.EatLayer.from_workload(lw, 300, gpu_params(OLMOE_S))
+        x = W.make_tokens(OLMOE_S, 300).cuda()
+        ys = [layer.forward(x, 0) for _ in range(3)]
+        outs.append((ys, layer.accounts()))
+        layer.close()
+    for a, b in zip(outs[0][0], outs[1][0]):
+        assert torch.equal(a, b)
+    for a, b in zip(outs[0][1], outs[1][1]):
+        assert torch.equal(a, b)
+
+
+# ------------------------------------------------------------------ full-size layers (sampled)
+def _big(shape, layer_id=0):
+    return W.make_layer(shape, layer_id, device="cuda")
+
+
+def test_full_mixtral_decode_batches():
+    """Mixtral-8x7B-shaped layer, decode at batch 1 / 16 / 64 (the benchmarked configuration)."""
+    lw = _big(W.MIXTRAL)
+    L = oracle_layer_lazy(lw)
+    for B in (1, 16, 64):
+        layer = eat.EatLayer.from_workload(lw, 64, gpu_params(W.MIXTRAL))
+        run_parity(W.MIXTRAL, lw, [B] * 3, layer=layer, L=L, sample=8, x_device="cuda")
+        layer.close()
+
+
+def test_full_olmoe_prefill_then_decode():
+    lw = _big(W.OLMOE)
+    L = oracle_layer_lazy(lw)
+    layer = eat.EatLayer.from_workload(lw, 4096, gpu_params(W.OLMOE))
+    run_parity(W.OLMOE, lw, [4096, 32, 32], layer=layer, L=L, sample=12, x_device="cuda")
+    layer.close()
+
+
+def test_full_qwen_prefill():
+    lw = _big(W.QWEN)
+    L = oracle_layer_lazy(lw)
+    layer = eat.EatLayer.from_workload(lw, 8192, gpu_params(W.QWEN))
+    run_parity(W.QWEN, lw, [8192], layer=layer, L=L, sample=8, x_device="cuda")
+    layer.close()
+
+
+def test_full_dsv2l_layer_prefill_then_decode():
+    lw = _big(W.DSV2L, 25)
+    L = oracle_layer_lazy(lw)
+    layer = eat.EatLayer.from_workload(lw, 16384, gpu_params(W.DSV2L))
+    run_parity(W.DSV2L, lw, [16384, 128], layer=layer, L=L, sample=8, x_device="cuda")
+    layer.close()
