@@ -28,7 +28,7 @@ struct eat_handle {
   double* st_p = nullptr;
   double* st_norm = nullptr;
   long long* counters = nullptr;  // [4] on the device: calls, sum |union|, sum k, spare
-  float* logit_part = nullptr;
+  double* logit_part = nullptr;
   int32_t* idx = nullptr;
   float* w = nullptr;
   int32_t* k = nullptr;
@@ -330,7 +330,7 @@ eat_status eat_create(const eat_layer_desc* desc, const eat_params* params, eat_
   add(&h->st_p, sizeof(double) * h->E);
   add(&h->st_norm, sizeof(double) * h->E);
   add(&h->counters, sizeof(long long) * 4);
-  add(&h->logit_part, sizeof(float) * (size_t)max_lsplit * h->E);
+  add(&h->logit_part, sizeof(double) * (size_t)max_lsplit * h->E);
   add(&h->idx, sizeof(int32_t) * rows);
   add(&h->w, sizeof(float) * rows);
   add(&h->k, sizeof(int32_t) * h->Tmax);

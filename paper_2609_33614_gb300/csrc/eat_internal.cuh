@@ -21,11 +21,11 @@ struct RouteParams {
   int clamp, c_mode;
 };
 
-// Partial router logits: part[s][t][e] = sum over the s-th slice of d of x[t, j] * Wr[e, j].
+// Partial router logits (fp64): part[s][t][e] = sum over the s-th slice of d of x[t,j] Wr[e,j].
 cudaError_t launch_router_logits(const void* x, int x_bf16, const float* w_router, int T, int d,
-                                 int E, int n_split, float* part, cudaStream_t st);
+                                 int E, int n_split, double* part, cudaStream_t st);
 // Warp-per-token softmax + history score + threshold + selection + renormalisation.
-cudaError_t launch_route_select(const float* part, int n_split, const float* b_router, int T,
+cudaError_t launch_route_select(const double* part, int n_split, const float* b_router, int T,
                                 int E, int K, const int64_t* accN, const double* accP,
                                 const double* accC, RouteParams rp, int32_t* idx, float* w,
                                 int32_t* k, float* psel, cudaStream_t st);

@@ -1,8 +1,9 @@
 // Router and EAT selection (§3.1-§3.4 of the EAT paper, Eq. 1-8).
 //
-//  router_logits_kernel: partial router scores x . w_r over slices of d, fp32 FMA in a fixed
-//      order (a [T, E] GEMM too small and too precision-sensitive for the bf16 tensor path:
-//      the selection compares I against tau at 1e-5).
+//  router_logits_kernel: partial router scores x . w_r over slices of d: fp32 FMA inside
+//      32-wide chunks, chunk sums accumulated in fp64, so the logits carry ~1e-7 absolute error
+//      (the selection compares I against tau at 1e-5 and P_total sums p at 1e-6 relative; a
+//      [T, E] GEMM this small and this precision-sensitive stays off the bf16 tensor path).
 //  route_select_kernel: one warp per token.  Each lane owns experts lane, lane+32, ...; the warp
 //      does the softmax (§3.2), importance (Eq. 2), mean / population std (Eq. 3-4), tau (Eq. 5),
 //      PPL factor and smoothing (§3.3), the clamp to the type-7 q_lo / q_hi quantiles of p
@@ -36,7 +37,7 @@ int logits_tile_tokens(int E) {
 template <typename TX>
 __global__ void __launch_bounds__(kLogitThreads)
 router_logits_kernel(const TX* __restrict__ x, const float* __restrict__ wr, int T, int d, int E,
-                     int TT, int d_per_split, float* __restrict__ part) {
+                     int TT, int d_per_split, double* __restrict__ part) {
   extern __shared__ float sm[];
   float* xs = sm;                        // [TT][kChunk + 1]
   float* ws = sm + TT * (kChunk + 1);    // [E][kChunk + 1]
@@ -45,9 +46,9 @@ router_logits_kernel(const TX* __restrict__ x, const float* __restrict__ wr, int
   const int dbeg = blockIdx.y * d_per_split;
   const int dend = min(d, dbeg + d_per_split);
   const int n_out = TT * E;
-  float acc[kMaxOut];
+  double acc[kMaxOut];
 #pragma unroll
-  for (int q = 0; q < kMaxOut; ++q) acc[q] = 0.f;
+  for (int q = 0; q < kMaxOut; ++q) acc[q] = 0.0;
 
   for (int j0 = dbeg; j0 < dend; j0 += kChunk) {
     for (int i = tid; i < TT * kChunk; i += kLogitThreads) {
@@ -68,10 +69,10 @@ router_logits_kernel(const TX* __restrict__ x, const float* __restrict__ wr, int
         const int tt = o / E, e = o % E;
         const float* xr = xs + tt * (kChunk + 1);
         const float* wrow = ws + e * (kChunk + 1);
-        float a = acc[q];
+        float a = 0.f;
 #pragma unroll
         for (int jj = 0; jj < kChunk; ++jj) a = fmaf(xr[jj], wrow[jj], a);
-        acc[q] = a;
+        acc[q] += (double)a;
       }
     }
     __syncthreads();
@@ -154,7 +155,7 @@ __device__ __forceinline__ float order_stat(const float (&p)[EPL], const int (&r
 
 template <int EPL>
 __global__ void __launch_bounds__(kSelectThreads)
-route_select_kernel(const float* __restrict__ part, int n_split, const float* __restrict__ bias,
+route_select_kernel(const double* __restrict__ part, int n_split, const float* __restrict__ bias,
                     int T, int E, int K, const int64_t* __restrict__ accN,
                     const double* __restrict__ accP, const double* __restrict__ accC,
                     RouteParams rp, int32_t* __restrict__ out_idx, float* __restrict__ out_w,
@@ -178,10 +179,10 @@ route_select_kernel(const float* __restrict__ part, int n_split, const float* __
     valid[i] = e < E;
     float z = -INFINITY;
     if (valid[i]) {
-      float s = 0.f;
+      double s = 0.0;
       for (int sp = 0; sp < n_split; ++sp) s += part[((size_t)sp * T + t) * E + e];
-      if (bias) s += bias[e];
-      z = s / rp.temperature;
+      if (bias) s += (double)bias[e];
+      z = (float)(s / (double)rp.temperature);
     }
     p[i] = z;
     lmax = fmaxf(lmax, z);
@@ -340,7 +341,7 @@ int router_split(int T, int d, int E) {
 }
 
 cudaError_t launch_router_logits(const void* x, int x_bf16, const float* w_router, int T, int d,
-                                 int E, int n_split, float* part, cudaStream_t st) {
+                                 int E, int n_split, double* part, cudaStream_t st) {
   const int TT = logits_tile_tokens(E);
   int per = (d + n_split - 1) / n_split;
   per = (per + kChunk - 1) / kChunk * kChunk;
@@ -355,7 +356,7 @@ cudaError_t launch_router_logits(const void* x, int x_bf16, const float* w_route
   return cudaGetLastError();
 }
 
-cudaError_t launch_route_select(const float* part, int n_split, const float* b_router, int T,
+cudaError_t launch_route_select(const double* part, int n_split, const float* b_router, int T,
                                 int E, int K, const int64_t* accN, const double* accP,
                                 const double* accC, RouteParams rp, int32_t* idx, float* w,
                                 int32_t* k, float* psel, cudaStream_t st) {

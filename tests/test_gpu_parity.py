@@ -29,6 +29,12 @@ def _built():
 
 
 def oracle_params(shape, **kw):
+    """The oracle's Params for the same settings as the C ABI's eat_params overrides."""
+    kw = dict(kw)
+    if "c_mode" in kw:
+        kw["c_mode"] = "raw" if kw["c_mode"] == eat.EAT_C_RAW else "sum"
+    if "clamp_enabled" in kw:
+        kw["clamp"] = bool(kw.pop("clamp_enabled"))
     return orc.Params(max_k=shape.max_k, temperature=shape.temperature, **kw)
 
 
@@ -71,14 +77,14 @@ def run_parity(shape, lw, Ts, signs=None, prm_kw=None, layer=None, L=None, sampl
         amb, _ = par.check_routing(routing, sel_gpu, w.cpu().numpy(), shape.max_k)
         sel = par.substituted(routing, sel_gpu, amb, prm.eps)
         y_gpu = np64(y)
+        # outputs of every token, with the GPU's (validated) selection on the ambiguous ones
         if sample is None:
             y_ref, norms = par.oracle_outputs_batched(x64, L, routing, sel, prm.eps)
-            toks = [t for t in range(T) if t not in amb]
-            err = par.rel_err_rows(y_gpu[toks], y_ref[toks])
+            toks = list(range(T))
+            err = par.rel_err_rows(y_gpu, y_ref)
             norms_ref = norms
         else:
-            toks = sorted(set(rng.choice(T, size=min(sample, T), replace=False).tolist()) -
-                          set(amb))
+            toks = sorted(set(rng.choice(T, size=min(sample, T), replace=False).tolist()))
             yd, _ = par.oracle_outputs(x64, L, routing, sel, prm.eps, toks)
             err = par.rel_err_rows(y_gpu[toks], np.stack([yd[t] for t in toks]))
             norms_ref = None
