@@ -124,6 +124,31 @@ eat_status eat_moe_forward(eat_handle* h, const void* x, int32_t T, int32_t ppl_
 eat_status eat_moe_forward_host(eat_handle* h, const void* x_host, int32_t T, int32_t ppl_sign,
                                 void* y_host, void* stream);
 
+/* Size of the fixed device scratch eat_route_noalloc uses (1 MiB = 131072 fp64 router scores). */
+#define EAT_NOALLOC_SCRATCH_BYTES (1u << 20)
+
+/* Routing for callers that cannot allocate device memory.  The paper has no counterpart: this is a
+ * deployment variant of eat_route.  Some callers cannot call cudaMalloc -- a serving process that
+ * reserved nearly all HBM for its own pool, a decode loop that must not take cudaMalloc's implicit
+ * device synchronisation, a framework that forbids allocations outside its own allocator -- and so
+ * cannot create a handle.  This call computes exactly what eat_route computes (Eq. 1-8) from
+ * caller-owned device buffers: x [T, d_model] (xdtype), w_router [E, d_model] fp32, b_router [E]
+ * fp32 or NULL, accounts N [E] int64, P [E] fp64, C [E] fp64 (read only), and writes idx / w / k
+ * as eat_route does.  It allocates nothing: its only scratch is a fixed 1 MiB array compiled into
+ * the library, which every GPU that loads the library holds until the process exits.
+ *  - T * n_experts must be <= 131072 (EAT_NOALLOC_SCRATCH_BYTES / 8), else EAT_ERR_INVALID_ARG;
+ *    larger batches are routed in several calls.
+ *  - The first call on each device looks up the scratch's device address (a one-time set-up per
+ *    device, done with that device current); make that first call before any stream capture.
+ *  - Calls share the scratch: two calls that may overlap on the GPU (different streams or host
+ *    threads) race on it and must be serialised by the caller.
+ * Errors are reported through eat_last_error(NULL). */
+eat_status eat_route_noalloc(const void* x, int32_t T, int32_t d_model, int32_t n_experts,
+                             int32_t xdtype, const float* w_router, const float* b_router,
+                             const int64_t* N, const double* P, const double* C,
+                             const eat_params* params, int32_t ppl_sign, int32_t* idx, float* w,
+                             int32_t* k, void* stream);
+
 /* Free everything the handle owns.  Synchronises the device first.  NULL is accepted. */
 eat_status eat_destroy(eat_handle* h);
 

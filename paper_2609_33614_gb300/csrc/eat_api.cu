@@ -539,3 +539,7 @@ const char* eat_status_string(eat_status s) {
 }
 
 }  // extern "C"
+
+namespace eat {
+void set_thread_error(const char* msg) { g_err = msg ? msg : ""; }
+}  // namespace eat

@@ -84,4 +84,8 @@ cudaError_t launch_account(const int32_t* offs, const float* perm_p, const float
                            double alpha, int64_t* N, double* P, double* C, int32_t* st_n,
                            double* st_p, double* st_norm, long long* counters, cudaStream_t st);
 
+// Records msg as the text eat_last_error(NULL) returns on this thread (entry points without a
+// handle).
+void set_thread_error(const char* msg);
+
 }  // namespace eat

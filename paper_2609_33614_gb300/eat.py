@@ -53,6 +53,8 @@ _SIGS = {
     "eat_route": (c_i32, [c_vp, c_vp, c_i32, c_i32, c_vp, c_vp, c_vp, c_vp]),
     "eat_moe_forward": (c_i32, [c_vp, c_vp, c_i32, c_i32, c_vp, c_vp, c_vp, c_vp, c_vp]),
     "eat_moe_forward_host": (c_i32, [c_vp, c_vp, c_i32, c_i32, c_vp, c_vp]),
+    "eat_route_noalloc": (c_i32, [c_vp, c_i32, c_i32, c_i32, c_i32, c_vp, c_vp, c_vp, c_vp, c_vp,
+                                  ctypes.POINTER(eat_params), c_i32, c_vp, c_vp, c_vp, c_vp]),
     "eat_destroy": (c_i32, [c_vp]),
     "eat_get_accounts": (c_i32, [c_vp, c_vp, c_vp, c_vp, c_vp]),
     "eat_set_accounts": (c_i32, [c_vp, c_vp, c_vp, c_vp, c_vp]),
@@ -134,6 +136,15 @@ def eat_moe_forward(h, x, T, ppl_sign, y, idx=None, w=None, k=None, stream=None)
 def eat_moe_forward_host(h, x_host, T, ppl_sign, y_host, stream=None):
     _check(lib().eat_moe_forward_host(h, _ptr(x_host), T, ppl_sign, _ptr(y_host),
                                       _stream(stream)), h)
+
+
+def eat_route_noalloc(x, T, d_model, n_experts, xdtype, w_router, b_router, N, P, C, params,
+                      ppl_sign, idx, w, k, stream=None):
+    """Routing with no device allocation (see include/eat.h): every buffer is the caller's."""
+    _check(lib().eat_route_noalloc(_ptr(x), T, d_model, n_experts, xdtype, _ptr(w_router),
+                                   _ptr(b_router), _ptr(N), _ptr(P), _ptr(C),
+                                   ctypes.byref(params), ppl_sign, _ptr(idx), _ptr(w), _ptr(k),
+                                   _stream(stream)))
 
 
 def eat_destroy(h):
