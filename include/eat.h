@@ -104,6 +104,7 @@ eat_status eat_reset_accounts(eat_handle* h, void* stream);
 /* Routing only (§3.2-§3.4, Eq. 1-8) for T tokens x [T, d] (xdtype), 1 <= T <= max_tokens,
  * reading the current accounts and never changing them.  ppl_sign is the sign of
  * PPL_curr - PPL_prev (§3.3): +1 -> factor ppl_up, -1 -> ppl_down, 0 -> no signal (factor 1).
+ * x must be 16-byte aligned.
  * Outputs: idx [T, K] int32 selected experts in ascending index order, -1 after the k-th;
  * w [T, K] fp32 renormalised gates g_norm (Eq. 7), 0 after the k-th; k [T] int32 count. */
 eat_status eat_route(eat_handle* h, const void* x, int32_t T, int32_t ppl_sign,
@@ -168,7 +169,8 @@ eat_status eat_get_call_stats(eat_handle* h, int32_t* n_e, double* sum_p, double
  * (synchronises the device):
  *   out[0] forward calls, out[1] sum over calls of the number of distinct activated experts,
  *   out[2] sum over calls of the activations (sum_t k_t), out[3] kernel launches issued by this
- *   handle (all entry points). */
+ *   handle (all entry points), out[4] the device status word: 0, or the bits of kernel waits that
+ *   expired (a kernel that gives up on a wait returns early and its outputs are invalid). */
 eat_status eat_get_counters(eat_handle* h, int64_t* out, int32_t n);
 
 /* Per-kernel device timing.  eat_profile_begin(h, capacity) makes every later launch of this

@@ -41,7 +41,9 @@ struct eat_handle {
   float* sout = nullptr;  // [S*Tmax, d]
   void* xstage = nullptr; // [Tmax, d]
   void* ystage = nullptr; // [Tmax, d]
-  int max_split = 1;      // split-K slices of the routed down projection held in opart
+  void* xperm = nullptr;  // [Tmax*K, d] gathered token rows (tensor-core path)
+  unsigned int* status = nullptr;  // device status word: bounded waits that expired
+  long long opart_rows = 0;
 
   TcLayer tc{};
 
@@ -124,6 +126,8 @@ eat_status check_call(eat_handle* h, const void* x, int32_t T, int32_t ppl_sign)
                     "]");
   if (ppl_sign < -1 || ppl_sign > 1)
     return fail(h, EAT_ERR_INVALID_ARG, "ppl_sign must be -1, 0 or +1");
+  if (((uintptr_t)x & 15) != 0)
+    return fail(h, EAT_ERR_INVALID_ARG, "x must be 16-byte aligned");
   return EAT_OK;
 }
 
@@ -160,12 +164,15 @@ eat_status run_forward(eat_handle* h, const void* x, int T, int ppl_sign, void* 
     c.offs = h->perm.offs;
     c.tile_offs = h->perm.tile_offs;
     c.perm_tok = h->perm.perm_tok;
+    c.xperm = h->xperm;
     c.act = h->act;
     c.opart = h->opart;
     c.sact = h->sact;
     c.sout = h->sout;
-    c.max_split = h->max_split;
+    c.status = h->status;
     n_split = tc_down_split(h->tc, T);
+    EAT_TRY(launch(h, kPermute, st, "gather rows",
+                   [&] { return tc_launch_gather(h->tc, c, st); }));
     EAT_TRY(launch(h, kUp, st, "tc gate/up", [&] { return tc_launch_up(h->tc, c, false, st); }));
     EAT_TRY(launch(h, kDown, st, "tc down",
                    [&] { return tc_launch_down(h->tc, c, false, n_split, st); }));
@@ -199,7 +206,7 @@ eat_status run_forward(eat_handle* h, const void* x, int T, int ppl_sign, void* 
     }
   }
   EAT_TRY(launch(h, kCombine, st, "combine", [&] {
-    return launch_combine(h->bf16, h->opart, n_split, h->Tmax * h->K, h->perm.slot_of, h->w,
+    return launch_combine(h->bf16, h->opart, n_split, rows, h->perm.slot_of, h->w,
                           h->k, h->sout, h->S, T, h->K, h->d, y, h->onorm, st);
   }));
   EAT_TRY(launch(h, kAccount, st, "account update", [&] {
@@ -303,16 +310,17 @@ eat_status eat_create(const eat_layer_desc* desc, const eat_params* params, eat_
   h->K = Pm.max_k;
   h->bf16 = D.wdtype == EAT_BF16;
   h->elt = h->bf16 ? 2 : 4;
-  h->backend = 0;
+  h->backend = h->bf16 ? 1 : 0;
+  h->opart_rows = (long long)h->Tmax * h->K;
 
   if (h->backend == 1) {
     const char* msg = nullptr;
-    if (tc_init(h->tc, D, h->K, h->Tmax, &msg) != 0) {
+    if (tc_configure(h->tc, D, h->K, h->Tmax, &msg) != 0) {
       std::string m = msg ? msg : "tensor-core setup failed";
       free_handle(h);
-      return fail(nullptr, EAT_ERR_CUDA, m);
+      return fail(nullptr, EAT_ERR_UNSUPPORTED, m);
     }
-    h->max_split = tc_max_split(h->tc);
+    h->opart_rows = tc_opart_rows(h->tc);
   }
 
   int max_lsplit = 0;
@@ -330,6 +338,7 @@ eat_status eat_create(const eat_layer_desc* desc, const eat_params* params, eat_
   add(&h->st_p, sizeof(double) * h->E);
   add(&h->st_norm, sizeof(double) * h->E);
   add(&h->counters, sizeof(long long) * 4);
+  add(&h->status, sizeof(unsigned int) * 4);
   add(&h->logit_part, sizeof(double) * (size_t)max_lsplit * h->E);
   add(&h->idx, sizeof(int32_t) * rows);
   add(&h->w, sizeof(float) * rows);
@@ -343,12 +352,13 @@ eat_status eat_create(const eat_layer_desc* desc, const eat_params* params, eat_
   add(&h->perm.perm_p, sizeof(float) * rows);
   add(&h->perm.active, sizeof(int32_t) * (h->E + 1));
   add(&h->act, h->elt * rows * h->F);
-  add(&h->opart, sizeof(float) * (size_t)h->max_split * rows * h->d);
+  add(&h->opart, sizeof(float) * (size_t)h->opart_rows * h->d);
   add(&h->onorm, sizeof(float) * rows);
   if (h->S > 0) {
     add(&h->sact, h->elt * (size_t)h->S * h->Tmax * h->Fs);
     add(&h->sout, sizeof(float) * (size_t)h->S * h->Tmax * h->d);
   }
+  if (h->backend == 1) add(&h->xperm, h->elt * rows * h->d);
   add(&h->xstage, h->elt * (size_t)h->Tmax * h->d);
   add(&h->ystage, h->elt * (size_t)h->Tmax * h->d);
   size_t total = 0;
@@ -372,6 +382,14 @@ eat_status eat_create(const eat_layer_desc* desc, const eat_params* params, eat_
     free_handle(h);
     return fail(nullptr, EAT_ERR_CUDA, std::string("workspace init: ") + cudaGetErrorString(e));
   }
+  if (h->backend == 1) {
+    const char* msg = nullptr;
+    if (tc_bind(h->tc, D, h->xperm, h->act, h->sact, &msg) != 0) {
+      std::string m = msg ? msg : "tensor map setup failed";
+      free_handle(h);
+      return fail(nullptr, EAT_ERR_CUDA, m);
+    }
+  }
   *out = h;
   return EAT_OK;
 }
@@ -383,6 +401,7 @@ eat_status eat_reset_accounts(eat_handle* h, void* stream) {
   if (e == cudaSuccess) e = cudaMemsetAsync(h->P, 0, sizeof(double) * h->E, st);
   if (e == cudaSuccess) e = cudaMemsetAsync(h->C, 0, sizeof(double) * h->E, st);
   if (e == cudaSuccess) e = cudaMemsetAsync(h->counters, 0, sizeof(long long) * 4, st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(h->status, 0, sizeof(unsigned int) * 4, st);
   if (e != cudaSuccess) return cuda_fail(h, e, "reset accounts");
   h->launches = 0;
   return EAT_OK;
@@ -471,11 +490,13 @@ eat_status eat_get_counters(eat_handle* h, int64_t* out, int32_t n) {
   if (!h) return fail(nullptr, EAT_ERR_INVALID_ARG, "null handle");
   if (!out || n < 0) return fail(h, EAT_ERR_INVALID_ARG, "out is NULL or n < 0");
   long long dev[4] = {0, 0, 0, 0};
+  unsigned int stw = 0;
   cudaError_t e = cudaDeviceSynchronize();
   if (e == cudaSuccess) e = cudaMemcpy(dev, h->counters, sizeof(dev), cudaMemcpyDeviceToHost);
+  if (e == cudaSuccess) e = cudaMemcpy(&stw, h->status, sizeof(stw), cudaMemcpyDeviceToHost);
   if (e != cudaSuccess) return cuda_fail(h, e, "get counters");
-  const long long vals[4] = {dev[0], dev[1], dev[2], h->launches};
-  for (int i = 0; i < n && i < 4; ++i) out[i] = vals[i];
+  const long long vals[5] = {dev[0], dev[1], dev[2], h->launches, (long long)stw};
+  for (int i = 0; i < n && i < 5; ++i) out[i] = vals[i];
   return EAT_OK;
 }
 

@@ -1,22 +1,652 @@
-// Placeholder until the tcgen05 kernels land: every entry reports "unsupported".
+// Tensor-core expert FFN kernels for bf16 layers (the dominant cost of the EAT MoE layer): grouped
+// SwiGLU expert GEMMs over the activated experts only (§3.4: "only activated experts ...
+// participate"), written for sm_103a with tcgen05.mma (accumulators in TMEM), TMA tile loads into
+// 128B-swizzled shared memory and mbarrier pipelines.
+//
+// Orientation ("swap AB"): a tile is 128 weight rows (output features of one expert) x BN tokens
+// (16..128 rows of that expert's slot list), so decode calls with a handful of tokens still issue
+// full M = 128 MMAs and simply stream the activated experts' weights; prefill calls use BN = 128.
+//   gate/up kernel: D_gate = Wg[e, f0:f0+128, :] . Xperm[slots]^T and D_up likewise, both in TMEM;
+//       the epilogue writes act[slot, f] = silu(D_gate) * D_up in bf16 (fp32 accumulation).
+//   down kernel:    D = Wd[e, c0:c0+128, :] . act[slots]^T over a K slice (split-K for decode),
+//       fp32 partials opart[split][slot][c] summed in fixed order by the combine kernel.
+// Persistent CTAs (one per SM) walk the work units (token tile, feature tile, K slice) of all
+// groups; the group sizes live on the device (written by the permute kernel), so no host sync.
+// Warp roles: warp 0 lane 0 issues TMA; warp 1 owns TMEM and lane 0 issues MMAs; warps 2-5 drain
+// TMEM (double-buffered accumulators, so the epilogue of tile i overlaps the MMAs of tile i + 1).
+// Every mbarrier wait is bounded (2 s); on expiry the kernel records an error in the device status
+// word, lets in-flight copies and MMAs finish, frees its TMEM and returns.
 #include "ffn_tc.cuh"
+
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <cstring>
+#include <mutex>
+#include <vector>
 
 namespace eat {
 
-int tc_init(TcLayer& L, const eat_layer_desc&, int, int, const char** msg) {
+namespace {
+
+constexpr int kBM = 128;                  // weight rows per tile (MMA M)
+constexpr int kBK = 64;                   // 64 bf16 = 128 B: one 128B-swizzle row
+constexpr int kThreadsTc = 192;           // 6 warps
+constexpr int kBNs[4] = {16, 32, 64, 128};
+constexpr unsigned long long kWaitLimitNs = 2000000000ull;
+constexpr int kSmemBudget = 220 * 1024;
+
+// -------------------------------------------------------------------------------- PTX wrappers
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+__device__ __forceinline__ unsigned long long globaltimer() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count));
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Bounded wait on the phase with the given parity.  Returns false when it gave up: because another
+// role raised the CTA's abort flag (check_abort), or after kWaitLimitNs (then it raises the flag and
+// records `code` in the device status word).
+__device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                       unsigned int* err, unsigned int code, bool check_abort) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const unsigned long long t0 = globaltimer();
+  for (;;) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (check_abort && *abort_flag) return false;
+    if (globaltimer() - t0 > kWaitLimitNs) {
+      *abort_flag = 1;
+      atomicOr(err, code);
+      return false;
+    }
+  }
+}
+
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar,
+                                            int c0, int c1) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(map), "r"(smem_u32(bar)), "r"(c0), "r"(c1)
+      : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_alloc(uint32_t* slot, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                   smem_u32(slot)),
+               "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+// D[tmem] (+)= A[smem desc] . B[smem desc]^T, both K-major, kind::f16 (bf16 in, fp32 accumulate)
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                         uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// Arrive on `bar` once every MMA this thread issued so far has completed.
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+          smem_u32(bar))
+      : "memory");
+}
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, "
+      "%12, %13, %14, %15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_wait_ld() {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Shared-memory matrix descriptor: K-major operand, 128B swizzle, rows of 128 B, 8-row groups
+// 1024 B apart (SBO); LBO unused for swizzled K-major layouts; version field 1 (bit 46).
+__device__ __forceinline__ uint64_t sdesc_k128(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFF) >> 4);
+  d |= (uint64_t)1 << 16;
+  d |= (uint64_t)(1024 >> 4) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;
+  return d;
+}
+// Instruction descriptor, kind::f16: D fp32, A and B bf16, both K-major, M = 128, N = n.
+__host__ __device__ constexpr uint32_t idesc_bf16(int n) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) |
+         ((uint32_t)(kBM >> 4) << 24);
+}
+
+__host__ __device__ constexpr int tmem_cols_for(int c) {
+  return c <= 32 ? 32 : c <= 64 ? 64 : c <= 128 ? 128 : c <= 256 ? 256 : 512;
+}
+
+template <int BN, bool GATEUP>
+struct Cfg {
+  static constexpr int kNA = GATEUP ? 2 : 1;
+  static constexpr int kABytes = kBM * kBK * 2;
+  static constexpr int kBBytes = BN * kBK * 2;
+  static constexpr int kStageBytes = kNA * kABytes + kBBytes;
+  static constexpr int kStagesRaw = (kSmemBudget - 2048) / kStageBytes;
+  static constexpr int kStages = kStagesRaw > 12 ? 12 : kStagesRaw;
+  static constexpr int kAccCols = kNA * BN;
+  static constexpr int kTmemCols = tmem_cols_for(2 * kAccCols);
+  static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + 256;
+};
+
+struct TcArgs {
+  int n_groups;
+  const int32_t* row_offs;   // [G+1] slot ranges per group, or nullptr: uniform_rows each
+  const int32_t* tile_offs;  // [G+1] prefix of token tiles, or nullptr: uniform
+  int uniform_rows;
+  int b_shift_per_group;     // B row = slot - g * b_shift_per_group
+  int a_rows_per_group;      // A row = g * a_rows_per_group + m0
+  int M;                     // output features per group
+  int m_tiles;
+  int kblocks;
+  int n_split;
+  int kb_per_split;
+  void* out;
+  long long split_stride;    // elements between split slices of the fp32 output
+  unsigned int* err;
+};
+
+struct Unit {
+  int g, slot0, nrows, m0, kb0, kb1, split;
+};
+
+template <int BN>
+__device__ __forceinline__ Unit decode_unit(const TcArgs& a, int u) {
+  Unit w;
+  w.split = u % a.n_split;
+  const int r = u / a.n_split;
+  const int mi = r % a.m_tiles;
+  const int tl = r / a.m_tiles;
+  int g, j;
+  if (a.tile_offs) {
+    int lo = 0, hi = a.n_groups - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (a.tile_offs[mid] <= tl) lo = mid;
+      else hi = mid - 1;
+    }
+    g = lo;
+    j = tl - a.tile_offs[lo];
+  } else {
+    const int tpg = (a.uniform_rows + BN - 1) / BN;
+    g = tl / tpg;
+    j = tl % tpg;
+  }
+  const int beg = a.row_offs ? a.row_offs[g] : g * a.uniform_rows;
+  const int end = a.row_offs ? a.row_offs[g + 1] : (g + 1) * a.uniform_rows;
+  w.g = g;
+  w.slot0 = beg + j * BN;
+  w.nrows = min(BN, end - w.slot0);
+  w.m0 = mi * kBM;
+  w.kb0 = w.split * a.kb_per_split;
+  w.kb1 = min(a.kblocks, w.kb0 + a.kb_per_split);
+  return w;
+}
+
+__device__ __forceinline__ float silu_f(float g) { return g / (1.0f + expf(-g)); }
+
+template <int BN, bool GATEUP>
+__global__ void __launch_bounds__(kThreadsTc, 1)
+tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__ CUtensorMap mapA1,
+              const __grid_constant__ CUtensorMap mapB, const TcArgs args) {
+  using C = Cfg<BN, GATEUP>;
+  constexpr int S = C::kStages;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  uint64_t* full = (uint64_t*)(smem + S * C::kStageBytes);
+  uint64_t* empty = full + S;
+  uint64_t* tfull = empty + S;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* mma_done = tempty + 2;
+  uint32_t* tmem_slot = (uint32_t*)(mma_done + 1);
+  volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&tfull[b], 1);
+      mbar_init(&tempty[b], 4);
+    }
+    mbar_init(mma_done, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, C::kTmemCols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const int total_tiles = args.tile_offs
+                              ? args.tile_offs[args.n_groups]
+                              : args.n_groups * ((args.uniform_rows + BN - 1) / BN);
+  const int units = total_tiles * args.m_tiles * args.n_split;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------------------ TMA producer
+      int stage = 0;
+      uint32_t phase = 0;
+      long long issued = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
+        const Unit w = decode_unit<BN>(args, u);
+        const int a_row = w.g * args.a_rows_per_group + w.m0;
+        const int b_row = w.slot0 - w.g * args.b_shift_per_group;
+        for (int kb = w.kb0; kb < w.kb1; ++kb) {
+          if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, args.err, 1u, true)) {
+            ok = false;
+            break;
+          }
+          uint8_t* st = smem + stage * C::kStageBytes;
+          mbar_expect_tx(&full[stage], C::kStageBytes);
+          tma_load_2d(st, &mapA0, &full[stage], kb * kBK, a_row);
+          if (GATEUP) tma_load_2d(st + C::kABytes, &mapA1, &full[stage], kb * kBK, a_row);
+          tma_load_2d(st + C::kNA * C::kABytes, &mapB, &full[stage], kb * kBK, b_row);
+          ++issued;
+          if (++stage == S) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      // let the copies still in flight land before the CTA may exit
+      const long long first = issued > S ? issued - S : 0;
+      for (long long i = first; i < issued; ++i)
+        mbar_wait(&full[i % S], (uint32_t)((i / S) & 1), abort_flag, args.err, 2u, false);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ------------------------------------------------------------ MMA issuer
+      constexpr uint32_t idesc = idesc_bf16(BN);
+      int stage = 0;
+      uint32_t phase = 0;
+      int local = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++local) {
+        const Unit w = decode_unit<BN>(args, u);
+        const int buf = local & 1;
+        const uint32_t tph = (uint32_t)((local >> 1) & 1);
+        if (!mbar_wait(&tempty[buf], tph ^ 1u, abort_flag, args.err, 4u, true)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d0 = tmem_base + (uint32_t)(buf * C::kAccCols);
+        const uint32_t d1 = d0 + BN;
+        for (int kb = w.kb0; kb < w.kb1; ++kb) {
+          if (!mbar_wait(&full[stage], phase, abort_flag, args.err, 8u, true)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa0 = smem_u32(smem + stage * C::kStageBytes);
+          const uint32_t sa1 = sa0 + C::kABytes;
+          const uint32_t sb = sa0 + C::kNA * C::kABytes;
+#pragma unroll
+          for (int k = 0; k < kBK / 16; ++k) {
+            const uint64_t db = sdesc_k128(sb + k * 32);
+            const uint32_t acc = (kb > w.kb0 || k > 0) ? 1u : 0u;
+            mma_bf16(d0, sdesc_k128(sa0 + k * 32), db, idesc, acc);
+            if (GATEUP) mma_bf16(d1, sdesc_k128(sa1 + k * 32), db, idesc, acc);
+          }
+          mma_commit(&empty[stage]);
+          if (++stage == S) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        mma_commit(&tfull[buf]);
+      }
+      // no MMA may still be running when TMEM is freed
+      mma_commit(mma_done);
+      mbar_wait(mma_done, 0u, abort_flag, args.err, 16u, false);
+    }
+  } else {
+    // -------------------------------------------------------------- epilogue (warps 2..5)
+    const int q = warp & 3;  // TMEM lane quarter this warp may access
+    const int row = 32 * q + lane;
+    int local = 0;
+    for (int u = blockIdx.x; u < units; u += gridDim.x, ++local) {
+      const Unit w = decode_unit<BN>(args, u);
+      const int buf = local & 1;
+      const uint32_t tph = (uint32_t)((local >> 1) & 1);
+      if (!mbar_wait(&tfull[buf], tph, abort_flag, args.err, 32u, true)) break;
+      tc_fence_after();
+      const uint32_t tbase = tmem_base + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * C::kAccCols);
+      const int f = w.m0 + row;
+      const bool fok = f < args.M;
+      for (int c0 = 0; c0 < BN && c0 < w.nrows; c0 += 16) {
+        uint32_t g[16], up[16];
+        tmem_ld16(tbase + c0, g);
+        if (GATEUP) tmem_ld16(tbase + BN + c0, up);
+        tmem_wait_ld();
+        if (fok) {
+#pragma unroll
+          for (int c = 0; c < 16; ++c) {
+            if (c0 + c < w.nrows) {
+              const size_t slot = (size_t)(w.slot0 + c0 + c);
+              if (GATEUP) {
+                const float h = silu_f(__uint_as_float(g[c])) * __uint_as_float(up[c]);
+                ((__nv_bfloat16*)args.out)[slot * args.M + f] = __float2bfloat16_rn(h);
+              } else {
+                ((float*)args.out)[(size_t)w.split * args.split_stride + slot * args.M + f] =
+                    __uint_as_float(g[c]);
+              }
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tempty[buf]);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem_base, C::kTmemCols);
+}
+
+// Xperm[slot] = x[perm_tok[slot]] for every slot of the call (16-byte copies).
+__global__ void gather_rows_kernel(const uint4* __restrict__ x, const int32_t* __restrict__ perm_tok,
+                                   const int32_t* __restrict__ n_rows, int row_vecs,
+                                   uint4* __restrict__ xperm) {
+  const int slot = blockIdx.x;
+  if (slot >= *n_rows) return;
+  const size_t src = (size_t)perm_tok[slot] * row_vecs;
+  const size_t dst = (size_t)slot * row_vecs;
+  for (int i = threadIdx.x; i < row_vecs; i += blockDim.x) xperm[dst + i] = x[src + i];
+}
+
+// -------------------------------------------------------------------------------- host side
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = (PFN_cuTensorMapEncodeTiled_v12000)p;
+  });
+  return fn;
+}
+
+// 2D bf16 tensor [rows, cols] (row-major), box {64 cols, box_rows}, 128B swizzle, OOB -> 0.
+bool encode_2d(CUtensorMap* m, const void* ptr, long long rows, long long cols, int box_rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
+  cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+struct Maps {
+  CUtensorMap wg, wu, wd, wsg, wsu, wsd;
+  CUtensorMap xperm[4], act[4], sact[4];
+};
+
+int bn_index(int bn) {
+  for (int i = 0; i < 4; ++i)
+    if (kBNs[i] == bn) return i;
+  return 3;
+}
+
+template <int BN, bool GATEUP>
+cudaError_t launch_tc(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& b,
+                      const TcArgs& args, int grid, cudaStream_t st) {
+  using C = Cfg<BN, GATEUP>;
+  static std::once_flag once;
+  static cudaError_t attr_err = cudaSuccess;
+  std::call_once(once, [] {
+    attr_err = cudaFuncSetAttribute(tc_ffn_kernel<BN, GATEUP>,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
+  });
+  if (attr_err != cudaSuccess) return attr_err;
+  if (grid <= 0) return cudaSuccess;
+  tc_ffn_kernel<BN, GATEUP><<<grid, kThreadsTc, C::kSmemBytes, st>>>(a0, a1, b, args);
+  return cudaGetLastError();
+}
+
+template <bool GATEUP>
+cudaError_t launch_bn(int bn, const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& b,
+                      const TcArgs& args, int grid, cudaStream_t st) {
+  switch (bn) {
+    case 16: return launch_tc<16, GATEUP>(a0, a1, b, args, grid, st);
+    case 32: return launch_tc<32, GATEUP>(a0, a1, b, args, grid, st);
+    case 64: return launch_tc<64, GATEUP>(a0, a1, b, args, grid, st);
+    default: return launch_tc<128, GATEUP>(a0, a1, b, args, grid, st);
+  }
+}
+
+}  // namespace
+
+int tc_tile_rows(const TcLayer&, int T) {
+  // the largest group of a call has at most T rows (each token picks an expert once)
+  for (int i = 0; i < 4; ++i)
+    if (T <= kBNs[i]) return kBNs[i];
+  return 128;
+}
+
+static int split_for(const TcLayer& L, int T) {
+  const int m_tiles = (L.d + kBM - 1) / kBM;
+  const int kblocks = L.F / kBK;
+  long long est = (long long)std::min(L.E, T * L.K) * m_tiles;
+  int split = 1;
+  while (est * split < 2LL * L.num_sms && kblocks / (split * 2) >= 8 && split < 16) split *= 2;
+  return split;
+}
+
+// Split count with no empty K slice: n slices of ceil(kblocks / split) k-blocks each.
+int tc_down_split(const TcLayer& L, int T) {
+  const int kblocks = L.F / kBK;
+  const int split = split_for(L, T);
+  const int per = (kblocks + split - 1) / split;
+  return (kblocks + per - 1) / per;
+}
+
+long long tc_opart_rows(const TcLayer& L) {
+  long long best = (long long)L.Tmax * L.K;
+  for (int T = 1; T <= L.Tmax; ++T) {
+    const int s = split_for(L, T);
+    if (s == 1 && T > 4096) break;  // split is 1 from here on
+    best = std::max(best, (long long)s * T * L.K);
+  }
+  return best;
+}
+
+int tc_configure(TcLayer& L, const eat_layer_desc& D, int K, int Tmax, const char** msg) {
+  L.E = D.n_experts;
+  L.d = D.d_model;
+  L.F = D.d_ff;
+  L.S = D.n_shared;
+  L.Fs = D.n_shared > 0 ? D.d_ff_shared : 0;
+  L.K = K;
+  L.Tmax = Tmax;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceProp prop;
+  if (cudaGetDeviceProperties(&prop, dev) != cudaSuccess) {
+    if (msg) *msg = "cudaGetDeviceProperties failed";
+    return 1;
+  }
+  if (prop.major != 10 || prop.minor != 3) {
+    if (msg) *msg = "the tensor-core kernels are built for sm_103a (GB300)";
+    return 1;
+  }
+  L.num_sms = prop.multiProcessorCount;
+  if (!encode_fn()) {
+    if (msg) *msg = "cuTensorMapEncodeTiled is unavailable";
+    return 1;
+  }
+  return 0;
+}
+
+int tc_bind(TcLayer& L, const eat_layer_desc& D, void* xperm, void* act, void* sact,
+            const char** msg) {
+  Maps* m = new Maps();
+  std::memset(m, 0, sizeof(Maps));
+  const long long rows = (long long)L.Tmax * L.K;
+  bool ok = encode_2d(&m->wg, D.w_gate, (long long)L.E * L.F, L.d, kBM) &&
+            encode_2d(&m->wu, D.w_up, (long long)L.E * L.F, L.d, kBM) &&
+            encode_2d(&m->wd, D.w_down, (long long)L.E * L.d, L.F, kBM);
+  if (ok && L.S > 0)
+    ok = encode_2d(&m->wsg, D.ws_gate, (long long)L.S * L.Fs, L.d, kBM) &&
+         encode_2d(&m->wsu, D.ws_up, (long long)L.S * L.Fs, L.d, kBM) &&
+         encode_2d(&m->wsd, D.ws_down, (long long)L.S * L.d, L.Fs, kBM);
+  for (int i = 0; i < 4 && ok; ++i) {
+    ok = encode_2d(&m->xperm[i], xperm, rows, L.d, kBNs[i]) &&
+         encode_2d(&m->act[i], act, rows, L.F, kBNs[i]);
+    if (ok && L.S > 0) ok = encode_2d(&m->sact[i], sact, (long long)L.S * L.Tmax, L.Fs, kBNs[i]);
+  }
+  if (!ok) {
+    delete m;
+    if (msg) *msg = "cuTensorMapEncodeTiled rejected a weight or workspace tensor";
+    return 1;
+  }
+  L.maps = m;
+  L.ready = true;
+  return 0;
+}
+
+void tc_destroy(TcLayer& L) {
+  delete (Maps*)L.maps;
+  L.maps = nullptr;
   L.ready = false;
-  if (msg) *msg = "tensor-core FFN kernels not built";
-  return 1;
 }
-void tc_destroy(TcLayer&) {}
-int tc_tile_rows(const TcLayer&, int) { return kSimtTileRows; }
-int tc_down_split(const TcLayer&, int) { return 1; }
-int tc_max_split(const TcLayer&) { return 1; }
-cudaError_t tc_launch_up(const TcLayer&, const TcCall&, bool, cudaStream_t) {
-  return cudaErrorNotSupported;
+
+cudaError_t tc_launch_gather(const TcLayer& L, const TcCall& c, cudaStream_t st) {
+  const int rows = c.T * L.K;
+  const int vecs = L.d / 8;
+  gather_rows_kernel<<<rows, std::min(256, vecs), 0, st>>>(
+      (const uint4*)c.x, c.perm_tok, c.offs + L.E, vecs, (uint4*)c.xperm);
+  return cudaGetLastError();
 }
-cudaError_t tc_launch_down(const TcLayer&, const TcCall&, bool, int, cudaStream_t) {
-  return cudaErrorNotSupported;
+
+cudaError_t tc_launch_up(const TcLayer& L, const TcCall& c, bool shared, cudaStream_t st) {
+  const Maps* m = (const Maps*)L.maps;
+  TcArgs a;
+  std::memset(&a, 0, sizeof(a));
+  const int bn = c.tile_rows;
+  a.M = shared ? L.Fs : L.F;
+  a.m_tiles = (a.M + kBM - 1) / kBM;
+  a.kblocks = L.d / kBK;
+  a.n_split = 1;
+  a.kb_per_split = a.kblocks;
+  a.a_rows_per_group = a.M;
+  a.err = c.status;
+  long long max_tiles;
+  if (shared) {
+    CUtensorMap xm;
+    if (!encode_2d(&xm, c.x, c.T, L.d, bn)) return cudaErrorInvalidValue;
+    a.n_groups = L.S;
+    a.uniform_rows = c.T;
+    a.b_shift_per_group = c.T;
+    a.out = c.sact;
+    max_tiles = (long long)L.S * ((c.T + bn - 1) / bn);
+    const long long units = max_tiles * a.m_tiles;
+    const int grid = (int)std::min<long long>(L.num_sms, units);
+    return launch_bn<true>(bn, m->wsg, m->wsu, xm, a, grid, st);
+  }
+  a.n_groups = L.E;
+  a.row_offs = c.offs;
+  a.tile_offs = c.tile_offs;
+  a.out = c.act;
+  max_tiles = (long long)(c.T * L.K + bn - 1) / bn + L.E;
+  const long long units = max_tiles * a.m_tiles;
+  const int grid = (int)std::min<long long>(L.num_sms, units);
+  return launch_bn<true>(bn, m->wg, m->wu, m->xperm[bn_index(bn)], a, grid, st);
+}
+
+cudaError_t tc_launch_down(const TcLayer& L, const TcCall& c, bool shared, int n_split,
+                           cudaStream_t st) {
+  const Maps* m = (const Maps*)L.maps;
+  TcArgs a;
+  std::memset(&a, 0, sizeof(a));
+  const int bn = c.tile_rows;
+  const int Kdim = shared ? L.Fs : L.F;
+  a.M = L.d;
+  a.m_tiles = (L.d + kBM - 1) / kBM;
+  a.kblocks = Kdim / kBK;
+  a.n_split = n_split;
+  a.kb_per_split = (a.kblocks + n_split - 1) / n_split;
+  a.a_rows_per_group = L.d;
+  a.err = c.status;
+  long long max_tiles;
+  if (shared) {
+    a.n_groups = L.S;
+    a.uniform_rows = c.T;
+    a.out = c.sout;
+    a.split_stride = 0;
+    max_tiles = (long long)L.S * ((c.T + bn - 1) / bn);
+    const long long units = max_tiles * a.m_tiles;
+    const int grid = (int)std::min<long long>(L.num_sms, units);
+    return launch_bn<false>(bn, m->wsd, m->wsd, m->sact[bn_index(bn)], a, grid, st);
+  }
+  a.n_groups = L.E;
+  a.row_offs = c.offs;
+  a.tile_offs = c.tile_offs;
+  a.out = c.opart;
+  a.split_stride = (long long)c.T * L.K * L.d;
+  max_tiles = (long long)(c.T * L.K + bn - 1) / bn + L.E;
+  const long long units = max_tiles * a.m_tiles * n_split;
+  const int grid = (int)std::min<long long>(L.num_sms, units);
+  return launch_bn<false>(bn, m->wd, m->wd, m->act[bn_index(bn)], a, grid, st);
 }
 
 }  // namespace eat

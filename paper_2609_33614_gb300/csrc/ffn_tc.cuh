@@ -9,29 +9,35 @@ namespace eat {
 struct TcLayer {
   bool ready = false;
   int E = 0, d = 0, F = 0, S = 0, Fs = 0, K = 0, Tmax = 0;
+  int num_sms = 0;
   void* maps = nullptr;  // host copy of the tensor maps (see ffn_tc.cu)
 };
 
 struct TcCall {
-  const void* x = nullptr;
+  const void* x = nullptr;         // [T, d] bf16 hidden states of the call
   int T = 0;
-  int tile_rows = 0;
-  const int32_t* offs = nullptr;
+  int tile_rows = 0;               // BN: token rows per tile
+  const int32_t* offs = nullptr;   // [E+1] slot offsets
   const int32_t* tile_offs = nullptr;
   const int32_t* perm_tok = nullptr;
-  void* act = nullptr;
-  float* opart = nullptr;
-  void* sact = nullptr;
-  float* sout = nullptr;
-  int max_split = 1;
+  void* xperm = nullptr;           // [Tmax*K, d] gathered rows in slot order
+  void* act = nullptr;             // [Tmax*K, F] bf16
+  float* opart = nullptr;          // [split][T*K, d] fp32
+  void* sact = nullptr;            // [S*T, Fs] bf16
+  float* sout = nullptr;           // [S*T, d] fp32
+  unsigned int* status = nullptr;  // device status word (bounded-wait failures)
 };
 
-// 0 on success; *msg explains a failure.
-int tc_init(TcLayer& L, const eat_layer_desc& D, int K, int Tmax, const char** msg);
+// Device checks and the tensor-map encoder; 0 on success, *msg explains a failure.
+int tc_configure(TcLayer& L, const eat_layer_desc& D, int K, int Tmax, const char** msg);
+// Tensor maps over the weights and the handle's workspace buffers.
+int tc_bind(TcLayer& L, const eat_layer_desc& D, void* xperm, void* act, void* sact,
+            const char** msg);
 void tc_destroy(TcLayer& L);
 int tc_tile_rows(const TcLayer& L, int T);   // token rows per tile for a call of T tokens
 int tc_down_split(const TcLayer& L, int T);  // split-K slices of the routed down projection
-int tc_max_split(const TcLayer& L);
+long long tc_opart_rows(const TcLayer& L);   // rows of fp32 partials the workspace must hold
+cudaError_t tc_launch_gather(const TcLayer& L, const TcCall& c, cudaStream_t st);
 cudaError_t tc_launch_up(const TcLayer& L, const TcCall& c, bool shared, cudaStream_t st);
 cudaError_t tc_launch_down(const TcLayer& L, const TcCall& c, bool shared, int n_split,
                            cudaStream_t st);

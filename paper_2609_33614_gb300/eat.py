@@ -165,9 +165,10 @@ def eat_get_call_stats(h, n_e=None, sum_p=None, sum_norm=None, stream=None):
 
 
 def eat_get_counters(h) -> dict:
-    out = (c_i64 * 4)()
-    _check(lib().eat_get_counters(h, out, 4), h)
-    return {"calls": out[0], "union_sum": out[1], "activations": out[2], "launches": out[3]}
+    out = (c_i64 * 5)()
+    _check(lib().eat_get_counters(h, out, 5), h)
+    return {"calls": out[0], "union_sum": out[1], "activations": out[2], "launches": out[3],
+            "status": out[4]}
 
 
 def eat_profile_begin(h, capacity: int):
