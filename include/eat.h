@@ -115,7 +115,7 @@ eat_status eat_route(eat_handle* h, const void* x, int32_t T, int32_t ppl_sign,
  * the account update: N_e += n_e, P_total,e += sum of p over e's activations,
  * C_e <- (1 - alpha) C_e + alpha * mean ||E_e(x_t)||_2 when n_e > 0.
  * idx_opt / w_opt / k_opt may be NULL; when given they receive the routing as in eat_route.
- * y must not alias x. */
+ * y must not alias x; x and y must be 16-byte aligned. */
 eat_status eat_moe_forward(eat_handle* h, const void* x, int32_t T, int32_t ppl_sign, void* y,
                            int32_t* idx_opt, float* w_opt, int32_t* k_opt, void* stream);
 

@@ -5,6 +5,7 @@
 
 #include <algorithm>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <new>
 #include <string>
@@ -36,7 +37,8 @@ struct eat_handle {
   PermuteOut perm{};
   void* act = nullptr;    // [Tmax*K, F]
   float* opart = nullptr; // [splits][Tmax*K, d]
-  float* onorm = nullptr; // [Tmax*K]
+  float* nrm_part = nullptr; // [Tmax*K, column blocks] partial sums of squares of expert rows
+  int nb = 1;                 // column blocks per row in the combine kernel
   void* sact = nullptr;   // [S*Tmax, Fs]
   float* sout = nullptr;  // [S*Tmax, d]
   void* xstage = nullptr; // [Tmax, d]
@@ -207,11 +209,11 @@ eat_status run_forward(eat_handle* h, const void* x, int T, int ppl_sign, void* 
   }
   EAT_TRY(launch(h, kCombine, st, "combine", [&] {
     return launch_combine(h->bf16, h->opart, n_split, rows, h->perm.slot_of, h->w,
-                          h->k, h->sout, h->S, T, h->K, h->d, y, h->onorm, st);
+                          h->k, h->sout, h->S, T, h->K, h->d, y, h->nrm_part, st);
   }));
   EAT_TRY(launch(h, kAccount, st, "account update", [&] {
-    return launch_account(h->perm.offs, h->perm.perm_p, h->onorm, h->E, h->prm.alpha, h->N, h->P,
-                          h->C, h->st_n, h->st_p, h->st_norm, h->counters, st);
+    return launch_account(h->perm.offs, h->perm.perm_p, h->nrm_part, h->nb, h->E, h->prm.alpha,
+                          h->N, h->P, h->C, h->st_n, h->st_p, h->st_norm, h->counters, st);
   }));
   if (idx_opt || w_opt || k_opt) {
     cudaError_t e = cudaSuccess;
@@ -353,7 +355,8 @@ eat_status eat_create(const eat_layer_desc* desc, const eat_params* params, eat_
   add(&h->perm.active, sizeof(int32_t) * (h->E + 1));
   add(&h->act, h->elt * rows * h->F);
   add(&h->opart, sizeof(float) * (size_t)h->opart_rows * h->d);
-  add(&h->onorm, sizeof(float) * rows);
+  h->nb = combine_col_blocks(h->d);
+  add(&h->nrm_part, sizeof(float) * rows * h->nb);
   if (h->S > 0) {
     add(&h->sact, h->elt * (size_t)h->S * h->Tmax * h->Fs);
     add(&h->sout, sizeof(float) * (size_t)h->S * h->Tmax * h->d);
@@ -419,6 +422,7 @@ eat_status eat_moe_forward(eat_handle* h, const void* x, int32_t T, int32_t ppl_
   EAT_TRY(check_call(h, x, T, ppl_sign));
   if (!y) return fail(h, EAT_ERR_INVALID_ARG, "y is NULL");
   if (y == x) return fail(h, EAT_ERR_INVALID_ARG, "y must not alias x");
+  if (((uintptr_t)y & 15) != 0) return fail(h, EAT_ERR_INVALID_ARG, "y must be 16-byte aligned");
   return run_forward(h, x, T, ppl_sign, y, idx_opt, w_opt, k_opt, (cudaStream_t)stream);
 }
 
@@ -563,4 +567,14 @@ const char* eat_status_string(eat_status s) {
 
 namespace eat {
 void set_thread_error(const char* msg) { g_err = msg ? msg : ""; }
+}  // namespace eat
+
+namespace eat {
+bool pdl_enabled() {
+  static const bool on = [] {
+    const char* v = getenv("EAT_PDL");
+    return !(v && v[0] == '0');
+  }();
+  return on;
+}
 }  // namespace eat

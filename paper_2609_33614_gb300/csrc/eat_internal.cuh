@@ -9,6 +9,32 @@
 
 namespace eat {
 
+// Programmatic dependent launch: every kernel of the chain waits for its predecessor's results
+// with griddepcontrol.wait before touching global data, and lets its successor be scheduled early
+// (the successor's CTAs then only run their local prologue until the wait returns).
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+bool pdl_enabled();
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t st, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = pdl_enabled() ? 1 : 0;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, ((KArgs)args)...);
+}
+
 constexpr int kMaxExperts = 256;
 constexpr int kMaxK = 16;
 
@@ -76,12 +102,13 @@ constexpr int kSimtTileRows = 32;
 // ---------------------------------------------------------------------------------------------
 // Combine / unpermute and account update
 // ---------------------------------------------------------------------------------------------
+int combine_col_blocks(int d);  // column blocks per token row in the combine kernel
 cudaError_t launch_combine(int y_bf16, const float* opart, int n_split, int split_stride_rows,
                            const int32_t* slot_of, const float* w, const int32_t* k,
-                           const float* sout, int S, int T, int K, int d, void* y, float* onorm,
-                           cudaStream_t st);
-cudaError_t launch_account(const int32_t* offs, const float* perm_p, const float* onorm, int E,
-                           double alpha, int64_t* N, double* P, double* C, int32_t* st_n,
+                           const float* sout, int S, int T, int K, int d, void* y,
+                           float* nrm_part, cudaStream_t st);
+cudaError_t launch_account(const int32_t* offs, const float* perm_p, const float* nrm_part, int nb,
+                           int E, double alpha, int64_t* N, double* P, double* C, int32_t* st_n,
                            double* st_p, double* st_norm, long long* counters, cudaStream_t st);
 
 // Records msg as the text eat_last_error(NULL) returns on this thread (entry points without a

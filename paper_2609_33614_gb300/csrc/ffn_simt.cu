@@ -72,6 +72,8 @@ ffn_simt_kernel(const TW* __restrict__ in, const TW* __restrict__ w0, const TW* 
   __shared__ float ws0[BF][BK + 1];
   __shared__ float ws1[GATEUP ? BF : 1][BK + 1];
   __shared__ int rows[BR];
+  pdl_wait();
+  pdl_launch_dependents();
   const TileInfo ti = find_tile(gm, blockIdx.y);
   if (!ti.ok) return;
   const int f0 = blockIdx.x * BF;
@@ -139,13 +141,11 @@ cudaError_t launch_ffn_gateup_simt(int dtype_bf16, const void* in, const void* w
   dim3 grid((Fout + BF - 1) / BF, gm.max_tiles);
   if (grid.y == 0) return cudaSuccess;
   if (dtype_bf16)
-    ffn_simt_kernel<__nv_bfloat16, true><<<grid, kThreads, 0, st>>>(
-        (const __nv_bfloat16*)in, (const __nv_bfloat16*)wg, (const __nv_bfloat16*)wu, Fout, Kdim,
-        gm, act);
-  else
-    ffn_simt_kernel<float, true><<<grid, kThreads, 0, st>>>(
-        (const float*)in, (const float*)wg, (const float*)wu, Fout, Kdim, gm, act);
-  return cudaGetLastError();
+    return launch_pdl(ffn_simt_kernel<__nv_bfloat16, true>, grid, dim3(kThreads), 0, st,
+                      (const __nv_bfloat16*)in, (const __nv_bfloat16*)wg,
+                      (const __nv_bfloat16*)wu, Fout, Kdim, gm, act);
+  return launch_pdl(ffn_simt_kernel<float, true>, grid, dim3(kThreads), 0, st, (const float*)in,
+                    (const float*)wg, (const float*)wu, Fout, Kdim, gm, act);
 }
 
 cudaError_t launch_ffn_down_simt(int dtype_bf16, const void* act, const void* wd, int Dout,
@@ -155,12 +155,12 @@ cudaError_t launch_ffn_down_simt(int dtype_bf16, const void* act, const void* wd
   GroupMap g2 = gm;
   g2.row_mode = kRowSlot;  // the down projection reads act rows in slot order
   if (dtype_bf16)
-    ffn_simt_kernel<__nv_bfloat16, false><<<grid, kThreads, 0, st>>>(
-        (const __nv_bfloat16*)act, (const __nv_bfloat16*)wd, nullptr, Dout, Kdim, g2, out);
-  else
-    ffn_simt_kernel<float, false><<<grid, kThreads, 0, st>>>(
-        (const float*)act, (const float*)wd, nullptr, Dout, Kdim, g2, out);
-  return cudaGetLastError();
+    return launch_pdl(ffn_simt_kernel<__nv_bfloat16, false>, grid, dim3(kThreads), 0, st,
+                      (const __nv_bfloat16*)act, (const __nv_bfloat16*)wd,
+                      (const __nv_bfloat16*)nullptr, Dout, Kdim, g2, (void*)out);
+  return launch_pdl(ffn_simt_kernel<float, false>, grid, dim3(kThreads), 0, st,
+                    (const float*)act, (const float*)wd, (const float*)nullptr, Dout, Kdim, g2,
+                    (void*)out);
 }
 
 }  // namespace eat

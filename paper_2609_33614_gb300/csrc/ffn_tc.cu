@@ -260,10 +260,17 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 1) tmem_alloc(tmem_slot, C::kTmemCols);
+  if (threadIdx.x == 32) {
+    asm volatile("prefetch.tensormap [%0];" ::"l"(&mapA0) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(&mapB) : "memory");
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  // everything above is local to the CTA; from here on it reads what earlier kernels wrote
+  pdl_wait();
+  pdl_launch_dependents();
 
   const int total_tiles = args.tile_offs
                               ? args.tile_offs[args.n_groups]
@@ -401,6 +408,8 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
 __global__ void gather_rows_kernel(const uint4* __restrict__ x, const int32_t* __restrict__ perm_tok,
                                    const int32_t* __restrict__ n_rows, int row_vecs,
                                    uint4* __restrict__ xperm) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int slot = blockIdx.x;
   if (slot >= *n_rows) return;
   const size_t src = (size_t)perm_tok[slot] * row_vecs;
@@ -459,8 +468,8 @@ cudaError_t launch_tc(const CUtensorMap& a0, const CUtensorMap& a1, const CUtens
   });
   if (attr_err != cudaSuccess) return attr_err;
   if (grid <= 0) return cudaSuccess;
-  tc_ffn_kernel<BN, GATEUP><<<grid, kThreadsTc, C::kSmemBytes, st>>>(a0, a1, b, args);
-  return cudaGetLastError();
+  return launch_pdl(tc_ffn_kernel<BN, GATEUP>, dim3(grid), dim3(kThreadsTc), C::kSmemBytes, st,
+                    a0, a1, b, args);
 }
 
 template <bool GATEUP>
@@ -483,12 +492,18 @@ int tc_tile_rows(const TcLayer&, int T) {
   return 128;
 }
 
+// Split-K of the routed down projection: enough work units for ~8 waves of the persistent grid
+// (so the last, partial wave is a small fraction of a memory-bound launch), each K slice at least
+// 8 k-blocks (128 KB of weights per tile).  Estimated units = (token tiles + groups) x feature
+// tiles; prefill calls already have plenty and keep one slice.
 static int split_for(const TcLayer& L, int T) {
   const int m_tiles = (L.d + kBM - 1) / kBM;
   const int kblocks = L.F / kBK;
-  long long est = (long long)std::min(L.E, T * L.K) * m_tiles;
+  const int bn = tc_tile_rows(L, T);
+  const long long rows = (long long)T * L.K;
+  const long long est = ((rows + bn - 1) / bn + std::min<long long>(L.E, rows)) * m_tiles;
   int split = 1;
-  while (est * split < 2LL * L.num_sms && kblocks / (split * 2) >= 8 && split < 16) split *= 2;
+  while (est * split < 8LL * L.num_sms && kblocks / (split * 2) >= 8 && split < 32) split *= 2;
   return split;
 }
 
@@ -573,9 +588,8 @@ void tc_destroy(TcLayer& L) {
 cudaError_t tc_launch_gather(const TcLayer& L, const TcCall& c, cudaStream_t st) {
   const int rows = c.T * L.K;
   const int vecs = L.d / 8;
-  gather_rows_kernel<<<rows, std::min(256, vecs), 0, st>>>(
-      (const uint4*)c.x, c.perm_tok, c.offs + L.E, vecs, (uint4*)c.xperm);
-  return cudaGetLastError();
+  return launch_pdl(gather_rows_kernel, dim3(rows), dim3(std::min(256, vecs)), 0, st,
+                    (const uint4*)c.x, c.perm_tok, c.offs + L.E, vecs, (uint4*)c.xperm);
 }
 
 cudaError_t tc_launch_up(const TcLayer& L, const TcCall& c, bool shared, cudaStream_t st) {

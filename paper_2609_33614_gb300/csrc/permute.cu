@@ -43,6 +43,8 @@ __global__ void __launch_bounds__(kPermThreads)
 permute_kernel(const int32_t* __restrict__ idx, const int32_t* __restrict__ kk,
                const float* __restrict__ psel, int T, int K, int E, int tile_rows, PermuteOut o) {
   extern __shared__ int sm[];
+  pdl_wait();
+  pdl_launch_dependents();
   int* cnt = sm;                      // [E]
   int* cursor = cnt + E;              // [E]
   int* wcnt = cursor + E;             // [kPermWarps][E]
@@ -114,8 +116,8 @@ permute_kernel(const int32_t* __restrict__ idx, const int32_t* __restrict__ kk,
 cudaError_t launch_permute(const int32_t* idx, const int32_t* k, const float* psel, int T, int K,
                            int E, int tile_rows, PermuteOut o, cudaStream_t st) {
   const size_t smem = (size_t)(2 * E + kPermWarps * E) * sizeof(int);
-  permute_kernel<<<1, kPermThreads, smem, st>>>(idx, k, psel, T, K, E, tile_rows, o);
-  return cudaGetLastError();
+  return launch_pdl(permute_kernel, dim3(1), dim3(kPermThreads), smem, st, idx, k, psel, T, K, E,
+                    tile_rows, o);
 }
 
 }  // namespace eat

@@ -1,7 +1,8 @@
 // Router and EAT selection (§3.1-§3.4 of the EAT paper, Eq. 1-8).
 //
-//  router_logits_kernel: partial router scores x . w_r over slices of d: fp32 FMA inside
-//      32-wide chunks, chunk sums accumulated in fp64, so the logits carry ~1e-7 absolute error
+//  router_logits_small_kernel (T <= 128, decode) / router_logits_kernel (tiled through shared
+//      memory, prefill): partial router scores x . w_r over slices of d: fp32 FMA inside
+//      16- or 32-wide chunks, chunk sums accumulated in fp64, so the logits carry ~1e-7 absolute error
 //      (the selection compares I against tau at 1e-5 and P_total sums p at 1e-6 relative; a
 //      [T, E] GEMM this small and this precision-sensitive stays off the bf16 tensor path).
 //  route_select_kernel: one warp per token.  Each lane owns experts lane, lane+32, ...; the warp
@@ -39,6 +40,8 @@ __global__ void __launch_bounds__(kLogitThreads)
 router_logits_kernel(const TX* __restrict__ x, const float* __restrict__ wr, int T, int d, int E,
                      int TT, int d_per_split, double* __restrict__ part) {
   extern __shared__ float sm[];
+  pdl_wait();
+  pdl_launch_dependents();
   float* xs = sm;                        // [TT][kChunk + 1]
   float* ws = sm + TT * (kChunk + 1);    // [E][kChunk + 1]
   const int tid = threadIdx.x;
@@ -85,6 +88,58 @@ router_logits_kernel(const TX* __restrict__ x, const float* __restrict__ wr, int
       const int t = t0 + tt;
       if (t < T) part[((size_t)blockIdx.y * T + t) * E + e] = acc[q];
     }
+  }
+}
+
+// Router scores for small T (decode): block (t, s) computes part[s][t][e] for every expert over
+// the s-th slice of d; warp w takes experts w, w + 8, ...; lanes read float4 pieces of the weight
+// row and of x (coalesced), multiply in fp32, fold each 16 products into an fp64 lane sum, and the
+// 32 lane sums are added in fp64 (a fixed tree).
+constexpr int kSmallT = 128;
+constexpr int kSmallSlice = 512;
+
+__device__ __forceinline__ float4 load_x4(const float* p) { return *(const float4*)p; }
+__device__ __forceinline__ float4 load_x4(const __nv_bfloat16* p) {
+  const uint2 u = *(const uint2*)p;
+  const __nv_bfloat162 a = *(const __nv_bfloat162*)&u.x;
+  const __nv_bfloat162 b = *(const __nv_bfloat162*)&u.y;
+  const float2 fa = __bfloat1622float2(a), fb = __bfloat1622float2(b);
+  return make_float4(fa.x, fa.y, fb.x, fb.y);
+}
+
+template <typename TX>
+__global__ void __launch_bounds__(kLogitThreads)
+router_logits_small_kernel(const TX* __restrict__ x, const float* __restrict__ wr, int T, int d,
+                           int E, int d_per_split, double* __restrict__ part) {
+  pdl_wait();
+  pdl_launch_dependents();
+  const int t = blockIdx.x, s = blockIdx.y;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int beg = s * d_per_split;
+  const int end = min(d, beg + d_per_split);
+  const TX* xr = x + (size_t)t * d;
+  for (int e = warp; e < E; e += kLogitThreads / 32) {
+    const float* wrow = wr + (size_t)e * d;
+    double dacc = 0.0;
+    float acc = 0.f;
+    int cnt = 0;
+    for (int c = beg + lane * 4; c < end; c += 128) {
+      const float4 wv = *(const float4*)(wrow + c);
+      const float4 xv = load_x4(xr + c);
+      acc = fmaf(xv.x, wv.x, acc);
+      acc = fmaf(xv.y, wv.y, acc);
+      acc = fmaf(xv.z, wv.z, acc);
+      acc = fmaf(xv.w, wv.w, acc);
+      if (++cnt == 4) {
+        dacc += (double)acc;
+        acc = 0.f;
+        cnt = 0;
+      }
+    }
+    dacc += (double)acc;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) dacc += __shfl_xor_sync(0xffffffffu, dacc, o);
+    if (lane == 0) part[((size_t)s * T + t) * E + e] = dacc;
   }
 }
 
@@ -161,6 +216,8 @@ route_select_kernel(const double* __restrict__ part, int n_split, const float* _
                     RouteParams rp, int32_t* __restrict__ out_idx, float* __restrict__ out_w,
                     int32_t* __restrict__ out_k, float* __restrict__ out_p) {
   __shared__ float s_h[kMaxExperts];
+  pdl_wait();
+  pdl_launch_dependents();
   history_score_block(accN, accP, accC, E, rp, s_h);
 
   const int lane = threadIdx.x & 31;
@@ -332,7 +389,8 @@ route_select_kernel(const double* __restrict__ part, int n_split, const float* _
 }  // namespace
 
 int router_split(int T, int d, int E) {
-  // Enough blocks to cover the SMs when T is small; each slice at least 256 of d.
+  if (T <= kSmallT) return (d + kSmallSlice - 1) / kSmallSlice;
+  // Enough blocks to cover the SMs; each slice at least 256 of d.
   const int tt = logits_tile_tokens(E);
   const int tblocks = (T + tt - 1) / tt;
   int split = 1;
@@ -342,18 +400,27 @@ int router_split(int T, int d, int E) {
 
 cudaError_t launch_router_logits(const void* x, int x_bf16, const float* w_router, int T, int d,
                                  int E, int n_split, double* part, cudaStream_t st) {
+  const bool vec_ok = d % 4 == 0 && ((uintptr_t)x & 15) == 0 && ((uintptr_t)w_router & 15) == 0;
+  if (T <= kSmallT && vec_ok) {
+    int per = (d + n_split - 1) / n_split;
+    per = (per + 127) / 128 * 128;
+    dim3 grid(T, n_split);
+    if (x_bf16)
+      return launch_pdl(router_logits_small_kernel<__nv_bfloat16>, grid, dim3(kLogitThreads), 0,
+                        st, (const __nv_bfloat16*)x, w_router, T, d, E, per, part);
+    return launch_pdl(router_logits_small_kernel<float>, grid, dim3(kLogitThreads), 0, st,
+                      (const float*)x, w_router, T, d, E, per, part);
+  }
   const int TT = logits_tile_tokens(E);
   int per = (d + n_split - 1) / n_split;
   per = (per + kChunk - 1) / kChunk * kChunk;
   dim3 grid((T + TT - 1) / TT, n_split);
   const size_t smem = (size_t)(TT + E) * (kChunk + 1) * sizeof(float);
   if (x_bf16)
-    router_logits_kernel<__nv_bfloat16><<<grid, kLogitThreads, smem, st>>>(
-        (const __nv_bfloat16*)x, w_router, T, d, E, TT, per, part);
-  else
-    router_logits_kernel<float><<<grid, kLogitThreads, smem, st>>>((const float*)x, w_router, T,
-                                                                    d, E, TT, per, part);
-  return cudaGetLastError();
+    return launch_pdl(router_logits_kernel<__nv_bfloat16>, grid, dim3(kLogitThreads), smem, st,
+                      (const __nv_bfloat16*)x, w_router, T, d, E, TT, per, part);
+  return launch_pdl(router_logits_kernel<float>, grid, dim3(kLogitThreads), smem, st,
+                    (const float*)x, w_router, T, d, E, TT, per, part);
 }
 
 cudaError_t launch_route_select(const double* part, int n_split, const float* b_router, int T,
@@ -362,16 +429,14 @@ cudaError_t launch_route_select(const double* part, int n_split, const float* b_
                                 int32_t* k, float* psel, cudaStream_t st) {
   const int warps = kSelectThreads / 32;
   dim3 grid((T + warps - 1) / warps);
-#define EAT_SELECT(EPL)                                                                         \
-  route_select_kernel<EPL><<<grid, kSelectThreads, 0, st>>>(part, n_split, b_router, T, E, K,  \
-                                                            accN, accP, accC, rp, idx, w, k,   \
-                                                            psel)
-  if (E <= 32) EAT_SELECT(1);
-  else if (E <= 64) EAT_SELECT(2);
-  else if (E <= 128) EAT_SELECT(4);
-  else EAT_SELECT(8);
+#define EAT_SELECT(EPL)                                                                    \
+  launch_pdl(route_select_kernel<EPL>, grid, dim3(kSelectThreads), 0, st, part, n_split,    \
+             b_router, T, E, K, accN, accP, accC, rp, idx, w, k, psel)
+  if (E <= 32) return EAT_SELECT(1);
+  if (E <= 64) return EAT_SELECT(2);
+  if (E <= 128) return EAT_SELECT(4);
+  return EAT_SELECT(8);
 #undef EAT_SELECT
-  return cudaGetLastError();
 }
 
 }  // namespace eat
