@@ -45,6 +45,7 @@ struct eat_handle {
   void* ystage = nullptr; // [Tmax, d]
   void* xperm = nullptr;  // [Tmax*K, d] gathered token rows (tensor-core path)
   unsigned int* status = nullptr;  // device status word: bounded waits that expired
+  int32_t* chunk_cnt = nullptr;    // [permute chunks][E]
   long long opart_rows = 0;
 
   TcLayer tc{};
@@ -136,15 +137,15 @@ eat_status check_call(eat_handle* h, const void* x, int32_t T, int32_t ppl_sign)
 // Router + selection into (idx, w, k, psel).
 eat_status run_route(eat_handle* h, const void* x, int T, int ppl_sign, int32_t* idx, float* w,
                      int32_t* k, float* psel, cudaStream_t st) {
+  const RouteParams rp = route_params(h->prm, ppl_sign);
   const int split = router_split(T, h->d, h->E);
   EAT_TRY(launch(h, kRoute, st, "router logits", [&] {
     return launch_router_logits(x, h->bf16, h->desc.w_router, T, h->d, h->E, split,
                                 h->logit_part, st);
   }));
-  const RouteParams rp = route_params(h->prm, ppl_sign);
   EAT_TRY(launch(h, kRoute, st, "route select", [&] {
-    return launch_route_select(h->logit_part, split, h->desc.b_router, T, h->E, h->K, h->N, h->P,
-                               h->C, rp, idx, w, k, psel, st);
+    return launch_route_select(h->logit_part, split, h->desc.b_router, T, h->E, h->K, h->N,
+                               h->P, h->C, rp, idx, w, k, psel, st);
   }));
   return EAT_OK;
 }
@@ -154,7 +155,8 @@ eat_status run_forward(eat_handle* h, const void* x, int T, int ppl_sign, void* 
   EAT_TRY(run_route(h, x, T, ppl_sign, h->idx, h->w, h->k, h->psel, st));
   const int tile_rows = h->backend == 1 ? tc_tile_rows(h->tc, T) : kSimtTileRows;
   EAT_TRY(launch(h, kPermute, st, "permute", [&] {
-    return launch_permute(h->idx, h->k, h->psel, T, h->K, h->E, tile_rows, h->perm, st);
+    return launch_permute(h->idx, h->k, h->psel, T, h->K, h->E, tile_rows, h->perm, h->chunk_cnt,
+                          st);
   }));
   const int rows = T * h->K;
   int n_split = 1;
@@ -361,7 +363,10 @@ eat_status eat_create(const eat_layer_desc* desc, const eat_params* params, eat_
     add(&h->sact, h->elt * (size_t)h->S * h->Tmax * h->Fs);
     add(&h->sout, sizeof(float) * (size_t)h->S * h->Tmax * h->d);
   }
-  if (h->backend == 1) add(&h->xperm, h->elt * rows * h->d);
+  if (h->backend == 1) {
+    add(&h->xperm, h->elt * rows * h->d);
+  }
+  add(&h->chunk_cnt, sizeof(int32_t) * (size_t)permute_chunks(h->Tmax) * h->E);
   add(&h->xstage, h->elt * (size_t)h->Tmax * h->d);
   add(&h->ystage, h->elt * (size_t)h->Tmax * h->d);
   size_t total = 0;

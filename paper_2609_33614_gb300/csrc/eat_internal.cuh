@@ -50,11 +50,13 @@ struct RouteParams {
 // Partial router logits (fp64): part[s][t][e] = sum over the s-th slice of d of x[t,j] Wr[e,j].
 cudaError_t launch_router_logits(const void* x, int x_bf16, const float* w_router, int T, int d,
                                  int E, int n_split, double* part, cudaStream_t st);
-// Warp-per-token softmax + history score + threshold + selection + renormalisation.
+// Warp-per-token softmax + history score + threshold + selection + renormalisation; the router
+// scores are the sum over the n_split slices of part (fp64 [split][T][E]).
 cudaError_t launch_route_select(const double* part, int n_split, const float* b_router, int T,
                                 int E, int K, const int64_t* accN, const double* accP,
                                 const double* accC, RouteParams rp, int32_t* idx, float* w,
                                 int32_t* k, float* psel, cudaStream_t st);
+constexpr int kSmallRouterT = 128;  // calls up to this many tokens use the GEMV-style router
 int router_split(int T, int d, int E);
 
 // ---------------------------------------------------------------------------------------------
@@ -69,8 +71,10 @@ struct PermuteOut {
   float* perm_p;       // [T*K] p of each slot
   int32_t* active;     // [E+1] ascending active experts, active[E] = count
 };
+int permute_chunks(int T);  // CTAs (1024-token chunks) of the permute; chunk_cnt holds [chunks][E]
 cudaError_t launch_permute(const int32_t* idx, const int32_t* k, const float* psel, int T, int K,
-                           int E, int tile_rows, PermuteOut o, cudaStream_t st);
+                           int E, int tile_rows, PermuteOut o, int32_t* chunk_cnt,
+                           cudaStream_t st);
 
 // ---------------------------------------------------------------------------------------------
 // Expert FFNs

@@ -1,10 +1,11 @@
 // Permute by expert: groups the selected (token, expert) pairs of one call by expert so that the
 // expert FFNs read contiguous row lists ("only activated experts participate", §3.4).
 //
-// One CTA of 1024 threads.  Pass 1 counts n_e with shared-memory atomics (integer, order-free)
-// and scans them into slot offsets and row-tile offsets.  Pass 2 walks the tokens in chunks of
-// 1024 and gives every pair a STABLE slot (tokens ascending inside each expert): each warp finds
-// the experts present among its 32 tokens with ballots, counts them per warp, the counts are
+// Tokens are split in chunks of 1024, one CTA each (a call of at most 1024 tokens runs as a single
+// CTA that also counts).  Counts n_e come from shared-memory atomics (integers, order-free); each
+// chunk's first slot per expert is the expert's offset plus the counts of the earlier chunks.
+// Inside a chunk every pair gets a STABLE slot (tokens ascending inside each expert): each warp
+// finds the experts present among its 32 tokens with ballots, counts them per warp, the counts are
 // scanned across warps per expert, and the same ballots give each lane its rank.  Stable slots
 // make every later per-expert sum (P_total, the EMA norm mean) run in a fixed order.
 #include "eat_internal.cuh"
@@ -39,47 +40,92 @@ __device__ __forceinline__ void for_each_warp_expert(const int* ex, int K, Fn fn
   }
 }
 
+// Per-chunk expert counts (large calls): chunk_cnt[c][e] = activations of expert e among tokens
+// [c * 1024, (c + 1) * 1024).
 __global__ void __launch_bounds__(kPermThreads)
-permute_kernel(const int32_t* __restrict__ idx, const int32_t* __restrict__ kk,
-               const float* __restrict__ psel, int T, int K, int E, int tile_rows, PermuteOut o) {
+permute_count_kernel(const int32_t* __restrict__ idx, int T, int K, int E,
+                     int32_t* __restrict__ chunk_cnt) {
+  extern __shared__ int cnt[];
+  pdl_wait();
+  pdl_launch_dependents();
+  const int tid = threadIdx.x, c = blockIdx.x;
+  for (int e = tid; e < E; e += kPermThreads) cnt[e] = 0;
+  __syncthreads();
+  const int t0 = c * kPermThreads, t1 = min(T, t0 + kPermThreads);
+  for (int i = t0 * K + tid; i < t1 * K; i += kPermThreads) {
+    const int e = idx[i];
+    if (e >= 0) atomicAdd(&cnt[e], 1);
+  }
+  __syncthreads();
+  for (int e = tid; e < E; e += kPermThreads) chunk_cnt[(size_t)c * E + e] = cnt[e];
+}
+
+// Slot assignment of one chunk of 1024 tokens.  With chunk_cnt == nullptr the kernel runs as a
+// single CTA over a call of at most 1024 tokens and counts in place.
+__global__ void __launch_bounds__(kPermThreads)
+permute_assign_kernel(const int32_t* __restrict__ idx, const int32_t* __restrict__ kk,
+                      const float* __restrict__ psel, int T, int K, int E, int tile_rows,
+                      const int32_t* __restrict__ chunk_cnt, int n_chunks, PermuteOut o) {
   extern __shared__ int sm[];
   pdl_wait();
   pdl_launch_dependents();
-  int* cnt = sm;                      // [E]
-  int* cursor = cnt + E;              // [E]
+  int* cnt = sm;                      // [E] activations of each expert in the whole call
+  int* cursor = cnt + E;              // [E] first slot of each expert for this chunk
   int* wcnt = cursor + E;             // [kPermWarps][E]
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int c = blockIdx.x;
   const unsigned lt = (1u << lane) - 1u;
 
-  for (int e = tid; e < E; e += kPermThreads) cnt[e] = 0;
-  __syncthreads();
-  for (int i = tid; i < T * K; i += kPermThreads) {
-    const int e = idx[i];
-    if (e >= 0) atomicAdd(&cnt[e], 1);
+  if (chunk_cnt == nullptr) {
+    for (int e = tid; e < E; e += kPermThreads) {
+      cnt[e] = 0;
+      cursor[e] = 0;
+    }
+    __syncthreads();
+    for (int i = tid; i < T * K; i += kPermThreads) {
+      const int e = idx[i];
+      if (e >= 0) atomicAdd(&cnt[e], 1);
+    }
+  } else {
+    for (int e = tid; e < E; e += kPermThreads) {
+      int tot = 0, before = 0;
+      for (int cc = 0; cc < n_chunks; ++cc) {
+        const int v = chunk_cnt[(size_t)cc * E + e];
+        tot += v;
+        if (cc < c) before += v;
+      }
+      cnt[e] = tot;
+      cursor[e] = before;
+    }
   }
   __syncthreads();
   if (tid == 0) {
     int s = 0, ts = 0, na = 0;
     for (int e = 0; e < E; ++e) {
-      o.offs[e] = s;
-      o.tile_offs[e] = ts;
-      o.n_e[e] = cnt[e];
-      cursor[e] = s;
-      if (cnt[e] > 0) o.active[na++] = e;
+      if (c == 0) {
+        o.offs[e] = s;
+        o.tile_offs[e] = ts;
+        o.n_e[e] = cnt[e];
+        if (cnt[e] > 0) o.active[na++] = e;
+      }
+      cursor[e] += s;
       s += cnt[e];
       ts += (cnt[e] + tile_rows - 1) / tile_rows;
     }
-    o.offs[E] = s;
-    o.tile_offs[E] = ts;
-    for (int e = na; e < E; ++e) o.active[e] = -1;
-    o.active[E] = na;
+    if (c == 0) {
+      o.offs[E] = s;
+      o.tile_offs[E] = ts;
+      for (int e = na; e < E; ++e) o.active[e] = -1;
+      o.active[E] = na;
+    }
   }
   __syncthreads();
 
   int ex[kMaxK];
-  for (int c0 = 0; c0 < T; c0 += kPermThreads) {
+  const int c_end = chunk_cnt == nullptr ? T : min(T, (c + 1) * kPermThreads);
+  for (int c0 = c * kPermThreads; c0 < c_end; c0 += kPermThreads) {
     const int t = c0 + tid;
-    const int kt = t < T ? kk[t] : 0;
+    const int kt = t < c_end ? kk[t] : 0;
     for (int j = 0; j < K; ++j) ex[j] = (j < kt) ? idx[(size_t)t * K + j] : -1;
     for (int e = lane; e < E; e += 32) wcnt[warp * E + e] = 0;
     __syncwarp();
@@ -90,9 +136,9 @@ permute_kernel(const int32_t* __restrict__ idx, const int32_t* __restrict__ kk,
     for (int e = tid; e < E; e += kPermThreads) {
       int run = cursor[e];
       for (int w = 0; w < kPermWarps; ++w) {
-        const int c = wcnt[w * E + e];
+        const int v = wcnt[w * E + e];
         wcnt[w * E + e] = run;
-        run += c;
+        run += v;
       }
       cursor[e] = run;
     }
@@ -105,7 +151,7 @@ permute_kernel(const int32_t* __restrict__ idx, const int32_t* __restrict__ kk,
         o.perm_p[slot] = psel[(size_t)t * K + jj];
       }
     });
-    if (t < T)
+    if (t < c_end)
       for (int j = kt; j < K; ++j) o.slot_of[(size_t)t * K + j] = -1;
     __syncthreads();
   }
@@ -113,11 +159,21 @@ permute_kernel(const int32_t* __restrict__ idx, const int32_t* __restrict__ kk,
 
 }  // namespace
 
+int permute_chunks(int T) { return (T + kPermThreads - 1) / kPermThreads; }
+
 cudaError_t launch_permute(const int32_t* idx, const int32_t* k, const float* psel, int T, int K,
-                           int E, int tile_rows, PermuteOut o, cudaStream_t st) {
+                           int E, int tile_rows, PermuteOut o, int32_t* chunk_cnt,
+                           cudaStream_t st) {
   const size_t smem = (size_t)(2 * E + kPermWarps * E) * sizeof(int);
-  return launch_pdl(permute_kernel, dim3(1), dim3(kPermThreads), smem, st, idx, k, psel, T, K, E,
-                    tile_rows, o);
+  const int n_chunks = permute_chunks(T);
+  if (n_chunks == 1)
+    return launch_pdl(permute_assign_kernel, dim3(1), dim3(kPermThreads), smem, st, idx, k, psel,
+                      T, K, E, tile_rows, (const int32_t*)nullptr, 1, o);
+  cudaError_t e = launch_pdl(permute_count_kernel, dim3(n_chunks), dim3(kPermThreads),
+                             (size_t)E * sizeof(int), st, idx, T, K, E, chunk_cnt);
+  if (e != cudaSuccess) return e;
+  return launch_pdl(permute_assign_kernel, dim3(n_chunks), dim3(kPermThreads), smem, st, idx, k,
+                    psel, T, K, E, tile_rows, (const int32_t*)chunk_cnt, n_chunks, o);
 }
 
 }  // namespace eat

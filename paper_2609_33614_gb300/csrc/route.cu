@@ -1,10 +1,11 @@
 // Router and EAT selection (§3.1-§3.4 of the EAT paper, Eq. 1-8).
 //
-//  router_logits_small_kernel (T <= 128, decode) / router_logits_kernel (tiled through shared
-//      memory, prefill): partial router scores x . w_r over slices of d: fp32 FMA inside
-//      16- or 32-wide chunks, chunk sums accumulated in fp64, so the logits carry ~1e-7 absolute error
-//      (the selection compares I against tau at 1e-5 and P_total sums p at 1e-6 relative; a
-//      [T, E] GEMM this small and this precision-sensitive stays off the bf16 tensor path).
+//  router_logits_small_kernel (T <= 128, decode) / router_logits_kernel (register-tiled through
+//      shared memory, prefill): partial router scores x . w_r over slices of d: fp32 FMA inside
+//      16- or 32-wide chunks, chunk sums accumulated in fp64 or Kahan-compensated fp32, so the
+//      logits carry ~1e-7 absolute error (the selection compares I against tau at 1e-5 and P_total
+//      sums p at 1e-6 relative).  The scores stay off the tensor cores: their fp32 accumulation
+//      biased the scores enough to move P_total by ~1e-6 relative.
 //  route_select_kernel: one warp per token.  Each lane owns experts lane, lane+32, ...; the warp
 //      does the softmax (§3.2), importance (Eq. 2), mean / population std (Eq. 3-4), tau (Eq. 5),
 //      PPL factor and smoothing (§3.3), the clamp to the type-7 q_lo / q_hi quantiles of p
@@ -19,74 +20,86 @@ namespace eat {
 
 namespace {
 
-constexpr int kChunk = 32;
 constexpr int kLogitThreads = 256;
-constexpr int kMaxOut = 8;  // outputs per thread in the logits kernel
 
 __device__ __forceinline__ float load_x(const float* p, size_t i) { return p[i]; }
 __device__ __forceinline__ float load_x(const __nv_bfloat16* p, size_t i) {
   return __bfloat162float(p[i]);
 }
 
-int logits_tile_tokens(int E) {
-  int tt = (kLogitThreads * kMaxOut) / E;
-  if (tt > 32) tt = 32;
-  if (tt < 1) tt = 1;
-  return tt;
+
+// Router scores for large T: CTA tile of 64 tokens x 64 experts over one slice of d, 256 threads
+// with 4 tokens x 4 experts each.  x and W_r chunks of 32 columns are staged transposed in shared
+// memory; every output takes 32 fp32 FMAs per chunk and the chunk sums are added with Kahan
+// compensation (fp32), so the score carries about the error of an fp64 sum of fp32 products.
+constexpr int kTileT = 64, kTileE = 64, kChunkK = 32;
+
+__device__ __forceinline__ void kahan_add(float& sum, float& comp, float v) {
+  const float y = v - comp;
+  const float t = sum + y;
+  comp = (t - sum) - y;
+  sum = t;
 }
 
 template <typename TX>
 __global__ void __launch_bounds__(kLogitThreads)
 router_logits_kernel(const TX* __restrict__ x, const float* __restrict__ wr, int T, int d, int E,
-                     int TT, int d_per_split, double* __restrict__ part) {
-  extern __shared__ float sm[];
+                     int d_per_split, double* __restrict__ part) {
+  __shared__ float xs[kChunkK][kTileT + 4];
+  __shared__ float ws[kChunkK][kTileE + 4];
   pdl_wait();
   pdl_launch_dependents();
-  float* xs = sm;                        // [TT][kChunk + 1]
-  float* ws = sm + TT * (kChunk + 1);    // [E][kChunk + 1]
   const int tid = threadIdx.x;
-  const int t0 = blockIdx.x * TT;
-  const int dbeg = blockIdx.y * d_per_split;
+  const int tx = tid & 15, ty = tid >> 4;
+  const int t0 = blockIdx.x * kTileT, e0 = blockIdx.y * kTileE;
+  const int dbeg = blockIdx.z * d_per_split;
   const int dend = min(d, dbeg + d_per_split);
-  const int n_out = TT * E;
-  double acc[kMaxOut];
+  float sum[4][4], comp[4][4];
 #pragma unroll
-  for (int q = 0; q < kMaxOut; ++q) acc[q] = 0.0;
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) sum[i][j] = comp[i][j] = 0.f;
 
-  for (int j0 = dbeg; j0 < dend; j0 += kChunk) {
-    for (int i = tid; i < TT * kChunk; i += kLogitThreads) {
-      const int tt = i / kChunk, jj = i % kChunk;
-      const int t = t0 + tt, j = j0 + jj;
-      xs[tt * (kChunk + 1) + jj] = (t < T && j < dend) ? load_x(x, (size_t)t * d + j) : 0.f;
-    }
-    for (int i = tid; i < E * kChunk; i += kLogitThreads) {
-      const int e = i / kChunk, jj = i % kChunk;
-      const int j = j0 + jj;
-      ws[e * (kChunk + 1) + jj] = (j < dend) ? wr[(size_t)e * d + j] : 0.f;
+  for (int k0 = dbeg; k0 < dend; k0 += kChunkK) {
+    // stage: 64 rows x 32 columns of x and of W_r, transposed (column-major in shared memory)
+    for (int i = tid; i < kTileT * kChunkK; i += kLogitThreads) {
+      const int r = i / kChunkK, kk = i % kChunkK;
+      const int t = t0 + r, k = k0 + kk;
+      xs[kk][r] = (t < T && k < dend) ? load_x(x, (size_t)t * d + k) : 0.f;
+      const int e = e0 + r;
+      ws[kk][r] = (e < E && k < dend) ? wr[(size_t)e * d + k] : 0.f;
     }
     __syncthreads();
+    float acc[4][4];
 #pragma unroll
-    for (int q = 0; q < kMaxOut; ++q) {
-      const int o = tid + q * kLogitThreads;
-      if (o < n_out) {
-        const int tt = o / E, e = o % E;
-        const float* xr = xs + tt * (kChunk + 1);
-        const float* wrow = ws + e * (kChunk + 1);
-        float a = 0.f;
+    for (int i = 0; i < 4; ++i)
 #pragma unroll
-        for (int jj = 0; jj < kChunk; ++jj) a = fmaf(xr[jj], wrow[jj], a);
-        acc[q] += (double)a;
-      }
+      for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
+#pragma unroll 8
+    for (int kk = 0; kk < kChunkK; ++kk) {
+      const float4 a = *(const float4*)&xs[kk][ty * 4];
+      const float4 b = *(const float4*)&ws[kk][tx * 4];
+      const float av[4] = {a.x, a.y, a.z, a.w}, bv[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
     }
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+      for (int j = 0; j < 4; ++j) kahan_add(sum[i][j], comp[i][j], acc[i][j]);
     __syncthreads();
   }
 #pragma unroll
-  for (int q = 0; q < kMaxOut; ++q) {
-    const int o = tid + q * kLogitThreads;
-    if (o < n_out) {
-      const int tt = o / E, e = o % E;
-      const int t = t0 + tt;
-      if (t < T) part[((size_t)blockIdx.y * T + t) * E + e] = acc[q];
+  for (int i = 0; i < 4; ++i) {
+    const int t = t0 + ty * 4 + i;
+    if (t >= T) continue;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int e = e0 + tx * 4 + j;
+      if (e < E)
+        part[((size_t)blockIdx.z * T + t) * E + e] = (double)sum[i][j] - (double)comp[i][j];
     }
   }
 }
@@ -95,8 +108,9 @@ router_logits_kernel(const TX* __restrict__ x, const float* __restrict__ wr, int
 // the s-th slice of d; warp w takes experts w, w + 8, ...; lanes read float4 pieces of the weight
 // row and of x (coalesced), multiply in fp32, fold each 16 products into an fp64 lane sum, and the
 // 32 lane sums are added in fp64 (a fixed tree).
-constexpr int kSmallT = 128;
+constexpr int kSmallT = kSmallRouterT;
 constexpr int kSmallSlice = 512;
+
 
 __device__ __forceinline__ float4 load_x4(const float* p) { return *(const float4*)p; }
 __device__ __forceinline__ float4 load_x4(const __nv_bfloat16* p) {
@@ -390,11 +404,10 @@ route_select_kernel(const double* __restrict__ part, int n_split, const float* _
 
 int router_split(int T, int d, int E) {
   if (T <= kSmallT) return (d + kSmallSlice - 1) / kSmallSlice;
-  // Enough blocks to cover the SMs; each slice at least 256 of d.
-  const int tt = logits_tile_tokens(E);
-  const int tblocks = (T + tt - 1) / tt;
+  // enough CTAs for two waves, each slice at least 256 columns of d
+  const long long tiles = (long long)((T + kTileT - 1) / kTileT) * ((E + kTileE - 1) / kTileE);
   int split = 1;
-  while (tblocks * split < 2 * 152 && d / (split * 2) >= 256 && split < 64) split *= 2;
+  while (tiles * split < 2 * 152 && d / (split * 2) >= 256 && split < 64) split *= 2;
   return split;
 }
 
@@ -411,16 +424,14 @@ cudaError_t launch_router_logits(const void* x, int x_bf16, const float* w_route
     return launch_pdl(router_logits_small_kernel<float>, grid, dim3(kLogitThreads), 0, st,
                       (const float*)x, w_router, T, d, E, per, part);
   }
-  const int TT = logits_tile_tokens(E);
   int per = (d + n_split - 1) / n_split;
-  per = (per + kChunk - 1) / kChunk * kChunk;
-  dim3 grid((T + TT - 1) / TT, n_split);
-  const size_t smem = (size_t)(TT + E) * (kChunk + 1) * sizeof(float);
+  per = (per + kChunkK - 1) / kChunkK * kChunkK;
+  dim3 grid((T + kTileT - 1) / kTileT, (E + kTileE - 1) / kTileE, n_split);
   if (x_bf16)
-    return launch_pdl(router_logits_kernel<__nv_bfloat16>, grid, dim3(kLogitThreads), smem, st,
-                      (const __nv_bfloat16*)x, w_router, T, d, E, TT, per, part);
-  return launch_pdl(router_logits_kernel<float>, grid, dim3(kLogitThreads), smem, st,
-                    (const float*)x, w_router, T, d, E, TT, per, part);
+    return launch_pdl(router_logits_kernel<__nv_bfloat16>, grid, dim3(kLogitThreads), 0, st,
+                      (const __nv_bfloat16*)x, w_router, T, d, E, per, part);
+  return launch_pdl(router_logits_kernel<float>, grid, dim3(kLogitThreads), 0, st,
+                    (const float*)x, w_router, T, d, E, per, part);
 }
 
 cudaError_t launch_route_select(const double* part, int n_split, const float* b_router, int T,
