@@ -199,9 +199,10 @@ def kernel_flops(kind, shape, acts, T):
     raise KeyError(kind)
 
 
-def traffic_for(kind, workload):
-    """DRAM bytes per launch from the committed ncu summary, if it was taken on the current
-    kernel sources (its source hash matches); else None."""
+def traffic_for(kind, workload, experts_per_launch):
+    """DRAM bytes per launch from the committed ncu summary (profiles/traffic.json), if it was
+    taken on the current kernel sources (its source hash matches); else None.  Decode captures are
+    stored per activated expert and scaled by this run's mean activated experts per launch."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         from paper_2609_33614_gb300 import build
@@ -209,6 +210,8 @@ def traffic_for(kind, workload):
             tr = json.load(fh)
         ent = tr.get(workload, {}).get(kind)
         if ent and ent.get("source_hash") == build._stamp():
+            if "dram_bytes_per_expert" in ent:
+                return ent["dram_bytes_per_expert"] * experts_per_launch
             return ent["dram_bytes_per_launch"]
     except Exception:
         pass
@@ -320,6 +323,9 @@ def run_ours(args, world, rank, local):
                 k = kinds.setdefault(kind, {"ms": 0.0, "launches": 0, "bytes": 0.0, "flops": 0.0})
                 k["ms"] += kms
                 k["launches"] += n
+                k.setdefault("union", 0.0)
+                if n and dC:
+                    k["union"] += n * dU / dC
                 if kind in ("ffn_up", "ffn_down", "shared_up", "shared_down") and n:
                     # per-launch average union / activations of this handle
                     k["bytes"] += n * kernel_bytes(kind, shape, dU / max(1, dC), dA / max(1, dC), B)
@@ -335,12 +341,12 @@ def run_ours(args, world, rank, local):
         achieved = dk["bytes"] / max(1, dk["launches"]) / avg_launch_s / 1e9
         roof = {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
                 "frac": achieved / hbm, "peak_source": peak_src,
-                "traffic": traffic_for(dom, args.workload)}
+                "traffic": traffic_for(dom, args.workload, dk["union"] / max(1, dk["launches"]))}
     else:
         achieved = dk["flops"] / max(1, dk["launches"]) / avg_launch_s / 1e12
         roof = {"bound": "tensor", "achieved": achieved, "peak": bf16_sus, "unit": "TFLOP/s",
                 "frac": achieved / bf16_sus, "peak_source": peak_src + " sustained",
-                "traffic": traffic_for(dom, args.workload)}
+                "traffic": traffic_for(dom, args.workload, dk["union"] / max(1, dk["launches"]))}
     roof.update({"kernel": dom, "kernel_share": dk["ms"] / total_kernel_ms,
                  "avg_launch_us": avg_launch_s * 1e6,
                  "algorithmic_bytes_per_launch": dk["bytes"] / max(1, dk["launches"])})
