@@ -176,8 +176,9 @@ eat_status eat_get_counters(eat_handle* h, int64_t* out, int32_t n);
 /* Per-kernel device timing.  eat_profile_begin(h, capacity) makes every later launch of this
  * handle record a CUDA event pair (capacity = max launches recorded); eat_profile_end
  * synchronises, writes for each kernel kind i < n the summed milliseconds ms[i] and the launch
- * count launches[i], and stops recording.  Kernel kinds: 0 route, 1 permute, 2 routed
- * gate/up FFN, 3 routed down FFN, 4 shared gate/up, 5 shared down, 6 combine, 7 account. */
+ * count launches[i], and stops recording.  Kernel kinds: 0 router scores, 1 permute, 2 routed
+ * gate/up FFN, 3 routed down FFN, 4 shared gate/up, 5 shared down, 6 combine, 7 account,
+ * 8 selection (softmax / threshold / Eq. 6-8), 9 token-row gather. */
 eat_status eat_profile_begin(eat_handle* h, int32_t capacity);
 eat_status eat_profile_end(eat_handle* h, double* ms, int64_t* launches, int32_t n);
 

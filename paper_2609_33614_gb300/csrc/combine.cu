@@ -1,7 +1,7 @@
 // Weighted combine / unpermute (§3.4: the layer output is the g_norm-weighted sum of the activated
 // experts' outputs) and the expert-account update (§3.2).
 //
-//  combine_kernel: one block per (token, 1024-column block).  For each of the token's k_t slots
+//  combine_kernel: one block per (token, 2048-column block).  For each of the token's k_t slots
 //      it sums the expert output partials (split-K slices, fixed order), accumulates g_norm * o into
 //      y in the order j = 0..k_t-1, adds the always-on shared experts with weight 1, and writes the
 //      partial sum of squares of every slot (||o||_2 of the unweighted expert output feeds C_s).
@@ -16,30 +16,61 @@ namespace eat {
 namespace {
 
 constexpr int kCombThreads = 256;
-constexpr int kAccThreads = 128;
+constexpr int kAccThreads = 512;
 
-__device__ __forceinline__ void store_y4(float* y, float4 v) { *(float4*)y = v; }
-__device__ __forceinline__ void store_y4(__nv_bfloat16* y, float4 v) {
-  __nv_bfloat162 a = __floats2bfloat162_rn(v.x, v.y);
-  __nv_bfloat162 b = __floats2bfloat162_rn(v.z, v.w);
-  uint2 u;
-  u.x = *(uint32_t*)&a;
-  u.y = *(uint32_t*)&b;
-  *(uint2*)y = u;
+
+// 8 consecutive values as fp32, from fp32 (two 16-byte loads) or bf16 (one 16-byte load).
+struct V8 {
+  float v[8];
+};
+__device__ __forceinline__ V8 load8(const void* base, bool bf16, size_t i) {
+  V8 r;
+  if (bf16) {
+    const uint4 u = *(const uint4*)((const __nv_bfloat16*)base + i);
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float2 f = __bfloat1622float2(*(const __nv_bfloat162*)&w[q]);
+      r.v[2 * q] = f.x;
+      r.v[2 * q + 1] = f.y;
+    }
+  } else {
+    const float4 a = *(const float4*)((const float*)base + i);
+    const float4 b = *(const float4*)((const float*)base + i + 4);
+    r.v[0] = a.x; r.v[1] = a.y; r.v[2] = a.z; r.v[3] = a.w;
+    r.v[4] = b.x; r.v[5] = b.y; r.v[6] = b.z; r.v[7] = b.w;
+  }
+  return r;
+}
+__device__ __forceinline__ void store8(float* y, const float (&a)[8]) {
+  *(float4*)y = make_float4(a[0], a[1], a[2], a[3]);
+  *(float4*)(y + 4) = make_float4(a[4], a[5], a[6], a[7]);
+}
+__device__ __forceinline__ void store8(__nv_bfloat16* y, const float (&a)[8]) {
+  uint4 u;
+  uint32_t* w = (uint32_t*)&u;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const __nv_bfloat162 h = __floats2bfloat162_rn(a[2 * q], a[2 * q + 1]);
+    w[q] = *(const uint32_t*)&h;
+  }
+  *(uint4*)y = u;
 }
 
-// Column block of one token: 4 consecutive columns per thread (float4 loads), so a token's row
-// is spread over ceil(d / 1024) blocks; every block writes the partial sum of squares of each of
-// the token's slots over its columns (nrm_part[slot][block]), which the account kernel sums.
-template <typename TY>
+// Column block of one token: 8 consecutive columns per thread (16-byte loads), so a token's row
+// spans ceil(d / 2048) blocks; every block writes the partial sum of squares of each of the
+// token's slots over its columns (nrm_part[slot][block]), which the account kernel sums.  Expert
+// outputs are fp32 split-K partials (o_bf16 = 0) or, without split-K, bf16 rows; the shared
+// experts' outputs likewise (s_bf16).  All of a token's slot rows are loaded before any use.
+template <typename TY, int KM>
 __global__ void __launch_bounds__(kCombThreads)
-combine_kernel(const float* __restrict__ opart, int n_split, size_t split_stride,
+combine_kernel(const void* __restrict__ opart, int o_bf16, int n_split, size_t split_stride,
                const int32_t* __restrict__ slot_of, const float* __restrict__ w,
-               const int32_t* __restrict__ kk, const float* __restrict__ sout, int S, int T, int K,
-               int d, TY* __restrict__ y, float* __restrict__ nrm_part) {
-  __shared__ int slots[kMaxK];
-  __shared__ float gw[kMaxK];
-  __shared__ float red[kCombThreads / 32][kMaxK];
+               const int32_t* __restrict__ kk, const void* __restrict__ sout, int s_bf16, int S,
+               int T, int K, int d, TY* __restrict__ y, float* __restrict__ nrm_part) {
+  __shared__ int slots[KM];
+  __shared__ float gw[KM];
+  __shared__ float red[kCombThreads / 32][KM];
   pdl_wait();
   pdl_launch_dependents();
   const int t = blockIdx.x;
@@ -51,43 +82,48 @@ combine_kernel(const float* __restrict__ opart, int n_split, size_t split_stride
     gw[tid] = tid < kt ? w[(size_t)t * K + tid] : 0.f;
   }
   __syncthreads();
-  float nrm[kMaxK];
+  float nrm[KM];
 #pragma unroll
-  for (int j = 0; j < kMaxK; ++j) nrm[j] = 0.f;
-  const int c = (cb * kCombThreads + tid) * 4;
+  for (int j = 0; j < KM; ++j) nrm[j] = 0.f;
+  const int c = (cb * kCombThreads + tid) * 8;
   if (c < d) {
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    V8 o[KM];
 #pragma unroll
-    for (int j = 0; j < kMaxK; ++j) {
-      if (j < kt) {
-        const float* src = opart + (size_t)slots[j] * d + c;
-        float4 o = *(const float4*)src;
-        for (int sp = 1; sp < n_split; ++sp) {
-          const float4 q = *(const float4*)(src + sp * split_stride);
-          o.x += q.x;
-          o.y += q.y;
-          o.z += q.z;
-          o.w += q.w;
+    for (int j = 0; j < KM; ++j)
+      if (j < kt) o[j] = load8(opart, o_bf16, (size_t)slots[j] * d + c);
+    for (int sp = 1; sp < n_split; ++sp) {
+#pragma unroll
+      for (int j = 0; j < KM; ++j) {
+        if (j < kt) {
+          const V8 q = load8(opart, false, sp * split_stride + (size_t)slots[j] * d + c);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) o[j].v[i] += q.v[i];
         }
+      }
+    }
+    float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int j = 0; j < KM; ++j) {
+      if (j < kt) {
         const float g = gw[j];
-        acc.x = fmaf(g, o.x, acc.x);
-        acc.y = fmaf(g, o.y, acc.y);
-        acc.z = fmaf(g, o.z, acc.z);
-        acc.w = fmaf(g, o.w, acc.w);
-        nrm[j] = fmaf(o.x, o.x, fmaf(o.y, o.y, fmaf(o.z, o.z, fmaf(o.w, o.w, nrm[j]))));
+        float n = 0.f;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          acc[i] = fmaf(g, o[j].v[i], acc[i]);
+          n = fmaf(o[j].v[i], o[j].v[i], n);
+        }
+        nrm[j] = n;
       }
     }
     for (int s = 0; s < S; ++s) {
-      const float4 q = *(const float4*)(sout + ((size_t)s * T + t) * d + c);
-      acc.x += q.x;
-      acc.y += q.y;
-      acc.z += q.z;
-      acc.w += q.w;
+      const V8 q = load8(sout, s_bf16, ((size_t)s * T + t) * d + c);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) acc[i] += q.v[i];
     }
-    store_y4(y + (size_t)t * d + c, acc);
+    store8(y + (size_t)t * d + c, acc);
   }
 #pragma unroll
-  for (int j = 0; j < kMaxK; ++j) {
+  for (int j = 0; j < KM; ++j) {
     if (j < kt) {
       float v = nrm[j];
 #pragma unroll
@@ -115,13 +151,23 @@ account_kernel(const int32_t* __restrict__ offs, const float* __restrict__ perm_
   const int e = blockIdx.x;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int beg = offs[e], end = offs[e + 1];
-  double sp = 0.0, sn = 0.0;
-  for (int i = beg + tid; i < end; i += kAccThreads) {
-    sp += (double)perm_p[i];
-    double sq = 0.0;
-    for (int b = 0; b < nb; ++b) sq += (double)nrm_part[(size_t)i * nb + b];
-    sn += sqrt(sq);
+  // four independent slot streams per thread keep enough loads in flight for an expert that
+  // holds most of a large call's tokens
+  double sp4[4] = {0.0, 0.0, 0.0, 0.0}, sn4[4] = {0.0, 0.0, 0.0, 0.0};
+  for (int i0 = beg + tid; i0 < end; i0 += 4 * kAccThreads) {
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int i = i0 + u * kAccThreads;
+      if (i < end) {
+        sp4[u] += (double)perm_p[i];
+        double sq = 0.0;
+        for (int b = 0; b < nb; ++b) sq += (double)nrm_part[(size_t)i * nb + b];
+        sn4[u] += sqrt(sq);
+      }
+    }
   }
+  double sp = (sp4[0] + sp4[1]) + (sp4[2] + sp4[3]);
+  double sn = (sn4[0] + sn4[1]) + (sn4[2] + sn4[3]);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     sp += __shfl_xor_sync(0xffffffffu, sp, o);
@@ -145,22 +191,50 @@ account_kernel(const int32_t* __restrict__ offs, const float* __restrict__ perm_
   }
 }
 
+
 }  // namespace
 
-int combine_col_blocks(int d) { return (d + 4 * kCombThreads - 1) / (4 * kCombThreads); }
+int combine_col_blocks(int d) { return (d + 8 * kCombThreads - 1) / (8 * kCombThreads); }
 
-cudaError_t launch_combine(int y_bf16, const float* opart, int n_split, int split_stride_rows,
-                           const int32_t* slot_of, const float* w, const int32_t* k,
-                           const float* sout, int S, int T, int K, int d, void* y,
-                           float* nrm_part, cudaStream_t st) {
+namespace {
+
+template <typename TY, int KM>
+cudaError_t launch_combine_t(dim3 grid, cudaStream_t st, const void* opart, int o_bf16,
+                             int n_split, size_t stride, const int32_t* slot_of, const float* w,
+                             const int32_t* k, const void* sout, int s_bf16, int S, int T, int K,
+                             int d, void* y, float* nrm_part) {
+  return launch_pdl(combine_kernel<TY, KM>, grid, dim3(kCombThreads), 0, st, opart, o_bf16,
+                    n_split, stride, slot_of, w, k, sout, s_bf16, S, T, K, d, (TY*)y, nrm_part);
+}
+
+template <typename TY>
+cudaError_t launch_combine_k(dim3 grid, cudaStream_t st, const void* opart, int o_bf16,
+                             int n_split, size_t stride, const int32_t* slot_of, const float* w,
+                             const int32_t* k, const void* sout, int s_bf16, int S, int T, int K,
+                             int d, void* y, float* nrm_part) {
+#define EAT_COMB(KM)                                                                            \
+  launch_combine_t<TY, KM>(grid, st, opart, o_bf16, n_split, stride, slot_of, w, k, sout, s_bf16, \
+                           S, T, K, d, y, nrm_part)
+  if (K <= 2) return EAT_COMB(2);
+  if (K <= 4) return EAT_COMB(4);
+  if (K <= 8) return EAT_COMB(8);
+  return EAT_COMB(16);
+#undef EAT_COMB
+}
+
+}  // namespace
+
+cudaError_t launch_combine(int y_bf16, const void* opart, int o_bf16, int n_split,
+                           int split_stride_rows, const int32_t* slot_of, const float* w,
+                           const int32_t* k, const void* sout, int s_bf16, int S, int T, int K,
+                           int d, void* y, float* nrm_part, cudaStream_t st) {
   const size_t stride = (size_t)split_stride_rows * d;
   dim3 grid(T, combine_col_blocks(d));
   if (y_bf16)
-    return launch_pdl(combine_kernel<__nv_bfloat16>, grid, dim3(kCombThreads), 0, st, opart,
-                      n_split, stride, slot_of, w, k, sout, S, T, K, d, (__nv_bfloat16*)y,
-                      nrm_part);
-  return launch_pdl(combine_kernel<float>, grid, dim3(kCombThreads), 0, st, opart, n_split,
-                    stride, slot_of, w, k, sout, S, T, K, d, (float*)y, nrm_part);
+    return launch_combine_k<__nv_bfloat16>(grid, st, opart, o_bf16, n_split, stride, slot_of, w,
+                                           k, sout, s_bf16, S, T, K, d, y, nrm_part);
+  return launch_combine_k<float>(grid, st, opart, o_bf16, n_split, stride, slot_of, w, k, sout,
+                                 s_bf16, S, T, K, d, y, nrm_part);
 }
 
 cudaError_t launch_account(const int32_t* offs, const float* perm_p, const float* nrm_part, int nb,

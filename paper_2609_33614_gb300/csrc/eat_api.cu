@@ -40,7 +40,7 @@ struct eat_handle {
   float* nrm_part = nullptr; // [Tmax*K, column blocks] partial sums of squares of expert rows
   int nb = 1;                 // column blocks per row in the combine kernel
   void* sact = nullptr;   // [S*Tmax, Fs]
-  float* sout = nullptr;  // [S*Tmax, d]
+  float* sout = nullptr;  // [S*Tmax, d] (fp32; bf16 on the tensor-core path)
   void* xstage = nullptr; // [Tmax, d]
   void* ystage = nullptr; // [Tmax, d]
   void* xperm = nullptr;  // [Tmax*K, d] gathered token rows (tensor-core path)
@@ -74,7 +74,9 @@ eat_status cuda_fail(eat_handle* h, cudaError_t e, const char* what) {
   return fail(h, EAT_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
 }
 
-enum Kind { kRoute = 0, kPermute, kUp, kDown, kSUp, kSDown, kCombine, kAccount, kKinds };
+enum Kind {
+  kRoute = 0, kPermute, kUp, kDown, kSUp, kSDown, kCombine, kAccount, kSelect, kGather, kKinds
+};
 
 // Run one launch, optionally bracketed by CUDA events for the per-kernel profile.
 template <typename Fn>
@@ -143,7 +145,7 @@ eat_status run_route(eat_handle* h, const void* x, int T, int ppl_sign, int32_t*
     return launch_router_logits(x, h->bf16, h->desc.w_router, T, h->d, h->E, split,
                                 h->logit_part, st);
   }));
-  EAT_TRY(launch(h, kRoute, st, "route select", [&] {
+  EAT_TRY(launch(h, kSelect, st, "route select", [&] {
     return launch_route_select(h->logit_part, split, h->desc.b_router, T, h->E, h->K, h->N,
                                h->P, h->C, rp, idx, w, k, psel, st);
   }));
@@ -175,7 +177,7 @@ eat_status run_forward(eat_handle* h, const void* x, int T, int ppl_sign, void* 
     c.sout = h->sout;
     c.status = h->status;
     n_split = tc_down_split(h->tc, T);
-    EAT_TRY(launch(h, kPermute, st, "gather rows",
+    EAT_TRY(launch(h, kGather, st, "gather rows",
                    [&] { return tc_launch_gather(h->tc, c, st); }));
     EAT_TRY(launch(h, kUp, st, "tc gate/up", [&] { return tc_launch_up(h->tc, c, false, st); }));
     EAT_TRY(launch(h, kDown, st, "tc down",
@@ -204,14 +206,15 @@ eat_status run_forward(eat_handle* h, const void* x, int T, int ppl_sign, void* 
                                       gs, h->sact, st);
       }));
       EAT_TRY(launch(h, kSDown, st, "shared down", [&] {
-        return launch_ffn_down_simt(h->bf16, h->sact, h->desc.ws_down, h->d, h->Fs, gs, h->sout,
-                                    st);
+        return launch_ffn_down_simt(h->bf16, h->sact, h->desc.ws_down, h->d, h->Fs, gs,
+                                    (float*)h->sout, st);
       }));
     }
   }
   EAT_TRY(launch(h, kCombine, st, "combine", [&] {
-    return launch_combine(h->bf16, h->opart, n_split, rows, h->perm.slot_of, h->w,
-                          h->k, h->sout, h->S, T, h->K, h->d, y, h->nrm_part, st);
+    const int tc = h->backend == 1;
+    return launch_combine(h->bf16, h->opart, tc && n_split == 1, n_split, rows, h->perm.slot_of,
+                          h->w, h->k, h->sout, tc, h->S, T, h->K, h->d, y, h->nrm_part, st);
   }));
   EAT_TRY(launch(h, kAccount, st, "account update", [&] {
     return launch_account(h->perm.offs, h->perm.perm_p, h->nrm_part, h->nb, h->E, h->prm.alpha,

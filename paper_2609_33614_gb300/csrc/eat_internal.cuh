@@ -107,10 +107,10 @@ constexpr int kSimtTileRows = 32;
 // Combine / unpermute and account update
 // ---------------------------------------------------------------------------------------------
 int combine_col_blocks(int d);  // column blocks per token row in the combine kernel
-cudaError_t launch_combine(int y_bf16, const float* opart, int n_split, int split_stride_rows,
-                           const int32_t* slot_of, const float* w, const int32_t* k,
-                           const float* sout, int S, int T, int K, int d, void* y,
-                           float* nrm_part, cudaStream_t st);
+cudaError_t launch_combine(int y_bf16, const void* opart, int o_bf16, int n_split,
+                           int split_stride_rows, const int32_t* slot_of, const float* w,
+                           const int32_t* k, const void* sout, int s_bf16, int S, int T, int K,
+                           int d, void* y, float* nrm_part, cudaStream_t st);
 cudaError_t launch_account(const int32_t* offs, const float* perm_p, const float* nrm_part, int nb,
                            int E, double alpha, int64_t* N, double* P, double* C, int32_t* st_n,
                            double* st_p, double* st_norm, long long* counters, cudaStream_t st);

@@ -8,8 +8,9 @@
 // full M = 128 MMAs and simply stream the activated experts' weights; prefill calls use BN = 128.
 //   gate/up kernel: D_gate = Wg[e, f0:f0+128, :] . Xperm[slots]^T and D_up likewise, both in TMEM;
 //       the epilogue writes act[slot, f] = silu(D_gate) * D_up in bf16 (fp32 accumulation).
-//   down kernel:    D = Wd[e, c0:c0+128, :] . act[slots]^T over a K slice (split-K for decode),
-//       fp32 partials opart[split][slot][c] summed in fixed order by the combine kernel.
+//   down kernel:    D = Wd[e, c0:c0+128, :] . act[slots]^T over a K slice: with split-K (decode)
+//       fp32 partials opart[split][slot][c], summed in fixed order by the combine kernel; without
+//       it, bf16 rows O[slot][c].
 // Persistent CTAs (one per SM) walk the work units (token tile, feature tile, K slice) of all
 // groups; the group sizes live on the device (written by the permute kernel), so no host sync.
 // Warp roles: warp 0 lane 0 issues TMA; warp 1 owns TMEM and lane 0 issues MMAs; warps 2-5 drain
@@ -187,6 +188,7 @@ struct TcArgs {
   int kb_per_split;
   void* out;
   long long split_stride;    // elements between split slices of the fp32 output
+  int out_bf16;              // down kernel without split-K: write bf16 rows instead of fp32
   unsigned int* err;
 };
 
@@ -385,6 +387,9 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
               if (GATEUP) {
                 const float h = silu_f(__uint_as_float(g[c])) * __uint_as_float(up[c]);
                 ((__nv_bfloat16*)args.out)[slot * args.M + f] = __float2bfloat16_rn(h);
+              } else if (args.out_bf16) {
+                ((__nv_bfloat16*)args.out)[slot * args.M + f] =
+                    __float2bfloat16_rn(__uint_as_float(g[c]));
               } else {
                 ((float*)args.out)[(size_t)w.split * args.split_stride + slot * args.M + f] =
                     __uint_as_float(g[c]);
@@ -646,6 +651,7 @@ cudaError_t tc_launch_down(const TcLayer& L, const TcCall& c, bool shared, int n
     a.n_groups = L.S;
     a.uniform_rows = c.T;
     a.out = c.sout;
+    a.out_bf16 = 1;
     a.split_stride = 0;
     max_tiles = (long long)L.S * ((c.T + bn - 1) / bn);
     const long long units = max_tiles * a.m_tiles;
@@ -656,6 +662,7 @@ cudaError_t tc_launch_down(const TcLayer& L, const TcCall& c, bool shared, int n
   a.row_offs = c.offs;
   a.tile_offs = c.tile_offs;
   a.out = c.opart;
+  a.out_bf16 = n_split == 1 ? 1 : 0;
   a.split_stride = (long long)c.T * L.K * L.d;
   max_tiles = (long long)(c.T * L.K + bn - 1) / bn + L.E;
   const long long units = max_tiles * a.m_tiles * n_split;

@@ -22,9 +22,9 @@ struct TcCall {
   const int32_t* perm_tok = nullptr;
   void* xperm = nullptr;           // [Tmax*K, d] gathered rows in slot order
   void* act = nullptr;             // [Tmax*K, F] bf16
-  float* opart = nullptr;          // [split][T*K, d] fp32
+  float* opart = nullptr;          // [split][T*K, d] fp32, or [T*K, d] bf16 without split-K
   void* sact = nullptr;            // [S*T, Fs] bf16
-  float* sout = nullptr;           // [S*T, d] fp32
+  void* sout = nullptr;            // [S*T, d] bf16
   unsigned int* status = nullptr;  // device status word (bounded-wait failures)
 };
 

@@ -1,8 +1,8 @@
 // Permute by expert: groups the selected (token, expert) pairs of one call by expert so that the
 // expert FFNs read contiguous row lists ("only activated experts participate", §3.4).
 //
-// Tokens are split in chunks of 1024, one CTA each (a call of at most 1024 tokens runs as a single
-// CTA that also counts).  Counts n_e come from shared-memory atomics (integers, order-free); each
+// A call of at most 1024 tokens runs as a single 1024-thread CTA that also counts; larger calls
+// are split in chunks of 256 tokens, one CTA each, after a counting pass.  Counts n_e come from shared-memory atomics (integers, order-free); each
 // chunk's first slot per expert is the expert's offset plus the counts of the earlier chunks.
 // Inside a chunk every pair gets a STABLE slot (tokens ascending inside each expert): each warp
 // finds the experts present among its 32 tokens with ballots, counts them per warp, the counts are
@@ -14,8 +14,8 @@ namespace eat {
 
 namespace {
 
-constexpr int kPermThreads = 1024;
-constexpr int kPermWarps = kPermThreads / 32;
+constexpr int kPermThreads = 1024;   // single-CTA calls (T <= 1024)
+constexpr int kChunkThreads = 256;   // tokens (and threads) per CTA of a multi-CTA call
 
 // For the calling lane's experts ex[0..K) (-1 = none), iterate over the distinct experts present
 // in the warp; fn(e, mask_of_lanes_with_e, j_of_this_lane_or_-1).
@@ -40,29 +40,29 @@ __device__ __forceinline__ void for_each_warp_expert(const int* ex, int K, Fn fn
   }
 }
 
-// Per-chunk expert counts (large calls): chunk_cnt[c][e] = activations of expert e among tokens
-// [c * 1024, (c + 1) * 1024).
-__global__ void __launch_bounds__(kPermThreads)
+// Per-chunk expert counts (large calls): chunk_cnt[c][e] = activations of expert e among the
+// chunk's tokens [c * 256, (c + 1) * 256).
+__global__ void __launch_bounds__(kChunkThreads)
 permute_count_kernel(const int32_t* __restrict__ idx, int T, int K, int E,
                      int32_t* __restrict__ chunk_cnt) {
   extern __shared__ int cnt[];
   pdl_wait();
   pdl_launch_dependents();
-  const int tid = threadIdx.x, c = blockIdx.x;
-  for (int e = tid; e < E; e += kPermThreads) cnt[e] = 0;
+  const int tid = threadIdx.x, c = blockIdx.x, nt = blockDim.x;
+  for (int e = tid; e < E; e += nt) cnt[e] = 0;
   __syncthreads();
-  const int t0 = c * kPermThreads, t1 = min(T, t0 + kPermThreads);
-  for (int i = t0 * K + tid; i < t1 * K; i += kPermThreads) {
+  const int t0 = c * nt, t1 = min(T, t0 + nt);
+  for (int i = t0 * K + tid; i < t1 * K; i += nt) {
     const int e = idx[i];
     if (e >= 0) atomicAdd(&cnt[e], 1);
   }
   __syncthreads();
-  for (int e = tid; e < E; e += kPermThreads) chunk_cnt[(size_t)c * E + e] = cnt[e];
+  for (int e = tid; e < E; e += nt) chunk_cnt[(size_t)c * E + e] = cnt[e];
 }
 
-// Slot assignment of one chunk of 1024 tokens.  With chunk_cnt == nullptr the kernel runs as a
-// single CTA over a call of at most 1024 tokens and counts in place.
-__global__ void __launch_bounds__(kPermThreads)
+// Slot assignment of one chunk of blockDim.x tokens.  With chunk_cnt == nullptr the kernel runs
+// as a single CTA over a call of at most 1024 tokens and counts in place.
+__global__ void __launch_bounds__(1024)
 permute_assign_kernel(const int32_t* __restrict__ idx, const int32_t* __restrict__ kk,
                       const float* __restrict__ psel, int T, int K, int E, int tile_rows,
                       const int32_t* __restrict__ chunk_cnt, int n_chunks, PermuteOut o) {
@@ -71,23 +71,24 @@ permute_assign_kernel(const int32_t* __restrict__ idx, const int32_t* __restrict
   pdl_launch_dependents();
   int* cnt = sm;                      // [E] activations of each expert in the whole call
   int* cursor = cnt + E;              // [E] first slot of each expert for this chunk
-  int* wcnt = cursor + E;             // [kPermWarps][E]
+  int* wcnt = cursor + E;             // [warps][E]
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int nt = blockDim.x, n_warps = nt >> 5;
   const int c = blockIdx.x;
   const unsigned lt = (1u << lane) - 1u;
 
   if (chunk_cnt == nullptr) {
-    for (int e = tid; e < E; e += kPermThreads) {
+    for (int e = tid; e < E; e += nt) {
       cnt[e] = 0;
       cursor[e] = 0;
     }
     __syncthreads();
-    for (int i = tid; i < T * K; i += kPermThreads) {
+    for (int i = tid; i < T * K; i += nt) {
       const int e = idx[i];
       if (e >= 0) atomicAdd(&cnt[e], 1);
     }
   } else {
-    for (int e = tid; e < E; e += kPermThreads) {
+    for (int e = tid; e < E; e += nt) {
       int tot = 0, before = 0;
       for (int cc = 0; cc < n_chunks; ++cc) {
         const int v = chunk_cnt[(size_t)cc * E + e];
@@ -122,8 +123,8 @@ permute_assign_kernel(const int32_t* __restrict__ idx, const int32_t* __restrict
   __syncthreads();
 
   int ex[kMaxK];
-  const int c_end = chunk_cnt == nullptr ? T : min(T, (c + 1) * kPermThreads);
-  for (int c0 = c * kPermThreads; c0 < c_end; c0 += kPermThreads) {
+  const int c_end = chunk_cnt == nullptr ? T : min(T, (c + 1) * nt);
+  for (int c0 = c * nt; c0 < c_end; c0 += nt) {
     const int t = c0 + tid;
     const int kt = t < c_end ? kk[t] : 0;
     for (int j = 0; j < K; ++j) ex[j] = (j < kt) ? idx[(size_t)t * K + j] : -1;
@@ -133,9 +134,9 @@ permute_assign_kernel(const int32_t* __restrict__ idx, const int32_t* __restrict
       if (lane == 0) wcnt[warp * E + e] = __popc(m);
     });
     __syncthreads();
-    for (int e = tid; e < E; e += kPermThreads) {
+    for (int e = tid; e < E; e += nt) {
       int run = cursor[e];
-      for (int w = 0; w < kPermWarps; ++w) {
+      for (int w = 0; w < n_warps; ++w) {
         const int v = wcnt[w * E + e];
         wcnt[w * E + e] = run;
         run += v;
@@ -159,20 +160,24 @@ permute_assign_kernel(const int32_t* __restrict__ idx, const int32_t* __restrict
 
 }  // namespace
 
-int permute_chunks(int T) { return (T + kPermThreads - 1) / kPermThreads; }
+int permute_chunks(int T) {
+  return T <= kPermThreads ? 1 : (T + kChunkThreads - 1) / kChunkThreads;
+}
 
 cudaError_t launch_permute(const int32_t* idx, const int32_t* k, const float* psel, int T, int K,
                            int E, int tile_rows, PermuteOut o, int32_t* chunk_cnt,
                            cudaStream_t st) {
-  const size_t smem = (size_t)(2 * E + kPermWarps * E) * sizeof(int);
   const int n_chunks = permute_chunks(T);
-  if (n_chunks == 1)
+  if (n_chunks == 1) {
+    const size_t smem = (size_t)(2 * E + (kPermThreads / 32) * E) * sizeof(int);
     return launch_pdl(permute_assign_kernel, dim3(1), dim3(kPermThreads), smem, st, idx, k, psel,
                       T, K, E, tile_rows, (const int32_t*)nullptr, 1, o);
-  cudaError_t e = launch_pdl(permute_count_kernel, dim3(n_chunks), dim3(kPermThreads),
+  }
+  cudaError_t e = launch_pdl(permute_count_kernel, dim3(n_chunks), dim3(kChunkThreads),
                              (size_t)E * sizeof(int), st, idx, T, K, E, chunk_cnt);
   if (e != cudaSuccess) return e;
-  return launch_pdl(permute_assign_kernel, dim3(n_chunks), dim3(kPermThreads), smem, st, idx, k,
+  const size_t smem = (size_t)(2 * E + (kChunkThreads / 32) * E) * sizeof(int);
+  return launch_pdl(permute_assign_kernel, dim3(n_chunks), dim3(kChunkThreads), smem, st, idx, k,
                     psel, T, K, E, tile_rows, (const int32_t*)chunk_cnt, n_chunks, o);
 }
 

@@ -17,7 +17,7 @@ EAT_OK, EAT_ERR_INVALID_ARG, EAT_ERR_UNSUPPORTED, EAT_ERR_OOM, EAT_ERR_CUDA, EAT
 EAT_F32, EAT_BF16 = 0, 1
 EAT_C_SUM, EAT_C_RAW = 0, 1
 KERNEL_KINDS = ("route", "permute", "ffn_up", "ffn_down", "shared_up", "shared_down", "combine",
-                "account")
+                "account", "select", "gather")
 
 c_i32, c_i64, c_dbl, c_vp = ctypes.c_int32, ctypes.c_int64, ctypes.c_double, ctypes.c_void_p
 
