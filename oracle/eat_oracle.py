@@ -14,7 +14,8 @@ Paper: "EAT: Expert Account Tracker for Efficient MoE Inference" (arxiv 2609.336
   * §3.3  threshold tau (Eq. 3-5), PPL adjustment, boundedness, smoothing
   * §3.4  candidate set / K cap (Eq. 6), mask and renormalisation (Eq. 7-8)
   * Table 1  hyper-parameter defaults
-  * §4.1  Top-P comparison router (P = 0.6 / 0.2 / 0.4)
+  * §3.5  OPD inference reweighting of the routing probabilities (scales supplied by the caller)
+  * §4.1  Top-P comparison router (P = 0.6 / 0.2 / 0.4) and the vanilla fixed Top-K router
 
 Readings taken where the paper is silent or ambiguous (each is also listed in the design notes):
   R1  the "raw router gating score g" of §3.3 is the softmax probability p of §3.2 (g == p).
@@ -75,6 +76,8 @@ class Params:
     max_k: int = 2           # K of Eq. 6 (Table 1: 2 for Mixtral/Phi, 8 for Qwen)
     clamp: bool = True       # boundedness enforcement on/off
     c_mode: str = "sum"      # reading R3: "sum" or "raw"
+    router: str = "eat"      # "eat" (§3.2-§3.4), or the baselines "topk" / "topp" (§4.1)
+    top_p: float = 0.6       # P of the Top-P baseline (§4.1: 0.6 / 0.2 / 0.4)
 
     def with_(self, **kw) -> "Params":
         return replace(self, **kw)
@@ -109,6 +112,7 @@ class Layer:
     ws_gate: np.ndarray | None = None
     ws_up: np.ndarray | None = None
     ws_down: np.ndarray | None = None
+    opd_scale: np.ndarray | None = None   # [E] per-expert OPD reweighting scales (§3.5)
 
     @property
     def n_experts(self) -> int:
@@ -125,6 +129,15 @@ def router_logits(x: np.ndarray, w_router: np.ndarray, b_router: np.ndarray | No
     if b_router is not None:
         z = z + np.asarray(b_router, F64)[None, :]
     return z / F64(temperature)
+
+
+def opd_reweight(p: np.ndarray, scale: np.ndarray | None) -> np.ndarray:
+    """§3.5 OPD inference reweighting: scale each routing probability by the expert's factor and
+    renormalise the distribution, p'_i = s_i p_i / sum_j s_j p_j (identity without scales)."""
+    if scale is None:
+        return np.asarray(p, F64)
+    q = np.asarray(p, F64) * np.asarray(scale, F64)[None, :]
+    return q / q.sum(axis=-1, keepdims=True)
 
 
 def softmax(z: np.ndarray) -> np.ndarray:
@@ -270,17 +283,25 @@ class Routing:
 
 
 def route(x: np.ndarray, layer: Layer, acc: Accounts, prm: Params, ppl_sign: int = 0) -> Routing:
-    """Router -> softmax -> S_h -> I -> tau_final -> E_final -> g_norm for every token, all from
-    the same account snapshot (reading R10)."""
+    """Router -> softmax (-> OPD reweighting, §3.5) -> S_h -> I -> tau_final -> E_final -> g_norm
+    for every token, all from the same account snapshot (reading R10).  With router "topk" /
+    "topp" the selection is the §4.1 baseline instead of Eq. 6; everything else is unchanged."""
     z = router_logits(x, layer.w_router, layer.b_router, prm.temperature)
-    p = softmax(z)
+    p = opd_reweight(softmax(z), layer.opd_scale)
     s_h = history_score(acc, prm)
     I = importance(p, s_h[None, :], prm.beta)
     ths, sels = [], []
     g_norm = np.zeros_like(p)
     for t in range(p.shape[0]):
         th = threshold(p[t], prm, ppl_sign)
-        sel = select(I[t], th.tau_final, prm.max_k)
+        if prm.router == "eat":
+            sel = select(I[t], th.tau_final, prm.max_k)
+        elif prm.router == "topk":
+            sel = topk_select(p[t], prm.max_k)
+        elif prm.router == "topp":
+            sel = topp_select(p[t], prm.top_p, prm.max_k)
+        else:
+            raise ValueError(f"unknown router {prm.router!r}")
         ths.append(th)
         sels.append(sel)
         g_norm[t] = renormalize(p[t], sel, prm.eps)
@@ -379,15 +400,25 @@ def token_output(x_t: np.ndarray, layer: Layer, routing: Routing, t: int) -> tup
 # ----------------------------------------------------------------------------------------------
 # Comparison router of §4.1 (Top-P, Huang et al.) -- oracle only
 # ----------------------------------------------------------------------------------------------
-def topp_select(p: np.ndarray, P: float) -> list[int]:
+def topp_select(p: np.ndarray, P: float, K: int | None = None) -> list[int]:
     """Top-P routing: take experts in descending probability (index ascending on ties) until
-    their cumulative probability reaches P; the smallest such prefix.  Ascending indices."""
+    their cumulative probability reaches P; the smallest such prefix, at most K experts when K is
+    given.  Ascending indices."""
     p = np.asarray(p, F64)
     order = sorted(range(p.shape[0]), key=lambda i: (-p[i], i))
     chosen, acc = [], 0.0
     for i in order:
+        if K is not None and len(chosen) == K:
+            break
         chosen.append(i)
         acc += p[i]
         if acc >= P:
             break
     return sorted(chosen)
+
+
+def topk_select(p: np.ndarray, K: int) -> list[int]:
+    """Vanilla fixed Top-K routing (§2, §4.1): the K largest probabilities, index ascending on
+    ties.  Ascending indices."""
+    p = np.asarray(p, F64)
+    return sorted(sorted(range(p.shape[0]), key=lambda i: (-p[i], i))[:K])

@@ -479,3 +479,44 @@ def test_planted_mistake_is_caught(name, monkeypatch):
     assert _pins(orc) == []
     monkeypatch.setattr(orc, attr, repl)
     assert _pins(orc) != [], f"mutant {name} survived every pin"
+
+
+# ---------------------------------------------------------------- baselines and OPD (§3.5, §4.1)
+def test_topk_router_equals_degenerate_eat():
+    """router "topk" and the degenerate EAT setting (beta 0, alpha1 0, alpha2 huge, no clamp)
+    are two formulations of vanilla Top-K: same selections and gates."""
+    rng = np.random.default_rng(31)
+    E, d = 12, 9
+    layer = orc.Layer(rng.normal(size=(E, d)), rng.normal(size=E), None, None, None)
+    x = rng.normal(size=(40, d))
+    acc = random_accounts(rng, E)
+    a = orc.route(x, layer, acc, orc.Params(router="topk", max_k=3), 1)
+    b = orc.route(x, layer, acc, orc.Params(beta=0.0, alpha1=0.0, alpha2=1e30, clamp=False,
+                                            max_k=3), 0)
+    assert a.selected == b.selected
+    assert close(a.g_norm, b.g_norm)
+
+
+def test_topp_router_hand_and_cap():
+    p = np.array([0.1, 0.5, 0.3, 0.1])
+    assert orc.topp_select(p, 0.6) == [1, 2]            # 0.5 < 0.6, 0.5 + 0.3 >= 0.6
+    assert orc.topp_select(p, 0.85, K=2) == [1, 2]      # would need a third expert; capped at K
+    assert orc.topp_select(p, 0.85) == [0, 1, 2]        # ties 0.1/0.1 -> lower index first
+    layer = orc.Layer(np.zeros((4, 1)), np.log(p), None, None, None)
+    r = orc.route(np.zeros((1, 1)), layer, orc.Accounts.zeros(4),
+                  orc.Params(router="topp", top_p=0.6, max_k=4))
+    assert r.selected == [[1, 2]]
+    assert close(r.g_norm[0], [0.0, 0.5 / (0.8 + 1e-8), 0.3 / (0.8 + 1e-8), 0.0])
+
+
+def test_opd_reweighting():
+    p = np.array([[0.5, 0.5], [0.2, 0.8]])
+    assert close(orc.opd_reweight(p, np.array([3.0, 1.0])), [[0.75, 0.25], [3 * 0.2 / 1.4, 0.8 / 1.4]])
+    assert close(orc.opd_reweight(p, np.array([2.0, 2.0])), p)   # uniform scales: identity
+    assert close(orc.opd_reweight(p, None), p)
+    # the reweighted distribution drives selection: a large scale on expert 0 flips token 2
+    layer = orc.Layer(np.zeros((2, 1)), np.log(np.array([0.2, 0.8])), None, None, None,
+                      opd_scale=np.array([9.0, 1.0]))
+    r = orc.route(np.zeros((1, 1)), layer, orc.Accounts.zeros(2), orc.Params(router="topk",
+                                                                             max_k=1))
+    assert r.selected == [[0]] and close(r.p[0], [1.8 / 2.6, 0.8 / 2.6])
