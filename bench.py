@@ -234,10 +234,14 @@ def run_ours(args, world, rank, local):
     # layers (weights drawn on the GPU generator) and one handle per (layer, batch)
     layer_w = [W.make_layer(shape, l, device="cuda") for l in range(n_layers)]
     handles = []  # [layer][batch]
+    mode = {"eat": eat.EAT_ROUTER_EAT, "topk": eat.EAT_ROUTER_TOPK,
+            "topp": eat.EAT_ROUTER_TOPP}[args.router]
     for lw in layer_w:
         row = []
         for B in batches:
-            row.append(eat.EatLayer.from_workload(lw, B))
+            prm = eat.eat_default_params(shape.max_k, temperature=shape.temperature,
+                                         router_mode=mode, top_p=args.top_p)
+            row.append(eat.EatLayer.from_workload(lw, B, prm))
         handles.append(row)
     # inputs resident in HBM before the timed region
     xs = {B: [W.make_tokens(shape, B, step=s, device="cuda") for s in range(min(n_steps_total, 64))]
@@ -379,7 +383,9 @@ def run_ours(args, world, rank, local):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": job_ms / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded N(0,1) hidden states, N(0,0.02^2) weights)",
-        "config": {"workload": spec["desc"], "d_model": shape.d_model,
+        "config": {"workload": spec["desc"], "router": args.router,
+                   **({"top_p": args.top_p} if args.router == "topp" else {}),
+                   "d_model": shape.d_model,
                    "n_experts": shape.n_experts, "d_ff": shape.d_ff, "n_shared": shape.n_shared,
                    "max_k": shape.max_k, "layers": n_layers, "batches": batches,
                    "l2": "inputs larger than L2 (expert weights > 129 MB), no flush"},
@@ -494,6 +500,9 @@ def main(argv=None):
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="mixtral-decode")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--router", default="eat", choices=["eat", "topk", "topp"],
+                    help="selection rule: EAT (default) or the paper's Top-K / Top-P baselines")
+    ap.add_argument("--top-p", type=float, default=0.6)
     args = ap.parse_args(argv)
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

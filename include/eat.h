@@ -44,6 +44,17 @@ typedef enum eat_status {
 
 typedef enum eat_dtype { EAT_F32 = 0, EAT_BF16 = 1 } eat_dtype;
 
+/* Expert selection rule.  EAT_ROUTER_EAT: the adaptive threshold of §3.3-§3.4 (Eq. 3-8).  The
+ * baselines the paper compares with (§4.1), computed by the same kernels from the same
+ * probabilities: EAT_ROUTER_TOPK, the K largest p (index ascending on ties); EAT_ROUTER_TOPP, the
+ * smallest descending-p prefix whose cumulative probability reaches top_p, at most K experts.
+ * Gates are always Eq. 7; the accounts are updated in every mode. */
+typedef enum eat_router_mode {
+  EAT_ROUTER_EAT = 0,
+  EAT_ROUTER_TOPK = 1,
+  EAT_ROUTER_TOPP = 2
+} eat_router_mode;
+
 /* How the EMA contribution C_s enters Eq. 1 (§3.2).  EAT_C_SUM: as the share C_i / sum_j C_j,
  * on the same [0, 1] scale as the other two terms (default).  EAT_C_RAW: the literal C_i. */
 typedef enum eat_c_mode { EAT_C_SUM = 0, EAT_C_RAW = 1 } eat_c_mode;
@@ -66,16 +77,21 @@ typedef struct eat_params {
   int32_t max_k;       /* K of Eq. 6: at most K experts per token, 1 <= K <= min(E, 16) */
   int32_t clamp_enabled; /* 1: apply the [q_lo, q_hi] bounds; 0: skip them */
   int32_t c_mode;      /* eat_c_mode */
+  int32_t router_mode; /* eat_router_mode (EAT_ROUTER_EAT) */
+  double top_p;        /* P of EAT_ROUTER_TOPP, in (0, 1] (0.6) */
 } eat_params;
 
-/* Fill *p with the defaults above and max_k = 2.  Returns EAT_ERR_INVALID_ARG if p is NULL. */
+/* Fill *p with the defaults above, max_k = 2, router_mode EAT_ROUTER_EAT, top_p 0.6.  Returns
+ * EAT_ERR_INVALID_ARG if p is NULL. */
 eat_status eat_default_params(eat_params* p);
 
 /* One MoE layer.  Shapes use nn.Linear layout (out_features x in_features), row-major:
  *   w_router [E, d] fp32, b_router [E] fp32 or NULL;
  *   w_gate, w_up [E, F, d], w_down [E, d, F] in wdtype;
  *   ws_gate, ws_up [S, Fs, d], ws_down [S, d, Fs] in wdtype, all NULL when n_shared == 0
- *   (always-on shared experts, added with weight 1, not routed, no account).
+ *   (always-on shared experts, added with weight 1, not routed, no account);
+ *   opd_scale [E] fp32 or NULL: OPD inference reweighting (§3.5) -- the routing probabilities
+ *   become p'_i = s_i p_i / sum_j s_j p_j before selection, and p' is used everywhere p is.
  * Supported: 1 <= E <= 256; d, F, Fs multiples of 64; (wdtype, xdtype) both EAT_F32 or both
  * EAT_BF16; 1 <= max_tokens <= 65536.  All weight pointers 16-byte aligned. */
 typedef struct eat_layer_desc {
@@ -89,6 +105,7 @@ typedef struct eat_layer_desc {
   const void* ws_gate;
   const void* ws_up;
   const void* ws_down;
+  const float* opd_scale;
 } eat_layer_desc;
 
 typedef struct eat_handle eat_handle;

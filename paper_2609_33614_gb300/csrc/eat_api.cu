@@ -117,6 +117,9 @@ RouteParams route_params(const eat_params& p, int ppl_sign) {
   r.temperature = (float)p.temperature;
   r.clamp = p.clamp_enabled;
   r.c_mode = p.c_mode;
+  r.mode = p.router_mode;
+  r.top_p = (float)p.top_p;
+  r.opd_scale = nullptr;
   return r;
 }
 
@@ -139,7 +142,8 @@ eat_status check_call(eat_handle* h, const void* x, int32_t T, int32_t ppl_sign)
 // Router + selection into (idx, w, k, psel).
 eat_status run_route(eat_handle* h, const void* x, int T, int ppl_sign, int32_t* idx, float* w,
                      int32_t* k, float* psel, cudaStream_t st) {
-  const RouteParams rp = route_params(h->prm, ppl_sign);
+  RouteParams rp = route_params(h->prm, ppl_sign);
+  rp.opd_scale = h->desc.opd_scale;
   const int split = router_split(T, h->d, h->E);
   EAT_TRY(launch(h, kRoute, st, "router logits", [&] {
     return launch_router_logits(x, h->bf16, h->desc.w_router, T, h->d, h->E, split,
@@ -265,6 +269,8 @@ eat_status eat_default_params(eat_params* p) {
   p->max_k = 2;
   p->clamp_enabled = 1;
   p->c_mode = EAT_C_SUM;
+  p->router_mode = EAT_ROUTER_EAT;
+  p->top_p = 0.6;
   return EAT_OK;
 }
 
@@ -303,6 +309,10 @@ eat_status eat_create(const eat_layer_desc* desc, const eat_params* params, eat_
     return fail(nullptr, EAT_ERR_INVALID_ARG, "need 0 <= q_lo <= q_hi <= 1");
   if (Pm.c_mode != EAT_C_SUM && Pm.c_mode != EAT_C_RAW)
     return fail(nullptr, EAT_ERR_INVALID_ARG, "bad c_mode");
+  if (Pm.router_mode < EAT_ROUTER_EAT || Pm.router_mode > EAT_ROUTER_TOPP)
+    return fail(nullptr, EAT_ERR_INVALID_ARG, "bad router_mode");
+  if (Pm.router_mode == EAT_ROUTER_TOPP && !(Pm.top_p > 0.0 && Pm.top_p <= 1.0))
+    return fail(nullptr, EAT_ERR_INVALID_ARG, "top_p must be in (0, 1]");
 
   eat_handle* h = new (std::nothrow) eat_handle();
   if (!h) return fail(nullptr, EAT_ERR_OOM, "host allocation failed");

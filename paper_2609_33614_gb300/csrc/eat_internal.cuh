@@ -43,8 +43,9 @@ constexpr int kMaxK = 16;
 // ---------------------------------------------------------------------------------------------
 struct RouteParams {
   float w1, w2, w3, beta, alpha1, alpha2, kappa1, kappa2, ppl_factor, q_lo, q_hi, eps,
-      temperature;
-  int clamp, c_mode;
+      temperature, top_p;
+  int clamp, c_mode, mode;
+  const float* opd_scale;  // [E] or nullptr
 };
 
 // Partial router logits (fp64): part[s][t][e] = sum over the s-th slice of d of x[t,j] Wr[e,j].

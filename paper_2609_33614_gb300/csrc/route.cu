@@ -273,6 +273,22 @@ route_select_kernel(const double* __restrict__ part, int n_split, const float* _
     p[i] = valid[i] ? p[i] / ssum : 0.f;
     psum += p[i];
   }
+  if (rp.opd_scale) {
+    // §3.5 OPD reweighting: p'_i = s_i p_i / sum_j s_j p_j replaces p from here on
+    float qs = 0.f;
+#pragma unroll
+    for (int i = 0; i < EPL; ++i) {
+      p[i] = valid[i] ? p[i] * rp.opd_scale[lane + 32 * i] : 0.f;
+      qs += p[i];
+    }
+    qs = warp_sum(qs);
+    psum = 0.f;
+#pragma unroll
+    for (int i = 0; i < EPL; ++i) {
+      p[i] = valid[i] ? p[i] / qs : 0.f;
+      psum += p[i];
+    }
+  }
   // Eq. 3-4: mean and population standard deviation of g = p
   const float mu = warp_sum(psum) * inv_e;
   float dev = 0.f;
@@ -329,7 +345,37 @@ route_select_kernel(const double* __restrict__ part, int n_split, const float* _
     ncand += __popc(__ballot_sync(full, cand[i]));
   }
   bool sel[EPL];
-  if (ncand == 0) {
+  if (rp.mode != EAT_ROUTER_EAT) {
+    // §4.1 baselines: rank by (p desc, index asc); Top-K keeps ranks < K, Top-P keeps the
+    // smallest prefix whose cumulative probability reaches top_p (at most K)
+    int r[EPL];
+    float cum[EPL];
+#pragma unroll
+    for (int i = 0; i < EPL; ++i) {
+      r[i] = 0;
+      cum[i] = 0.f;
+    }
+#pragma unroll
+    for (int jb = 0; jb < EPL; ++jb) {
+      for (int jl = 0; jl < 32; ++jl) {
+        const int ej = jb * 32 + jl;
+        const float pj = __shfl_sync(full, p[jb], jl);
+        if (ej < E) {
+#pragma unroll
+          for (int i = 0; i < EPL; ++i) {
+            const int ei = lane + 32 * i;
+            if (pj > p[i] || (pj == p[i] && ej < ei)) {
+              r[i] += 1;
+              cum[i] += pj;
+            }
+          }
+        }
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < EPL; ++i)
+      sel[i] = valid[i] && r[i] < K && (rp.mode == EAT_ROUTER_TOPK || cum[i] < rp.top_p);
+  } else if (ncand == 0) {
     // argmax I, lowest index on ties
     float bv = -INFINITY;
     int be = 0x7fffffff;

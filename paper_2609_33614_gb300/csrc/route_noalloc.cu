@@ -83,6 +83,9 @@ extern "C" eat_status eat_route_noalloc(const void* x, int32_t T, int32_t d_mode
   if (!(p.q_lo >= 0.0 && p.q_lo <= p.q_hi && p.q_hi <= 1.0))
     return bad("eat_route_noalloc: need 0 <= q_lo <= q_hi <= 1");
   if (p.c_mode != EAT_C_SUM && p.c_mode != EAT_C_RAW) return bad("eat_route_noalloc: bad c_mode");
+  if (p.router_mode < EAT_ROUTER_EAT || p.router_mode > EAT_ROUTER_TOPP ||
+      (p.router_mode == EAT_ROUTER_TOPP && !(p.top_p > 0.0 && p.top_p <= 1.0)))
+    return bad("eat_route_noalloc: bad router_mode or top_p");
   if ((size_t)T * (size_t)n_experts > kScratchDoubles)
     return bad("eat_route_noalloc: T * n_experts exceeds the 131072 router scores its fixed "
                "1 MiB scratch holds; split the call into smaller token batches");
@@ -110,6 +113,9 @@ extern "C" eat_status eat_route_noalloc(const void* x, int32_t T, int32_t d_mode
   rp.temperature = (float)p.temperature;
   rp.clamp = p.clamp_enabled;
   rp.c_mode = p.c_mode;
+  rp.mode = p.router_mode;
+  rp.top_p = (float)p.top_p;
+  rp.opd_scale = nullptr;
 
   cudaStream_t st = (cudaStream_t)stream;
   cudaError_t e = eat::launch_router_logits(x, xdtype == EAT_BF16, w_router, T, d_model,

@@ -16,6 +16,7 @@ LIB_PATH = os.path.join(PKG, "libeat.so")
 EAT_OK, EAT_ERR_INVALID_ARG, EAT_ERR_UNSUPPORTED, EAT_ERR_OOM, EAT_ERR_CUDA, EAT_ERR_STATE = range(6)
 EAT_F32, EAT_BF16 = 0, 1
 EAT_C_SUM, EAT_C_RAW = 0, 1
+EAT_ROUTER_EAT, EAT_ROUTER_TOPK, EAT_ROUTER_TOPP = 0, 1, 2
 KERNEL_KINDS = ("route", "permute", "ffn_up", "ffn_down", "shared_up", "shared_down", "combine",
                 "account", "select", "gather")
 
@@ -26,14 +27,15 @@ class eat_params(ctypes.Structure):
     _fields_ = [(n, c_dbl) for n in ("alpha", "w1", "w2", "w3", "beta", "alpha1", "alpha2",
                                      "kappa1", "kappa2", "ppl_up", "ppl_down", "q_lo", "q_hi",
                                      "eps", "temperature")] + \
-               [("max_k", c_i32), ("clamp_enabled", c_i32), ("c_mode", c_i32)]
+               [("max_k", c_i32), ("clamp_enabled", c_i32), ("c_mode", c_i32),
+                ("router_mode", c_i32), ("top_p", c_dbl)]
 
 
 class eat_layer_desc(ctypes.Structure):
     _fields_ = [(n, c_i32) for n in ("d_model", "n_experts", "d_ff", "n_shared", "d_ff_shared",
                                      "max_tokens", "wdtype", "xdtype")] + \
                [(n, c_vp) for n in ("w_router", "b_router", "w_gate", "w_up", "w_down",
-                                    "ws_gate", "ws_up", "ws_down")]
+                                    "ws_gate", "ws_up", "ws_down", "opd_scale")]
 
 
 class EatError(RuntimeError):
@@ -194,9 +196,10 @@ class EatLayer:
     """Owns an eat_handle for one MoE layer whose weights are CUDA tensors (kept referenced)."""
 
     def __init__(self, w_router, b_router, w_gate, w_up, w_down, max_tokens, params,
-                 ws_gate=None, ws_up=None, ws_down=None):
+                 ws_gate=None, ws_up=None, ws_down=None, opd_scale=None):
         import torch
-        self._keep = [w_router, b_router, w_gate, w_up, w_down, ws_gate, ws_up, ws_down]
+        self._keep = [w_router, b_router, w_gate, w_up, w_down, ws_gate, ws_up, ws_down,
+                      opd_scale]
         bf16 = w_gate.dtype == torch.bfloat16
         E, F, d = w_gate.shape
         S = 0 if ws_gate is None else ws_gate.shape[0]
@@ -207,18 +210,19 @@ class EatLayer:
         desc = eat_layer_desc(d, E, F, S, Fs, max_tokens, EAT_BF16 if bf16 else EAT_F32,
                               EAT_BF16 if bf16 else EAT_F32, _ptr(w_router), _ptr(b_router),
                               _ptr(w_gate), _ptr(w_up), _ptr(w_down), _ptr(ws_gate), _ptr(ws_up),
-                              _ptr(ws_down))
+                              _ptr(ws_down), _ptr(opd_scale))
         self.params = params
         self.h = eat_create(desc, params)
 
     @classmethod
-    def from_workload(cls, lw, max_tokens, params=None, device="cuda"):
+    def from_workload(cls, lw, max_tokens, params=None, device="cuda", opd_scale=None):
         """Build from a workloads.LayerWeights (moved to ``device`` if needed)."""
         if params is None:
             params = eat_default_params(lw.shape.max_k, temperature=lw.shape.temperature)
         mv = lambda t: None if t is None else t.to(device).contiguous()
         return cls(mv(lw.w_router), mv(lw.b_router), mv(lw.w_gate), mv(lw.w_up), mv(lw.w_down),
-                   max_tokens, params, mv(lw.ws_gate), mv(lw.ws_up), mv(lw.ws_down))
+                   max_tokens, params, mv(lw.ws_gate), mv(lw.ws_up), mv(lw.ws_down),
+                   mv(opd_scale))
 
     def close(self):
         if getattr(self, "h", None):

@@ -73,15 +73,55 @@ def gpu_selection(idx: torch.Tensor, k: torch.Tensor) -> list:
     return [idx[t, :k[t]].tolist() for t in range(idx.shape[0])]
 
 
+def _desc(p):
+    return sorted(range(p.shape[0]), key=lambda i: (-p[i], i))
+
+
+def ambiguous_baseline(p: np.ndarray, K: int, mode: str, top_p: float) -> bool:
+    """Top-K: the K-th and (K+1)-th probabilities within delta.  Top-P: additionally any
+    cumulative probability before the first K + 1 ranks within delta of P."""
+    dl = 1e-5
+    order = _desc(p)
+    q = p[order]
+    if any(q[i] - q[i + 1] <= dl for i in range(min(K, q.size - 1))):
+        return True
+    if mode == "topp":
+        cum = np.concatenate([[0.0], np.cumsum(q)])
+        if np.any(np.abs(cum[:K + 1] - top_p) <= dl):
+            return True
+    return False
+
+
+def valid_baseline(sel: list, p: np.ndarray, K: int, mode: str, top_p: float) -> bool:
+    """A descending-p prefix (within delta) of admissible length."""
+    dl = 1e-5
+    L = len(sel)
+    if not 1 <= L <= K or len(set(sel)) != L:
+        return False
+    lo = min(p[i] for i in sel)
+    if any(p[j] > lo + dl for j in range(p.shape[0]) if j not in sel):
+        return False
+    if mode == "topk":
+        return L == K
+    tot = sum(p[i] for i in sel)
+    return (L == K or tot >= top_p - dl) and tot - lo < top_p + dl
+
+
 def check_routing(routing: orc.Routing, sel_gpu: list, w_gpu: np.ndarray, K: int,
-                  w_tol: float = 1e-5):
+                  w_tol: float = 1e-5, mode: str = "eat", top_p: float = 0.6):
     """Returns (ambiguous token list, max relative gate error on the others)."""
     amb = []
     max_w = 0.0
     for t, sel in enumerate(sel_gpu):
         I, tau = routing.I[t], routing.tau_final[t]
         assert sel == sorted(sel), f"token {t}: idx not ascending {sel}"
-        if ambiguous(I, tau, K):
+        if mode != "eat":
+            if ambiguous_baseline(routing.p[t], K, mode, top_p):
+                amb.append(t)
+                assert valid_baseline(sel, routing.p[t], K, mode, top_p), \
+                    f"token {t}: GPU {mode} selection {sel} invalid"
+                continue
+        elif ambiguous(I, tau, K):
             amb.append(t)
             assert valid_selection(sel, I, tau, K), \
                 f"token {t}: GPU selection {sel} invalid near the threshold (tau={tau})"

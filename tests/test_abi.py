@@ -37,13 +37,15 @@ def test_default_params_are_table1(lib):
     assert (p.alpha1, p.alpha2, p.kappa1, p.kappa2) == (0.5, 1.0, 0.7, 0.3)
     assert (p.ppl_up, p.ppl_down, p.q_lo, p.q_hi, p.eps) == (1.2, 0.9, 0.1, 0.9, 1e-8)
     assert (p.temperature, p.max_k, p.clamp_enabled, p.c_mode) == (1.0, 2, 1, eat.EAT_C_SUM)
+    assert (p.router_mode, p.top_p) == (eat.EAT_ROUTER_EAT, 0.6)
     assert lib.eat_default_params(None) == eat.EAT_ERR_INVALID_ARG
 
 
 def _desc(**kw):
     base = dict(d_model=256, n_experts=8, d_ff=512, n_shared=0, d_ff_shared=0, max_tokens=64,
                 wdtype=eat.EAT_F32, xdtype=eat.EAT_F32, w_router=16, b_router=None,
-                w_gate=4096, w_up=8192, w_down=12288, ws_gate=None, ws_up=None, ws_down=None)
+                w_gate=4096, w_up=8192, w_down=12288, ws_gate=None, ws_up=None, ws_down=None,
+                opd_scale=None)
     base.update(kw)
     return eat.eat_layer_desc(*[base[n] for n, _ in eat.eat_layer_desc._fields_])
 
@@ -65,6 +67,8 @@ def _desc(**kw):
     ({}, dict(q_lo=0.95), eat.EAT_ERR_INVALID_ARG),
     ({}, dict(c_mode=7), eat.EAT_ERR_INVALID_ARG),
     ({}, dict(alpha=1.5), eat.EAT_ERR_INVALID_ARG),
+    ({}, dict(router_mode=3), eat.EAT_ERR_INVALID_ARG),
+    ({}, dict(router_mode=eat.EAT_ROUTER_TOPP, top_p=0.0), eat.EAT_ERR_INVALID_ARG),
 ])
 def test_create_rejects_invalid_layers(lib, kw, params, status):
     h = ctypes.c_void_p(1234)

@@ -35,6 +35,9 @@ def oracle_params(shape, **kw):
         kw["c_mode"] = "raw" if kw["c_mode"] == eat.EAT_C_RAW else "sum"
     if "clamp_enabled" in kw:
         kw["clamp"] = bool(kw.pop("clamp_enabled"))
+    if "router_mode" in kw:
+        kw["router"] = {eat.EAT_ROUTER_EAT: "eat", eat.EAT_ROUTER_TOPK: "topk",
+                        eat.EAT_ROUTER_TOPP: "topp"}[kw.pop("router_mode")]
     return orc.Params(max_k=shape.max_k, temperature=shape.temperature, **kw)
 
 
@@ -48,7 +51,7 @@ def _acc(layer):
 
 
 def run_parity(shape, lw, Ts, signs=None, prm_kw=None, layer=None, L=None, sample=None,
-               x_device="cpu", max_tokens=None, inputs=None):
+               x_device="cpu", max_tokens=None, inputs=None, opd_scale=None):
     """Run len(Ts) steps and check each one.  sample: number of tokens whose outputs are checked
     (None: all).  inputs: optional list of x tensors replacing the seeded draws.  Returns the
     list of GPU outputs."""
@@ -56,9 +59,11 @@ def run_parity(shape, lw, Ts, signs=None, prm_kw=None, layer=None, L=None, sampl
     own = layer is None
     if own:
         layer = eat.EatLayer.from_workload(lw, max(Ts) if max_tokens is None else max_tokens,
-                                           gpu_params(shape, **prm_kw))
+                                           gpu_params(shape, **prm_kw), opd_scale=opd_scale)
     if L is None:
         L = oracle_layer(lw)
+    if opd_scale is not None:
+        L.opd_scale = np64(opd_scale)
     prm = oracle_params(shape, **prm_kw)
     outs = []
     rng = np.random.default_rng(99)
@@ -74,7 +79,8 @@ def run_parity(shape, lw, Ts, signs=None, prm_kw=None, layer=None, L=None, sampl
         x64 = np64(x)
         routing = orc.route(x64, L, acc0, prm, sign)
         sel_gpu = par.gpu_selection(idx, k)
-        amb, _ = par.check_routing(routing, sel_gpu, w.cpu().numpy(), shape.max_k)
+        amb, _ = par.check_routing(routing, sel_gpu, w.cpu().numpy(), shape.max_k,
+                                   mode=prm.router, top_p=prm.top_p)
         sel = par.substituted(routing, sel_gpu, amb, prm.eps)
         y_gpu = np64(y)
         # outputs of every token, with the GPU's (validated) selection on the ambiguous ones
@@ -241,6 +247,28 @@ def test_deterministic_repeat():
         assert torch.equal(a, b)
     for a, b in zip(outs[0][1], outs[1][1]):
         assert torch.equal(a, b)
+
+
+# ------------------------------------------------------------------ baselines and OPD (§4.1, §3.5)
+def test_topk_router_mode():
+    lw = W.make_layer(MIX_S)
+    run_parity(MIX_S, lw, [128, 7, 1], prm_kw={"router_mode": eat.EAT_ROUTER_TOPK})
+
+
+@pytest.mark.parametrize("top_p", [0.2, 0.4, 0.6])
+def test_topp_router_mode(top_p):
+    lw = W.make_layer(OLMOE_S)
+    run_parity(OLMOE_S, lw, [300, 32], prm_kw={"router_mode": eat.EAT_ROUTER_TOPP,
+                                                "top_p": top_p})
+
+
+def test_opd_reweighting_eat_and_topp():
+    lw = W.make_layer(QWEN_S)
+    g = torch.Generator().manual_seed(17)
+    scale = (torch.rand(60, generator=g) * 3 + 0.25).to(torch.float32)
+    run_parity(QWEN_S, lw, [200, 16], opd_scale=scale)
+    run_parity(QWEN_S, lw, [200], opd_scale=scale,
+               prm_kw={"router_mode": eat.EAT_ROUTER_TOPP, "top_p": 0.4})
 
 
 # ------------------------------------------------------------------ full-size layers (sampled)
