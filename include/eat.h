@@ -55,6 +55,11 @@ typedef enum eat_router_mode {
   EAT_ROUTER_TOPP = 2
 } eat_router_mode;
 
+/* Threshold smoothing of §3.3.  EAT_SMOOTH_CALL: the same-call blend kappa1 tau_PPL + kappa2 tau.
+ * EAT_SMOOTH_TEMPORAL: an EMA over calls of one token stream, kappa1 tau_PPL + kappa2 tau_prev,
+ * where tau_prev is that stream's tau_final of the previous call (see eat_set_tau_state). */
+typedef enum eat_smoothing { EAT_SMOOTH_CALL = 0, EAT_SMOOTH_TEMPORAL = 1 } eat_smoothing;
+
 /* How the EMA contribution C_s enters Eq. 1 (§3.2).  EAT_C_SUM: as the share C_i / sum_j C_j,
  * on the same [0, 1] scale as the other two terms (default).  EAT_C_RAW: the literal C_i. */
 typedef enum eat_c_mode { EAT_C_SUM = 0, EAT_C_RAW = 1 } eat_c_mode;
@@ -79,6 +84,7 @@ typedef struct eat_params {
   int32_t c_mode;      /* eat_c_mode */
   int32_t router_mode; /* eat_router_mode (EAT_ROUTER_EAT) */
   double top_p;        /* P of EAT_ROUTER_TOPP, in (0, 1] (0.6) */
+  int32_t smoothing_mode; /* eat_smoothing (EAT_SMOOTH_CALL) */
 } eat_params;
 
 /* Fill *p with the defaults above, max_k = 2, router_mode EAT_ROUTER_EAT, top_p 0.6.  Returns
@@ -160,12 +166,21 @@ eat_status eat_moe_forward_host(eat_handle* h, const void* x_host, int32_t T, in
  *    device, done with that device current); make that first call before any stream capture.
  *  - Calls share the scratch: two calls that may overlap on the GPU (different streams or host
  *    threads) race on it and must be serialised by the caller.
+ *  - There is no per-stream threshold state without a handle: EAT_SMOOTH_TEMPORAL is routed as
+ *    EAT_SMOOTH_CALL.
  * Errors are reported through eat_last_error(NULL). */
 eat_status eat_route_noalloc(const void* x, int32_t T, int32_t d_model, int32_t n_experts,
                              int32_t xdtype, const float* w_router, const float* b_router,
                              const int64_t* N, const double* P, const double* C,
                              const eat_params* params, int32_t ppl_sign, int32_t* idx, float* w,
                              int32_t* k, void* stream);
+
+/* Per-stream threshold state for EAT_SMOOTH_TEMPORAL: tau_state is a caller-owned device array
+ * of max_tokens fp32 values; row t of every call is token stream t (e.g. sequence t of a decode
+ * batch).  eat_route reads it; eat_moe_forward reads it and stores each token's tau_final back.
+ * NaN entries mean "no previous call" (the same-call blend is used).  NULL detaches the state
+ * (temporal mode then behaves as EAT_SMOOTH_CALL).  The array must stay alive while attached. */
+eat_status eat_set_tau_state(eat_handle* h, float* tau_state);
 
 /* Free everything the handle owns.  Synchronises the device first.  NULL is accepted. */
 eat_status eat_destroy(eat_handle* h);

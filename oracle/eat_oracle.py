@@ -24,6 +24,8 @@ Readings taken where the paper is silent or ambiguous (each is also listed in th
       c_mode "raw": the literal C_i.
   R4  tau_PPL = f * tau (f = 1.2 after a PPL rise, 0.9 otherwise, 1 without a signal) and the
       smoothing is the same-call blend kappa1 * tau_PPL + kappa2 * tau.
+  R4' (optional, smoothing "temporal") the smoothing is an EMA over calls of one token stream:
+      kappa1 * tau_PPL + kappa2 * (that stream's previous tau_final).
   R5  tau_min / tau_max are the linear-interpolation ("type 7") 10th / 90th percentiles of the
       token's E routing probabilities, applied after smoothing so tau_final lies in range.
   R6  argmax ties (empty candidate set) go to the lowest expert index.
@@ -78,6 +80,7 @@ class Params:
     c_mode: str = "sum"      # reading R3: "sum" or "raw"
     router: str = "eat"      # "eat" (§3.2-§3.4), or the baselines "topk" / "topp" (§4.1)
     top_p: float = 0.6       # P of the Top-P baseline (§4.1: 0.6 / 0.2 / 0.4)
+    smoothing: str = "call"  # reading R4 ("call") or the temporal reading ("temporal", R4')
 
     def with_(self, **kw) -> "Params":
         return replace(self, **kw)
@@ -213,18 +216,26 @@ class Threshold:
     tau_final: float
 
 
-def threshold(g: np.ndarray, prm: Params, ppl_sign: int = 0) -> Threshold:
+def threshold(g: np.ndarray, prm: Params, ppl_sign: int = 0,
+              tau_prev: float | None = None) -> Threshold:
     """§3.3 for one token's gating scores g [E] (g = p, reading R1):
     mu = mean g (Eq. 3), sigma = population std (Eq. 4), tau = max(a1 mu, mu - a2 sigma) (Eq. 5),
     tau_PPL = f tau, smoothed kappa1 tau_PPL + kappa2 tau (R4), then clamped to the
-    [q_lo, q_hi] quantiles of g (R5)."""
+    [q_lo, q_hi] quantiles of g (R5).  Temporal reading (R4', smoothing "temporal"): the second
+    term is the previous call's tau_final of the same token stream, kappa1 tau_PPL + kappa2
+    tau_prev; without a previous value (None or NaN) it falls back to tau."""
     g = np.asarray(g, F64)
     n = g.shape[0]
     mu = g.sum() / n
     sigma = math.sqrt(((g - mu) ** 2).sum() / n)
     tau = max(prm.alpha1 * mu, mu - prm.alpha2 * sigma)
     tau_ppl = ppl_factor(ppl_sign, prm) * tau
-    tau_s = prm.kappa1 * tau_ppl + prm.kappa2 * tau
+    second = tau
+    if prm.smoothing == "temporal" and tau_prev is not None and not math.isnan(tau_prev):
+        second = float(tau_prev)
+    elif prm.smoothing not in ("call", "temporal"):
+        raise ValueError(f"unknown smoothing {prm.smoothing!r}")
+    tau_s = prm.kappa1 * tau_ppl + prm.kappa2 * second
     lo = quantile_type7(g, prm.q_lo)
     hi = quantile_type7(g, prm.q_hi)
     tau_final = min(max(tau_s, lo), hi) if prm.clamp else tau_s
@@ -282,10 +293,12 @@ class Routing:
         return np.array([t.tau_final for t in self.thresholds], F64)
 
 
-def route(x: np.ndarray, layer: Layer, acc: Accounts, prm: Params, ppl_sign: int = 0) -> Routing:
+def route(x: np.ndarray, layer: Layer, acc: Accounts, prm: Params, ppl_sign: int = 0,
+          tau_prev: np.ndarray | None = None) -> Routing:
     """Router -> softmax (-> OPD reweighting, §3.5) -> S_h -> I -> tau_final -> E_final -> g_norm
     for every token, all from the same account snapshot (reading R10).  With router "topk" /
-    "topp" the selection is the §4.1 baseline instead of Eq. 6; everything else is unchanged."""
+    "topp" the selection is the §4.1 baseline instead of Eq. 6; everything else is unchanged.
+    tau_prev [T]: previous tau_final per token stream for the temporal smoothing (NaN: none)."""
     z = router_logits(x, layer.w_router, layer.b_router, prm.temperature)
     p = opd_reweight(softmax(z), layer.opd_scale)
     s_h = history_score(acc, prm)
@@ -293,7 +306,7 @@ def route(x: np.ndarray, layer: Layer, acc: Accounts, prm: Params, ppl_sign: int
     ths, sels = [], []
     g_norm = np.zeros_like(p)
     for t in range(p.shape[0]):
-        th = threshold(p[t], prm, ppl_sign)
+        th = threshold(p[t], prm, ppl_sign, None if tau_prev is None else float(tau_prev[t]))
         if prm.router == "eat":
             sel = select(I[t], th.tau_final, prm.max_k)
         elif prm.router == "topk":
@@ -362,11 +375,11 @@ class ForwardResult:
 
 
 def moe_forward(x: np.ndarray, layer: Layer, acc: Accounts, prm: Params,
-                ppl_sign: int = 0) -> ForwardResult:
+                ppl_sign: int = 0, tau_prev: np.ndarray | None = None) -> ForwardResult:
     """One MoE layer call: y_t = sum_{e in E_final(t)} g_norm,t,e E_e(x_t) + shared(x_t), then the
     account update.  One call is one EMA timestep t of §3.2."""
     x = np.asarray(x, F64)
-    r = route(x, layer, acc, prm, ppl_sign)
+    r = route(x, layer, acc, prm, ppl_sign, tau_prev)
     T = x.shape[0]
     y = np.zeros((T, layer.w_router.shape[1]), F64)
     norms = {}

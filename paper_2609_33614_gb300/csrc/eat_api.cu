@@ -47,6 +47,7 @@ struct eat_handle {
   unsigned int* status = nullptr;  // device status word: bounded waits that expired
   int32_t* chunk_cnt = nullptr;    // [permute chunks][E]
   long long opart_rows = 0;
+  float* tau_state = nullptr;  // caller-owned [Tmax] previous tau_final per stream, or null
 
   TcLayer tc{};
 
@@ -119,7 +120,10 @@ RouteParams route_params(const eat_params& p, int ppl_sign) {
   r.c_mode = p.c_mode;
   r.mode = p.router_mode;
   r.top_p = (float)p.top_p;
+  r.smoothing = p.smoothing_mode;
   r.opd_scale = nullptr;
+  r.tau_in = nullptr;
+  r.tau_out = nullptr;
   return r;
 }
 
@@ -141,9 +145,13 @@ eat_status check_call(eat_handle* h, const void* x, int32_t T, int32_t ppl_sign)
 
 // Router + selection into (idx, w, k, psel).
 eat_status run_route(eat_handle* h, const void* x, int T, int ppl_sign, int32_t* idx, float* w,
-                     int32_t* k, float* psel, cudaStream_t st) {
+                     int32_t* k, float* psel, bool write_tau, cudaStream_t st) {
   RouteParams rp = route_params(h->prm, ppl_sign);
   rp.opd_scale = h->desc.opd_scale;
+  if (h->prm.smoothing_mode == EAT_SMOOTH_TEMPORAL && h->tau_state) {
+    rp.tau_in = h->tau_state;
+    rp.tau_out = write_tau ? h->tau_state : nullptr;
+  }
   const int split = router_split(T, h->d, h->E);
   EAT_TRY(launch(h, kRoute, st, "router logits", [&] {
     return launch_router_logits(x, h->bf16, h->desc.w_router, T, h->d, h->E, split,
@@ -158,7 +166,7 @@ eat_status run_route(eat_handle* h, const void* x, int T, int ppl_sign, int32_t*
 
 eat_status run_forward(eat_handle* h, const void* x, int T, int ppl_sign, void* y,
                        int32_t* idx_opt, float* w_opt, int32_t* k_opt, cudaStream_t st) {
-  EAT_TRY(run_route(h, x, T, ppl_sign, h->idx, h->w, h->k, h->psel, st));
+  EAT_TRY(run_route(h, x, T, ppl_sign, h->idx, h->w, h->k, h->psel, true, st));
   const int tile_rows = h->backend == 1 ? tc_tile_rows(h->tc, T) : kSimtTileRows;
   EAT_TRY(launch(h, kPermute, st, "permute", [&] {
     return launch_permute(h->idx, h->k, h->psel, T, h->K, h->E, tile_rows, h->perm, h->chunk_cnt,
@@ -271,6 +279,7 @@ eat_status eat_default_params(eat_params* p) {
   p->c_mode = EAT_C_SUM;
   p->router_mode = EAT_ROUTER_EAT;
   p->top_p = 0.6;
+  p->smoothing_mode = EAT_SMOOTH_CALL;
   return EAT_OK;
 }
 
@@ -309,6 +318,8 @@ eat_status eat_create(const eat_layer_desc* desc, const eat_params* params, eat_
     return fail(nullptr, EAT_ERR_INVALID_ARG, "need 0 <= q_lo <= q_hi <= 1");
   if (Pm.c_mode != EAT_C_SUM && Pm.c_mode != EAT_C_RAW)
     return fail(nullptr, EAT_ERR_INVALID_ARG, "bad c_mode");
+  if (Pm.smoothing_mode != EAT_SMOOTH_CALL && Pm.smoothing_mode != EAT_SMOOTH_TEMPORAL)
+    return fail(nullptr, EAT_ERR_INVALID_ARG, "bad smoothing_mode");
   if (Pm.router_mode < EAT_ROUTER_EAT || Pm.router_mode > EAT_ROUTER_TOPP)
     return fail(nullptr, EAT_ERR_INVALID_ARG, "bad router_mode");
   if (Pm.router_mode == EAT_ROUTER_TOPP && !(Pm.top_p > 0.0 && Pm.top_p <= 1.0))
@@ -432,7 +443,7 @@ eat_status eat_route(eat_handle* h, const void* x, int32_t T, int32_t ppl_sign, 
                      float* w, int32_t* k, void* stream) {
   EAT_TRY(check_call(h, x, T, ppl_sign));
   if (!idx || !w || !k) return fail(h, EAT_ERR_INVALID_ARG, "idx, w and k must be non-NULL");
-  return run_route(h, x, T, ppl_sign, idx, w, k, nullptr, (cudaStream_t)stream);
+  return run_route(h, x, T, ppl_sign, idx, w, k, nullptr, false, (cudaStream_t)stream);
 }
 
 eat_status eat_moe_forward(eat_handle* h, const void* x, int32_t T, int32_t ppl_sign, void* y,
@@ -456,6 +467,14 @@ eat_status eat_moe_forward_host(eat_handle* h, const void* x_host, int32_t T, in
   e = cudaMemcpyAsync(y_host, h->ystage, bytes, cudaMemcpyDeviceToHost, st);
   if (e == cudaSuccess) e = cudaStreamSynchronize(st);
   if (e != cudaSuccess) return cuda_fail(h, e, "y device-to-host copy");
+  return EAT_OK;
+}
+
+eat_status eat_set_tau_state(eat_handle* h, float* tau_state) {
+  if (!h) return fail(nullptr, EAT_ERR_INVALID_ARG, "null handle");
+  if (((uintptr_t)tau_state & 3) != 0)
+    return fail(h, EAT_ERR_INVALID_ARG, "tau_state must be 4-byte aligned");
+  h->tau_state = tau_state;
   return EAT_OK;
 }
 

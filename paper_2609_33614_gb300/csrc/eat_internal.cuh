@@ -44,8 +44,10 @@ constexpr int kMaxK = 16;
 struct RouteParams {
   float w1, w2, w3, beta, alpha1, alpha2, kappa1, kappa2, ppl_factor, q_lo, q_hi, eps,
       temperature, top_p;
-  int clamp, c_mode, mode;
+  int clamp, c_mode, mode, smoothing;
   const float* opd_scale;  // [E] or nullptr
+  const float* tau_in;     // [T] previous tau_final per token stream (temporal smoothing) or null
+  float* tau_out;          // [T] tau_final written back (temporal smoothing, forward calls) or null
 };
 
 // Partial router logits (fp64): part[s][t][e] = sum over the s-th slice of d of x[t,j] Wr[e,j].

@@ -300,7 +300,12 @@ route_select_kernel(const double* __restrict__ part, int n_split, const float* _
   const float sigma = sqrtf(warp_sum(dev) * inv_e);
   // Eq. 5, PPL adjustment and smoothing (§3.3)
   const float tau = fmaxf(rp.alpha1 * mu, mu - rp.alpha2 * sigma);
-  float tau_f = rp.kappa1 * (rp.ppl_factor * tau) + rp.kappa2 * tau;
+  float second = tau;  // same-call blend, or the stream's previous tau_final (temporal reading)
+  if (rp.smoothing == EAT_SMOOTH_TEMPORAL && rp.tau_in) {
+    const float prev = rp.tau_in[t];
+    if (!isnan(prev)) second = prev;
+  }
+  float tau_f = rp.kappa1 * (rp.ppl_factor * tau) + rp.kappa2 * second;
 
   int rank[EPL];
 #pragma unroll
@@ -333,6 +338,8 @@ route_select_kernel(const double* __restrict__ part, int n_split, const float* _
     const float q_hi = v_hi0 + (h_hi - (float)hi0) * (v_hi1 - v_hi0);
     tau_f = fminf(fmaxf(tau_f, q_lo), q_hi);
   }
+
+  if (rp.tau_out && lane == 0) rp.tau_out[t] = tau_f;
 
   // Eq. 2 importance and Eq. 6 candidate set
   bool cand[EPL];

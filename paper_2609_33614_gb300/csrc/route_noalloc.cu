@@ -115,7 +115,10 @@ extern "C" eat_status eat_route_noalloc(const void* x, int32_t T, int32_t d_mode
   rp.c_mode = p.c_mode;
   rp.mode = p.router_mode;
   rp.top_p = (float)p.top_p;
+  rp.smoothing = EAT_SMOOTH_CALL;  // no per-stream state without a handle
   rp.opd_scale = nullptr;
+  rp.tau_in = nullptr;
+  rp.tau_out = nullptr;
 
   cudaStream_t st = (cudaStream_t)stream;
   cudaError_t e = eat::launch_router_logits(x, xdtype == EAT_BF16, w_router, T, d_model,

@@ -17,6 +17,7 @@ EAT_OK, EAT_ERR_INVALID_ARG, EAT_ERR_UNSUPPORTED, EAT_ERR_OOM, EAT_ERR_CUDA, EAT
 EAT_F32, EAT_BF16 = 0, 1
 EAT_C_SUM, EAT_C_RAW = 0, 1
 EAT_ROUTER_EAT, EAT_ROUTER_TOPK, EAT_ROUTER_TOPP = 0, 1, 2
+EAT_SMOOTH_CALL, EAT_SMOOTH_TEMPORAL = 0, 1
 KERNEL_KINDS = ("route", "permute", "ffn_up", "ffn_down", "shared_up", "shared_down", "combine",
                 "account", "select", "gather")
 
@@ -28,7 +29,7 @@ class eat_params(ctypes.Structure):
                                      "kappa1", "kappa2", "ppl_up", "ppl_down", "q_lo", "q_hi",
                                      "eps", "temperature")] + \
                [("max_k", c_i32), ("clamp_enabled", c_i32), ("c_mode", c_i32),
-                ("router_mode", c_i32), ("top_p", c_dbl)]
+                ("router_mode", c_i32), ("top_p", c_dbl), ("smoothing_mode", c_i32)]
 
 
 class eat_layer_desc(ctypes.Structure):
@@ -57,6 +58,7 @@ _SIGS = {
     "eat_moe_forward_host": (c_i32, [c_vp, c_vp, c_i32, c_i32, c_vp, c_vp]),
     "eat_route_noalloc": (c_i32, [c_vp, c_i32, c_i32, c_i32, c_i32, c_vp, c_vp, c_vp, c_vp, c_vp,
                                   ctypes.POINTER(eat_params), c_i32, c_vp, c_vp, c_vp, c_vp]),
+    "eat_set_tau_state": (c_i32, [c_vp, c_vp]),
     "eat_destroy": (c_i32, [c_vp]),
     "eat_get_accounts": (c_i32, [c_vp, c_vp, c_vp, c_vp, c_vp]),
     "eat_set_accounts": (c_i32, [c_vp, c_vp, c_vp, c_vp, c_vp]),
@@ -147,6 +149,29 @@ def eat_route_noalloc(x, T, d_model, n_experts, xdtype, w_router, b_router, N, P
                                    _ptr(b_router), _ptr(N), _ptr(P), _ptr(C),
                                    ctypes.byref(params), ppl_sign, _ptr(idx), _ptr(w), _ptr(k),
                                    _stream(stream)))
+
+
+def eat_set_tau_state(h, tau_state):
+    _check(lib().eat_set_tau_state(h, _ptr(tau_state)), h)
+
+
+def ppl_sign(ppl_prev: float, ppl_curr: float) -> int:
+    """The sign eat_route / eat_moe_forward take for the §3.3 adjustment from two perplexities of
+    the model (e.g. exp of the mean token negative log-likelihood over the last two windows):
+    +1 if PPL rose, -1 otherwise; 0 when no previous value exists."""
+    if ppl_prev is None:
+        return 0
+    return 1 if ppl_curr - ppl_prev > 0 else -1
+
+
+def layer_policy(layer: int, n_layers: int, max_k: int) -> dict:
+    """Per-layer EAT settings after §5.2 (lower layers tolerate far fewer experts, the top ~quarter
+    of the stack needs close to the full K): the lower three quarters route with at most
+    max(1, max_k // 3) experts and a doubled threshold floor, the upper layers use the defaults.
+    Returns eat_params overrides."""
+    if layer < (3 * n_layers) // 4:
+        return {"max_k": max(1, max_k // 3), "alpha1": 1.0}
+    return {"max_k": max_k}
 
 
 def eat_destroy(h):

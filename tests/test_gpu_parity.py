@@ -35,6 +35,9 @@ def oracle_params(shape, **kw):
         kw["c_mode"] = "raw" if kw["c_mode"] == eat.EAT_C_RAW else "sum"
     if "clamp_enabled" in kw:
         kw["clamp"] = bool(kw.pop("clamp_enabled"))
+    if "smoothing_mode" in kw:
+        kw["smoothing"] = "temporal" if kw.pop("smoothing_mode") == eat.EAT_SMOOTH_TEMPORAL \
+            else "call"
     if "router_mode" in kw:
         kw["router"] = {eat.EAT_ROUTER_EAT: "eat", eat.EAT_ROUTER_TOPK: "topk",
                         eat.EAT_ROUTER_TOPP: "topp"}[kw.pop("router_mode")]
@@ -51,7 +54,7 @@ def _acc(layer):
 
 
 def run_parity(shape, lw, Ts, signs=None, prm_kw=None, layer=None, L=None, sample=None,
-               x_device="cpu", max_tokens=None, inputs=None, opd_scale=None):
+               x_device="cpu", max_tokens=None, inputs=None, opd_scale=None, tau_state=None):
     """Run len(Ts) steps and check each one.  sample: number of tokens whose outputs are checked
     (None: all).  inputs: optional list of x tensors replacing the seeded draws.  Returns the
     list of GPU outputs."""
@@ -65,6 +68,8 @@ def run_parity(shape, lw, Ts, signs=None, prm_kw=None, layer=None, L=None, sampl
     if opd_scale is not None:
         L.opd_scale = np64(opd_scale)
     prm = oracle_params(shape, **prm_kw)
+    if tau_state is not None:
+        eat.eat_set_tau_state(layer.h, tau_state)
     outs = []
     rng = np.random.default_rng(99)
     for step, T in enumerate(Ts):
@@ -72,12 +77,17 @@ def run_parity(shape, lw, Ts, signs=None, prm_kw=None, layer=None, L=None, sampl
         x = inputs[step] if inputs is not None else W.make_tokens(shape, T, step=step,
                                                                   device=x_device)
         acc0 = _acc(layer)
+        tau_prev = None if tau_state is None else tau_state[:T].cpu().numpy().astype(np.float64)
         y, idx, w, k = layer.forward(x.cuda(), sign, with_routing=True)
         torch.cuda.synchronize()
         n_e, s_p, s_n = (t.cpu().numpy() for t in layer.call_stats())
         N1, P1, C1 = (t.cpu().numpy() for t in layer.accounts())
         x64 = np64(x)
-        routing = orc.route(x64, L, acc0, prm, sign)
+        routing = orc.route(x64, L, acc0, prm, sign, tau_prev)
+        if tau_state is not None:
+            got = tau_state[:T].cpu().numpy().astype(np.float64)
+            assert np.allclose(got, routing.tau_final, rtol=1e-5, atol=1e-9), \
+                f"step {step}: stored tau_final differs from the oracle"
         sel_gpu = par.gpu_selection(idx, k)
         amb, _ = par.check_routing(routing, sel_gpu, w.cpu().numpy(), shape.max_k,
                                    mode=prm.router, top_p=prm.top_p)
@@ -269,6 +279,35 @@ def test_opd_reweighting_eat_and_topp():
     run_parity(QWEN_S, lw, [200, 16], opd_scale=scale)
     run_parity(QWEN_S, lw, [200], opd_scale=scale,
                prm_kw={"router_mode": eat.EAT_ROUTER_TOPP, "top_p": 0.4})
+
+
+# ------------------------------------------------------------------ threshold variants, layer policy
+def test_temporal_smoothing_state():
+    """EMA of tau_final over calls of each token stream (decode batch of 24 streams)."""
+    lw = W.make_layer(OLMOE_S)
+    state = torch.full((64,), float("nan"), device="cuda")
+    run_parity(OLMOE_S, lw, [24] * 6, signs=[0, 1, 1, -1, 0, -1], max_tokens=64,
+               prm_kw={"smoothing_mode": eat.EAT_SMOOTH_TEMPORAL}, tau_state=state)
+
+
+def test_reversed_ppl_factors():
+    """The other reading of §3.3's PPL adjustment (a PPL rise lowers the threshold)."""
+    lw = W.make_layer(MIX_S)
+    run_parity(MIX_S, lw, [64] * 4, signs=[1, -1, 1, 1], prm_kw={"ppl_up": 0.8, "ppl_down": 1.1})
+
+
+def test_layer_policy_stack():
+    """Per-layer parameters on a stack (§5.2: lower layers sparser, upper layers up to full K)."""
+    from paper_2609_33614_gb300.eat import layer_policy
+    T, n = 64, 4
+    sh = W.scaled(W.DSV2L, "dsv2l-policy", d_model=256, d_ff=192, n_layers=n)
+    x = W.make_tokens(sh, T)
+    for l in range(n):
+        kw = layer_policy(l, n, sh.max_k)
+        lw = W.make_layer(sh, l)
+        outs = run_parity(W.scaled(sh, "p", max_k=kw["max_k"]), lw, [T], inputs=[x],
+                          prm_kw={k: v for k, v in kw.items() if k != "max_k"})
+        x = (x.cuda().float() + outs[0].float()).to(torch.bfloat16).cpu()
 
 
 # ------------------------------------------------------------------ full-size layers (sampled)

@@ -520,3 +520,29 @@ def test_opd_reweighting():
     r = orc.route(np.zeros((1, 1)), layer, orc.Accounts.zeros(2), orc.Params(router="topk",
                                                                              max_k=1))
     assert r.selected == [[0]] and close(r.p[0], [1.8 / 2.6, 0.8 / 2.6])
+
+
+# ---------------------------------------------------------------- temporal smoothing (W5)
+def check_w5(m):
+    w = GOLD["W5"]
+    p = np.array(w["p"])
+    prm = P0.with_(smoothing="temporal")
+    I = m.importance(p, np.zeros(4), prm.beta)
+    for case in w["cases"]:
+        prev = float("nan") if case["tau_prev"] is None else case["tau_prev"]
+        th = m.threshold(p, prm, 0, prev)
+        assert close(th.tau_final, case["tau_final"])
+        assert m.select(I, th.tau_final, prm.max_k) == case["selected"]
+
+
+def test_w5_temporal_smoothing():
+    check_w5(orc)
+
+
+def test_temporal_equals_call_when_prev_is_tau():
+    rng = np.random.default_rng(44)
+    for _ in range(20):
+        p = orc.softmax(rng.normal(size=(1, 8)))[0]
+        a = orc.threshold(p, P0, 1)
+        b = orc.threshold(p, P0.with_(smoothing="temporal"), 1, a.tau)
+        assert close(a.tau_final, b.tau_final)
