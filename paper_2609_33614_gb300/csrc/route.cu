@@ -157,6 +157,132 @@ router_logits_small_kernel(const TX* __restrict__ x, const float* __restrict__ w
   }
 }
 
+// Router scores for large T, vectorised variant (d a multiple of 32, 16-byte aligned x and W_r):
+// CTA tile of 128 tokens x 64 experts, 256 threads with 8 tokens x 4 experts each.  Each 32-column
+// chunk of x and W_r is loaded with 16-byte loads into registers one chunk ahead of the compute
+// (the global latency overlaps the FMAs of the current chunk) and stored transposed into shared
+// memory (lanes of a warp take consecutive rows, so the transposed stores hit distinct banks).
+// Chunk sums are added with Kahan compensation, as in router_logits_kernel.
+constexpr int kVT = 128, kVE = 64;
+
+__device__ __forceinline__ void load8(const __nv_bfloat16* p, float (&v)[8]) {
+  const uint4 u = *(const uint4*)p;
+  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const float2 f = __bfloat1622float2(*(const __nv_bfloat162*)&w[q]);
+    v[2 * q] = f.x;
+    v[2 * q + 1] = f.y;
+  }
+}
+__device__ __forceinline__ void load8(const float* p, float (&v)[8]) {
+  const float4 a = *(const float4*)p, b = *(const float4*)(p + 4);
+  v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+  v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+}
+
+template <typename TX>
+__global__ void __launch_bounds__(kLogitThreads, 1)
+router_logits_vec_kernel(const TX* __restrict__ x, const float* __restrict__ wr, int T, int d,
+                         int E, int d_per_split, double* __restrict__ part) {
+  __shared__ __align__(16) float xs[kChunkK][kVT + 4];
+  __shared__ __align__(16) float ws[kChunkK][kVE + 4];
+  pdl_wait();
+  pdl_launch_dependents();
+  const int tid = threadIdx.x;
+  const int tx = tid & 15, ty = tid >> 4;
+  const int t0 = blockIdx.x * kVT, e0 = blockIdx.y * kVE;
+  const int dbeg = blockIdx.z * d_per_split;
+  const int dend = min(d, dbeg + d_per_split);
+  // loader mapping: x -- 128 rows x 4 pieces of 8 columns, 2 pieces per thread (row = q % 128);
+  // W_r -- 64 rows x 8 pieces of 4 columns, 2 per thread (row = q % 64)
+  float xv[2][8], wv[2][4];
+  auto load_chunk = [&](int k0) {
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      const int q = tid + r * kLogitThreads;
+      const int row = q % kVT, c8 = (q / kVT) * 8;
+      const int t = t0 + row;
+      if (t < T && k0 + c8 < dend) {
+        load8(x + (size_t)t * d + k0 + c8, xv[r]);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) xv[r][i] = 0.f;
+      }
+      const int erow = q % kVE, c4 = (q / kVE) * 4;
+      const int e = e0 + erow;
+      if (e < E && k0 + c4 < dend) {
+        const float4 v = *(const float4*)(wr + (size_t)e * d + k0 + c4);
+        wv[r][0] = v.x; wv[r][1] = v.y; wv[r][2] = v.z; wv[r][3] = v.w;
+      } else {
+        wv[r][0] = wv[r][1] = wv[r][2] = wv[r][3] = 0.f;
+      }
+    }
+  };
+  auto store_chunk = [&]() {
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      const int q = tid + r * kLogitThreads;
+      const int row = q % kVT, c8 = (q / kVT) * 8;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) xs[c8 + i][row] = xv[r][i];
+      const int erow = q % kVE, c4 = (q / kVE) * 4;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) ws[c4 + i][erow] = wv[r][i];
+    }
+  };
+  float sum[8][4], comp[8][4];
+#pragma unroll
+  for (int i = 0; i < 8; ++i)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) sum[i][j] = comp[i][j] = 0.f;
+
+  if (dbeg < dend) {
+    load_chunk(dbeg);
+    store_chunk();
+  }
+  __syncthreads();
+  for (int k0 = dbeg; k0 < dend; k0 += kChunkK) {
+    const bool more = k0 + kChunkK < dend;
+    if (more) load_chunk(k0 + kChunkK);
+    float acc[8][4];
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+#pragma unroll
+      for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
+#pragma unroll 4
+    for (int kk = 0; kk < kChunkK; ++kk) {
+      const float4 a0 = *(const float4*)&xs[kk][ty * 8];
+      const float4 a1 = *(const float4*)&xs[kk][ty * 8 + 4];
+      const float4 b = *(const float4*)&ws[kk][tx * 4];
+      const float av[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+      const float bv[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+      for (int i = 0; i < 8; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
+    }
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+#pragma unroll
+      for (int j = 0; j < 4; ++j) kahan_add(sum[i][j], comp[i][j], acc[i][j]);
+    __syncthreads();
+    if (more) store_chunk();
+    __syncthreads();
+  }
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const int t = t0 + ty * 8 + i;
+    if (t >= T) continue;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int e = e0 + tx * 4 + j;
+      if (e < E)
+        part[((size_t)blockIdx.z * T + t) * E + e] = (double)sum[i][j] - (double)comp[i][j];
+    }
+  }
+}
+
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
@@ -457,6 +583,13 @@ route_select_kernel(const double* __restrict__ part, int n_split, const float* _
 
 int router_split(int T, int d, int E) {
   if (T <= kSmallT) return (d + kSmallSlice - 1) / kSmallSlice;
+  if (d % kChunkK == 0) {
+    // vectorised kernel (one 256-thread CTA per SM): about one full wave of long CTAs
+    const long long tiles = (long long)((T + kVT - 1) / kVT) * ((E + kVE - 1) / kVE);
+    int split = 1;
+    while (tiles * split * 2 <= 152 && d / (split * 2) >= 512 && split < 64) split *= 2;
+    return split;
+  }
   // enough CTAs for two waves, each slice at least 256 columns of d
   const long long tiles = (long long)((T + kTileT - 1) / kTileT) * ((E + kTileE - 1) / kTileE);
   int split = 1;
@@ -479,6 +612,14 @@ cudaError_t launch_router_logits(const void* x, int x_bf16, const float* w_route
   }
   int per = (d + n_split - 1) / n_split;
   per = (per + kChunkK - 1) / kChunkK * kChunkK;
+  if (d % kChunkK == 0 && vec_ok) {
+    dim3 grid((T + kVT - 1) / kVT, (E + kVE - 1) / kVE, n_split);
+    if (x_bf16)
+      return launch_pdl(router_logits_vec_kernel<__nv_bfloat16>, grid, dim3(kLogitThreads), 0,
+                        st, (const __nv_bfloat16*)x, w_router, T, d, E, per, part);
+    return launch_pdl(router_logits_vec_kernel<float>, grid, dim3(kLogitThreads), 0, st,
+                      (const float*)x, w_router, T, d, E, per, part);
+  }
   dim3 grid((T + kTileT - 1) / kTileT, (E + kTileE - 1) / kTileE, n_split);
   if (x_bf16)
     return launch_pdl(router_logits_kernel<__nv_bfloat16>, grid, dim3(kLogitThreads), 0, st,
