@@ -168,9 +168,10 @@ eat_status run_forward(eat_handle* h, const void* x, int T, int ppl_sign, void* 
                        int32_t* idx_opt, float* w_opt, int32_t* k_opt, cudaStream_t st) {
   EAT_TRY(run_route(h, x, T, ppl_sign, h->idx, h->w, h->k, h->psel, true, st));
   const int tile_rows = h->backend == 1 ? tc_tile_rows(h->tc, T) : kSimtTileRows;
+  const int tile_rows_down = h->backend == 1 ? tc_tile_rows_down(h->tc, T) : kSimtTileRows;
   EAT_TRY(launch(h, kPermute, st, "permute", [&] {
-    return launch_permute(h->idx, h->k, h->psel, T, h->K, h->E, tile_rows, h->perm, h->chunk_cnt,
-                          st);
+    return launch_permute(h->idx, h->k, h->psel, T, h->K, h->E, tile_rows, tile_rows_down,
+                          h->perm, h->chunk_cnt, st);
   }));
   const int rows = T * h->K;
   int n_split = 1;
@@ -179,8 +180,10 @@ eat_status run_forward(eat_handle* h, const void* x, int T, int ppl_sign, void* 
     c.x = x;
     c.T = T;
     c.tile_rows = tile_rows;
+    c.tile_rows_down = tile_rows_down;
     c.offs = h->perm.offs;
     c.tile_offs = h->perm.tile_offs;
+    c.tile_offs_down = h->perm.tile_offs2;
     c.perm_tok = h->perm.perm_tok;
     c.xperm = h->xperm;
     c.act = h->act;
@@ -375,6 +378,7 @@ eat_status eat_create(const eat_layer_desc* desc, const eat_params* params, eat_
   add(&h->perm.n_e, sizeof(int32_t) * h->E);
   add(&h->perm.offs, sizeof(int32_t) * (h->E + 1));
   add(&h->perm.tile_offs, sizeof(int32_t) * (h->E + 1));
+  add(&h->perm.tile_offs2, sizeof(int32_t) * (h->E + 1));
   add(&h->perm.perm_tok, sizeof(int32_t) * rows);
   add(&h->perm.slot_of, sizeof(int32_t) * rows);
   add(&h->perm.perm_p, sizeof(float) * rows);

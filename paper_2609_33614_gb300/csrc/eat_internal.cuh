@@ -69,6 +69,7 @@ struct PermuteOut {
   int32_t* n_e;        // [E]
   int32_t* offs;       // [E+1] slot offsets per expert
   int32_t* tile_offs;  // [E+1] prefix of ceil(n_e / tile_rows)
+  int32_t* tile_offs2; // [E+1] prefix of ceil(n_e / tile_rows2) (a second tile size), or null
   int32_t* perm_tok;   // [T*K] token of each slot
   int32_t* slot_of;    // [T*K] slot of (t, j), -1 for j >= k_t
   float* perm_p;       // [T*K] p of each slot
@@ -76,7 +77,7 @@ struct PermuteOut {
 };
 int permute_chunks(int T);  // CTAs (1024-token chunks) of the permute; chunk_cnt holds [chunks][E]
 cudaError_t launch_permute(const int32_t* idx, const int32_t* k, const float* psel, int T, int K,
-                           int E, int tile_rows, PermuteOut o, int32_t* chunk_cnt,
+                           int E, int tile_rows, int tile_rows2, PermuteOut o, int32_t* chunk_cnt,
                            cudaStream_t st);
 
 // ---------------------------------------------------------------------------------------------

@@ -33,7 +33,8 @@ namespace {
 constexpr int kBM = 128;                  // weight rows per tile (MMA M)
 constexpr int kBK = 64;                   // 64 bf16 = 128 B: one 128B-swizzle row
 constexpr int kThreadsTc = 192;           // 6 warps
-constexpr int kBNs[4] = {16, 32, 64, 128};
+constexpr int kNumBN = 5;
+constexpr int kBNs[kNumBN] = {16, 32, 64, 128, 256};
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;
 constexpr int kSmemBudget = 220 * 1024;
 
@@ -182,6 +183,7 @@ struct TcArgs {
   int b_shift_per_group;     // B row = slot - g * b_shift_per_group
   int a_rows_per_group;      // A row = g * a_rows_per_group + m0
   int M;                     // output features per group
+  int m_tile;                // output features per unit (128, or 64 for interleaved gate/up)
   int m_tiles;
   int kblocks;
   int n_split;
@@ -223,7 +225,7 @@ __device__ __forceinline__ Unit decode_unit(const TcArgs& a, int u) {
   w.g = g;
   w.slot0 = beg + j * BN;
   w.nrows = min(BN, end - w.slot0);
-  w.m0 = mi * kBM;
+  w.m0 = mi * a.m_tile;
   w.kb0 = w.split * a.kb_per_split;
   w.kb1 = min(a.kblocks, w.kb0 + a.kb_per_split);
   return w;
@@ -315,7 +317,6 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
   } else if (warp == 1) {
     if (lane == 0) {
       // ------------------------------------------------------------ MMA issuer
-      constexpr uint32_t idesc = idesc_bf16(BN);
       int stage = 0;
       uint32_t phase = 0;
       int local = 0;
@@ -331,6 +332,8 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
         tc_fence_after();
         const uint32_t d0 = tmem_base + (uint32_t)(buf * C::kAccCols);
         const uint32_t d1 = d0 + BN;
+        // MMA width: the tile's rows rounded up to 16 (a partial tile computes no padding)
+        const uint32_t idesc = idesc_bf16(min(BN, (w.nrows + 15) & ~15));
         for (int kb = w.kb0; kb < w.kb1; ++kb) {
           if (!mbar_wait(&full[stage], phase, abort_flag, args.err, 8u, true)) {
             ok = false;
@@ -452,13 +455,13 @@ bool encode_2d(CUtensorMap* m, const void* ptr, long long rows, long long cols, 
 
 struct Maps {
   CUtensorMap wg, wu, wd, wsg, wsu, wsd;
-  CUtensorMap xperm[4], act[4], sact[4];
+  CUtensorMap xperm[kNumBN], act[kNumBN], sact[kNumBN];
 };
 
 int bn_index(int bn) {
-  for (int i = 0; i < 4; ++i)
+  for (int i = 0; i < kNumBN; ++i)
     if (kBNs[i] == bn) return i;
-  return 3;
+  return kNumBN - 1;
 }
 
 template <int BN, bool GATEUP>
@@ -484,17 +487,26 @@ cudaError_t launch_bn(int bn, const CUtensorMap& a0, const CUtensorMap& a1, cons
     case 16: return launch_tc<16, GATEUP>(a0, a1, b, args, grid, st);
     case 32: return launch_tc<32, GATEUP>(a0, a1, b, args, grid, st);
     case 64: return launch_tc<64, GATEUP>(a0, a1, b, args, grid, st);
-    default: return launch_tc<128, GATEUP>(a0, a1, b, args, grid, st);
+    case 128: return launch_tc<128, GATEUP>(a0, a1, b, args, grid, st);
+    default: return launch_tc<256, GATEUP>(a0, a1, b, args, grid, st);
   }
 }
 
 }  // namespace
 
+// The largest group of a call has at most T rows (each token picks an expert once).  In large
+// calls the down projection takes 256-token tiles (M = 128 x N = 256 MMAs read 25% fewer shared-
+// memory operand bytes per flop than N = 128; measured 1.3-1.5x faster); the gate/up kernel keeps
+// 128 (its two accumulators of 256 columns would leave no second TMEM buffer).
 int tc_tile_rows(const TcLayer&, int T) {
-  // the largest group of a call has at most T rows (each token picks an expert once)
   for (int i = 0; i < 4; ++i)
     if (T <= kBNs[i]) return kBNs[i];
   return 128;
+}
+int tc_tile_rows_down(const TcLayer&, int T) {
+  for (int i = 0; i < 4; ++i)
+    if (T <= kBNs[i]) return kBNs[i];
+  return T >= 2048 ? 256 : 128;
 }
 
 // Split-K of the routed down projection: enough work units for ~8 waves of the persistent grid
@@ -504,7 +516,7 @@ int tc_tile_rows(const TcLayer&, int T) {
 static int split_for(const TcLayer& L, int T) {
   const int m_tiles = (L.d + kBM - 1) / kBM;
   const int kblocks = L.F / kBK;
-  const int bn = tc_tile_rows(L, T);
+  const int bn = tc_tile_rows_down(L, T);
   const long long rows = (long long)T * L.K;
   const long long est = ((rows + bn - 1) / bn + std::min<long long>(L.E, rows)) * m_tiles;
   int split = 1;
@@ -569,7 +581,7 @@ int tc_bind(TcLayer& L, const eat_layer_desc& D, void* xperm, void* act, void* s
     ok = encode_2d(&m->wsg, D.ws_gate, (long long)L.S * L.Fs, L.d, kBM) &&
          encode_2d(&m->wsu, D.ws_up, (long long)L.S * L.Fs, L.d, kBM) &&
          encode_2d(&m->wsd, D.ws_down, (long long)L.S * L.d, L.Fs, kBM);
-  for (int i = 0; i < 4 && ok; ++i) {
+  for (int i = 0; i < kNumBN && ok; ++i) {
     ok = encode_2d(&m->xperm[i], xperm, rows, L.d, kBNs[i]) &&
          encode_2d(&m->act[i], act, rows, L.F, kBNs[i]);
     if (ok && L.S > 0) ok = encode_2d(&m->sact[i], sact, (long long)L.S * L.Tmax, L.Fs, kBNs[i]);
@@ -603,7 +615,8 @@ cudaError_t tc_launch_up(const TcLayer& L, const TcCall& c, bool shared, cudaStr
   std::memset(&a, 0, sizeof(a));
   const int bn = c.tile_rows;
   a.M = shared ? L.Fs : L.F;
-  a.m_tiles = (a.M + kBM - 1) / kBM;
+  a.m_tile = kBM;
+  a.m_tiles = (a.M + a.m_tile - 1) / a.m_tile;
   a.kblocks = L.d / kBK;
   a.n_split = 1;
   a.kb_per_split = a.kblocks;
@@ -637,9 +650,10 @@ cudaError_t tc_launch_down(const TcLayer& L, const TcCall& c, bool shared, int n
   const Maps* m = (const Maps*)L.maps;
   TcArgs a;
   std::memset(&a, 0, sizeof(a));
-  const int bn = c.tile_rows;
+  const int bn = c.tile_rows_down;
   const int Kdim = shared ? L.Fs : L.F;
   a.M = L.d;
+  a.m_tile = kBM;
   a.m_tiles = (L.d + kBM - 1) / kBM;
   a.kblocks = Kdim / kBK;
   a.n_split = n_split;
@@ -660,7 +674,7 @@ cudaError_t tc_launch_down(const TcLayer& L, const TcCall& c, bool shared, int n
   }
   a.n_groups = L.E;
   a.row_offs = c.offs;
-  a.tile_offs = c.tile_offs;
+  a.tile_offs = c.tile_offs_down;
   a.out = c.opart;
   a.out_bf16 = n_split == 1 ? 1 : 0;
   a.split_stride = (long long)c.T * L.K * L.d;

@@ -16,9 +16,11 @@ struct TcLayer {
 struct TcCall {
   const void* x = nullptr;         // [T, d] bf16 hidden states of the call
   int T = 0;
-  int tile_rows = 0;               // BN: token rows per tile
+  int tile_rows = 0;               // BN of the gate/up kernel (token rows per tile)
+  int tile_rows_down = 0;          // BN of the down kernel
   const int32_t* offs = nullptr;   // [E+1] slot offsets
-  const int32_t* tile_offs = nullptr;
+  const int32_t* tile_offs = nullptr;       // tile prefix for tile_rows
+  const int32_t* tile_offs_down = nullptr;  // tile prefix for tile_rows_down
   const int32_t* perm_tok = nullptr;
   void* xperm = nullptr;           // [Tmax*K, d] gathered rows in slot order
   void* act = nullptr;             // [Tmax*K, F] bf16
@@ -34,7 +36,8 @@ int tc_configure(TcLayer& L, const eat_layer_desc& D, int K, int Tmax, const cha
 int tc_bind(TcLayer& L, const eat_layer_desc& D, void* xperm, void* act, void* sact,
             const char** msg);
 void tc_destroy(TcLayer& L);
-int tc_tile_rows(const TcLayer& L, int T);   // token rows per tile for a call of T tokens
+int tc_tile_rows(const TcLayer& L, int T);       // gate/up token rows per tile, call of T tokens
+int tc_tile_rows_down(const TcLayer& L, int T);  // down-projection token rows per tile
 int tc_down_split(const TcLayer& L, int T);  // split-K slices of the routed down projection
 long long tc_opart_rows(const TcLayer& L);   // rows of fp32 partials the workspace must hold
 cudaError_t tc_launch_gather(const TcLayer& L, const TcCall& c, cudaStream_t st);

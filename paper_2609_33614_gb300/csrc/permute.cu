@@ -65,7 +65,8 @@ permute_count_kernel(const int32_t* __restrict__ idx, int T, int K, int E,
 __global__ void __launch_bounds__(1024)
 permute_assign_kernel(const int32_t* __restrict__ idx, const int32_t* __restrict__ kk,
                       const float* __restrict__ psel, int T, int K, int E, int tile_rows,
-                      const int32_t* __restrict__ chunk_cnt, int n_chunks, PermuteOut o) {
+                      int tile_rows2, const int32_t* __restrict__ chunk_cnt, int n_chunks,
+                      PermuteOut o) {
   extern __shared__ int sm[];
   pdl_wait();
   pdl_launch_dependents();
@@ -101,21 +102,24 @@ permute_assign_kernel(const int32_t* __restrict__ idx, const int32_t* __restrict
   }
   __syncthreads();
   if (tid == 0) {
-    int s = 0, ts = 0, na = 0;
+    int s = 0, ts = 0, ts2 = 0, na = 0;
     for (int e = 0; e < E; ++e) {
       if (c == 0) {
         o.offs[e] = s;
         o.tile_offs[e] = ts;
+        if (o.tile_offs2) o.tile_offs2[e] = ts2;
         o.n_e[e] = cnt[e];
         if (cnt[e] > 0) o.active[na++] = e;
       }
       cursor[e] += s;
       s += cnt[e];
       ts += (cnt[e] + tile_rows - 1) / tile_rows;
+      ts2 += (cnt[e] + tile_rows2 - 1) / tile_rows2;
     }
     if (c == 0) {
       o.offs[E] = s;
       o.tile_offs[E] = ts;
+      if (o.tile_offs2) o.tile_offs2[E] = ts2;
       for (int e = na; e < E; ++e) o.active[e] = -1;
       o.active[E] = na;
     }
@@ -165,20 +169,21 @@ int permute_chunks(int T) {
 }
 
 cudaError_t launch_permute(const int32_t* idx, const int32_t* k, const float* psel, int T, int K,
-                           int E, int tile_rows, PermuteOut o, int32_t* chunk_cnt,
+                           int E, int tile_rows, int tile_rows2, PermuteOut o, int32_t* chunk_cnt,
                            cudaStream_t st) {
   const int n_chunks = permute_chunks(T);
   if (n_chunks == 1) {
     const size_t smem = (size_t)(2 * E + (kPermThreads / 32) * E) * sizeof(int);
     return launch_pdl(permute_assign_kernel, dim3(1), dim3(kPermThreads), smem, st, idx, k, psel,
-                      T, K, E, tile_rows, (const int32_t*)nullptr, 1, o);
+                      T, K, E, tile_rows, tile_rows2, (const int32_t*)nullptr, 1, o);
   }
   cudaError_t e = launch_pdl(permute_count_kernel, dim3(n_chunks), dim3(kChunkThreads),
                              (size_t)E * sizeof(int), st, idx, T, K, E, chunk_cnt);
   if (e != cudaSuccess) return e;
   const size_t smem = (size_t)(2 * E + (kChunkThreads / 32) * E) * sizeof(int);
   return launch_pdl(permute_assign_kernel, dim3(n_chunks), dim3(kChunkThreads), smem, st, idx, k,
-                    psel, T, K, E, tile_rows, (const int32_t*)chunk_cnt, n_chunks, o);
+                    psel, T, K, E, tile_rows, tile_rows2, (const int32_t*)chunk_cnt, n_chunks,
+                    o);
 }
 
 }  // namespace eat
