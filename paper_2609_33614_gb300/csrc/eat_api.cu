@@ -192,8 +192,9 @@ eat_status run_forward(eat_handle* h, const void* x, int T, int ppl_sign, void* 
     c.sout = h->sout;
     c.status = h->status;
     n_split = tc_down_split(h->tc, T);
-    EAT_TRY(launch(h, kGather, st, "gather rows",
-                   [&] { return tc_launch_gather(h->tc, c, st); }));
+    if (!tc_gathers_in_kernel(h->tc, T))
+      EAT_TRY(launch(h, kGather, st, "gather rows",
+                     [&] { return tc_launch_gather(h->tc, c, st); }));
     EAT_TRY(launch(h, kUp, st, "tc gate/up", [&] { return tc_launch_up(h->tc, c, false, st); }));
     EAT_TRY(launch(h, kDown, st, "tc down",
                    [&] { return tc_launch_down(h->tc, c, false, n_split, st); }));

@@ -95,6 +95,21 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, u
       "l"(map), "r"(smem_u32(bar)), "r"(c0), "r"(c1)
       : "memory");
 }
+// 16-byte global -> shared copy (generic proxy), its group commit / wait, and the proxy fence that
+// orders the copied bytes before the tensor core reads them (async proxy).
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+__device__ __forceinline__ void fence_proxy_async() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
 __device__ __forceinline__ void tc_fence_before() {
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
 }
@@ -191,6 +206,8 @@ struct TcArgs {
   void* out;
   long long split_stride;    // elements between split slices of the fp32 output
   int out_bf16;              // down kernel without split-K: write bf16 rows instead of fp32
+  const int32_t* b_rows;     // gather mode: slot -> token; B rows are copied from bx by the warp
+  const __nv_bfloat16* bx;   // gather mode: token rows [T, row stride kblocks * 64]
   unsigned int* err;
 };
 
@@ -252,7 +269,7 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
-      mbar_init(&full[s], 1);
+      mbar_init(&full[s], args.b_rows ? 2 : 1);  // + the gathered rows' arrival
       mbar_init(&empty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
@@ -281,7 +298,80 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
                               : args.n_groups * ((args.uniform_rows + BN - 1) / BN);
   const int units = total_tiles * args.m_tiles * args.n_split;
 
-  if (warp == 0) {
+  if (warp == 0 && args.b_rows) {
+    // ------------------------------------------------------------ producer, gathered tokens:
+    // lane 0 issues the weight TMA; all lanes copy the tile's token rows from x with 16-byte
+    // cp.async into the 128B-swizzled B tile (lane l: column chunk l % 8 of rows l / 8 + 4 i).
+    // A stage's rows are released LAG stages later: wait for the lane's own copies, fence the
+    // async proxy, and one arrive per warp on the stage's full barrier.
+    constexpr int PER = BN / 4;
+    constexpr int LAG = S > 2 ? S - 2 : 1;
+    const unsigned fullmask = 0xffffffffu;
+    const int cc = lane & 7, r0 = lane >> 3;
+    const size_t ld = (size_t)args.kblocks * kBK;
+    int stage = 0;
+    uint32_t phase = 0;
+    long long it = 0, released = 0;
+    bool ok = true;
+    for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
+      const Unit w = decode_unit<BN>(args, u);
+      const int a_row = w.g * args.a_rows_per_group + w.m0;
+      int tok[PER];
+#pragma unroll
+      for (int i = 0; i < PER; ++i) {
+        const int r = r0 + 4 * i;
+        tok[i] = r < w.nrows ? args.b_rows[w.slot0 + r] : -1;
+      }
+      for (int kb = w.kb0; kb < w.kb1; ++kb) {
+        bool okw = true;
+        if (lane == 0) okw = mbar_wait(&empty[stage], phase ^ 1u, abort_flag, args.err, 1u, true);
+        okw = __shfl_sync(fullmask, okw ? 1 : 0, 0) != 0;
+        if (!okw) {
+          ok = false;
+          break;
+        }
+        uint8_t* st = smem + stage * C::kStageBytes;
+        if (lane == 0) {
+          mbar_expect_tx(&full[stage], C::kNA * C::kABytes);
+          tma_load_2d(st, &mapA0, &full[stage], kb * kBK, a_row);
+          if (GATEUP) tma_load_2d(st + C::kABytes, &mapA1, &full[stage], kb * kBK, a_row);
+        }
+        const uint32_t sb = smem_u32(st + C::kNA * C::kABytes);
+#pragma unroll
+        for (int i = 0; i < PER; ++i) {
+          if (tok[i] >= 0) {
+            const int r = r0 + 4 * i;
+            cp_async16(sb + r * 128 + ((cc ^ (r & 7)) << 4),
+                       args.bx + (size_t)tok[i] * ld + kb * kBK + cc * 8);
+          }
+        }
+        cp_async_commit();
+        ++it;
+        if (it - released > LAG) {
+          cp_async_wait<LAG>();
+          fence_proxy_async();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&full[released % S]);
+          ++released;
+        }
+        if (++stage == S) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+    }
+    // release the stages still held (also on abort, so their barriers can complete), then let the
+    // weight copies in flight land before the CTA may exit
+    cp_async_wait<0>();
+    fence_proxy_async();
+    __syncwarp();
+    if (lane == 0) {
+      for (; released < it; ++released) mbar_arrive(&full[released % S]);
+      const long long first = it > S ? it - S : 0;
+      for (long long i = first; i < it; ++i)
+        mbar_wait(&full[i % S], (uint32_t)((i / S) & 1), abort_flag, args.err, 2u, false);
+    }
+  } else if (warp == 0) {
     if (lane == 0) {
       // ------------------------------------------------------------ TMA producer
       int stage = 0;
@@ -503,6 +593,11 @@ int tc_tile_rows(const TcLayer&, int T) {
     if (T <= kBNs[i]) return kBNs[i];
   return 128;
 }
+// Small calls gather their token rows inside the gate/up kernel (one launch and one HBM round
+// trip fewer); large calls copy them to Xperm first: there the shared-memory-bound gate/up kernel
+// loses more to the warp's cp.async traffic than the separate gather costs.
+bool tc_gathers_in_kernel(const TcLayer&, int T) { return T <= 128; }
+
 int tc_tile_rows_down(const TcLayer&, int T) {
   for (int i = 0; i < 4; ++i)
     if (T <= kBNs[i]) return kBNs[i];
@@ -642,6 +737,12 @@ cudaError_t tc_launch_up(const TcLayer& L, const TcCall& c, bool shared, cudaStr
   max_tiles = (long long)(c.T * L.K + bn - 1) / bn + L.E;
   const long long units = max_tiles * a.m_tiles;
   const int grid = (int)std::min<long long>(L.num_sms, units);
+  if (tc_gathers_in_kernel(L, c.T)) {
+    // small call: the token rows are gathered from x inside the kernel
+    a.b_rows = c.perm_tok;
+    a.bx = (const __nv_bfloat16*)c.x;
+    return launch_bn<true>(bn, m->wg, m->wu, m->wg, a, grid, st);
+  }
   return launch_bn<true>(bn, m->wg, m->wu, m->xperm[bn_index(bn)], a, grid, st);
 }
 

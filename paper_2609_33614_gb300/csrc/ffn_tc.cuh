@@ -38,6 +38,7 @@ int tc_bind(TcLayer& L, const eat_layer_desc& D, void* xperm, void* act, void* s
 void tc_destroy(TcLayer& L);
 int tc_tile_rows(const TcLayer& L, int T);       // gate/up token rows per tile, call of T tokens
 int tc_tile_rows_down(const TcLayer& L, int T);  // down-projection token rows per tile
+bool tc_gathers_in_kernel(const TcLayer& L, int T);  // gate/up gathers x rows itself (no Xperm)
 int tc_down_split(const TcLayer& L, int T);  // split-K slices of the routed down projection
 long long tc_opart_rows(const TcLayer& L);   // rows of fp32 partials the workspace must hold
 cudaError_t tc_launch_gather(const TcLayer& L, const TcCall& c, cudaStream_t st);
