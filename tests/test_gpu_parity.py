@@ -310,6 +310,36 @@ def test_layer_policy_stack():
         x = (x.cuda().float() + outs[0].float()).to(torch.bfloat16).cpu()
 
 
+# ------------------------------------------------------------------ CUDA graph capture
+def test_forward_replays_as_cuda_graph():
+    """A layer call has no host synchronisation and decides its expert schedule on the device, so
+    it can be captured once and replayed: the replays must match direct calls bit for bit, accounts
+    included (two handles on the same weights, same inputs)."""
+    lw = W.make_layer(MIX_S)
+    a = eat.EatLayer.from_workload(lw, 64, gpu_params(MIX_S))
+    b = eat.EatLayer.from_workload(lw, 64, gpu_params(MIX_S))
+    x = W.make_tokens(MIX_S, 64).cuda()
+    y_graph = torch.empty_like(x)
+    stream = torch.cuda.Stream()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(stream):
+        eat.eat_moe_forward(a.h, x, 64, 0, y_graph, stream=stream.cuda_stream)  # warm-up call
+        torch.cuda.current_stream().synchronize()
+        with torch.cuda.graph(g, stream=stream):
+            eat.eat_moe_forward(a.h, x, 64, 0, y_graph, stream=stream.cuda_stream)
+    torch.cuda.synchronize()
+    ys = [b.forward(x, 0)]  # matches the warm-up call of a
+    for _ in range(4):
+        g.replay()
+        torch.cuda.synchronize()
+        y_direct = b.forward(x, 0)
+        assert torch.equal(y_graph, y_direct)
+    for u, v in zip(a.accounts(), b.accounts()):
+        assert torch.equal(u, v)
+    a.close()
+    b.close()
+
+
 # ------------------------------------------------------------------ full-size layers (sampled)
 def _big(shape, layer_id=0):
     return W.make_layer(shape, layer_id, device="cuda")
