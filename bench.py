@@ -54,6 +54,19 @@ def workload_spec(name):
     return specs[name]
 
 
+def bench_config(args, spec):
+    """The `config` object of the JSON line (identical for both arms)."""
+    shape = spec["shape"]
+    cfg = {"workload": spec["desc"], "router": args.router, "cuda_graph": args.graph}
+    if args.router == "topp":
+        cfg["top_p"] = args.top_p
+    cfg.update({"d_model": shape.d_model, "n_experts": shape.n_experts, "d_ff": shape.d_ff,
+                "n_shared": shape.n_shared, "max_k": shape.max_k, "layers": spec["layers"],
+                "batches": spec["batches"],
+                "l2": "inputs larger than L2 (expert weights > 129 MB), no flush"})
+    return cfg
+
+
 def load_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -81,7 +94,7 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.Q}",
-                 "--format=csv,noheader,nounits", "-lms", "100"],
+                 "--format=csv,noheader,nounits", "-lms", "50"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.t = threading.Thread(target=self._read, daemon=True)
             self.t.start()
@@ -404,12 +417,7 @@ def run_ours(args, world, rank, local):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": job_ms / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded N(0,1) hidden states, N(0,0.02^2) weights)",
-        "config": {"workload": spec["desc"], "router": args.router, "cuda_graph": args.graph,
-                   **({"top_p": args.top_p} if args.router == "topp" else {}),
-                   "d_model": shape.d_model,
-                   "n_experts": shape.n_experts, "d_ff": shape.d_ff, "n_shared": shape.n_shared,
-                   "max_k": shape.max_k, "layers": n_layers, "batches": batches,
-                   "l2": "inputs larger than L2 (expert weights > 129 MB), no flush"},
+        "config": bench_config(args, spec),
         "roofline": roof,
         "experts_per_token": acts / max(1, sum(B * args.steps for B in batches) * n_layers),
         "union_per_call": unions,
@@ -486,7 +494,8 @@ def run_reference(args, world, rank):
     import oracle.eat_oracle as orc
     L = _oracle_layer(lw)
     del lw
-    prm = orc.Params(max_k=shape.max_k, temperature=shape.temperature)
+    prm = orc.Params(max_k=shape.max_k, temperature=shape.temperature, router=args.router,
+                     top_p=args.top_p)
     acc = orc.Accounts.zeros(shape.n_experts)
     toks, el = 0, 0.0
     for s in range(args.warmup + args.steps):
@@ -505,7 +514,7 @@ def run_reference(args, world, rank):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": el * 1e3 / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic", "impl": "reference",
-            "config": {"workload": spec["desc"], "sample": f"batch {bs} per step"},
+            "config": bench_config(args, spec),
             "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores,
                              "kind": "oracle",
                              "sample": f"{args.steps} timed oracle layer calls at batch {bs}"},
@@ -516,8 +525,8 @@ def run_reference(args, world, rank):
 def main(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=64)
-    ap.add_argument("--warmup", type=int, default=8)
+    ap.add_argument("--steps", type=int, default=256)
+    ap.add_argument("--warmup", type=int, default=16)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="mixtral-decode")
     ap.add_argument("--no-cpu-baseline", action="store_true")

@@ -218,6 +218,12 @@ eat_status eat_profile_end(eat_handle* h, double* ms, int64_t* launches, int32_t
  * tensor-core kernels (bf16 layers).  -1 on a NULL handle. */
 int32_t eat_ffn_backend(const eat_handle* h);
 
+/* Diagnostic of the failure path: runs one kernel thread that waits, with the bounded wait the
+ * tensor-core kernels use, on a barrier nothing arrives on.  After limit_ns (1 us .. 1 s) the wait
+ * gives up, sets bit 64 in a device status word and the kernel returns; *status_out receives the
+ * word (64 when the bound works) and the context stays usable.  Synchronous; allocates 4 bytes. */
+eat_status eat_selftest_bounded_wait(int64_t limit_ns, uint32_t* status_out);
+
 /* Last error on the handle (never NULL), or a generic text for a NULL handle. */
 const char* eat_last_error(const eat_handle* h);
 const char* eat_status_string(eat_status s);

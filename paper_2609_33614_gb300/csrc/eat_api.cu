@@ -588,6 +588,23 @@ eat_status eat_profile_end(eat_handle* h, double* ms, int64_t* launches, int32_t
 
 int32_t eat_ffn_backend(const eat_handle* h) { return h ? h->backend : -1; }
 
+eat_status eat_selftest_bounded_wait(int64_t limit_ns, uint32_t* status_out) {
+  if (!status_out || limit_ns < 1000 || limit_ns > 1000000000LL)
+    return fail(nullptr, EAT_ERR_INVALID_ARG, "need status_out and 1 us <= limit_ns <= 1 s");
+  unsigned int* dev = nullptr;
+  cudaError_t e = cudaMalloc(&dev, sizeof(unsigned int));
+  if (e == cudaSuccess) e = cudaMemset(dev, 0, sizeof(unsigned int));
+  if (e == cudaSuccess) e = tc_selftest_bounded_wait((unsigned long long)limit_ns, dev, nullptr);
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  unsigned int v = 0;
+  if (e == cudaSuccess) e = cudaMemcpy(&v, dev, sizeof(v), cudaMemcpyDeviceToHost);
+  if (dev) cudaFree(dev);
+  if (e != cudaSuccess) return fail(nullptr, EAT_ERR_CUDA, std::string("self-test: ") +
+                                                              cudaGetErrorString(e));
+  *status_out = v;
+  return EAT_OK;
+}
+
 const char* eat_last_error(const eat_handle* h) {
   if (!h) return g_err.empty() ? "no error recorded" : g_err.c_str();
   return h->err.empty() ? "no error recorded" : h->err.c_str();

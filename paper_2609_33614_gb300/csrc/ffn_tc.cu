@@ -73,13 +73,14 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 // role raised the CTA's abort flag (check_abort), or after kWaitLimitNs (then it raises the flag and
 // records `code` in the device status word).
 __device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
-                                       unsigned int* err, unsigned int code, bool check_abort) {
+                                       unsigned int* err, unsigned int code, bool check_abort,
+                                       unsigned long long limit_ns = kWaitLimitNs) {
   if (mbar_try_wait(bar, parity)) return true;
   const unsigned long long t0 = globaltimer();
   for (;;) {
     if (mbar_try_wait(bar, parity)) return true;
     if (check_abort && *abort_flag) return false;
-    if (globaltimer() - t0 > kWaitLimitNs) {
+    if (globaltimer() - t0 > limit_ns) {
       *abort_flag = 1;
       atomicOr(err, code);
       return false;
@@ -515,6 +516,18 @@ __global__ void gather_rows_kernel(const uint4* __restrict__ x, const int32_t* _
   for (int i = threadIdx.x; i < row_vecs; i += blockDim.x) xperm[dst + i] = x[src + i];
 }
 
+// Self-test of the bounded wait: one thread waits on an mbarrier that nothing arrives on; after
+// limit_ns the wait gives up, records bit 64 in the status word and the kernel returns normally.
+__global__ void bounded_wait_selftest_kernel(unsigned long long limit_ns, unsigned int* err) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x != 0) return;
+  abort_flag = 0;
+  mbar_init(&bar, 1);
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  mbar_wait(&bar, 0u, &abort_flag, err, 64u, false, limit_ns);
+}
+
 // -------------------------------------------------------------------------------- host side
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
@@ -783,6 +796,12 @@ cudaError_t tc_launch_down(const TcLayer& L, const TcCall& c, bool shared, int n
   const long long units = max_tiles * a.m_tiles * n_split;
   const int grid = (int)std::min<long long>(L.num_sms, units);
   return launch_bn<false>(bn, m->wd, m->wd, m->act[bn_index(bn)], a, grid, st);
+}
+
+cudaError_t tc_selftest_bounded_wait(unsigned long long limit_ns, unsigned int* dev_status,
+                                     cudaStream_t st) {
+  bounded_wait_selftest_kernel<<<1, 32, 0, st>>>(limit_ns, dev_status);
+  return cudaGetLastError();
 }
 
 }  // namespace eat

@@ -43,6 +43,10 @@ int tc_down_split(const TcLayer& L, int T);  // split-K slices of the routed dow
 long long tc_opart_rows(const TcLayer& L);   // rows of fp32 partials the workspace must hold
 cudaError_t tc_launch_gather(const TcLayer& L, const TcCall& c, cudaStream_t st);
 cudaError_t tc_launch_up(const TcLayer& L, const TcCall& c, bool shared, cudaStream_t st);
+// Launches one thread waiting on an mbarrier nobody arrives on, bounded by limit_ns (the wait the
+// tensor-core kernels use); the expiry sets bit 64 in *dev_status.
+cudaError_t tc_selftest_bounded_wait(unsigned long long limit_ns, unsigned int* dev_status,
+                                     cudaStream_t st);
 cudaError_t tc_launch_down(const TcLayer& L, const TcCall& c, bool shared, int n_split,
                            cudaStream_t st);
 

@@ -67,6 +67,7 @@ _SIGS = {
     "eat_profile_begin": (c_i32, [c_vp, c_i32]),
     "eat_profile_end": (c_i32, [c_vp, ctypes.POINTER(c_dbl), ctypes.POINTER(c_i64), c_i32]),
     "eat_ffn_backend": (c_i32, [c_vp]),
+    "eat_selftest_bounded_wait": (c_i32, [c_i64, ctypes.POINTER(ctypes.c_uint32)]),
     "eat_last_error": (ctypes.c_char_p, [c_vp]),
     "eat_status_string": (ctypes.c_char_p, [c_i32]),
 }
@@ -212,6 +213,12 @@ def eat_profile_end(h) -> dict:
 
 def eat_ffn_backend(h) -> int:
     return lib().eat_ffn_backend(h)
+
+
+def eat_selftest_bounded_wait(limit_ns: int) -> int:
+    out = ctypes.c_uint32(0)
+    _check(lib().eat_selftest_bounded_wait(limit_ns, ctypes.byref(out)))
+    return out.value
 
 
 # ------------------------------------------------------------------------------------------------

@@ -89,6 +89,9 @@ def test_null_handle_calls(lib):
     assert lib.eat_ffn_backend(None) == -1
     assert lib.eat_status_string(eat.EAT_ERR_CUDA) == b"EAT_ERR_CUDA"
     assert lib.eat_status_string(99) == b"EAT_UNKNOWN_STATUS"
+    out = ctypes.c_uint32(7)
+    assert lib.eat_selftest_bounded_wait(10, ctypes.byref(out)) == eat.EAT_ERR_INVALID_ARG
+    assert lib.eat_selftest_bounded_wait(10**6, None) == eat.EAT_ERR_INVALID_ARG
 
 
 def test_binding_raises_with_message(lib):

@@ -310,6 +310,22 @@ def test_layer_policy_stack():
         x = (x.cuda().float() + outs[0].float()).to(torch.bfloat16).cpu()
 
 
+# ------------------------------------------------------------------ failure path
+def test_bounded_wait_expires_and_context_survives():
+    """A kernel wait that nothing satisfies gives up after its bound, reports through the status
+    word, and the context keeps working (no trap, no hang)."""
+    import time
+    t0 = time.time()
+    assert eat.eat_selftest_bounded_wait(20_000_000) == 64       # 20 ms bound
+    assert time.time() - t0 < 10.0
+    lw = W.make_layer(MIX_S)
+    run_parity(MIX_S, lw, [16])
+    layer = eat.EatLayer.from_workload(lw, 16, gpu_params(MIX_S))
+    layer.forward(W.make_tokens(MIX_S, 16).cuda(), 0)
+    assert eat.eat_get_counters(layer.h)["status"] == 0
+    layer.close()
+
+
 # ------------------------------------------------------------------ CUDA graph capture
 def test_forward_replays_as_cuda_graph():
     """A layer call has no host synchronisation and decides its expert schedule on the device, so
