@@ -176,6 +176,22 @@ def test_k_equals_e():
     run_parity(sh, lw, [50, 50, 50])
 
 
+@pytest.mark.parametrize("E,K,T", [(256, 8, 300), (100, 16, 130), (33, 5, 77)])
+def test_expert_counts_and_max_k(E, K, T):
+    """Up to 256 experts (8 per lane of the selection warp), a ragged lane layout, K = 16."""
+    sh = W.scaled(W.OLMOE, f"e{E}", d_model=256, n_experts=E, d_ff=128, max_k=K)
+    lw = W.make_layer(sh)
+    run_parity(sh, lw, [T, 1, T // 3])
+
+
+def test_partial_feature_tiles():
+    """d = 320 and d_ff = 192: feature tiles of 128 end half-full in both expert GEMMs."""
+    sh = W.scaled(W.QWEN, "ragged-d", d_model=320, n_experts=16, d_ff=192, n_shared=1,
+                  d_ff_shared=320, max_k=3)
+    lw = W.make_layer(sh)
+    run_parity(sh, lw, [97, 3000, 5])
+
+
 def test_degenerate_fixed_topk_on_gpu():
     """beta = 0, alpha1 = 0, alpha2 huge, no clamp: vanilla Top-K by p (index tie-break)."""
     kw = {"beta": 0.0, "alpha1": 0.0, "alpha2": 1e30, "clamp_enabled": 0}
