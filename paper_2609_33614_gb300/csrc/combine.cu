@@ -1,23 +1,26 @@
 // Weighted combine / unpermute (§3.4: the layer output is the g_norm-weighted sum of the activated
 // experts' outputs) and the expert-account update (§3.2).
 //
-//  combine_kernel: one block per (token, 2048-column block).  For each of the token's k_t slots
-//      it sums the expert output partials (split-K slices, fixed order), accumulates g_norm * o into
-//      y in the order j = 0..k_t-1, adds the always-on shared experts with weight 1, and writes the
-//      partial sum of squares of every slot (||o||_2 of the unweighted expert output feeds C_s).
-//  account_kernel: one block per expert.  Finishes ||o||_2 of each slot from the column-block
-//      partials, sums p and ||o||_2 over the expert's slots (tokens ascending, a fixed tree) in
-//      fp64 and applies N += n_e, P_total += sum p,
-//      C_s <- (1 - alpha) C_s + alpha * mean ||o||_2 when n_e > 0.
+//  combine_kernel: one warp per (token, 256-column segment), 8 columns per lane, no shared memory
+//      and no block barrier, so each warp's loads go out as soon as it starts.  For each of the
+//      token's k_t slots it sums the expert output partials (split-K slices, fixed order),
+//      accumulates g_norm * o into y in the order j = 0..k_t-1, adds the always-on shared experts
+//      with weight 1, and writes the segment's sum of squares of every slot (||o||_2 of the
+//      unweighted expert output feeds C_s) to nrm_part[slot][segment].
+//  account_kernel: one block per expert.  Finishes ||o||_2 of each slot from its segment sums
+//      (fp32, fixed order), sums p and ||o||_2 over the expert's slots in fp64 (a fixed tree) and
+//      applies N += n_e, P_total += sum p, C_s <- (1 - alpha) C_s + alpha * mean ||o||_2 when
+//      n_e > 0.  Only additions run in fp64: GB300's fp64 pipe is narrow, and an fp64 square
+//      root per slot made the block of a heavily used expert the longest of the step.
 #include "eat_internal.cuh"
 
 namespace eat {
 
 namespace {
 
-constexpr int kCombThreads = 256;
-constexpr int kAccThreads = 512;
-
+constexpr int kCombThreads = 256;  // 8 warps: 8 (token, segment) tasks per block
+constexpr int kSegCols = 256;      // columns per warp task, 8 per lane
+constexpr int kAccThreads = 256;
 
 // 8 consecutive values as fp32, from fp32 (two 16-byte loads) or bf16 (one 16-byte load).
 struct V8 {
@@ -57,64 +60,110 @@ __device__ __forceinline__ void store8(__nv_bfloat16* y, const float (&a)[8]) {
   *(uint4*)y = u;
 }
 
-// Column block of one token: 8 consecutive columns per thread (16-byte loads), so a token's row
-// spans ceil(d / 2048) blocks; every block writes the partial sum of squares of each of the
-// token's slots over its columns (nrm_part[slot][block]), which the account kernel sums.  Expert
-// outputs are fp32 split-K partials (o_bf16 = 0) or, without split-K, bf16 rows; the shared
-// experts' outputs likewise (s_bf16).  All of a token's slot rows are loaded before any use.
-template <typename TY, int KM>
+// Sum over the warp of v[0..N) (N a power of two <= 32), fixed order.  Each step exchanges half
+// of the remaining values with the partner lane, so N sums take N - 1 + 5 - log2 N shuffles
+// instead of 5 N.  On return every lane holds the total of value j = lane / (32 / N).
+template <int N>
+__device__ __forceinline__ float warp_sum_many(float (&v)[N], int lane) {
+  const unsigned full = 0xffffffffu;
+#pragma unroll
+  for (int n = N, m = 16; n > 1; n >>= 1, m >>= 1) {
+    const bool upper = (lane & m) != 0;
+#pragma unroll
+    for (int i = 0; i < n / 2; ++i) {
+      const float send = upper ? v[i] : v[i + n / 2];
+      const float keep = upper ? v[i + n / 2] : v[i];
+      v[i] = keep + __shfl_xor_sync(full, send, m);
+    }
+  }
+  float r = v[0];
+#pragma unroll
+  for (int m = 16 / N; m > 0; m >>= 1) r += __shfl_xor_sync(full, r, m);
+  return r;
+}
+
+// Expert outputs are bf16 rows (OB, no split-K) or fp32 split-K partials; the shared experts'
+// outputs bf16 (s_bf16) or fp32.  Slots past k_t are -1 with gate 0.  All of a token's slot rows
+// are loaded before any use.
+template <typename TY, int KM, bool OB>
 __global__ void __launch_bounds__(kCombThreads)
-combine_kernel(const void* __restrict__ opart, int o_bf16, int n_split, size_t split_stride,
+combine_kernel(const void* __restrict__ opart, int n_split, size_t split_stride,
                const int32_t* __restrict__ slot_of, const float* __restrict__ w,
-               const int32_t* __restrict__ kk, const void* __restrict__ sout, int s_bf16, int S,
-               int T, int K, int d, TY* __restrict__ y, float* __restrict__ nrm_part) {
-  __shared__ int slots[KM];
-  __shared__ float gw[KM];
-  __shared__ float red[kCombThreads / 32][KM];
+               const void* __restrict__ sout, int s_bf16, int S, int T, int K, int d, int nseg,
+               TY* __restrict__ y, float* __restrict__ nrm_part) {
   pdl_wait();
   pdl_launch_dependents();
-  const int t = blockIdx.x;
-  const int nb = gridDim.y, cb = blockIdx.y;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int kt = kk[t];
-  if (tid < K) {
-    slots[tid] = tid < kt ? slot_of[(size_t)t * K + tid] : -1;
-    gw[tid] = tid < kt ? w[(size_t)t * K + tid] : 0.f;
+  const unsigned full = 0xffffffffu;
+  const int lane = threadIdx.x & 31;
+  const int task = blockIdx.x * (kCombThreads / 32) + (threadIdx.x >> 5);
+  if (task >= T * nseg) return;
+  const int t = task / nseg, sg = task - t * nseg;
+  int my_slot = -1;
+  float my_w = 0.f;
+  if (lane < K) {
+    my_slot = slot_of[(size_t)t * K + lane];
+    my_w = w[(size_t)t * K + lane];
   }
-  __syncthreads();
-  float nrm[KM];
+  int slots[KM];
+  float g[KM];
 #pragma unroll
-  for (int j = 0; j < KM; ++j) nrm[j] = 0.f;
-  const int c = (cb * kCombThreads + tid) * 8;
-  if (c < d) {
+  for (int j = 0; j < KM; ++j) {
+    slots[j] = __shfl_sync(full, my_slot, j);
+    g[j] = __shfl_sync(full, my_w, j);
+  }
+  const int c = sg * kSegCols + lane * 8;
+  const bool in = c < d;
+  float nrm[KM];
+  float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  if constexpr (OB) {
+    uint4 raw[KM];
+#pragma unroll
+    for (int j = 0; j < KM; ++j)
+      if (in && slots[j] >= 0)
+        raw[j] = *(const uint4*)((const __nv_bfloat16*)opart + (size_t)slots[j] * d + c);
+#pragma unroll
+    for (int j = 0; j < KM; ++j) {
+      nrm[j] = 0.f;
+      if (in && slots[j] >= 0) {
+        const uint32_t wd[4] = {raw[j].x, raw[j].y, raw[j].z, raw[j].w};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const float2 f = __bfloat1622float2(*(const __nv_bfloat162*)&wd[q]);
+          acc[2 * q] = fmaf(g[j], f.x, acc[2 * q]);
+          acc[2 * q + 1] = fmaf(g[j], f.y, acc[2 * q + 1]);
+          nrm[j] = fmaf(f.x, f.x, nrm[j]);
+          nrm[j] = fmaf(f.y, f.y, nrm[j]);
+        }
+      }
+    }
+  } else {
     V8 o[KM];
 #pragma unroll
     for (int j = 0; j < KM; ++j)
-      if (j < kt) o[j] = load8(opart, o_bf16, (size_t)slots[j] * d + c);
+      if (in && slots[j] >= 0) o[j] = load8(opart, false, (size_t)slots[j] * d + c);
     for (int sp = 1; sp < n_split; ++sp) {
 #pragma unroll
       for (int j = 0; j < KM; ++j) {
-        if (j < kt) {
+        if (in && slots[j] >= 0) {
           const V8 q = load8(opart, false, sp * split_stride + (size_t)slots[j] * d + c);
 #pragma unroll
           for (int i = 0; i < 8; ++i) o[j].v[i] += q.v[i];
         }
       }
     }
-    float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
     for (int j = 0; j < KM; ++j) {
-      if (j < kt) {
-        const float g = gw[j];
-        float n = 0.f;
+      nrm[j] = 0.f;
+      if (in && slots[j] >= 0) {
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
-          acc[i] = fmaf(g, o[j].v[i], acc[i]);
-          n = fmaf(o[j].v[i], o[j].v[i], n);
+          acc[i] = fmaf(g[j], o[j].v[i], acc[i]);
+          nrm[j] = fmaf(o[j].v[i], o[j].v[i], nrm[j]);
         }
-        nrm[j] = n;
       }
     }
+  }
+  if (in) {
     for (int s = 0; s < S; ++s) {
       const V8 q = load8(sout, s_bf16, ((size_t)s * T + t) * d + c);
 #pragma unroll
@@ -122,21 +171,10 @@ combine_kernel(const void* __restrict__ opart, int o_bf16, int n_split, size_t s
     }
     store8(y + (size_t)t * d + c, acc);
   }
-#pragma unroll
-  for (int j = 0; j < KM; ++j) {
-    if (j < kt) {
-      float v = nrm[j];
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-      if (lane == 0) red[warp][j] = v;
-    }
-  }
-  __syncthreads();
-  if (tid < kt) {
-    float v = 0.f;
-    for (int wi = 0; wi < kCombThreads / 32; ++wi) v += red[wi][tid];
-    nrm_part[(size_t)slots[tid] * nb + cb] = v;
-  }
+  const float r = warp_sum_many<KM>(nrm, lane);
+  const int jm = lane / (32 / KM);
+  const int sm = __shfl_sync(full, my_slot, jm);
+  if (lane % (32 / KM) == 0 && sm >= 0) nrm_part[(size_t)sm * nseg + sg] = r;
 }
 
 __global__ void __launch_bounds__(kAccThreads)
@@ -151,23 +189,40 @@ account_kernel(const int32_t* __restrict__ offs, const float* __restrict__ perm_
   const int e = blockIdx.x;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int beg = offs[e], end = offs[e + 1];
-  // four independent slot streams per thread keep enough loads in flight for an expert that
-  // holds most of a large call's tokens
-  double sp4[4] = {0.0, 0.0, 0.0, 0.0}, sn4[4] = {0.0, 0.0, 0.0, 0.0};
+  const bool vec = (nb & 3) == 0;
+  double sp = 0.0, sn = 0.0;
+  // four slots per thread per pass, all loads issued before the sums
   for (int i0 = beg + tid; i0 < end; i0 += 4 * kAccThreads) {
+    float pv[4], nv[4];
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
       const int i = i0 + u * kAccThreads;
+      pv[u] = 0.f;
+      nv[u] = 0.f;
       if (i < end) {
-        sp4[u] += (double)perm_p[i];
-        double sq = 0.0;
-        for (int b = 0; b < nb; ++b) sq += (double)nrm_part[(size_t)i * nb + b];
-        sn4[u] += sqrt(sq);
+        pv[u] = perm_p[i];
+        const float* np = nrm_part + (size_t)i * nb;
+        float sq = 0.f;
+        if (vec) {
+          for (int b = 0; b < nb; b += 4) {
+            const float4 q = *(const float4*)(np + b);
+            sq += q.x;
+            sq += q.y;
+            sq += q.z;
+            sq += q.w;
+          }
+        } else {
+          for (int b = 0; b < nb; ++b) sq += np[b];
+        }
+        nv[u] = sq;
       }
     }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      sp += (double)pv[u];
+      sn += (double)sqrtf(nv[u]);
+    }
   }
-  double sp = (sp4[0] + sp4[1]) + (sp4[2] + sp4[3]);
-  double sn = (sn4[0] + sn4[1]) + (sn4[2] + sn4[3]);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     sp += __shfl_xor_sync(0xffffffffu, sp, o);
@@ -191,30 +246,37 @@ account_kernel(const int32_t* __restrict__ offs, const float* __restrict__ perm_
   }
 }
 
-
 }  // namespace
 
-int combine_col_blocks(int d) { return (d + 8 * kCombThreads - 1) / (8 * kCombThreads); }
+int combine_col_blocks(int d) { return (d + kSegCols - 1) / kSegCols; }
 
 namespace {
 
 template <typename TY, int KM>
-cudaError_t launch_combine_t(dim3 grid, cudaStream_t st, const void* opart, int o_bf16,
-                             int n_split, size_t stride, const int32_t* slot_of, const float* w,
-                             const int32_t* k, const void* sout, int s_bf16, int S, int T, int K,
-                             int d, void* y, float* nrm_part) {
-  return launch_pdl(combine_kernel<TY, KM>, grid, dim3(kCombThreads), 0, st, opart, o_bf16,
-                    n_split, stride, slot_of, w, k, sout, s_bf16, S, T, K, d, (TY*)y, nrm_part);
+cudaError_t launch_combine_t(int o_bf16, cudaStream_t st, const void* opart, int n_split,
+                             size_t stride, const int32_t* slot_of, const float* w,
+                             const void* sout, int s_bf16, int S, int T, int K, int d, void* y,
+                             float* nrm_part) {
+  const int nseg = combine_col_blocks(d);
+  const long long tasks = (long long)T * nseg;
+  const dim3 grid((unsigned)((tasks + kCombThreads / 32 - 1) / (kCombThreads / 32)));
+  if (o_bf16)
+    return launch_pdl(combine_kernel<TY, KM, true>, grid, dim3(kCombThreads), 0, st, opart,
+                      n_split, stride, slot_of, w, sout, s_bf16, S, T, K, d, nseg, (TY*)y,
+                      nrm_part);
+  return launch_pdl(combine_kernel<TY, KM, false>, grid, dim3(kCombThreads), 0, st, opart,
+                    n_split, stride, slot_of, w, sout, s_bf16, S, T, K, d, nseg, (TY*)y,
+                    nrm_part);
 }
 
 template <typename TY>
-cudaError_t launch_combine_k(dim3 grid, cudaStream_t st, const void* opart, int o_bf16,
-                             int n_split, size_t stride, const int32_t* slot_of, const float* w,
-                             const int32_t* k, const void* sout, int s_bf16, int S, int T, int K,
-                             int d, void* y, float* nrm_part) {
-#define EAT_COMB(KM)                                                                            \
-  launch_combine_t<TY, KM>(grid, st, opart, o_bf16, n_split, stride, slot_of, w, k, sout, s_bf16, \
-                           S, T, K, d, y, nrm_part)
+cudaError_t launch_combine_k(int o_bf16, cudaStream_t st, const void* opart, int n_split,
+                             size_t stride, const int32_t* slot_of, const float* w,
+                             const void* sout, int s_bf16, int S, int T, int K, int d, void* y,
+                             float* nrm_part) {
+#define EAT_COMB(KM)                                                                           \
+  launch_combine_t<TY, KM>(o_bf16, st, opart, n_split, stride, slot_of, w, sout, s_bf16, S, T, \
+                           K, d, y, nrm_part)
   if (K <= 2) return EAT_COMB(2);
   if (K <= 4) return EAT_COMB(4);
   if (K <= 8) return EAT_COMB(8);
@@ -226,15 +288,14 @@ cudaError_t launch_combine_k(dim3 grid, cudaStream_t st, const void* opart, int 
 
 cudaError_t launch_combine(int y_bf16, const void* opart, int o_bf16, int n_split,
                            int split_stride_rows, const int32_t* slot_of, const float* w,
-                           const int32_t* k, const void* sout, int s_bf16, int S, int T, int K,
-                           int d, void* y, float* nrm_part, cudaStream_t st) {
+                           const void* sout, int s_bf16, int S, int T, int K, int d, void* y,
+                           float* nrm_part, cudaStream_t st) {
   const size_t stride = (size_t)split_stride_rows * d;
-  dim3 grid(T, combine_col_blocks(d));
   if (y_bf16)
-    return launch_combine_k<__nv_bfloat16>(grid, st, opart, o_bf16, n_split, stride, slot_of, w,
-                                           k, sout, s_bf16, S, T, K, d, y, nrm_part);
-  return launch_combine_k<float>(grid, st, opart, o_bf16, n_split, stride, slot_of, w, k, sout,
-                                 s_bf16, S, T, K, d, y, nrm_part);
+    return launch_combine_k<__nv_bfloat16>(o_bf16, st, opart, n_split, stride, slot_of, w, sout,
+                                           s_bf16, S, T, K, d, y, nrm_part);
+  return launch_combine_k<float>(o_bf16, st, opart, n_split, stride, slot_of, w, sout, s_bf16, S,
+                                 T, K, d, y, nrm_part);
 }
 
 cudaError_t launch_account(const int32_t* offs, const float* perm_p, const float* nrm_part, int nb,

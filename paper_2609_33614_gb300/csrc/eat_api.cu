@@ -37,15 +37,15 @@ struct eat_handle {
   PermuteOut perm{};
   void* act = nullptr;    // [Tmax*K, F]
   float* opart = nullptr; // [splits][Tmax*K, d]
-  float* nrm_part = nullptr; // [Tmax*K, column blocks] partial sums of squares of expert rows
-  int nb = 1;                 // column blocks per row in the combine kernel
+  float* nrm_part = nullptr; // [Tmax*K, segments] partial sums of squares of expert rows
+  int nb = 1;                 // column segments per row in the combine kernel
   void* sact = nullptr;   // [S*Tmax, Fs]
   float* sout = nullptr;  // [S*Tmax, d] (fp32; bf16 on the tensor-core path)
   void* xstage = nullptr; // [Tmax, d]
   void* ystage = nullptr; // [Tmax, d]
   void* xperm = nullptr;  // [Tmax*K, d] gathered token rows (tensor-core path)
   unsigned int* status = nullptr;  // device status word: bounded waits that expired
-  int32_t* chunk_cnt = nullptr;    // [permute chunks][E]
+  int32_t* chunk_cnt = nullptr;    // permute scratch: ticket word, then [chunks][E] counts
   long long opart_rows = 0;
   float* tau_state = nullptr;  // caller-owned [Tmax] previous tau_final per stream, or null
 
@@ -230,7 +230,7 @@ eat_status run_forward(eat_handle* h, const void* x, int T, int ppl_sign, void* 
   EAT_TRY(launch(h, kCombine, st, "combine", [&] {
     const int tc = h->backend == 1;
     return launch_combine(h->bf16, h->opart, tc && n_split == 1, n_split, rows, h->perm.slot_of,
-                          h->w, h->k, h->sout, tc, h->S, T, h->K, h->d, y, h->nrm_part, st);
+                          h->w, h->sout, tc, h->S, T, h->K, h->d, y, h->nrm_part, st);
   }));
   EAT_TRY(launch(h, kAccount, st, "account update", [&] {
     return launch_account(h->perm.offs, h->perm.perm_p, h->nrm_part, h->nb, h->E, h->prm.alpha,
@@ -395,7 +395,7 @@ eat_status eat_create(const eat_layer_desc* desc, const eat_params* params, eat_
   if (h->backend == 1) {
     add(&h->xperm, h->elt * rows * h->d);
   }
-  add(&h->chunk_cnt, sizeof(int32_t) * (size_t)permute_chunks(h->Tmax) * h->E);
+  add(&h->chunk_cnt, sizeof(int32_t) * permute_scratch_ints(h->Tmax, h->E));
   add(&h->xstage, h->elt * (size_t)h->Tmax * h->d);
   add(&h->ystage, h->elt * (size_t)h->Tmax * h->d);
   size_t total = 0;

@@ -75,9 +75,12 @@ struct PermuteOut {
   float* perm_p;       // [T*K] p of each slot
   int32_t* active;     // [E+1] ascending active experts, active[E] = count
 };
-int permute_chunks(int T);  // CTAs (1024-token chunks) of the permute; chunk_cnt holds [chunks][E]
+int permute_chunks(int T);  // CTAs of the permute of a T-token call
+// int32 words of the permute's scratch (a ticket counter, zero between calls, and the per-chunk
+// expert counts) for calls of up to Tmax tokens
+size_t permute_scratch_ints(int Tmax, int E);
 cudaError_t launch_permute(const int32_t* idx, const int32_t* k, const float* psel, int T, int K,
-                           int E, int tile_rows, int tile_rows2, PermuteOut o, int32_t* chunk_cnt,
+                           int E, int tile_rows, int tile_rows2, PermuteOut o, int32_t* scratch,
                            cudaStream_t st);
 
 // ---------------------------------------------------------------------------------------------
@@ -110,11 +113,11 @@ constexpr int kSimtTileRows = 32;
 // ---------------------------------------------------------------------------------------------
 // Combine / unpermute and account update
 // ---------------------------------------------------------------------------------------------
-int combine_col_blocks(int d);  // column blocks per token row in the combine kernel
+int combine_col_blocks(int d);  // column segments per token row (norm partials per slot)
 cudaError_t launch_combine(int y_bf16, const void* opart, int o_bf16, int n_split,
                            int split_stride_rows, const int32_t* slot_of, const float* w,
-                           const int32_t* k, const void* sout, int s_bf16, int S, int T, int K,
-                           int d, void* y, float* nrm_part, cudaStream_t st);
+                           const void* sout, int s_bf16, int S, int T, int K, int d, void* y,
+                           float* nrm_part, cudaStream_t st);
 cudaError_t launch_account(const int32_t* offs, const float* perm_p, const float* nrm_part, int nb,
                            int E, double alpha, int64_t* N, double* P, double* C, int32_t* st_n,
                            double* st_p, double* st_norm, long long* counters, cudaStream_t st);

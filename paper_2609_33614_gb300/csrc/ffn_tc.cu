@@ -504,16 +504,30 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
 }
 
 // Xperm[slot] = x[perm_tok[slot]] for every slot of the call (16-byte copies).
-__global__ void gather_rows_kernel(const uint4* __restrict__ x, const int32_t* __restrict__ perm_tok,
-                                   const int32_t* __restrict__ n_rows, int row_vecs,
-                                   uint4* __restrict__ xperm) {
+__global__ void __launch_bounds__(256)
+gather_rows_kernel(const uint4* __restrict__ x, const int32_t* __restrict__ perm_tok,
+                   const int32_t* __restrict__ n_rows, int row_vecs, uint4* __restrict__ xperm) {
   pdl_wait();
   pdl_launch_dependents();
-  const int slot = blockIdx.x;
+  // one warp per row; each lane moves up to 8 16-byte pieces per pass, all loads before the stores
+  const int lane = threadIdx.x & 31;
+  const int slot = blockIdx.x * 8 + (threadIdx.x >> 5);
   if (slot >= *n_rows) return;
   const size_t src = (size_t)perm_tok[slot] * row_vecs;
   const size_t dst = (size_t)slot * row_vecs;
-  for (int i = threadIdx.x; i < row_vecs; i += blockDim.x) xperm[dst + i] = x[src + i];
+  for (int i0 = 0; i0 < row_vecs; i0 += 256) {
+    uint4 v[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int i = i0 + u * 32 + lane;
+      if (i < row_vecs) v[u] = x[src + i];
+    }
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int i = i0 + u * 32 + lane;
+      if (i < row_vecs) xperm[dst + i] = v[u];
+    }
+  }
 }
 
 // Self-test of the bounded wait: one thread waits on an mbarrier that nothing arrives on; after
@@ -713,7 +727,7 @@ void tc_destroy(TcLayer& L) {
 cudaError_t tc_launch_gather(const TcLayer& L, const TcCall& c, cudaStream_t st) {
   const int rows = c.T * L.K;
   const int vecs = L.d / 8;
-  return launch_pdl(gather_rows_kernel, dim3(rows), dim3(std::min(256, vecs)), 0, st,
+  return launch_pdl(gather_rows_kernel, dim3((rows + 7) / 8), dim3(256), 0, st,
                     (const uint4*)c.x, c.perm_tok, c.offs + L.E, vecs, (uint4*)c.xperm);
 }
 

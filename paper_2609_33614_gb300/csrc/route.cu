@@ -11,7 +11,7 @@
 //      PPL factor and smoothing (§3.3), the clamp to the type-7 q_lo / q_hi quantiles of p
 //      (order statistics by in-warp rank counting, no sort), the candidate set and K cap
 //      (Eq. 6, ties to the lower index) and the renormalised gates (Eq. 7-8), with shuffles only.
-//      The history score S_h (Eq. 1) is computed once per block in fp64 from the accounts.
+//      The history score S_h (Eq. 1) is computed once per block from the accounts.
 #include "eat_internal.cuh"
 
 #include <math.h>
@@ -296,8 +296,11 @@ __device__ __forceinline__ float warp_max(float v) {
 
 constexpr int kSelectThreads = 256;
 
-// S_h (Eq. 1) for all experts into smem, fp64 arithmetic, readings: empty-history terms are 0;
-// c_mode 0 uses C_i / sum C, c_mode 1 the raw C_i.
+// S_h (Eq. 1) for all experts into smem, readings: empty-history terms are 0; c_mode 0 uses
+// C_i / sum C, c_mode 1 the raw C_i.  The sums over experts are exact (int64) or fp64; the three
+// ratios are fp32 divisions of the fp32-rounded operands (relative error ~2e-7, far inside the
+// 1e-5 margin at which a token's selection counts as decided).  fp64 division is avoided: it is
+// a long sequence on GB300's narrow fp64 pipe.
 __device__ void history_score_block(const int64_t* accN, const double* accP, const double* accC,
                                     int E, const RouteParams& rp, float* s_h) {
   __shared__ long long red_n[kSelectThreads / 32];
@@ -324,16 +327,17 @@ __device__ void history_score_block(const int64_t* accN, const double* accP, con
     red_c[0] = b;
   }
   __syncthreads();
-  const double total_n = (double)red_n[0];
-  const double total_c = red_c[0];
+  const float total_n = (float)red_n[0];
+  const float total_c = (float)red_c[0];
   for (int e = tid; e < E; e += blockDim.x) {
-    const double n = (double)accN[e];
-    const double a = total_n > 0.0 ? n / total_n : 0.0;
-    const double b = n > 0.0 ? accP[e] / n : 0.0;
-    double c;
-    if (rp.c_mode == EAT_C_RAW) c = accC[e];
-    else c = total_c > 0.0 ? accC[e] / total_c : 0.0;
-    s_h[e] = (float)((double)rp.w1 * a + (double)rp.w2 * b + (double)rp.w3 * c);
+    const long long ni = accN[e];
+    const float n = (float)ni;
+    const float a = ni > 0 ? n / total_n : 0.f;
+    const float b = ni > 0 ? (float)accP[e] / n : 0.f;
+    float c;
+    if (rp.c_mode == EAT_C_RAW) c = (float)accC[e];
+    else c = total_c > 0.f ? (float)accC[e] / total_c : 0.f;
+    s_h[e] = rp.w1 * a + rp.w2 * b + rp.w3 * c;
   }
   __syncthreads();
 }
@@ -353,8 +357,9 @@ __global__ void __launch_bounds__(kSelectThreads)
 route_select_kernel(const double* __restrict__ part, int n_split, const float* __restrict__ bias,
                     int T, int E, int K, const int64_t* __restrict__ accN,
                     const double* __restrict__ accP, const double* __restrict__ accC,
-                    RouteParams rp, int32_t* __restrict__ out_idx, float* __restrict__ out_w,
-                    int32_t* __restrict__ out_k, float* __restrict__ out_p) {
+                    RouteParams rp, double inv_temp, int32_t* __restrict__ out_idx,
+                    float* __restrict__ out_w, int32_t* __restrict__ out_k,
+                    float* __restrict__ out_p) {
   __shared__ float s_h[kMaxExperts];
   pdl_wait();
   pdl_launch_dependents();
@@ -379,7 +384,7 @@ route_select_kernel(const double* __restrict__ part, int n_split, const float* _
       double s = 0.0;
       for (int sp = 0; sp < n_split; ++sp) s += part[((size_t)sp * T + t) * E + e];
       if (bias) s += (double)bias[e];
-      z = (float)(s / (double)rp.temperature);
+      z = (float)(s * inv_temp);
     }
     p[i] = z;
     lmax = fmaxf(lmax, z);
@@ -634,9 +639,10 @@ cudaError_t launch_route_select(const double* part, int n_split, const float* b_
                                 int32_t* k, float* psel, cudaStream_t st) {
   const int warps = kSelectThreads / 32;
   dim3 grid((T + warps - 1) / warps);
+  const double inv_temp = 1.0 / (double)rp.temperature;  // one host division, not one per score
 #define EAT_SELECT(EPL)                                                                    \
   launch_pdl(route_select_kernel<EPL>, grid, dim3(kSelectThreads), 0, st, part, n_split,    \
-             b_router, T, E, K, accN, accP, accC, rp, idx, w, k, psel)
+             b_router, T, E, K, accN, accP, accC, rp, inv_temp, idx, w, k, psel)
   if (E <= 32) return EAT_SELECT(1);
   if (E <= 64) return EAT_SELECT(2);
   if (E <= 128) return EAT_SELECT(4);
