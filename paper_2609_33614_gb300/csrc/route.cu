@@ -1,8 +1,8 @@
 // Router and EAT selection (§3.1-§3.4 of the EAT paper, Eq. 1-8).
 //
-//  router_logits_small_kernel (T <= 128, decode) / router_logits_kernel (register-tiled through
-//      shared memory, prefill): partial router scores x . w_r over slices of d: fp32 FMA inside
-//      16- or 32-wide chunks, chunk sums accumulated in fp64 or Kahan-compensated fp32, so the
+//  router_logits_small_kernel (T <= 128, decode) / router_logits_tile_kernel (bf16 x, prefill) /
+//      router_logits_kernel (other prefill calls; both tiled through shared memory): partial
+//      router scores x . w_r over slices of d: fp32 FMA inside 16- or 32-wide chunks, chunk sums accumulated in fp64 or Kahan-compensated fp32, so the
 //      logits carry ~1e-7 absolute error (the selection compares I against tau at 1e-5 and P_total
 //      sums p at 1e-6 relative).  The scores stay off the tensor cores: their fp32 accumulation
 //      biased the scores enough to move P_total by ~1e-6 relative.
@@ -157,16 +157,17 @@ router_logits_small_kernel(const TX* __restrict__ x, const float* __restrict__ w
   }
 }
 
-// Router scores for large T, vectorised variant (d a multiple of 32, 16-byte aligned x and W_r):
-// CTA tile of 128 tokens x 64 experts, 256 threads with 8 tokens x 4 experts each.  Each 32-column
-// chunk of x and W_r is loaded with 16-byte loads into registers one chunk ahead of the compute
-// (the global latency overlaps the FMAs of the current chunk) and stored transposed into shared
-// memory (lanes of a warp take consecutive rows, so the transposed stores hit distinct banks).
-// Chunk sums are added with Kahan compensation, as in router_logits_kernel.
-constexpr int kVT = 128, kVE = 64;
+// Router scores for large T with bf16 x (d a multiple of 32, 16-byte aligned x and W_r): CTA tile
+// of 64 tokens x 64 experts over one slice of d, 256 threads with 4 tokens x 4 experts each (the
+// experts tx, tx + 16, tx + 32, tx + 48, so a warp's weight reads cover 16 consecutive rows and
+// hit distinct bank groups).  Both operands sit row-major in shared memory as fp32 (row stride 36
+// floats), double-buffered by 32-column chunk: W_r rows arrive by cp.async, x rows are loaded
+// into registers one chunk ahead and converted when stored.  Each output takes 32 fp32 FMAs per
+// chunk and the chunk sums are added with Kahan compensation, as in router_logits_kernel.  With
+// 4 x 4 outputs a thread needs about 100 registers, so two CTAs (16 warps) share an SM.
+constexpr int kRT = 64, kRE = 64, kRS = kChunkK + 4;
 
-__device__ __forceinline__ void load8(const __nv_bfloat16* p, float (&v)[8]) {
-  const uint4 u = *(const uint4*)p;
+__device__ __forceinline__ void bf16x8_to_f32(const uint4& u, float (&v)[8]) {
   const uint32_t w[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
@@ -175,108 +176,107 @@ __device__ __forceinline__ void load8(const __nv_bfloat16* p, float (&v)[8]) {
     v[2 * q + 1] = f.y;
   }
 }
-__device__ __forceinline__ void load8(const float* p, float (&v)[8]) {
-  const float4 a = *(const float4*)p, b = *(const float4*)(p + 4);
-  v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
-  v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
-}
 
-template <typename TX>
-__global__ void __launch_bounds__(kLogitThreads, 1)
-router_logits_vec_kernel(const TX* __restrict__ x, const float* __restrict__ wr, int T, int d,
-                         int E, int d_per_split, double* __restrict__ part) {
-  __shared__ __align__(16) float xs[kChunkK][kVT + 4];
-  __shared__ __align__(16) float ws[kChunkK][kVE + 4];
+__global__ void __launch_bounds__(kLogitThreads, 2)
+router_logits_tile_kernel(const __nv_bfloat16* __restrict__ x, const float* __restrict__ wr,
+                          int T, int d, int E, int d_per_split, double* __restrict__ part) {
+  __shared__ __align__(16) float xs[2][kRT][kRS];
+  __shared__ __align__(16) float ws[2][kRE][kRS];
   pdl_wait();
   pdl_launch_dependents();
   const int tid = threadIdx.x;
   const int tx = tid & 15, ty = tid >> 4;
-  const int t0 = blockIdx.x * kVT, e0 = blockIdx.y * kVE;
+  const int t0 = blockIdx.x * kRT, e0 = blockIdx.y * kRE;
   const int dbeg = blockIdx.z * d_per_split;
   const int dend = min(d, dbeg + d_per_split);
-  // loader mapping: x -- 128 rows x 4 pieces of 8 columns, 2 pieces per thread (row = q % 128);
-  // W_r -- 64 rows x 8 pieces of 4 columns, 2 per thread (row = q % 64)
-  float xv[2][8], wv[2][4];
-  auto load_chunk = [&](int k0) {
+  const int n_chunks = dend > dbeg ? (dend - dbeg) / kChunkK : 0;
+  // x loader: row tid / 4, 8 columns at (tid % 4) * 8
+  const int xr = tid >> 2, xc = (tid & 3) * 8;
+  const bool x_ok = t0 + xr < T;
+  const __nv_bfloat16* xsrc = x + (size_t)(x_ok ? t0 + xr : 0) * d + xc;
+  uint4 xraw = make_uint4(0u, 0u, 0u, 0u);
+  auto load_x = [&](int k0) {
+    if (x_ok) xraw = *(const uint4*)(xsrc + k0);
+  };
+  auto store_x = [&](int b) {
+    float v[8];
+    bf16x8_to_f32(xraw, v);
+    *(float4*)&xs[b][xr][xc] = make_float4(v[0], v[1], v[2], v[3]);
+    *(float4*)&xs[b][xr][xc + 4] = make_float4(v[4], v[5], v[6], v[7]);
+  };
+  // W_r loader: pieces tid and tid + 256 -- row q / 8, 4 columns at (q % 8) * 4
+  auto load_w = [&](int k0, int b) {
 #pragma unroll
     for (int r = 0; r < 2; ++r) {
       const int q = tid + r * kLogitThreads;
-      const int row = q % kVT, c8 = (q / kVT) * 8;
-      const int t = t0 + row;
-      if (t < T && k0 + c8 < dend) {
-        load8(x + (size_t)t * d + k0 + c8, xv[r]);
-      } else {
-#pragma unroll
-        for (int i = 0; i < 8; ++i) xv[r][i] = 0.f;
-      }
-      const int erow = q % kVE, c4 = (q / kVE) * 4;
-      const int e = e0 + erow;
-      if (e < E && k0 + c4 < dend) {
-        const float4 v = *(const float4*)(wr + (size_t)e * d + k0 + c4);
-        wv[r][0] = v.x; wv[r][1] = v.y; wv[r][2] = v.z; wv[r][3] = v.w;
-      } else {
-        wv[r][0] = wv[r][1] = wv[r][2] = wv[r][3] = 0.f;
-      }
+      const int row = q >> 3, c4 = (q & 7) * 4;
+      const int e = e0 + row;
+      if (e < E)
+        cp_async16((uint32_t)__cvta_generic_to_shared(&ws[b][row][c4]),
+                   wr + (size_t)e * d + k0 + c4);
+      else
+        *(float4*)&ws[b][row][c4] = make_float4(0.f, 0.f, 0.f, 0.f);
     }
+    cp_async_commit();
   };
-  auto store_chunk = [&]() {
+  float sum[4][4], comp[4][4];
 #pragma unroll
-    for (int r = 0; r < 2; ++r) {
-      const int q = tid + r * kLogitThreads;
-      const int row = q % kVT, c8 = (q / kVT) * 8;
-#pragma unroll
-      for (int i = 0; i < 8; ++i) xs[c8 + i][row] = xv[r][i];
-      const int erow = q % kVE, c4 = (q / kVE) * 4;
-#pragma unroll
-      for (int i = 0; i < 4; ++i) ws[c4 + i][erow] = wv[r][i];
-    }
-  };
-  float sum[8][4], comp[8][4];
-#pragma unroll
-  for (int i = 0; i < 8; ++i)
+  for (int i = 0; i < 4; ++i)
 #pragma unroll
     for (int j = 0; j < 4; ++j) sum[i][j] = comp[i][j] = 0.f;
 
-  if (dbeg < dend) {
-    load_chunk(dbeg);
-    store_chunk();
+  if (n_chunks > 0) {
+    load_w(dbeg, 0);
+    load_x(dbeg);
+    store_x(0);
   }
-  __syncthreads();
-  for (int k0 = dbeg; k0 < dend; k0 += kChunkK) {
-    const bool more = k0 + kChunkK < dend;
-    if (more) load_chunk(k0 + kChunkK);
-    float acc[8][4];
+  for (int c = 0; c < n_chunks; ++c) {
+    const int cur = c & 1;
+    const bool more = c + 1 < n_chunks;
+    __syncthreads();  // chunk c - 1 consumed: buffer cur ^ 1 is free; xs[cur] is complete
+    if (more) {
+      load_w(dbeg + (c + 1) * kChunkK, cur ^ 1);
+      load_x(dbeg + (c + 1) * kChunkK);
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
+    }
+    __syncthreads();  // every thread's W_r pieces of chunk c have landed
+    float acc[4][4];
 #pragma unroll
-    for (int i = 0; i < 8; ++i)
+    for (int i = 0; i < 4; ++i)
 #pragma unroll
       for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
-#pragma unroll 4
-    for (int kk = 0; kk < kChunkK; ++kk) {
-      const float4 a0 = *(const float4*)&xs[kk][ty * 8];
-      const float4 a1 = *(const float4*)&xs[kk][ty * 8 + 4];
-      const float4 b = *(const float4*)&ws[kk][tx * 4];
-      const float av[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
-      const float bv[4] = {b.x, b.y, b.z, b.w};
 #pragma unroll
-      for (int i = 0; i < 8; ++i)
+    for (int kk = 0; kk < kChunkK; kk += 4) {
+      float4 a[4], b[4];
 #pragma unroll
-        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
+      for (int i = 0; i < 4; ++i) a[i] = *(const float4*)&xs[cur][ty * 4 + i][kk];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) b[j] = *(const float4*)&ws[cur][tx + 16 * j][kk];
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          acc[i][j] = fmaf(a[i].x, b[j].x, acc[i][j]);
+          acc[i][j] = fmaf(a[i].y, b[j].y, acc[i][j]);
+          acc[i][j] = fmaf(a[i].z, b[j].z, acc[i][j]);
+          acc[i][j] = fmaf(a[i].w, b[j].w, acc[i][j]);
+        }
     }
 #pragma unroll
-    for (int i = 0; i < 8; ++i)
+    for (int i = 0; i < 4; ++i)
 #pragma unroll
       for (int j = 0; j < 4; ++j) kahan_add(sum[i][j], comp[i][j], acc[i][j]);
-    __syncthreads();
-    if (more) store_chunk();
-    __syncthreads();
+    if (more) store_x(cur ^ 1);
   }
 #pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const int t = t0 + ty * 8 + i;
+  for (int i = 0; i < 4; ++i) {
+    const int t = t0 + ty * 4 + i;
     if (t >= T) continue;
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
-      const int e = e0 + tx * 4 + j;
+      const int e = e0 + tx + 16 * j;
       if (e < E)
         part[((size_t)blockIdx.z * T + t) * E + e] = (double)sum[i][j] - (double)comp[i][j];
     }
@@ -589,10 +589,10 @@ route_select_kernel(const double* __restrict__ part, int n_split, const float* _
 int router_split(int T, int d, int E) {
   if (T <= kSmallT) return (d + kSmallSlice - 1) / kSmallSlice;
   if (d % kChunkK == 0) {
-    // vectorised kernel (one 256-thread CTA per SM): about one full wave of long CTAs
-    const long long tiles = (long long)((T + kVT - 1) / kVT) * ((E + kVE - 1) / kVE);
+    // tile kernel (two 256-thread CTAs per SM): up to two waves, slices of at least 256 columns
+    const long long tiles = (long long)((T + kRT - 1) / kRT) * ((E + kRE - 1) / kRE);
     int split = 1;
-    while (tiles * split * 2 <= 152 && d / (split * 2) >= 512 && split < 64) split *= 2;
+    while (tiles * split * 2 <= 4 * 152 && d / (split * 2) >= 256 && split < 64) split *= 2;
     return split;
   }
   // enough CTAs for two waves, each slice at least 256 columns of d
@@ -617,13 +617,10 @@ cudaError_t launch_router_logits(const void* x, int x_bf16, const float* w_route
   }
   int per = (d + n_split - 1) / n_split;
   per = (per + kChunkK - 1) / kChunkK * kChunkK;
-  if (d % kChunkK == 0 && vec_ok) {
-    dim3 grid((T + kVT - 1) / kVT, (E + kVE - 1) / kVE, n_split);
-    if (x_bf16)
-      return launch_pdl(router_logits_vec_kernel<__nv_bfloat16>, grid, dim3(kLogitThreads), 0,
-                        st, (const __nv_bfloat16*)x, w_router, T, d, E, per, part);
-    return launch_pdl(router_logits_vec_kernel<float>, grid, dim3(kLogitThreads), 0, st,
-                      (const float*)x, w_router, T, d, E, per, part);
+  if (x_bf16 && d % kChunkK == 0 && vec_ok) {
+    dim3 grid((T + kRT - 1) / kRT, (E + kRE - 1) / kRE, n_split);
+    return launch_pdl(router_logits_tile_kernel, grid, dim3(kLogitThreads), 0, st,
+                      (const __nv_bfloat16*)x, w_router, T, d, E, per, part);
   }
   dim3 grid((T + kTileT - 1) / kTileT, (E + kTileE - 1) / kTileE, n_split);
   if (x_bf16)
