@@ -8,10 +8,11 @@
 //      with weight 1, and writes the segment's sum of squares of every slot (||o||_2 of the
 //      unweighted expert output feeds C_s) to nrm_part[slot][segment].
 //  account_kernel: one block per expert.  Finishes ||o||_2 of each slot from its segment sums
-//      (fp32, fixed order), sums p and ||o||_2 over the expert's slots in fp64 (a fixed tree) and
-//      applies N += n_e, P_total += sum p, C_s <- (1 - alpha) C_s + alpha * mean ||o||_2 when
-//      n_e > 0.  Only additions run in fp64: GB300's fp64 pipe is narrow, and an fp64 square
-//      root per slot made the block of a heavily used expert the longest of the step.
+//      (fp32, fixed order), sums p and ||o||_2 over the expert's slots with compensated fp32
+//      additions (a fixed tree; about fp64 accuracy) and applies, in fp64 on one thread,
+//      N += n_e, P_total += sum p, C_s <- (1 - alpha) C_s + alpha * mean ||o||_2 when n_e > 0.
+//      Per-slot work stays off GB300's narrow fp64 pipe: an fp64 square root per slot made the
+//      block of a heavily used expert the longest of the step.
 #include "eat_internal.cuh"
 
 namespace eat {
@@ -183,14 +184,14 @@ account_kernel(const int32_t* __restrict__ offs, const float* __restrict__ perm_
                double* __restrict__ P, double* __restrict__ C, int32_t* __restrict__ st_n,
                double* __restrict__ st_p, double* __restrict__ st_norm,
                unsigned long long* __restrict__ counters) {
-  __shared__ double rp[kAccThreads / 32], rn[kAccThreads / 32];
+  __shared__ float red[4][kAccThreads / 32];
   pdl_wait();
   pdl_launch_dependents();
   const int e = blockIdx.x;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int beg = offs[e], end = offs[e + 1];
   const bool vec = (nb & 3) == 0;
-  double sp = 0.0, sn = 0.0;
+  float p_hi = 0.f, p_lo = 0.f, n_hi = 0.f, n_lo = 0.f;
   // four slots per thread per pass, all loads issued before the sums
   for (int i0 = beg + tid; i0 < end; i0 += 4 * kAccThreads) {
     float pv[4], nv[4];
@@ -219,20 +220,33 @@ account_kernel(const int32_t* __restrict__ offs, const float* __restrict__ perm_
     }
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
-      sp += (double)pv[u];
-      sn += (double)sqrtf(nv[u]);
+      df_add(p_hi, p_lo, pv[u]);
+      df_add(n_hi, n_lo, sqrtf(nv[u]));
     }
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
-    sp += __shfl_xor_sync(0xffffffffu, sp, o);
-    sn += __shfl_xor_sync(0xffffffffu, sn, o);
+    const float a = __shfl_xor_sync(0xffffffffu, p_hi, o);
+    const float b = __shfl_xor_sync(0xffffffffu, p_lo, o);
+    const float c = __shfl_xor_sync(0xffffffffu, n_hi, o);
+    const float dd = __shfl_xor_sync(0xffffffffu, n_lo, o);
+    df_add(p_hi, p_lo, a, b);
+    df_add(n_hi, n_lo, c, dd);
   }
-  if (lane == 0) { rp[warp] = sp; rn[warp] = sn; }
+  if (lane == 0) {
+    red[0][warp] = p_hi;
+    red[1][warp] = p_lo;
+    red[2][warp] = n_hi;
+    red[3][warp] = n_lo;
+  }
   __syncthreads();
   if (tid == 0) {
-    double a = 0.0, b = 0.0;
-    for (int wi = 0; wi < kAccThreads / 32; ++wi) { a += rp[wi]; b += rn[wi]; }
+    float ah = 0.f, al = 0.f, bh = 0.f, bl = 0.f;
+    for (int wi = 0; wi < kAccThreads / 32; ++wi) {
+      df_add(ah, al, red[0][wi], red[1][wi]);
+      df_add(bh, bl, red[2][wi], red[3][wi]);
+    }
+    const double a = (double)ah + (double)al, b = (double)bh + (double)bl;
     const int n = end - beg;
     N[e] += n;
     P[e] += a;

@@ -29,7 +29,7 @@ struct eat_handle {
   double* st_p = nullptr;
   double* st_norm = nullptr;
   long long* counters = nullptr;  // [4] on the device: calls, sum |union|, sum k, spare
-  double* logit_part = nullptr;
+  float2* logit_part = nullptr;   // [split][T][E] partial router scores (fp32 pairs)
   int32_t* idx = nullptr;
   float* w = nullptr;
   int32_t* k = nullptr;
@@ -371,7 +371,7 @@ eat_status eat_create(const eat_layer_desc* desc, const eat_params* params, eat_
   add(&h->st_norm, sizeof(double) * h->E);
   add(&h->counters, sizeof(long long) * 4);
   add(&h->status, sizeof(unsigned int) * 4);
-  add(&h->logit_part, sizeof(double) * (size_t)max_lsplit * h->E);
+  add(&h->logit_part, sizeof(float2) * (size_t)max_lsplit * h->E);
   add(&h->idx, sizeof(int32_t) * rows);
   add(&h->w, sizeof(float) * rows);
   add(&h->k, sizeof(int32_t) * h->Tmax);

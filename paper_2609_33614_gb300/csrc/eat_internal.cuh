@@ -19,6 +19,30 @@ __device__ __forceinline__ void pdl_launch_dependents() {
 
 bool pdl_enabled();
 
+// Compensated fp32 sums ("double-float": a value is the unevaluated sum hi + lo).  GB300's fp64
+// pipe runs about two lanes per SM per clock, so one fp64 warp instruction occupies it for ~64
+// cycles; sums that need more than fp32 precision use these error-free fp32 steps instead.
+// two_sum (Knuth): s = fl(a + b) and s + e == a + b exactly.
+__device__ __forceinline__ void two_sum(float a, float b, float& s, float& e) {
+  s = a + b;
+  const float bb = s - a;
+  e = (a - (s - bb)) + (b - bb);
+}
+// (hi, lo) += v
+__device__ __forceinline__ void df_add(float& hi, float& lo, float v) {
+  float s, e;
+  two_sum(hi, v, s, e);
+  hi = s;
+  lo += e;
+}
+// (hi, lo) += (vhi, vlo)
+__device__ __forceinline__ void df_add(float& hi, float& lo, float vhi, float vlo) {
+  float s, e;
+  two_sum(hi, vhi, s, e);
+  hi = s;
+  lo += e + vlo;
+}
+
 // 16-byte global -> shared copy (cp.async, L2 only), its group commit and wait.
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
@@ -62,12 +86,13 @@ struct RouteParams {
   float* tau_out;          // [T] tau_final written back (temporal smoothing, forward calls) or null
 };
 
-// Partial router logits (fp64): part[s][t][e] = sum over the s-th slice of d of x[t,j] Wr[e,j].
+// Partial router logits: part[s][t][e] = sum over the s-th slice of d of x[t,j] Wr[e,j], as an
+// unevaluated fp32 pair (hi, lo) whose exact sum carries the slice's score (see df_add).
 cudaError_t launch_router_logits(const void* x, int x_bf16, const float* w_router, int T, int d,
-                                 int E, int n_split, double* part, cudaStream_t st);
+                                 int E, int n_split, float2* part, cudaStream_t st);
 // Warp-per-token softmax + history score + threshold + selection + renormalisation; the router
-// scores are the sum over the n_split slices of part (fp64 [split][T][E]).
-cudaError_t launch_route_select(const double* part, int n_split, const float* b_router, int T,
+// scores are the sum over the n_split slices of part ([split][T][E] fp32 pairs).
+cudaError_t launch_route_select(const float2* part, int n_split, const float* b_router, int T,
                                 int E, int K, const int64_t* accN, const double* accP,
                                 const double* accC, RouteParams rp, int32_t* idx, float* w,
                                 int32_t* k, float* psel, cudaStream_t st);

@@ -44,7 +44,7 @@ __device__ __forceinline__ void kahan_add(float& sum, float& comp, float v) {
 template <typename TX>
 __global__ void __launch_bounds__(kLogitThreads)
 router_logits_kernel(const TX* __restrict__ x, const float* __restrict__ wr, int T, int d, int E,
-                     int d_per_split, double* __restrict__ part) {
+                     int d_per_split, float2* __restrict__ part) {
   __shared__ float xs[kChunkK][kTileT + 4];
   __shared__ float ws[kChunkK][kTileE + 4];
   pdl_wait();
@@ -99,15 +99,15 @@ router_logits_kernel(const TX* __restrict__ x, const float* __restrict__ wr, int
     for (int j = 0; j < 4; ++j) {
       const int e = e0 + tx * 4 + j;
       if (e < E)
-        part[((size_t)blockIdx.z * T + t) * E + e] = (double)sum[i][j] - (double)comp[i][j];
+        part[((size_t)blockIdx.z * T + t) * E + e] = make_float2(sum[i][j], -comp[i][j]);
     }
   }
 }
 
 // Router scores for small T (decode): block (t, s) computes part[s][t][e] for every expert over
 // the s-th slice of d; warp w takes experts w, w + 8, ...; lanes read float4 pieces of the weight
-// row and of x (coalesced), multiply in fp32, fold each 16 products into an fp64 lane sum, and the
-// 32 lane sums are added in fp64 (a fixed tree).
+// row and of x (coalesced), multiply in fp32, fold each 16 products into a compensated lane sum,
+// and the 32 lane sums are added compensated (a fixed tree).
 constexpr int kSmallT = kSmallRouterT;
 constexpr int kSmallSlice = 512;
 
@@ -124,7 +124,7 @@ __device__ __forceinline__ float4 load_x4(const __nv_bfloat16* p) {
 template <typename TX>
 __global__ void __launch_bounds__(kLogitThreads)
 router_logits_small_kernel(const TX* __restrict__ x, const float* __restrict__ wr, int T, int d,
-                           int E, int d_per_split, double* __restrict__ part) {
+                           int E, int d_per_split, float2* __restrict__ part) {
   pdl_wait();
   pdl_launch_dependents();
   const int t = blockIdx.x, s = blockIdx.y;
@@ -134,7 +134,7 @@ router_logits_small_kernel(const TX* __restrict__ x, const float* __restrict__ w
   const TX* xr = x + (size_t)t * d;
   for (int e = warp; e < E; e += kLogitThreads / 32) {
     const float* wrow = wr + (size_t)e * d;
-    double dacc = 0.0;
+    float hi = 0.f, lo = 0.f;
     float acc = 0.f;
     int cnt = 0;
     for (int c = beg + lane * 4; c < end; c += 128) {
@@ -145,15 +145,19 @@ router_logits_small_kernel(const TX* __restrict__ x, const float* __restrict__ w
       acc = fmaf(xv.z, wv.z, acc);
       acc = fmaf(xv.w, wv.w, acc);
       if (++cnt == 4) {
-        dacc += (double)acc;
+        df_add(hi, lo, acc);
         acc = 0.f;
         cnt = 0;
       }
     }
-    dacc += (double)acc;
+    df_add(hi, lo, acc);
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) dacc += __shfl_xor_sync(0xffffffffu, dacc, o);
-    if (lane == 0) part[((size_t)s * T + t) * E + e] = dacc;
+    for (int o = 16; o > 0; o >>= 1) {
+      const float ohi = __shfl_xor_sync(0xffffffffu, hi, o);
+      const float olo = __shfl_xor_sync(0xffffffffu, lo, o);
+      df_add(hi, lo, ohi, olo);
+    }
+    if (lane == 0) part[((size_t)s * T + t) * E + e] = make_float2(hi, lo);
   }
 }
 
@@ -179,7 +183,7 @@ __device__ __forceinline__ void bf16x8_to_f32(const uint4& u, float (&v)[8]) {
 
 __global__ void __launch_bounds__(kLogitThreads, 2)
 router_logits_tile_kernel(const __nv_bfloat16* __restrict__ x, const float* __restrict__ wr,
-                          int T, int d, int E, int d_per_split, double* __restrict__ part) {
+                          int T, int d, int E, int d_per_split, float2* __restrict__ part) {
   __shared__ __align__(16) float xs[2][kRT][kRS];
   __shared__ __align__(16) float ws[2][kRE][kRS];
   pdl_wait();
@@ -278,7 +282,7 @@ router_logits_tile_kernel(const __nv_bfloat16* __restrict__ x, const float* __re
     for (int j = 0; j < 4; ++j) {
       const int e = e0 + tx + 16 * j;
       if (e < E)
-        part[((size_t)blockIdx.z * T + t) * E + e] = (double)sum[i][j] - (double)comp[i][j];
+        part[((size_t)blockIdx.z * T + t) * E + e] = make_float2(sum[i][j], -comp[i][j]);
     }
   }
 }
@@ -297,38 +301,47 @@ __device__ __forceinline__ float warp_max(float v) {
 constexpr int kSelectThreads = 256;
 
 // S_h (Eq. 1) for all experts into smem, readings: empty-history terms are 0; c_mode 0 uses
-// C_i / sum C, c_mode 1 the raw C_i.  The sums over experts are exact (int64) or fp64; the three
-// ratios are fp32 divisions of the fp32-rounded operands (relative error ~2e-7, far inside the
-// 1e-5 margin at which a token's selection counts as decided).  fp64 division is avoided: it is
-// a long sequence on GB300's narrow fp64 pipe.
+// C_i / sum C, c_mode 1 the raw C_i.  sum N is exact (int64), sum C a compensated fp32 sum of the
+// fp32-rounded C_i; the three ratios are fp32 divisions (relative error ~3e-7, far inside the
+// 1e-5 margin at which a token's selection counts as decided).  No fp64 arithmetic: it would run
+// on GB300's narrow fp64 pipe in every block.
 __device__ void history_score_block(const int64_t* accN, const double* accP, const double* accC,
                                     int E, const RouteParams& rp, float* s_h) {
   __shared__ long long red_n[kSelectThreads / 32];
-  __shared__ double red_c[kSelectThreads / 32];
+  __shared__ float red_c[2][kSelectThreads / 32];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   long long n_sum = 0;
-  double c_sum = 0.0;
+  float c_hi = 0.f, c_lo = 0.f;
   for (int e = tid; e < E; e += blockDim.x) {
     n_sum += (long long)accN[e];
-    c_sum += accC[e];
+    df_add(c_hi, c_lo, (float)accC[e]);
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     n_sum += __shfl_xor_sync(0xffffffffu, n_sum, o);
-    c_sum += __shfl_xor_sync(0xffffffffu, c_sum, o);
+    const float oh = __shfl_xor_sync(0xffffffffu, c_hi, o);
+    const float ol = __shfl_xor_sync(0xffffffffu, c_lo, o);
+    df_add(c_hi, c_lo, oh, ol);
   }
-  if (lane == 0) { red_n[warp] = n_sum; red_c[warp] = c_sum; }
+  if (lane == 0) {
+    red_n[warp] = n_sum;
+    red_c[0][warp] = c_hi;
+    red_c[1][warp] = c_lo;
+  }
   __syncthreads();
   if (tid == 0) {
     long long a = 0;
-    double b = 0.0;
-    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) { a += red_n[w]; b += red_c[w]; }
+    float bh = 0.f, bl = 0.f;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) {
+      a += red_n[w];
+      df_add(bh, bl, red_c[0][w], red_c[1][w]);
+    }
     red_n[0] = a;
-    red_c[0] = b;
+    red_c[0][0] = bh + bl;
   }
   __syncthreads();
   const float total_n = (float)red_n[0];
-  const float total_c = (float)red_c[0];
+  const float total_c = red_c[0][0];
   for (int e = tid; e < E; e += blockDim.x) {
     const long long ni = accN[e];
     const float n = (float)ni;
@@ -354,10 +367,10 @@ __device__ __forceinline__ float order_stat(const float (&p)[EPL], const int (&r
 
 template <int EPL>
 __global__ void __launch_bounds__(kSelectThreads)
-route_select_kernel(const double* __restrict__ part, int n_split, const float* __restrict__ bias,
+route_select_kernel(const float2* __restrict__ part, int n_split, const float* __restrict__ bias,
                     int T, int E, int K, const int64_t* __restrict__ accN,
                     const double* __restrict__ accP, const double* __restrict__ accC,
-                    RouteParams rp, double inv_temp, int32_t* __restrict__ out_idx,
+                    RouteParams rp, float inv_temp, int32_t* __restrict__ out_idx,
                     float* __restrict__ out_w, int32_t* __restrict__ out_k,
                     float* __restrict__ out_p) {
   __shared__ float s_h[kMaxExperts];
@@ -381,10 +394,13 @@ route_select_kernel(const double* __restrict__ part, int n_split, const float* _
     valid[i] = e < E;
     float z = -INFINITY;
     if (valid[i]) {
-      double s = 0.0;
-      for (int sp = 0; sp < n_split; ++sp) s += part[((size_t)sp * T + t) * E + e];
-      if (bias) s += (double)bias[e];
-      z = (float)(s * inv_temp);
+      float hi = 0.f, lo = 0.f;
+      for (int sp = 0; sp < n_split; ++sp) {
+        const float2 v = part[((size_t)sp * T + t) * E + e];
+        df_add(hi, lo, v.x, v.y);
+      }
+      if (bias) df_add(hi, lo, bias[e]);
+      z = (hi + lo) * inv_temp;
     }
     p[i] = z;
     lmax = fmaxf(lmax, z);
@@ -603,7 +619,7 @@ int router_split(int T, int d, int E) {
 }
 
 cudaError_t launch_router_logits(const void* x, int x_bf16, const float* w_router, int T, int d,
-                                 int E, int n_split, double* part, cudaStream_t st) {
+                                 int E, int n_split, float2* part, cudaStream_t st) {
   const bool vec_ok = d % 4 == 0 && ((uintptr_t)x & 15) == 0 && ((uintptr_t)w_router & 15) == 0;
   if (T <= kSmallT && vec_ok) {
     int per = (d + n_split - 1) / n_split;
@@ -630,13 +646,13 @@ cudaError_t launch_router_logits(const void* x, int x_bf16, const float* w_route
                     (const float*)x, w_router, T, d, E, per, part);
 }
 
-cudaError_t launch_route_select(const double* part, int n_split, const float* b_router, int T,
+cudaError_t launch_route_select(const float2* part, int n_split, const float* b_router, int T,
                                 int E, int K, const int64_t* accN, const double* accP,
                                 const double* accC, RouteParams rp, int32_t* idx, float* w,
                                 int32_t* k, float* psel, cudaStream_t st) {
   const int warps = kSelectThreads / 32;
   dim3 grid((T + warps - 1) / warps);
-  const double inv_temp = 1.0 / (double)rp.temperature;  // one host division, not one per score
+  const float inv_temp = (float)(1.0 / (double)rp.temperature);
 #define EAT_SELECT(EPL)                                                                    \
   launch_pdl(route_select_kernel<EPL>, grid, dim3(kSelectThreads), 0, st, part, n_split,    \
              b_router, T, E, K, accN, accP, accC, rp, inv_temp, idx, w, k, psel)

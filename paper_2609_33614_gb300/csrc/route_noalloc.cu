@@ -6,8 +6,8 @@
 // a latency-critical decode loop that must not pay cudaMalloc's implicit device synchronisation,
 // or a host framework whose rules route every device allocation through its own allocator.  They
 // cannot create an eat_handle (eat_create allocates the accounts and the workspace).  This entry
-// point takes every input and output from the caller and keeps its only scratch -- the fp64
-// partial router scores -- in a fixed array compiled into the library below.
+// point takes every input and output from the caller and keeps its only scratch -- the partial
+// router scores -- in a fixed array compiled into the library below.
 #include "eat_internal.cuh"
 
 #include <mutex>
@@ -15,12 +15,12 @@
 
 namespace {
 
-// Scratch of the partial router scores, [split][T][E] doubles.  Every GPU that loads the library
+// Scratch of the partial router scores, [split][T][E] fp32 pairs (8 bytes each).  Every GPU that loads the library
 // holds these 1 MiB until the process exits.  Calls share the array and it keeps the previous
 // call's contents; nothing in it needs to start at zero (the scores kernel writes every entry it
 // later reads).  Two calls that overlap on the GPU (different streams, or threads) race on it.
-constexpr size_t kScratchDoubles = EAT_NOALLOC_SCRATCH_BYTES / sizeof(double);
-static __device__ __align__(256) double g_route_scratch[kScratchDoubles];
+constexpr size_t kScratchScores = EAT_NOALLOC_SCRATCH_BYTES / sizeof(float2);
+static __device__ __align__(256) float2 g_route_scratch[kScratchScores];
 
 constexpr int kMaxDevices = 64;
 std::mutex g_mu;
@@ -29,7 +29,7 @@ void* g_scratch_ptr[kMaxDevices] = {};
 // Device address of the scratch on the current device, looked up once per device.  In host code
 // g_route_scratch names a host-side stand-in, not device memory, so only this address may be
 // handed to a kernel.
-eat_status scratch_address(double** out) {
+eat_status scratch_address(float2** out) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) {
@@ -51,7 +51,7 @@ eat_status scratch_address(double** out) {
     }
     g_scratch_ptr[dev] = p;
   }
-  *out = (double*)g_scratch_ptr[dev];
+  *out = (float2*)g_scratch_ptr[dev];
   return EAT_OK;
 }
 
@@ -86,16 +86,16 @@ extern "C" eat_status eat_route_noalloc(const void* x, int32_t T, int32_t d_mode
   if (p.router_mode < EAT_ROUTER_EAT || p.router_mode > EAT_ROUTER_TOPP ||
       (p.router_mode == EAT_ROUTER_TOPP && !(p.top_p > 0.0 && p.top_p <= 1.0)))
     return bad("eat_route_noalloc: bad router_mode or top_p");
-  if ((size_t)T * (size_t)n_experts > kScratchDoubles)
+  if ((size_t)T * (size_t)n_experts > kScratchScores)
     return bad("eat_route_noalloc: T * n_experts exceeds the 131072 router scores its fixed "
                "1 MiB scratch holds; split the call into smaller token batches");
 
-  double* scratch = nullptr;
+  float2* scratch = nullptr;
   const eat_status s = scratch_address(&scratch);
   if (s != EAT_OK) return s;
 
   int split = eat::router_split(T, d_model, n_experts);
-  while (split > 1 && (size_t)split * T * n_experts > kScratchDoubles) split /= 2;
+  while (split > 1 && (size_t)split * T * n_experts > kScratchScores) split /= 2;
 
   eat::RouteParams rp;
   rp.w1 = (float)p.w1;
