@@ -168,17 +168,28 @@ __host__ __device__ constexpr int tmem_cols_for(int c) {
   return c <= 32 ? 32 : c <= 64 ? 64 : c <= 128 ? 128 : c <= 256 ? 256 : 512;
 }
 
-template <int BN, bool GATEUP>
+// Kernel modes: the down projection (one A tile, plain epilogue); gate/up with two accumulators
+// (gate and up A tiles of 128 rows against one B tile); gate/up interleaved (one A tile of 64 gate
+// rows over 64 up rows of the same features, one accumulator: an M = 128 x N = BN MMA covers both
+// projections of 64 features, and the epilogue pairs the gate and up warps of each feature).
+enum : int { kModeDown = 0, kModeGateUp = 1, kModeGateUpIL = 2 };
+
+template <int BN, int MODE>
 struct Cfg {
-  static constexpr int kNA = GATEUP ? 2 : 1;
+  static constexpr bool kGateUp = MODE != kModeDown;
+  static constexpr bool kIL = MODE == kModeGateUpIL;
+  static constexpr int kNA = MODE == kModeGateUp ? 2 : 1;
   static constexpr int kABytes = kBM * kBK * 2;
   static constexpr int kBBytes = BN * kBK * 2;
   static constexpr int kStageBytes = kNA * kABytes + kBBytes;
-  static constexpr int kStagesRaw = (kSmemBudget - 2048) / kStageBytes;
+  // interleaved epilogue exchange: [2 pairs][2 buffers][2 directions][16 columns][32 lanes] fp32
+  static constexpr int kXchgFloats = kIL ? 2 * 2 * 2 * 16 * 32 : 0;
+  static constexpr int kStagesRaw = (kSmemBudget - 2048 - kXchgFloats * 4) / kStageBytes;
   static constexpr int kStages = kStagesRaw > 12 ? 12 : kStagesRaw;
   static constexpr int kAccCols = kNA * BN;
   static constexpr int kTmemCols = tmem_cols_for(2 * kAccCols);
-  static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + 256;
+  static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kXchgFloats * 4 + 256;
+  static_assert(2 * kAccCols <= 512, "two accumulator buffers must fit in TMEM");
 };
 
 struct TcArgs {
@@ -239,22 +250,29 @@ __device__ __forceinline__ Unit decode_unit(const TcArgs& a, int u) {
   return w;
 }
 
-__device__ __forceinline__ float silu_f(float g) { return g / (1.0f + expf(-g)); }
+// silu(g) = g / (1 + e^-g) with the hardware exponential and an approximate division: relative
+// error about 1e-6, far below the bf16 rounding of the activation it feeds (4e-3).  For g below
+// about -88 the denominator overflows to infinity and the quotient is 0, the function's limit.
+__device__ __forceinline__ float silu_f(float g) { return __fdividef(g, 1.0f + __expf(-g)); }
 
-template <int BN, bool GATEUP>
+template <int BN, int MODE>
 __global__ void __launch_bounds__(kThreadsTc, 1)
 tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__ CUtensorMap mapA1,
               const __grid_constant__ CUtensorMap mapB, const TcArgs args) {
-  using C = Cfg<BN, GATEUP>;
+  using C = Cfg<BN, MODE>;
+  constexpr bool GATEUP = C::kGateUp;
+  constexpr bool IL = C::kIL;
   constexpr int S = C::kStages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  uint64_t* full = (uint64_t*)(smem + S * C::kStageBytes);
+  float* xchg = (float*)(smem + S * C::kStageBytes);
+  uint64_t* full = (uint64_t*)(xchg + C::kXchgFloats);
   uint64_t* empty = full + S;
   uint64_t* tfull = empty + S;
   uint64_t* tempty = tfull + 2;
   uint64_t* mma_done = tempty + 2;
-  uint32_t* tmem_slot = (uint32_t*)(mma_done + 1);
+  uint64_t* xbar = mma_done + 1;  // [2 pairs][2 buffers], interleaved epilogue exchange
+  uint32_t* tmem_slot = (uint32_t*)(xbar + 4);
   volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -268,6 +286,7 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
       mbar_init(&tempty[b], 4);
     }
     mbar_init(mma_done, 1);
+    for (int i = 0; i < 4; ++i) mbar_init(&xbar[i], 2);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -283,6 +302,18 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
   // everything above is local to the CTA; from here on it reads what earlier kernels wrote
   pdl_wait();
   pdl_launch_dependents();
+
+  // A tile of one k-block: one 128-row box (or the gate and up boxes of the two-accumulator
+  // mode), or in the interleaved mode 64 gate rows over the 64 up rows of the same features
+  auto load_a = [&](uint8_t* st, uint64_t* bar, int kb, int a_row) {
+    if (IL) {
+      tma_load_2d(st, &mapA0, bar, kb * kBK, a_row);
+      tma_load_2d(st + C::kABytes / 2, &mapA1, bar, kb * kBK, a_row);
+    } else {
+      tma_load_2d(st, &mapA0, bar, kb * kBK, a_row);
+      if (GATEUP) tma_load_2d(st + C::kABytes, &mapA1, bar, kb * kBK, a_row);
+    }
+  };
 
   const int total_tiles = args.tile_offs
                               ? args.tile_offs[args.n_groups]
@@ -324,8 +355,7 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
         uint8_t* st = smem + stage * C::kStageBytes;
         if (lane == 0) {
           mbar_expect_tx(&full[stage], C::kNA * C::kABytes);
-          tma_load_2d(st, &mapA0, &full[stage], kb * kBK, a_row);
-          if (GATEUP) tma_load_2d(st + C::kABytes, &mapA1, &full[stage], kb * kBK, a_row);
+          load_a(st, &full[stage], kb, a_row);
         }
         const uint32_t sb = smem_u32(st + C::kNA * C::kABytes);
 #pragma unroll
@@ -380,8 +410,7 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
           }
           uint8_t* st = smem + stage * C::kStageBytes;
           mbar_expect_tx(&full[stage], C::kStageBytes);
-          tma_load_2d(st, &mapA0, &full[stage], kb * kBK, a_row);
-          if (GATEUP) tma_load_2d(st + C::kABytes, &mapA1, &full[stage], kb * kBK, a_row);
+          load_a(st, &full[stage], kb, a_row);
           tma_load_2d(st + C::kNA * C::kABytes, &mapB, &full[stage], kb * kBK, b_row);
           ++issued;
           if (++stage == S) {
@@ -429,7 +458,7 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
             const uint64_t db = sdesc_k128(sb + k * 32);
             const uint32_t acc = (kb > w.kb0 || k > 0) ? 1u : 0u;
             mma_bf16(d0, sdesc_k128(sa0 + k * 32), db, idesc, acc);
-            if (GATEUP) mma_bf16(d1, sdesc_k128(sa1 + k * 32), db, idesc, acc);
+            if (C::kNA == 2) mma_bf16(d1, sdesc_k128(sa1 + k * 32), db, idesc, acc);
           }
           mma_commit(&empty[stage]);
           if (++stage == S) {
@@ -443,6 +472,71 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
       // no MMA may still be running when TMEM is freed
       mma_commit(mma_done);
       mbar_wait(mma_done, 0u, abort_flag, args.err, 16u, false);
+    }
+  } else if (IL) {
+    // ------------------------------------------ epilogue, interleaved gate/up (warps 2..5)
+    // TMEM lanes 0-63 hold the gate rows and lanes 64-127 the up rows of the tile's 64 features;
+    // a warp may read lane quarter warp % 4, so quarters 0, 1 are gate and 2, 3 up of features
+    // 32 (q % 2) + lane.  The gate and up warps of a feature half trade half of every 32-column
+    // chunk through shared memory (double-buffered, one bounded mbarrier wait per chunk); the
+    // gate warp finishes columns 0-15 of the chunk, the up warp columns 16-31.
+    const int q = warp & 3;
+    const int half = q & 1;
+    const bool is_gate = q < 2;
+    float* xh = xchg + half * (2 * 2 * 16 * 32);
+    uint64_t* xb = xbar + half * 2;
+    int local = 0;
+    long long chunk = 0;
+    bool ok = true;
+    for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++local) {
+      const Unit w = decode_unit<BN>(args, u);
+      const int buf = local & 1;
+      const uint32_t tph = (uint32_t)((local >> 1) & 1);
+      if (!mbar_wait(&tfull[buf], tph, abort_flag, args.err, 32u, true)) break;
+      tc_fence_after();
+      const uint32_t tbase = tmem_base + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * C::kAccCols);
+      const int f = w.m0 + 32 * half + lane;
+      const bool fok = f < args.M;
+      const int keep = is_gate ? 0 : 16;  // chunk columns this warp finishes
+      for (int c0 = 0; c0 < BN && c0 < w.nrows; c0 += 32, ++chunk) {
+        uint32_t v0[16], v1[16];
+        tmem_ld16(tbase + c0, v0);
+        tmem_ld16(tbase + c0 + 16, v1);
+        tmem_wait_ld();
+        const int b = (int)(chunk & 1);
+        float* mine_out = xh + (b * 2 + (is_gate ? 0 : 1)) * 512;
+        const float* theirs = xh + (b * 2 + (is_gate ? 1 : 0)) * 512;
+        if (is_gate) {
+#pragma unroll
+          for (int j = 0; j < 16; ++j) mine_out[j * 32 + lane] = __uint_as_float(v1[j]);
+        } else {
+#pragma unroll
+          for (int j = 0; j < 16; ++j) mine_out[j * 32 + lane] = __uint_as_float(v0[j]);
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&xb[b]);
+        if (!mbar_wait(&xb[b], (uint32_t)((chunk >> 1) & 1), abort_flag, args.err, 128u, true)) {
+          ok = false;
+          break;
+        }
+        if (fok) {
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            const int col = c0 + keep + j;
+            if (col < w.nrows) {
+              const float o = theirs[j * 32 + lane];
+              const float m = __uint_as_float(is_gate ? v0[j] : v1[j]);
+              const float h = is_gate ? silu_f(m) * o : silu_f(o) * m;
+              ((__nv_bfloat16*)args.out)[(size_t)(w.slot0 + col) * args.M + f] =
+                  __float2bfloat16_rn(h);
+            }
+          }
+        }
+      }
+      if (!ok) break;
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tempty[buf]);
     }
   } else {
     // -------------------------------------------------------------- epilogue (warps 2..5)
@@ -491,6 +585,349 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
   __syncthreads();
   tc_fence_after();
   if (warp == 1) tmem_dealloc(tmem_base, C::kTmemCols);
+}
+
+// ------------------------------------------------------------ SM-pair kernels (cta_group::2)
+// Large calls run on pairs of SMs (2-CTA clusters).  The pair issues M = 256 x N = 256 MMAs: each
+// CTA holds 128 rows of A (weight rows) and 128 of the tile's 256 token rows of B, so a stage is
+// 32 KB per SM for the flops the single-SM kernel stages in 48 KB, and six stages are in flight
+// (the single-SM kernels, with four, wait on TMA latency about half the time).  Rank 0 of the pair
+// issues the MMAs (tcgen05.mma.cta_group::2) and commits them to the barriers of both CTAs; both
+// CTAs load their halves with TMA completing on rank 0's full barrier (rank 0 expects the bytes
+// of both); each CTA drains its own TMEM rows, and rank 0 reuses an accumulator buffer once the
+// epilogues of both CTAs released it.  Modes: the down projection (256 output features per unit)
+// and the interleaved gate/up (each CTA 64 gate rows over the 64 up rows of its features, 128
+// features per unit).  The MMA width is the unit's token rows rounded up to 32 (each CTA loads
+// half of it), so a partial tile computes no padding beyond that.
+constexpr int kPairBN = 256;
+constexpr int kPairRows = kPairBN / 2;
+
+template <int MODE>
+struct PairCfg {
+  static constexpr bool kIL = MODE == kModeGateUpIL;
+  static constexpr int kABytes = kBM * kBK * 2;
+  static constexpr int kBBytes = kPairRows * kBK * 2;
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr int kXchgFloats = kIL ? 2 * 2 * 2 * 16 * 32 : 0;
+  static constexpr int kStagesRaw = (kSmemBudget - 2048 - kXchgFloats * 4) / kStageBytes;
+  static constexpr int kStages = kStagesRaw > 8 ? 8 : kStagesRaw;
+  static constexpr int kAccCols = kPairBN;
+  static constexpr int kTmemCols = 512;
+  static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kXchgFloats * 4 + 256;
+  static constexpr int kFeat = kIL ? 64 : 128;  // output features of one CTA in a unit
+};
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// Address of the same shared variable in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t map_rank(uint32_t saddr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;"
+               ::: "memory");
+}
+// TMA load into this CTA's shared memory, completing on an mbarrier of either CTA of the pair.
+__device__ __forceinline__ void tma_load_2d_pair(void* dst, const CUtensorMap* map,
+                                                 uint32_t bar_cluster, int c0, int c1) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(map), "r"(bar_cluster), "r"(c0), "r"(c1)
+      : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar_cluster) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t* slot, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                   smem_u32(slot)),
+               "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void mma_bf16_pair(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                              uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// Arrive on `bar` of both CTAs of the pair once the MMAs issued so far completed.
+__device__ __forceinline__ void mma_commit_pair(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+      " [%0], %1;" ::"r"(smem_u32(bar)),
+      "h"((uint16_t)3)
+      : "memory");
+}
+__host__ __device__ constexpr uint32_t idesc_bf16_pair(int n) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(256 >> 4) << 24);
+}
+// MMA width of a pair unit: token rows rounded up to 32 (16 per CTA), at most 256.
+__device__ __forceinline__ int pair_n(int nrows) { return min(kPairBN, (nrows + 31) & ~31); }
+
+template <int MODE>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreadsTc, 1)
+tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__ CUtensorMap mapA1,
+               const __grid_constant__ CUtensorMap mapB, const TcArgs args) {
+  using C = PairCfg<MODE>;
+  constexpr bool IL = C::kIL;
+  constexpr int S = C::kStages;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  float* xchg = (float*)(smem + S * C::kStageBytes);
+  uint64_t* full = (uint64_t*)(xchg + C::kXchgFloats);
+  uint64_t* empty = full + S;
+  uint64_t* tfull = empty + S;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* mma_done = tempty + 2;
+  uint64_t* xbar = mma_done + 1;
+  uint32_t* tmem_slot = (uint32_t*)(xbar + 4);
+  volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
+
+  const uint32_t rank = cluster_rank();
+  const bool leader = rank == 0;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&tfull[b], 1);
+      mbar_init(&tempty[b], 8);  // the epilogue warps of both CTAs (rank 0's barrier is used)
+    }
+    mbar_init(mma_done, 1);
+    for (int i = 0; i < 4; ++i) mbar_init(&xbar[i], 2);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc_pair(tmem_slot, C::kTmemCols);
+  if (threadIdx.x == 32) {
+    asm volatile("prefetch.tensormap [%0];" ::"l"(&mapA0) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(&mapB) : "memory");
+  }
+  tc_fence_before();
+  cluster_sync_all();  // both CTAs' barriers exist before either signals the other
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  pdl_wait();
+  pdl_launch_dependents();
+
+  const int pair = blockIdx.x >> 1, n_pairs = gridDim.x >> 1;
+  const int total_tiles = args.tile_offs
+                              ? args.tile_offs[args.n_groups]
+                              : args.n_groups * ((args.uniform_rows + kPairBN - 1) / kPairBN);
+  const int units = total_tiles * args.m_tiles * args.n_split;
+  const uint32_t full0 = map_rank(smem_u32(full), 0);      // rank 0's full[0]
+  const uint32_t tempty0 = map_rank(smem_u32(tempty), 0);  // rank 0's tempty[0]
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------------------------------------------------- TMA producer (both CTAs)
+      int stage = 0;
+      uint32_t phase = 0;
+      long long issued = 0;
+      bool ok = true;
+      for (int u = pair; u < units && ok; u += n_pairs) {
+        const Unit w = decode_unit<kPairBN>(args, u);
+        const int n = pair_n(w.nrows);
+        const int a_row = w.g * args.a_rows_per_group + w.m0 + (int)rank * C::kFeat;
+        const int b_row = w.slot0 - w.g * args.b_shift_per_group + (int)rank * (n / 2);
+        for (int kb = w.kb0; kb < w.kb1; ++kb) {
+          if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, args.err, 1u, true)) {
+            ok = false;
+            break;
+          }
+          uint8_t* st = smem + stage * C::kStageBytes;
+          const uint32_t fb = full0 + 8u * (uint32_t)stage;
+          if (leader) mbar_expect_tx(&full[stage], 2 * C::kStageBytes);
+          if (IL) {
+            tma_load_2d_pair(st, &mapA0, fb, kb * kBK, a_row);
+            tma_load_2d_pair(st + C::kABytes / 2, &mapA1, fb, kb * kBK, a_row);
+          } else {
+            tma_load_2d_pair(st, &mapA0, fb, kb * kBK, a_row);
+          }
+          tma_load_2d_pair(st + C::kABytes, &mapB, fb, kb * kBK, b_row);
+          ++issued;
+          if (++stage == S) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      // rank 0: let the copies of both CTAs still in flight land before the pair may exit
+      if (leader) {
+        const long long first = issued > S ? issued - S : 0;
+        for (long long i = first; i < issued; ++i)
+          mbar_wait(&full[i % S], (uint32_t)((i / S) & 1), abort_flag, args.err, 2u, false);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && leader) {
+      // ---------------------------------------------------------- MMA issuer (rank 0)
+      int stage = 0;
+      uint32_t phase = 0;
+      int local = 0;
+      bool ok = true;
+      for (int u = pair; u < units && ok; u += n_pairs, ++local) {
+        const Unit w = decode_unit<kPairBN>(args, u);
+        const int buf = local & 1;
+        const uint32_t tph = (uint32_t)((local >> 1) & 1);
+        if (!mbar_wait(&tempty[buf], tph ^ 1u, abort_flag, args.err, 4u, true)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d0 = tmem_base + (uint32_t)(buf * C::kAccCols);
+        const uint32_t idesc = idesc_bf16_pair(pair_n(w.nrows));
+        for (int kb = w.kb0; kb < w.kb1; ++kb) {
+          if (!mbar_wait(&full[stage], phase, abort_flag, args.err, 8u, true)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(smem + stage * C::kStageBytes);
+          const uint32_t sb = sa + C::kABytes;
+#pragma unroll
+          for (int k = 0; k < kBK / 16; ++k)
+            mma_bf16_pair(d0, sdesc_k128(sa + k * 32), sdesc_k128(sb + k * 32), idesc,
+                          (kb > w.kb0 || k > 0) ? 1u : 0u);
+          mma_commit_pair(&empty[stage]);
+          if (++stage == S) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        mma_commit_pair(&tfull[buf]);
+      }
+      // no MMA may still be running when either CTA frees its TMEM
+      mma_commit_pair(mma_done);
+    }
+    if (lane == 0) mbar_wait(mma_done, 0u, abort_flag, args.err, 16u, false);
+  } else if (IL) {
+    // ---------------------------------------- epilogue, interleaved gate/up (warps 2..5)
+    const int q = warp & 3;
+    const int half = q & 1;
+    const bool is_gate = q < 2;
+    float* xh = xchg + half * (2 * 2 * 16 * 32);
+    uint64_t* xb = xbar + half * 2;
+    int local = 0;
+    long long chunk = 0;
+    bool ok = true;
+    for (int u = pair; u < units && ok; u += n_pairs, ++local) {
+      const Unit w = decode_unit<kPairBN>(args, u);
+      const int buf = local & 1;
+      const uint32_t tph = (uint32_t)((local >> 1) & 1);
+      if (!mbar_wait(&tfull[buf], tph, abort_flag, args.err, 32u, true)) break;
+      tc_fence_after();
+      const uint32_t tbase =
+          tmem_base + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * C::kAccCols);
+      const int f = w.m0 + (int)rank * C::kFeat + 32 * half + lane;
+      const bool fok = f < args.M;
+      const int keep = is_gate ? 0 : 16;
+      for (int c0 = 0; c0 < kPairBN && c0 < w.nrows; c0 += 32, ++chunk) {
+        uint32_t v0[16], v1[16];
+        tmem_ld16(tbase + c0, v0);
+        tmem_ld16(tbase + c0 + 16, v1);
+        tmem_wait_ld();
+        const int b = (int)(chunk & 1);
+        float* mine_out = xh + (b * 2 + (is_gate ? 0 : 1)) * 512;
+        const float* theirs = xh + (b * 2 + (is_gate ? 1 : 0)) * 512;
+        if (is_gate) {
+#pragma unroll
+          for (int j = 0; j < 16; ++j) mine_out[j * 32 + lane] = __uint_as_float(v1[j]);
+        } else {
+#pragma unroll
+          for (int j = 0; j < 16; ++j) mine_out[j * 32 + lane] = __uint_as_float(v0[j]);
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&xb[b]);
+        if (!mbar_wait(&xb[b], (uint32_t)((chunk >> 1) & 1), abort_flag, args.err, 128u, true)) {
+          ok = false;
+          break;
+        }
+        if (fok) {
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            const int col = c0 + keep + j;
+            if (col < w.nrows) {
+              const float o = theirs[j * 32 + lane];
+              const float m = __uint_as_float(is_gate ? v0[j] : v1[j]);
+              const float h = is_gate ? silu_f(m) * o : silu_f(o) * m;
+              ((__nv_bfloat16*)args.out)[(size_t)(w.slot0 + col) * args.M + f] =
+                  __float2bfloat16_rn(h);
+            }
+          }
+        }
+      }
+      if (!ok) break;
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) {
+        if (leader) mbar_arrive(&tempty[buf]);
+        else mbar_arrive_cluster(tempty0 + 8u * (uint32_t)buf);
+      }
+    }
+  } else {
+    // ---------------------------------------------------- epilogue, down projection (warps 2..5)
+    const int q = warp & 3;
+    int local = 0;
+    for (int u = pair; u < units; u += n_pairs, ++local) {
+      const Unit w = decode_unit<kPairBN>(args, u);
+      const int buf = local & 1;
+      const uint32_t tph = (uint32_t)((local >> 1) & 1);
+      if (!mbar_wait(&tfull[buf], tph, abort_flag, args.err, 32u, true)) break;
+      tc_fence_after();
+      const uint32_t tbase =
+          tmem_base + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * C::kAccCols);
+      const int f = w.m0 + (int)rank * C::kFeat + 32 * q + lane;
+      const bool fok = f < args.M;
+      for (int c0 = 0; c0 < kPairBN && c0 < w.nrows; c0 += 16) {
+        uint32_t g[16];
+        tmem_ld16(tbase + c0, g);
+        tmem_wait_ld();
+        if (fok) {
+#pragma unroll
+          for (int c = 0; c < 16; ++c) {
+            if (c0 + c < w.nrows) {
+              const size_t slot = (size_t)(w.slot0 + c0 + c);
+              if (args.out_bf16)
+                ((__nv_bfloat16*)args.out)[slot * args.M + f] =
+                    __float2bfloat16_rn(__uint_as_float(g[c]));
+              else
+                ((float*)args.out)[(size_t)w.split * args.split_stride + slot * args.M + f] =
+                    __uint_as_float(g[c]);
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) {
+        if (leader) mbar_arrive(&tempty[buf]);
+        else mbar_arrive_cluster(tempty0 + 8u * (uint32_t)buf);
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();  // neither CTA leaves while the other may still signal it
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc_pair(tmem_base, C::kTmemCols);
 }
 
 // Xperm[slot] = x[perm_tok[slot]] for every slot of the call (16-byte copies).
@@ -562,6 +999,7 @@ bool encode_2d(CUtensorMap* m, const void* ptr, long long rows, long long cols, 
 
 struct Maps {
   CUtensorMap wg, wu, wd, wsg, wsu, wsd;
+  CUtensorMap wg64, wu64, wsg64, wsu64;  // 64-row boxes for the interleaved gate/up A tile
   CUtensorMap xperm[kNumBN], act[kNumBN], sact[kNumBN];
 };
 
@@ -571,44 +1009,95 @@ int bn_index(int bn) {
   return kNumBN - 1;
 }
 
-template <int BN, bool GATEUP>
+template <int BN, int MODE>
 cudaError_t launch_tc(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& b,
                       const TcArgs& args, int grid, cudaStream_t st) {
-  using C = Cfg<BN, GATEUP>;
+  using C = Cfg<BN, MODE>;
   static std::once_flag once;
   static cudaError_t attr_err = cudaSuccess;
   std::call_once(once, [] {
-    attr_err = cudaFuncSetAttribute(tc_ffn_kernel<BN, GATEUP>,
+    attr_err = cudaFuncSetAttribute(tc_ffn_kernel<BN, MODE>,
                                     cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
   });
   if (attr_err != cudaSuccess) return attr_err;
   if (grid <= 0) return cudaSuccess;
-  return launch_pdl(tc_ffn_kernel<BN, GATEUP>, dim3(grid), dim3(kThreadsTc), C::kSmemBytes, st,
+  return launch_pdl(tc_ffn_kernel<BN, MODE>, dim3(grid), dim3(kThreadsTc), C::kSmemBytes, st,
                     a0, a1, b, args);
 }
 
-template <bool GATEUP>
-cudaError_t launch_bn(int bn, const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& b,
-                      const TcArgs& args, int grid, cudaStream_t st) {
+// SM-pair kernels: one 2-CTA cluster per pair of SMs, at most as many pairs as can be resident.
+template <int MODE>
+cudaError_t launch_pair(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& b,
+                        const TcArgs& args, long long units, int num_sms, cudaStream_t st) {
+  using C = PairCfg<MODE>;
+  static std::once_flag once;
+  static cudaError_t attr_err = cudaSuccess;
+  static int max_pairs = 0;
+  std::call_once(once, [num_sms] {
+    attr_err = cudaFuncSetAttribute(tc_pair_kernel<MODE>,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
+    if (attr_err != cudaSuccess) return;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(num_sms & ~1);
+    cfg.blockDim = dim3(kThreadsTc);
+    cfg.dynamicSmemBytes = C::kSmemBytes;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = 2;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, tc_pair_kernel<MODE>, &cfg) != cudaSuccess || n <= 0) {
+      cudaGetLastError();
+      n = num_sms / 2;
+    }
+    max_pairs = std::min(n, num_sms / 2);
+  });
+  if (attr_err != cudaSuccess) return attr_err;
+  const long long pairs = std::min<long long>(max_pairs, units);
+  if (pairs <= 0) return cudaSuccess;
+  return launch_pdl(tc_pair_kernel<MODE>, dim3((unsigned)(2 * pairs)), dim3(kThreadsTc),
+                    C::kSmemBytes, st, a0, a1, b, args);
+}
+
+// Gate/up: 256-token tiles run interleaved; narrower tiles keep the two accumulators.
+cudaError_t launch_up_bn(int bn, const CUtensorMap& a0, const CUtensorMap& a1,
+                         const CUtensorMap& b, const TcArgs& args, int grid, cudaStream_t st) {
   switch (bn) {
-    case 16: return launch_tc<16, GATEUP>(a0, a1, b, args, grid, st);
-    case 32: return launch_tc<32, GATEUP>(a0, a1, b, args, grid, st);
-    case 64: return launch_tc<64, GATEUP>(a0, a1, b, args, grid, st);
-    case 128: return launch_tc<128, GATEUP>(a0, a1, b, args, grid, st);
-    default: return launch_tc<256, GATEUP>(a0, a1, b, args, grid, st);
+    case 16: return launch_tc<16, kModeGateUp>(a0, a1, b, args, grid, st);
+    case 32: return launch_tc<32, kModeGateUp>(a0, a1, b, args, grid, st);
+    case 64: return launch_tc<64, kModeGateUp>(a0, a1, b, args, grid, st);
+    case 128: return launch_tc<128, kModeGateUp>(a0, a1, b, args, grid, st);
+    default: return launch_tc<256, kModeGateUpIL>(a0, a1, b, args, grid, st);
+  }
+}
+
+cudaError_t launch_down_bn(int bn, const CUtensorMap& a0, const CUtensorMap& b,
+                           const TcArgs& args, int grid, cudaStream_t st) {
+  switch (bn) {
+    case 16: return launch_tc<16, kModeDown>(a0, a0, b, args, grid, st);
+    case 32: return launch_tc<32, kModeDown>(a0, a0, b, args, grid, st);
+    case 64: return launch_tc<64, kModeDown>(a0, a0, b, args, grid, st);
+    case 128: return launch_tc<128, kModeDown>(a0, a0, b, args, grid, st);
+    default: return launch_tc<256, kModeDown>(a0, a0, b, args, grid, st);
   }
 }
 
 }  // namespace
 
-// The largest group of a call has at most T rows (each token picks an expert once).  In large
-// calls the down projection takes 256-token tiles (M = 128 x N = 256 MMAs read 25% fewer shared-
-// memory operand bytes per flop than N = 128; measured 1.3-1.5x faster); the gate/up kernel keeps
-// 128 (its two accumulators of 256 columns would leave no second TMEM buffer).
+// The largest group of a call has at most T rows (each token picks an expert once).  Calls of at
+// least kPairMinTokens run both expert GEMMs on SM pairs with 256-token tiles (interleaved gate/
+// up, 256-feature down tiles); smaller calls use single-SM kernels with tiles of the smallest
+// width that holds T, at most 128.  (On a single SM the interleaved 256-token gate/up moves the
+// same shared-memory bytes per flop as two 128-token accumulators and measured slower: OLMoE
+// prefill gate/up 294 -> 316 us.)
+constexpr int kPairMinTokens = 1024;
 int tc_tile_rows(const TcLayer&, int T) {
   for (int i = 0; i < 4; ++i)
     if (T <= kBNs[i]) return kBNs[i];
-  return 128;
+  return T >= kPairMinTokens ? kPairBN : 128;
 }
 // Small calls gather their token rows inside the gate/up kernel (one launch and one HBM round
 // trip fewer); large calls copy them to Xperm first: there the shared-memory-bound gate/up kernel
@@ -618,7 +1107,7 @@ bool tc_gathers_in_kernel(const TcLayer&, int T) { return T <= 128; }
 int tc_tile_rows_down(const TcLayer&, int T) {
   for (int i = 0; i < 4; ++i)
     if (T <= kBNs[i]) return kBNs[i];
-  return T >= 2048 ? 256 : 128;
+  return T >= kPairMinTokens ? kPairBN : 128;
 }
 
 // Split-K of the routed down projection: enough work units for ~8 waves of the persistent grid
@@ -688,10 +1177,14 @@ int tc_bind(TcLayer& L, const eat_layer_desc& D, void* xperm, void* act, void* s
   const long long rows = (long long)L.Tmax * L.K;
   bool ok = encode_2d(&m->wg, D.w_gate, (long long)L.E * L.F, L.d, kBM) &&
             encode_2d(&m->wu, D.w_up, (long long)L.E * L.F, L.d, kBM) &&
+            encode_2d(&m->wg64, D.w_gate, (long long)L.E * L.F, L.d, kBM / 2) &&
+            encode_2d(&m->wu64, D.w_up, (long long)L.E * L.F, L.d, kBM / 2) &&
             encode_2d(&m->wd, D.w_down, (long long)L.E * L.d, L.F, kBM);
   if (ok && L.S > 0)
     ok = encode_2d(&m->wsg, D.ws_gate, (long long)L.S * L.Fs, L.d, kBM) &&
          encode_2d(&m->wsu, D.ws_up, (long long)L.S * L.Fs, L.d, kBM) &&
+         encode_2d(&m->wsg64, D.ws_gate, (long long)L.S * L.Fs, L.d, kBM / 2) &&
+         encode_2d(&m->wsu64, D.ws_up, (long long)L.S * L.Fs, L.d, kBM / 2) &&
          encode_2d(&m->wsd, D.ws_down, (long long)L.S * L.d, L.Fs, kBM);
   for (int i = 0; i < kNumBN && ok; ++i) {
     ok = encode_2d(&m->xperm[i], xperm, rows, L.d, kBNs[i]) &&
@@ -726,6 +1219,7 @@ cudaError_t tc_launch_up(const TcLayer& L, const TcCall& c, bool shared, cudaStr
   TcArgs a;
   std::memset(&a, 0, sizeof(a));
   const int bn = c.tile_rows;
+  const bool pair = bn == kPairBN;  // SM pairs, interleaved gate/up: 128 features per unit
   a.M = shared ? L.Fs : L.F;
   a.m_tile = kBM;
   a.m_tiles = (a.M + a.m_tile - 1) / a.m_tile;
@@ -737,15 +1231,17 @@ cudaError_t tc_launch_up(const TcLayer& L, const TcCall& c, bool shared, cudaStr
   long long max_tiles;
   if (shared) {
     CUtensorMap xm;
-    if (!encode_2d(&xm, c.x, c.T, L.d, bn)) return cudaErrorInvalidValue;
+    if (!encode_2d(&xm, c.x, c.T, L.d, pair ? kPairRows : bn)) return cudaErrorInvalidValue;
     a.n_groups = L.S;
     a.uniform_rows = c.T;
     a.b_shift_per_group = c.T;
     a.out = c.sact;
     max_tiles = (long long)L.S * ((c.T + bn - 1) / bn);
     const long long units = max_tiles * a.m_tiles;
+    if (pair)
+      return launch_pair<kModeGateUpIL>(m->wsg64, m->wsu64, xm, a, units, L.num_sms, st);
     const int grid = (int)std::min<long long>(L.num_sms, units);
-    return launch_bn<true>(bn, m->wsg, m->wsu, xm, a, grid, st);
+    return launch_up_bn(bn, m->wsg, m->wsu, xm, a, grid, st);
   }
   a.n_groups = L.E;
   a.row_offs = c.offs;
@@ -758,9 +1254,12 @@ cudaError_t tc_launch_up(const TcLayer& L, const TcCall& c, bool shared, cudaStr
     // small call: the token rows are gathered from x inside the kernel
     a.b_rows = c.perm_tok;
     a.bx = (const __nv_bfloat16*)c.x;
-    return launch_bn<true>(bn, m->wg, m->wu, m->wg, a, grid, st);
+    return launch_up_bn(bn, m->wg, m->wu, m->wg, a, grid, st);
   }
-  return launch_bn<true>(bn, m->wg, m->wu, m->xperm[bn_index(bn)], a, grid, st);
+  if (pair)
+    return launch_pair<kModeGateUpIL>(m->wg64, m->wu64, m->xperm[bn_index(kPairRows)], a, units,
+                                      L.num_sms, st);
+  return launch_up_bn(bn, m->wg, m->wu, m->xperm[bn_index(bn)], a, grid, st);
 }
 
 cudaError_t tc_launch_down(const TcLayer& L, const TcCall& c, bool shared, int n_split,
@@ -769,10 +1268,11 @@ cudaError_t tc_launch_down(const TcLayer& L, const TcCall& c, bool shared, int n
   TcArgs a;
   std::memset(&a, 0, sizeof(a));
   const int bn = c.tile_rows_down;
+  const bool pair = bn == kPairBN;  // SM pairs: 256 output features per unit
   const int Kdim = shared ? L.Fs : L.F;
   a.M = L.d;
-  a.m_tile = kBM;
-  a.m_tiles = (L.d + kBM - 1) / kBM;
+  a.m_tile = pair ? 2 * kBM : kBM;
+  a.m_tiles = (L.d + a.m_tile - 1) / a.m_tile;
   a.kblocks = Kdim / kBK;
   a.n_split = n_split;
   a.kb_per_split = (a.kblocks + n_split - 1) / n_split;
@@ -787,8 +1287,11 @@ cudaError_t tc_launch_down(const TcLayer& L, const TcCall& c, bool shared, int n
     a.split_stride = 0;
     max_tiles = (long long)L.S * ((c.T + bn - 1) / bn);
     const long long units = max_tiles * a.m_tiles;
+    if (pair)
+      return launch_pair<kModeDown>(m->wsd, m->wsd, m->sact[bn_index(kPairRows)], a, units,
+                                    L.num_sms, st);
     const int grid = (int)std::min<long long>(L.num_sms, units);
-    return launch_bn<false>(bn, m->wsd, m->wsd, m->sact[bn_index(bn)], a, grid, st);
+    return launch_down_bn(bn, m->wsd, m->sact[bn_index(bn)], a, grid, st);
   }
   a.n_groups = L.E;
   a.row_offs = c.offs;
@@ -798,8 +1301,11 @@ cudaError_t tc_launch_down(const TcLayer& L, const TcCall& c, bool shared, int n
   a.split_stride = (long long)c.T * L.K * L.d;
   max_tiles = (long long)(c.T * L.K + bn - 1) / bn + L.E;
   const long long units = max_tiles * a.m_tiles * n_split;
+  if (pair)
+    return launch_pair<kModeDown>(m->wd, m->wd, m->act[bn_index(kPairRows)], a, units, L.num_sms,
+                                  st);
   const int grid = (int)std::min<long long>(L.num_sms, units);
-  return launch_bn<false>(bn, m->wd, m->wd, m->act[bn_index(bn)], a, grid, st);
+  return launch_down_bn(bn, m->wd, m->act[bn_index(bn)], a, grid, st);
 }
 
 cudaError_t tc_selftest_bounded_wait(unsigned long long limit_ns, unsigned int* dev_status,
