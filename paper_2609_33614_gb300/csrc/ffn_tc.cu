@@ -609,12 +609,15 @@ struct PairCfg {
   static constexpr int kBBytes = kPairRows * kBK * 2;
   static constexpr int kStageBytes = kABytes + kBBytes;
   static constexpr int kXchgFloats = kIL ? 2 * 2 * 2 * 16 * 32 : 0;
-  static constexpr int kStagesRaw = (kSmemBudget - 2048 - kXchgFloats * 4) / kStageBytes;
+  // the whole 227 KB a CTA may hold: 1 KB of alignment slack and 256 B of barriers besides the
+  // stages (seven for the down projection, six beside the gate/up exchange buffers)
+  static constexpr int kStagesRaw = (227 * 1024 - 1024 - 256 - kXchgFloats * 4) / kStageBytes;
   static constexpr int kStages = kStagesRaw > 8 ? 8 : kStagesRaw;
   static constexpr int kAccCols = kPairBN;
   static constexpr int kTmemCols = 512;
   static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kXchgFloats * 4 + 256;
   static constexpr int kFeat = kIL ? 64 : 128;  // output features of one CTA in a unit
+  static_assert(kSmemBytes <= 227 * 1024, "shared memory of one CTA");
 };
 
 __device__ __forceinline__ uint32_t cluster_rank() {
