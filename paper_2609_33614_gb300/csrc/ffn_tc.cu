@@ -5,7 +5,8 @@
 //
 // Orientation ("swap AB"): a tile is 128 weight rows (output features of one expert) x BN tokens
 // (16..128 rows of that expert's slot list), so decode calls with a handful of tokens still issue
-// full M = 128 MMAs and simply stream the activated experts' weights; prefill calls use BN = 128.
+// full M = 128 MMAs and simply stream the activated experts' weights.  Calls of 1024 tokens or more
+// run on SM pairs instead (tc_pair_kernel below: M = 256 weight rows x 256 tokens per MMA).
 //   gate/up kernel: D_gate = Wg[e, f0:f0+128, :] . Xperm[slots]^T and D_up likewise, both in TMEM;
 //       the epilogue writes act[slot, f] = silu(D_gate) * D_up in bf16 (fp32 accumulation).
 //   down kernel:    D = Wd[e, c0:c0+128, :] . act[slots]^T over a K slice: with split-K (decode)
@@ -33,8 +34,8 @@ namespace {
 constexpr int kBM = 128;                  // weight rows per tile (MMA M)
 constexpr int kBK = 64;                   // 64 bf16 = 128 B: one 128B-swizzle row
 constexpr int kThreadsTc = 192;           // 6 warps
-constexpr int kNumBN = 5;
-constexpr int kBNs[kNumBN] = {16, 32, 64, 128, 256};
+constexpr int kNumBN = 4;
+constexpr int kBNs[kNumBN] = {16, 32, 64, 128};  // single-SM token tiles; SM pairs load 128 per CTA
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;
 constexpr int kSmemBudget = 220 * 1024;
 
@@ -169,26 +170,25 @@ __host__ __device__ constexpr int tmem_cols_for(int c) {
 }
 
 // Kernel modes: the down projection (one A tile, plain epilogue); gate/up with two accumulators
-// (gate and up A tiles of 128 rows against one B tile); gate/up interleaved (one A tile of 64 gate
-// rows over 64 up rows of the same features, one accumulator: an M = 128 x N = BN MMA covers both
-// projections of 64 features, and the epilogue pairs the gate and up warps of each feature).
+// (gate and up A tiles of 128 rows against one B tile, single-SM kernel); gate/up interleaved (one
+// A tile of 64 gate rows over the 64 up rows of the same features, one accumulator: an MMA covers
+// both projections of 64 features, and the epilogue pairs the gate and up warps of each feature;
+// SM-pair kernel).
 enum : int { kModeDown = 0, kModeGateUp = 1, kModeGateUpIL = 2 };
 
 template <int BN, int MODE>
 struct Cfg {
-  static constexpr bool kGateUp = MODE != kModeDown;
-  static constexpr bool kIL = MODE == kModeGateUpIL;
-  static constexpr int kNA = MODE == kModeGateUp ? 2 : 1;
+  static_assert(MODE == kModeDown || MODE == kModeGateUp, "single-SM kernel modes");
+  static constexpr bool kGateUp = MODE == kModeGateUp;
+  static constexpr int kNA = kGateUp ? 2 : 1;
   static constexpr int kABytes = kBM * kBK * 2;
   static constexpr int kBBytes = BN * kBK * 2;
   static constexpr int kStageBytes = kNA * kABytes + kBBytes;
-  // interleaved epilogue exchange: [2 pairs][2 buffers][2 directions][16 columns][32 lanes] fp32
-  static constexpr int kXchgFloats = kIL ? 2 * 2 * 2 * 16 * 32 : 0;
-  static constexpr int kStagesRaw = (kSmemBudget - 2048 - kXchgFloats * 4) / kStageBytes;
+  static constexpr int kStagesRaw = (kSmemBudget - 2048) / kStageBytes;
   static constexpr int kStages = kStagesRaw > 12 ? 12 : kStagesRaw;
   static constexpr int kAccCols = kNA * BN;
   static constexpr int kTmemCols = tmem_cols_for(2 * kAccCols);
-  static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + kXchgFloats * 4 + 256;
+  static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + 256;
   static_assert(2 * kAccCols <= 512, "two accumulator buffers must fit in TMEM");
 };
 
@@ -261,18 +261,15 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
               const __grid_constant__ CUtensorMap mapB, const TcArgs args) {
   using C = Cfg<BN, MODE>;
   constexpr bool GATEUP = C::kGateUp;
-  constexpr bool IL = C::kIL;
   constexpr int S = C::kStages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  float* xchg = (float*)(smem + S * C::kStageBytes);
-  uint64_t* full = (uint64_t*)(xchg + C::kXchgFloats);
+  uint64_t* full = (uint64_t*)(smem + S * C::kStageBytes);
   uint64_t* empty = full + S;
   uint64_t* tfull = empty + S;
   uint64_t* tempty = tfull + 2;
   uint64_t* mma_done = tempty + 2;
-  uint64_t* xbar = mma_done + 1;  // [2 pairs][2 buffers], interleaved epilogue exchange
-  uint32_t* tmem_slot = (uint32_t*)(xbar + 4);
+  uint32_t* tmem_slot = (uint32_t*)(mma_done + 1);
   volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -286,7 +283,6 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
       mbar_init(&tempty[b], 4);
     }
     mbar_init(mma_done, 1);
-    for (int i = 0; i < 4; ++i) mbar_init(&xbar[i], 2);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -303,16 +299,10 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
   pdl_wait();
   pdl_launch_dependents();
 
-  // A tile of one k-block: one 128-row box (or the gate and up boxes of the two-accumulator
-  // mode), or in the interleaved mode 64 gate rows over the 64 up rows of the same features
+  // A tiles of one k-block: one 128-row box, or the gate and up boxes of the two accumulators
   auto load_a = [&](uint8_t* st, uint64_t* bar, int kb, int a_row) {
-    if (IL) {
-      tma_load_2d(st, &mapA0, bar, kb * kBK, a_row);
-      tma_load_2d(st + C::kABytes / 2, &mapA1, bar, kb * kBK, a_row);
-    } else {
-      tma_load_2d(st, &mapA0, bar, kb * kBK, a_row);
-      if (GATEUP) tma_load_2d(st + C::kABytes, &mapA1, bar, kb * kBK, a_row);
-    }
+    tma_load_2d(st, &mapA0, bar, kb * kBK, a_row);
+    if (GATEUP) tma_load_2d(st + C::kABytes, &mapA1, bar, kb * kBK, a_row);
   };
 
   const int total_tiles = args.tile_offs
@@ -472,71 +462,6 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
       // no MMA may still be running when TMEM is freed
       mma_commit(mma_done);
       mbar_wait(mma_done, 0u, abort_flag, args.err, 16u, false);
-    }
-  } else if (IL) {
-    // ------------------------------------------ epilogue, interleaved gate/up (warps 2..5)
-    // TMEM lanes 0-63 hold the gate rows and lanes 64-127 the up rows of the tile's 64 features;
-    // a warp may read lane quarter warp % 4, so quarters 0, 1 are gate and 2, 3 up of features
-    // 32 (q % 2) + lane.  The gate and up warps of a feature half trade half of every 32-column
-    // chunk through shared memory (double-buffered, one bounded mbarrier wait per chunk); the
-    // gate warp finishes columns 0-15 of the chunk, the up warp columns 16-31.
-    const int q = warp & 3;
-    const int half = q & 1;
-    const bool is_gate = q < 2;
-    float* xh = xchg + half * (2 * 2 * 16 * 32);
-    uint64_t* xb = xbar + half * 2;
-    int local = 0;
-    long long chunk = 0;
-    bool ok = true;
-    for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++local) {
-      const Unit w = decode_unit<BN>(args, u);
-      const int buf = local & 1;
-      const uint32_t tph = (uint32_t)((local >> 1) & 1);
-      if (!mbar_wait(&tfull[buf], tph, abort_flag, args.err, 32u, true)) break;
-      tc_fence_after();
-      const uint32_t tbase = tmem_base + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * C::kAccCols);
-      const int f = w.m0 + 32 * half + lane;
-      const bool fok = f < args.M;
-      const int keep = is_gate ? 0 : 16;  // chunk columns this warp finishes
-      for (int c0 = 0; c0 < BN && c0 < w.nrows; c0 += 32, ++chunk) {
-        uint32_t v0[16], v1[16];
-        tmem_ld16(tbase + c0, v0);
-        tmem_ld16(tbase + c0 + 16, v1);
-        tmem_wait_ld();
-        const int b = (int)(chunk & 1);
-        float* mine_out = xh + (b * 2 + (is_gate ? 0 : 1)) * 512;
-        const float* theirs = xh + (b * 2 + (is_gate ? 1 : 0)) * 512;
-        if (is_gate) {
-#pragma unroll
-          for (int j = 0; j < 16; ++j) mine_out[j * 32 + lane] = __uint_as_float(v1[j]);
-        } else {
-#pragma unroll
-          for (int j = 0; j < 16; ++j) mine_out[j * 32 + lane] = __uint_as_float(v0[j]);
-        }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&xb[b]);
-        if (!mbar_wait(&xb[b], (uint32_t)((chunk >> 1) & 1), abort_flag, args.err, 128u, true)) {
-          ok = false;
-          break;
-        }
-        if (fok) {
-#pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            const int col = c0 + keep + j;
-            if (col < w.nrows) {
-              const float o = theirs[j * 32 + lane];
-              const float m = __uint_as_float(is_gate ? v0[j] : v1[j]);
-              const float h = is_gate ? silu_f(m) * o : silu_f(o) * m;
-              ((__nv_bfloat16*)args.out)[(size_t)(w.slot0 + col) * args.M + f] =
-                  __float2bfloat16_rn(h);
-            }
-          }
-        }
-      }
-      if (!ok) break;
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&tempty[buf]);
     }
   } else {
     // -------------------------------------------------------------- epilogue (warps 2..5)
@@ -1065,15 +990,14 @@ cudaError_t launch_pair(const CUtensorMap& a0, const CUtensorMap& a1, const CUte
                     C::kSmemBytes, st, a0, a1, b, args);
 }
 
-// Gate/up: 256-token tiles run interleaved; narrower tiles keep the two accumulators.
+// Single-SM launches: token tiles of 16..128 rows (256-row tiles run on SM pairs).
 cudaError_t launch_up_bn(int bn, const CUtensorMap& a0, const CUtensorMap& a1,
                          const CUtensorMap& b, const TcArgs& args, int grid, cudaStream_t st) {
   switch (bn) {
     case 16: return launch_tc<16, kModeGateUp>(a0, a1, b, args, grid, st);
     case 32: return launch_tc<32, kModeGateUp>(a0, a1, b, args, grid, st);
     case 64: return launch_tc<64, kModeGateUp>(a0, a1, b, args, grid, st);
-    case 128: return launch_tc<128, kModeGateUp>(a0, a1, b, args, grid, st);
-    default: return launch_tc<256, kModeGateUpIL>(a0, a1, b, args, grid, st);
+    default: return launch_tc<128, kModeGateUp>(a0, a1, b, args, grid, st);
   }
 }
 
@@ -1083,8 +1007,7 @@ cudaError_t launch_down_bn(int bn, const CUtensorMap& a0, const CUtensorMap& b,
     case 16: return launch_tc<16, kModeDown>(a0, a0, b, args, grid, st);
     case 32: return launch_tc<32, kModeDown>(a0, a0, b, args, grid, st);
     case 64: return launch_tc<64, kModeDown>(a0, a0, b, args, grid, st);
-    case 128: return launch_tc<128, kModeDown>(a0, a0, b, args, grid, st);
-    default: return launch_tc<256, kModeDown>(a0, a0, b, args, grid, st);
+    default: return launch_tc<128, kModeDown>(a0, a0, b, args, grid, st);
   }
 }
 
