@@ -184,6 +184,24 @@ def test_expert_counts_and_max_k(E, K, T):
     run_parity(sh, lw, [T, 1, T // 3])
 
 
+@pytest.mark.parametrize("E,K,T", [(256, 8, 1500), (64, 2, 1100)])
+def test_sm_pair_small_groups(E, K, T):
+    """Calls of >= 1024 tokens run the SM-pair GEMMs; with many experts nearly every group is a
+    partial 256-token tile (MMA widths of 32..224, one CTA's half of the tile empty or partial),
+    and the all-tokens-one-expert call below makes one group span several full tiles."""
+    sh = W.scaled(W.OLMOE, f"pair{E}", d_model=256, n_experts=E, d_ff=384, max_k=K)
+    lw = W.make_layer(sh)
+    run_parity(sh, lw, [T, T])
+
+
+def test_sm_pair_one_large_group():
+    """One expert takes every token of a 2100-token call: 8 full SM-pair tiles and a partial one."""
+    lw = W.make_layer(OLMOE_S)
+    lw.b_router = torch.full_like(lw.b_router, -30.0)
+    lw.b_router[7] = 30.0
+    run_parity(OLMOE_S, lw, [2100])
+
+
 def test_partial_feature_tiles():
     """d = 320 and d_ff = 192: feature tiles of 128 end half-full in both expert GEMMs."""
     sh = W.scaled(W.QWEN, "ragged-d", d_model=320, n_experts=16, d_ff=192, n_shared=1,
