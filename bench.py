@@ -214,15 +214,16 @@ def kernel_flops(kind, shape, acts, T):
 
 def traffic_for(kind, workload, experts_per_launch):
     """DRAM bytes per launch from the committed ncu summary (profiles/traffic.json), if it was
-    taken on the current kernel sources (its source hash matches); else None.  Decode captures are
-    stored per activated expert and scaled by this run's mean activated experts per launch."""
+    taken on the current FFN kernel sources (its source hash equals build.ffn_source_hash());
+    else None.  Decode captures are stored per activated expert and scaled by this run's mean
+    activated experts per launch."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         from paper_2609_33614_gb300 import build
         with open(path) as fh:
             tr = json.load(fh)
         ent = tr.get(workload, {}).get(kind)
-        if ent and ent.get("source_hash") == build._stamp():
+        if ent and ent.get("source_hash") == build.ffn_source_hash():
             if "dram_bytes_per_expert" in ent:
                 return ent["dram_bytes_per_expert"] * experts_per_launch
             return ent["dram_bytes_per_launch"]

@@ -43,6 +43,21 @@ def _stamp() -> str:
     return h.hexdigest()
 
 
+# Sources that define the tensor-core FFN kernels: a DRAM-traffic capture of those kernels stays
+# valid while these files are unchanged (the rest of the library does not touch their code).
+FFN_SOURCES = ("ffn_tc.cu", "ffn_tc.cuh")
+
+
+def ffn_source_hash() -> str:
+    h = hashlib.sha256()
+    for name in FFN_SOURCES:
+        with open(os.path.join(CSRC, name), "rb") as fh:
+            h.update(name.encode())
+            h.update(fh.read())
+    h.update(" ".join(ARCH + FLAGS).encode())
+    return h.hexdigest()
+
+
 def build(verbose: bool = False, force: bool = False) -> str:
     """Compile and link libeat.so; returns its path."""
     os.makedirs(BUILD, exist_ok=True)
