@@ -49,12 +49,15 @@ FFN_SOURCES = ("ffn_tc.cu", "ffn_tc.cuh")
 
 
 def ffn_source_hash() -> str:
+    """Hash of the FFN kernel sources and the compile flags, independent of where the repository
+    lives (the include path enters relative to the repository root)."""
     h = hashlib.sha256()
     for name in FFN_SOURCES:
         with open(os.path.join(CSRC, name), "rb") as fh:
             h.update(name.encode())
             h.update(fh.read())
-    h.update(" ".join(ARCH + FLAGS).encode())
+    flags = [os.path.relpath(f, ROOT) if os.path.isabs(f) else f for f in ARCH + FLAGS]
+    h.update(" ".join(flags).encode())
     return h.hexdigest()
 
 
