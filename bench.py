@@ -50,6 +50,13 @@ def workload_spec(name):
                               desc="deepseek-v2-lite-shaped 26-layer MoE stack, prefill 16384"),
         "dsv2l-decode": dict(shape=W.DSV2L, batches=[128], layers=26,
                              desc="deepseek-v2-lite-shaped 26-layer MoE stack, decode batch 128"),
+        # e4m3 expert weights with per-row scales (hidden states bf16, expert GEMMs fp16 x fp16)
+        "mixtral-decode-fp8": dict(shape=W.MIXTRAL, batches=[1, 16, 64], layers=1, fp8=True,
+                                   desc="mixtral-8x7b-shaped MoE layer, e4m3 expert weights, "
+                                        "decode, batch 1+16+64 per step"),
+        "olmoe-decode-fp8": dict(shape=W.OLMOE, batches=[32], layers=1, fp8=True,
+                                 desc="olmoe-shaped MoE layer, e4m3 expert weights, decode "
+                                      "batch 32 per step"),
     }
     return specs[name]
 
@@ -60,6 +67,8 @@ def bench_config(args, spec):
     cfg = {"workload": spec["desc"], "router": args.router, "cuda_graph": args.graph}
     if args.router == "topp":
         cfg["top_p"] = args.top_p
+    if spec.get("fp8"):
+        cfg["expert_weights"] = "e4m3, fp32 scale per row (fp16 x fp16 -> fp32 GEMMs)"
     cfg.update({"d_model": shape.d_model, "n_experts": shape.n_experts, "d_ff": shape.d_ff,
                 "n_shared": shape.n_shared, "max_k": shape.max_k, "layers": spec["layers"],
                 "batches": spec["batches"],
@@ -182,20 +191,22 @@ def sum_over_ranks(value, world):
 
 
 # ------------------------------------------------------------------------------- roofline
-def kernel_bytes(kind, shape, union, acts, T):
-    """Algorithmic HBM bytes of one launch: weights of the activated experts plus the
-    activation rows the kernel must read and write (bf16 = 2 B, fp32 partials = 4 B)."""
+def kernel_bytes(kind, shape, union, acts, T, fp8=False):
+    """Algorithmic HBM bytes of one launch: weights of the activated experts (bf16 2 B, or e4m3
+    1 B plus a 4 B scale per row) plus the activation rows the kernel must read and write
+    (16-bit = 2 B, fp32 partials = 4 B)."""
     d, F = shape.d_model, shape.d_ff
+    wb = 1 if fp8 else 2
+    rs = 4 if fp8 else 0  # scale bytes per weight row
+    Fs = shape.d_ff_shared
     if kind == "ffn_up":
-        return union * 2 * F * d * 2 + acts * d * 2 + acts * F * 2
+        return union * 2 * F * (d * wb + rs) + acts * d * 2 + acts * F * 2
     if kind == "ffn_down":
-        return union * d * F * 2 + acts * F * 2 + acts * d * 4
+        return union * d * (F * wb + rs) + acts * F * 2 + acts * d * 4
     if kind == "shared_up":
-        return shape.n_shared * 2 * shape.d_ff_shared * d * 2 + T * d * 2 + \
-            shape.n_shared * T * shape.d_ff_shared * 2
+        return shape.n_shared * 2 * Fs * (d * wb + rs) + T * d * 2 + shape.n_shared * T * Fs * 2
     if kind == "shared_down":
-        return shape.n_shared * d * shape.d_ff_shared * 2 + \
-            shape.n_shared * T * (shape.d_ff_shared * 2 + d * 4)
+        return shape.n_shared * d * (Fs * wb + rs) + shape.n_shared * T * (Fs * 2 + d * 4)
     raise KeyError(kind)
 
 
@@ -247,6 +258,8 @@ def run_ours(args, world, rank, local):
 
     # layers (weights drawn on the GPU generator) and one handle per (layer, batch)
     layer_w = [W.make_layer(shape, l, device="cuda") for l in range(n_layers)]
+    if spec.get("fp8"):
+        layer_w = [W.to_fp8(lw) for lw in layer_w]
     handles = []  # [layer][batch]
     mode = {"eat": eat.EAT_ROUTER_EAT, "topk": eat.EAT_ROUTER_TOPK,
             "topp": eat.EAT_ROUTER_TOPP}[args.router]
@@ -367,7 +380,8 @@ def run_ours(args, world, rank, local):
                     k["union"] += n * dU / dC
                 if kind in ("ffn_up", "ffn_down", "shared_up", "shared_down") and n:
                     # per-launch average union / activations of this handle
-                    k["bytes"] += n * kernel_bytes(kind, shape, dU / max(1, dC), dA / max(1, dC), B)
+                    k["bytes"] += n * kernel_bytes(kind, shape, dU / max(1, dC), dA / max(1, dC), B,
+                                                   fp8=bool(spec.get("fp8")))
                     k["flops"] += n * kernel_flops(kind, shape, dA / max(1, dC), B)
     total_kernel_ms = sum(k["ms"] for k in kinds.values())
     dom = max((k for k in kinds if k.startswith("ffn") or k.startswith("shared")),
@@ -416,8 +430,10 @@ def run_ours(args, world, rank, local):
     result = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": job_ms / args.steps,
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-        "data": "synthetic (seeded N(0,1) hidden states, N(0,0.02^2) weights)",
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f16" if spec.get("fp8") else "bf16",
+        "data": "synthetic (seeded N(0,1) hidden states, N(0,0.02^2) weights"
+                + (", quantized to e4m3 per row)" if spec.get("fp8") else ")"),
         "config": bench_config(args, spec),
         "roofline": roof,
         "experts_per_token": acts / max(1, sum(B * args.steps for B in batches) * n_layers),
@@ -438,8 +454,11 @@ def run_ours(args, world, rank, local):
 
 # ------------------------------------------------------------------------------- oracle arm
 def _oracle_layer(lw):
+    """The oracle's fp64 layer (an fp8 layer's dequantized weights: what its GPU path uses)."""
     import torch
     import oracle.eat_oracle as orc
+    if hasattr(lw, "dequantized"):
+        lw = lw.dequantized()
     f = lambda t: None if t is None else t.detach().to("cpu").to(torch.float64).numpy()
     return orc.Layer(f(lw.w_router), f(lw.b_router), f(lw.w_gate), f(lw.w_up), f(lw.w_down),
                      f(lw.ws_gate), f(lw.ws_up), f(lw.ws_down))
@@ -490,6 +509,8 @@ def run_reference(args, world, rank):
     spec = workload_spec(args.workload)
     shape = spec["shape"]
     lw = W.make_layer(shape, 0, device="cuda" if torch.cuda.is_available() else "cpu")
+    if spec.get("fp8"):
+        lw = W.to_fp8(lw)
     # each step: one oracle layer call at batch 1 (bounded so K steps end in minutes)
     bs = [1] if spec["batches"][0] <= 256 else [64]
     import oracle.eat_oracle as orc

@@ -42,7 +42,10 @@ typedef enum eat_status {
   EAT_ERR_STATE = 5         /* handle not usable (e.g. device-side status word set) */
 } eat_status;
 
-typedef enum eat_dtype { EAT_F32 = 0, EAT_BF16 = 1 } eat_dtype;
+/* EAT_FP8_E4M3 is an expert-weight type only (wdtype, with xdtype EAT_BF16): OCP e4m3 bytes with
+ * one fp32 scale per weight row (see eat_layer_desc).  Not from the paper: a storage format that
+ * halves the weight bytes a decode call streams. */
+typedef enum eat_dtype { EAT_F32 = 0, EAT_BF16 = 1, EAT_FP8_E4M3 = 2 } eat_dtype;
 
 /* Expert selection rule.  EAT_ROUTER_EAT: the adaptive threshold of §3.3-§3.4 (Eq. 3-8).  The
  * baselines the paper compares with (§4.1), computed by the same kernels from the same
@@ -97,9 +100,15 @@ eat_status eat_default_params(eat_params* p);
  *   ws_gate, ws_up [S, Fs, d], ws_down [S, d, Fs] in wdtype, all NULL when n_shared == 0
  *   (always-on shared experts, added with weight 1, not routed, no account);
  *   opd_scale [E] fp32 or NULL: OPD inference reweighting (§3.5) -- the routing probabilities
- *   become p'_i = s_i p_i / sum_j s_j p_j before selection, and p' is used everywhere p is.
- * Supported: 1 <= E <= 256; d, F, Fs multiples of 64; (wdtype, xdtype) both EAT_F32 or both
- * EAT_BF16; 1 <= max_tokens <= 65536.  All weight pointers 16-byte aligned. */
+ *   become p'_i = s_i p_i / sum_j s_j p_j before selection, and p' is used everywhere p is;
+ *   w_gate_scale, w_up_scale [E, F], w_down_scale [E, d], ws_gate_scale, ws_up_scale [S, Fs],
+ *   ws_down_scale [S, d] fp32: with wdtype EAT_FP8_E4M3, weight row r of each matrix is
+ *   scale[r] * (its e4m3 bytes) (the shared ones NULL when n_shared == 0); ignored otherwise.
+ * Supported: 1 <= E <= 256; d, F, Fs multiples of 64; (wdtype, xdtype) both EAT_F32, both
+ * EAT_BF16, or EAT_FP8_E4M3 weights with EAT_BF16 hidden states; 1 <= max_tokens <= 65536.  All
+ * weight pointers 16-byte aligned.  fp8 layers compute the expert GEMMs in fp16 x fp16 -> fp32
+ * (the e4m3 values convert exactly; hidden states and SwiGLU activations round to fp16, so
+ * |x| above 65504 overflows) and always use the single-SM kernels. */
 typedef struct eat_layer_desc {
   int32_t d_model, n_experts, d_ff, n_shared, d_ff_shared, max_tokens;
   int32_t wdtype, xdtype;
@@ -112,6 +121,12 @@ typedef struct eat_layer_desc {
   const void* ws_up;
   const void* ws_down;
   const float* opd_scale;
+  const float* w_gate_scale;
+  const float* w_up_scale;
+  const float* w_down_scale;
+  const float* ws_gate_scale;
+  const float* ws_up_scale;
+  const float* ws_down_scale;
 } eat_layer_desc;
 
 typedef struct eat_handle eat_handle;

@@ -17,8 +17,9 @@ struct eat_handle {
   eat_layer_desc desc;
   eat_params prm;
   int E = 0, d = 0, F = 0, S = 0, Fs = 0, Tmax = 0, K = 0;
-  bool bf16 = false;
-  int backend = 0;  // 0 CUDA-core kernels (fp32 layers), 1 tcgen05 kernels (bf16 layers)
+  bool bf16 = false;  // hidden states and outputs in bf16
+  bool w8 = false;    // e4m3 expert weights (tensor-core kernels with fp16 operands)
+  int backend = 0;  // 0 CUDA-core kernels (fp32 layers), 1 tcgen05 kernels (bf16 / fp8 layers)
   size_t elt = 4;
 
   void* mem = nullptr;
@@ -41,6 +42,7 @@ struct eat_handle {
   int nb = 1;                 // column segments per row in the combine kernel
   void* sact = nullptr;   // [S*Tmax, Fs]
   float* sout = nullptr;  // [S*Tmax, d] (fp32; bf16 on the tensor-core path)
+  void* xh = nullptr;     // [Tmax, d] fp16 hidden states of the call (fp8 layers)
   void* xstage = nullptr; // [Tmax, d]
   void* ystage = nullptr; // [Tmax, d]
   void* xperm = nullptr;  // [Tmax*K, d] gathered token rows (tensor-core path)
@@ -178,6 +180,12 @@ eat_status run_forward(eat_handle* h, const void* x, int T, int ppl_sign, void* 
   if (h->backend == 1) {
     TcCall c;
     c.x = x;
+    if (h->w8) {
+      // fp8 layers multiply in fp16: the call's hidden states once in that type
+      EAT_TRY(launch(h, kGather, st, "hidden states to fp16",
+                     [&] { return tc_launch_to_f16(h->tc, x, h->xh, T, st); }));
+      c.x = h->xh;
+    }
     c.T = T;
     c.tile_rows = tile_rows;
     c.tile_rows_down = tile_rows_down;
@@ -302,8 +310,14 @@ eat_status eat_create(const eat_layer_desc* desc, const eat_params* params, eat_
   if (D.max_tokens < 1 || D.max_tokens > 65536)
     return fail(nullptr, EAT_ERR_INVALID_ARG, "max_tokens must be in [1, 65536]");
   if (!((D.wdtype == EAT_F32 && D.xdtype == EAT_F32) ||
-        (D.wdtype == EAT_BF16 && D.xdtype == EAT_BF16)))
-    return fail(nullptr, EAT_ERR_UNSUPPORTED, "wdtype and xdtype must both be F32 or both BF16");
+        (D.wdtype == EAT_BF16 && D.xdtype == EAT_BF16) ||
+        (D.wdtype == EAT_FP8_E4M3 && D.xdtype == EAT_BF16)))
+    return fail(nullptr, EAT_ERR_UNSUPPORTED,
+                "(wdtype, xdtype) must be (F32, F32), (BF16, BF16) or (FP8_E4M3, BF16)");
+  if (D.wdtype == EAT_FP8_E4M3 &&
+      (!D.w_gate_scale || !D.w_up_scale || !D.w_down_scale ||
+       (D.n_shared > 0 && (!D.ws_gate_scale || !D.ws_up_scale || !D.ws_down_scale))))
+    return fail(nullptr, EAT_ERR_INVALID_ARG, "fp8 weights need every per-row scale array");
   if (!D.w_router || !D.w_gate || !D.w_up || !D.w_down)
     return fail(nullptr, EAT_ERR_INVALID_ARG, "router or expert weight pointer is NULL");
   if (D.n_shared > 0 && (!D.ws_gate || !D.ws_up || !D.ws_down))
@@ -340,7 +354,8 @@ eat_status eat_create(const eat_layer_desc* desc, const eat_params* params, eat_
   h->Fs = D.n_shared > 0 ? D.d_ff_shared : 0;
   h->Tmax = D.max_tokens;
   h->K = Pm.max_k;
-  h->bf16 = D.wdtype == EAT_BF16;
+  h->bf16 = D.xdtype == EAT_BF16;  // hidden states (and y) in bf16
+  h->w8 = D.wdtype == EAT_FP8_E4M3;
   h->elt = h->bf16 ? 2 : 4;
   h->backend = h->bf16 ? 1 : 0;
   h->opart_rows = (long long)h->Tmax * h->K;
@@ -396,6 +411,7 @@ eat_status eat_create(const eat_layer_desc* desc, const eat_params* params, eat_
     add(&h->xperm, h->elt * rows * h->d);
   }
   add(&h->chunk_cnt, sizeof(int32_t) * permute_scratch_ints(h->Tmax, h->E));
+  if (h->w8) add(&h->xh, sizeof(uint16_t) * (size_t)h->Tmax * h->d);
   add(&h->xstage, h->elt * (size_t)h->Tmax * h->d);
   add(&h->ystage, h->elt * (size_t)h->Tmax * h->d);
   size_t total = 0;

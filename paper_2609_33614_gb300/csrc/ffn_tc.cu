@@ -89,6 +89,14 @@ __device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile 
   }
 }
 
+// The bounded wait by all lanes of a warp, with one outcome for the whole warp (a lane that gave
+// up makes every lane give up), so warp-synchronous code after it never sees diverged lanes.
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                          unsigned int* err, unsigned int code) {
+  const bool ok = mbar_wait(bar, parity, abort_flag, err, code, true);
+  return __all_sync(0xffffffffu, ok);
+}
+
 __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar,
                                             int c0, int c1) {
   asm volatile(
@@ -144,6 +152,31 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
         "=r"(r[14]), "=r"(r[15])
       : "r"(taddr));
 }
+// D[tmem] (+)= A[tmem] . B[smem desc]^T, kind::f16 (A: 128 lanes = rows, K pairs per column).
+__device__ __forceinline__ void mma_f16_ta(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc,
+                                           uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// This lane's 32 consecutive TMEM columns from r[0..31] (the warp's 32 lanes of its quarter).
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
+      "%11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, "
+      "%29, %30, %31, %32};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
+      "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]),
+      "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]),
+      "r"(r[29]), "r"(r[30]), "r"(r[31])
+      : "memory");
+}
+__device__ __forceinline__ void tmem_wait_st() {
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
 __device__ __forceinline__ void tmem_wait_ld() {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
@@ -164,6 +197,24 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int n) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) |
          ((uint32_t)(kBM >> 4) << 24);
 }
+// The same with A and B fp16 (fp8 layers: e4m3 weights widened to fp16, fp16 activations).
+__host__ __device__ constexpr uint32_t idesc_f16(int n) {
+  return (1u << 4) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
+}
+
+// 16 e4m3 values -> 16 fp16 values (exact: every e4m3 value is an fp16 value).
+__device__ __forceinline__ void e4m3x16_to_f16(const uint4& in, uint4& lo, uint4& hi) {
+  const uint32_t w[4] = {in.x, in.y, in.z, in.w};
+  uint32_t o[8];
+#pragma unroll
+  for (int q = 0; q < 4; ++q)
+    asm("{\n .reg .b16 l, h;\n mov.b32 {l, h}, %2;\n cvt.rn.f16x2.e4m3x2 %0, l;\n"
+        " cvt.rn.f16x2.e4m3x2 %1, h;\n}"
+        : "=r"(o[2 * q]), "=r"(o[2 * q + 1])
+        : "r"(w[q]));
+  lo = make_uint4(o[0], o[1], o[2], o[3]);
+  hi = make_uint4(o[4], o[5], o[6], o[7]);
+}
 
 __host__ __device__ constexpr int tmem_cols_for(int c) {
   return c <= 32 ? 32 : c <= 64 ? 64 : c <= 128 ? 128 : c <= 256 ? 256 : 512;
@@ -176,20 +227,32 @@ __host__ __device__ constexpr int tmem_cols_for(int c) {
 // SM-pair kernel).
 enum : int { kModeDown = 0, kModeGateUp = 1, kModeGateUpIL = 2 };
 
-template <int BN, int MODE>
+template <int BN, int MODE, bool W8 = false>
 struct Cfg {
   static_assert(MODE == kModeDown || MODE == kModeGateUp, "single-SM kernel modes");
   static constexpr bool kGateUp = MODE == kModeGateUp;
   static constexpr int kNA = kGateUp ? 2 : 1;
-  static constexpr int kABytes = kBM * kBK * 2;
+  static constexpr int kABytes = kBM * kBK * 2;              // 16-bit A tile the MMA reads
+  static constexpr int kAStage = W8 ? kBM * kBK : kABytes;   // A tile as a stage holds it (e4m3: 8 KB)
   static constexpr int kBBytes = BN * kBK * 2;
-  static constexpr int kStageBytes = kNA * kABytes + kBBytes;
-  static constexpr int kStagesRaw = (kSmemBudget - 2048) / kStageBytes;
-  static constexpr int kStages = kStagesRaw > 12 ? 12 : kStagesRaw;
+  static constexpr int kStageBytes = kNA * kAStage + kBBytes;
+  // fp8: widened A tiles live in TMEM (32 columns of fp16 pairs per 64-wide k-block and tile),
+  // as many k-blocks ahead of the MMAs as the columns beside the accumulators hold (at most 8)
+  static constexpr int kACols = 32;
   static constexpr int kAccCols = kNA * BN;
-  static constexpr int kTmemCols = tmem_cols_for(2 * kAccCols);
-  static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + 256;
-  static_assert(2 * kAccCols <= 512, "two accumulator buffers must fit in TMEM");
+  static constexpr int kCvtFit = (512 - 2 * kAccCols) / (kNA * kACols);
+  static constexpr int kCvtSlots = W8 ? (kCvtFit > 8 ? 8 : kCvtFit) : 0;
+  // fp8: each slot also keeps a copy of its k-block's B tile, so a stage is free as soon as the
+  // converters have read it
+  static constexpr int kBSlotsBytes = kCvtSlots * kBBytes;
+  static constexpr int kStagesRaw = (kSmemBudget - 2048 - kBSlotsBytes) / kStageBytes;
+  static constexpr int kStages = kStagesRaw > 12 ? 12 : kStagesRaw;
+  static constexpr int kTmemCols = W8 ? 512 : tmem_cols_for(2 * kAccCols);
+  static constexpr int kSmemBytes = 1024 + kBSlotsBytes + kStages * kStageBytes + 512;
+  static constexpr int kThreads = W8 ? 320 : kThreadsTc;      // + four converter warps (fp8)
+  static_assert(2 * kAccCols + kCvtSlots * kNA * kACols <= 512, "TMEM columns");
+  static_assert(!W8 || BN <= 64, "fp8 layers use token tiles of at most 64");
+  static_assert(kSmemBytes <= 227 * 1024, "shared memory of one CTA");
 };
 
 struct TcArgs {
@@ -209,7 +272,9 @@ struct TcArgs {
   long long split_stride;    // elements between split slices of the fp32 output
   int out_bf16;              // down kernel without split-K: write bf16 rows instead of fp32
   const int32_t* b_rows;     // gather mode: slot -> token; B rows are copied from bx by the warp
-  const __nv_bfloat16* bx;   // gather mode: token rows [T, row stride kblocks * 64]
+  const __nv_bfloat16* bx;   // gather mode: token rows [T, row stride kblocks * 64] (16-bit)
+  const float* scale0;       // fp8 weights: per-row scales of the A matrix (gate, or down)
+  const float* scale1;       // fp8 weights: per-row scales of the up matrix
   unsigned int* err;
 };
 
@@ -255,32 +320,44 @@ __device__ __forceinline__ Unit decode_unit(const TcArgs& a, int u) {
 // about -88 the denominator overflows to infinity and the quotient is 0, the function's limit.
 __device__ __forceinline__ float silu_f(float g) { return __fdividef(g, 1.0f + __expf(-g)); }
 
-template <int BN, int MODE>
-__global__ void __launch_bounds__(kThreadsTc, 1)
+// W8 (fp8 layers): the stages hold e4m3 A tiles (8 KB, 64B-swizzled); warps 6-9, one per TMEM
+// lane quarter, widen each thread's weight row to fp16 and store it into an A slot in tensor
+// memory (tcgen05.st; cready / cfree barriers) and copy the stage's B tile beside the slot, so the
+// stage is free as soon as the converters are done with it; the MMA takes A from TMEM and B from
+// the slot's copy, and the epilogue applies the per-row weight scales.
+template <int BN, int MODE, bool W8>
+__global__ void __launch_bounds__(Cfg<BN, MODE, W8>::kThreads, 1)
 tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__ CUtensorMap mapA1,
               const __grid_constant__ CUtensorMap mapB, const TcArgs args) {
-  using C = Cfg<BN, MODE>;
+  using C = Cfg<BN, MODE, W8>;
   constexpr bool GATEUP = C::kGateUp;
   constexpr int S = C::kStages;
   extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  uint8_t* bslots = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);  // fp8 only
+  uint8_t* smem = bslots + C::kBSlotsBytes;
   uint64_t* full = (uint64_t*)(smem + S * C::kStageBytes);
   uint64_t* empty = full + S;
   uint64_t* tfull = empty + S;
   uint64_t* tempty = tfull + 2;
   uint64_t* mma_done = tempty + 2;
-  uint32_t* tmem_slot = (uint32_t*)(mma_done + 1);
+  uint64_t* cready = mma_done + 1;  // [slots] converted A tiles of a slot written (fp8)
+  uint64_t* cfree = cready + 8;     // [slots] the MMAs of a slot completed (fp8)
+  uint32_t* tmem_slot = (uint32_t*)(cfree + 8);
   volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(&full[s], args.b_rows ? 2 : 1);  // + the gathered rows' arrival
-      mbar_init(&empty[s], 1);
+      mbar_init(&empty[s], W8 ? 4 : 1);          // fp8: the four converter warps
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tfull[b], 1);
       mbar_init(&tempty[b], 4);
+    }
+    for (int b = 0; b < C::kCvtSlots; ++b) {
+      mbar_init(&cready[b], 4);
+      mbar_init(&cfree[b], 1);
     }
     mbar_init(mma_done, 1);
     *abort_flag = 0;
@@ -300,9 +377,10 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
   pdl_launch_dependents();
 
   // A tiles of one k-block: one 128-row box, or the gate and up boxes of the two accumulators
+  // (e4m3 boxes of 64 bytes x 128 rows for fp8 weights)
   auto load_a = [&](uint8_t* st, uint64_t* bar, int kb, int a_row) {
     tma_load_2d(st, &mapA0, bar, kb * kBK, a_row);
-    if (GATEUP) tma_load_2d(st + C::kABytes, &mapA1, bar, kb * kBK, a_row);
+    if (GATEUP) tma_load_2d(st + C::kAStage, &mapA1, bar, kb * kBK, a_row);
   };
 
   const int total_tiles = args.tile_offs
@@ -344,10 +422,10 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
         }
         uint8_t* st = smem + stage * C::kStageBytes;
         if (lane == 0) {
-          mbar_expect_tx(&full[stage], C::kNA * C::kABytes);
+          mbar_expect_tx(&full[stage], C::kNA * C::kAStage);
           load_a(st, &full[stage], kb, a_row);
         }
-        const uint32_t sb = smem_u32(st + C::kNA * C::kABytes);
+        const uint32_t sb = smem_u32(st + C::kNA * C::kAStage);
 #pragma unroll
         for (int i = 0; i < PER; ++i) {
           if (tok[i] >= 0) {
@@ -401,7 +479,7 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
           uint8_t* st = smem + stage * C::kStageBytes;
           mbar_expect_tx(&full[stage], C::kStageBytes);
           load_a(st, &full[stage], kb, a_row);
-          tma_load_2d(st + C::kNA * C::kABytes, &mapB, &full[stage], kb * kBK, b_row);
+          tma_load_2d(st + C::kNA * C::kAStage, &mapB, &full[stage], kb * kBK, b_row);
           ++issued;
           if (++stage == S) {
             stage = 0;
@@ -419,6 +497,8 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
       // ------------------------------------------------------------ MMA issuer
       int stage = 0;
       uint32_t phase = 0;
+      int cs = 0;         // conversion slot (fp8)
+      uint32_t cph = 0;
       int local = 0;
       bool ok = true;
       for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++local) {
@@ -433,24 +513,48 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
         const uint32_t d0 = tmem_base + (uint32_t)(buf * C::kAccCols);
         const uint32_t d1 = d0 + BN;
         // MMA width: the tile's rows rounded up to 16 (a partial tile computes no padding)
-        const uint32_t idesc = idesc_bf16(min(BN, (w.nrows + 15) & ~15));
+        const int n_mma = min(BN, (w.nrows + 15) & ~15);
+        const uint32_t idesc = W8 ? idesc_f16(n_mma) : idesc_bf16(n_mma);
         for (int kb = w.kb0; kb < w.kb1; ++kb) {
-          if (!mbar_wait(&full[stage], phase, abort_flag, args.err, 8u, true)) {
+          // fp8: the slot's converted tiles (the converters waited for the stage's bytes)
+          if (!mbar_wait(W8 ? &cready[cs] : &full[stage], W8 ? cph : phase, abort_flag, args.err,
+                         8u, true)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t sa0 = smem_u32(smem + stage * C::kStageBytes);
-          const uint32_t sa1 = sa0 + C::kABytes;
-          const uint32_t sb = sa0 + C::kNA * C::kABytes;
+          const uint32_t st = smem_u32(smem + stage * C::kStageBytes);
+          const uint32_t sb = W8 ? smem_u32(bslots + cs * C::kBBytes) : st + C::kNA * C::kAStage;
+          if constexpr (W8) {
+            // A from the slot's TMEM columns: 8 columns (16 fp16 of K) per MMA
+            const uint32_t ta = tmem_base + (uint32_t)(2 * C::kAccCols + cs * C::kNA * C::kACols);
 #pragma unroll
-          for (int k = 0; k < kBK / 16; ++k) {
-            const uint64_t db = sdesc_k128(sb + k * 32);
-            const uint32_t acc = (kb > w.kb0 || k > 0) ? 1u : 0u;
-            mma_bf16(d0, sdesc_k128(sa0 + k * 32), db, idesc, acc);
-            if (C::kNA == 2) mma_bf16(d1, sdesc_k128(sa1 + k * 32), db, idesc, acc);
+            for (int k = 0; k < kBK / 16; ++k) {
+              const uint64_t db = sdesc_k128(sb + k * 32);
+              const uint32_t acc = (kb > w.kb0 || k > 0) ? 1u : 0u;
+              mma_f16_ta(d0, ta + 8 * k, db, idesc, acc);
+              if (C::kNA == 2) mma_f16_ta(d1, ta + C::kACols + 8 * k, db, idesc, acc);
+            }
+          } else {
+            const uint32_t sa0 = st;
+            const uint32_t sa1 = sa0 + C::kABytes;
+#pragma unroll
+            for (int k = 0; k < kBK / 16; ++k) {
+              const uint64_t db = sdesc_k128(sb + k * 32);
+              const uint32_t acc = (kb > w.kb0 || k > 0) ? 1u : 0u;
+              mma_bf16(d0, sdesc_k128(sa0 + k * 32), db, idesc, acc);
+              if (C::kNA == 2) mma_bf16(d1, sdesc_k128(sa1 + k * 32), db, idesc, acc);
+            }
           }
-          mma_commit(&empty[stage]);
+          if (W8) {
+            mma_commit(&cfree[cs]);  // frees the slot's TMEM columns and B copy
+            if (++cs == C::kCvtSlots) {
+              cs = 0;
+              cph ^= 1u;
+            }
+          } else {
+            mma_commit(&empty[stage]);
+          }
           if (++stage == S) {
             stage = 0;
             phase ^= 1u;
@@ -463,6 +567,69 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
       mma_commit(mma_done);
       mbar_wait(mma_done, 0u, abort_flag, args.err, 16u, false);
     }
+  } else if (W8 && warp >= 6) {
+    // ------------------------------------------- e4m3 -> fp16 converters (fp8 weights, warps 6-9)
+    // Warp w may store to TMEM lane quarter w % 4: its thread owns weight row 32 (w % 4) + lane of
+    // each A tile, reads the row's 64 e4m3 bytes (64B swizzle: 16-byte chunk c of row r sits at
+    // chunk c ^ ((r / 2) % 4)), widens them to fp16 pairs and stores the 32 columns of the row.
+    const int r = 32 * (warp & 3) + lane;
+    const uint32_t lane_base = tmem_base + ((uint32_t)(32 * (warp & 3)) << 16);
+    int stage = 0, cs = 0;
+    uint32_t phase = 0, cph = 0;
+    bool ok = true;
+    for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
+      const Unit w = decode_unit<BN>(args, u);
+      for (int kb = w.kb0; kb < w.kb1; ++kb) {
+        if (!warp_wait(&full[stage], phase, abort_flag, args.err, 8u) ||
+            !warp_wait(&cfree[cs], cph ^ 1u, abort_flag, args.err, 256u)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint8_t* src = smem + stage * C::kStageBytes + r * 64;
+#pragma unroll
+        for (int a = 0; a < C::kNA; ++a) {
+          uint32_t o[32];
+#pragma unroll
+          for (int c = 0; c < 4; ++c) {
+            const uint4 v = *(const uint4*)(src + a * C::kAStage + ((c ^ ((r >> 1) & 3)) << 4));
+            uint4 lo, hi;
+            e4m3x16_to_f16(v, lo, hi);
+            o[8 * c + 0] = lo.x;
+            o[8 * c + 1] = lo.y;
+            o[8 * c + 2] = lo.z;
+            o[8 * c + 3] = lo.w;
+            o[8 * c + 4] = hi.x;
+            o[8 * c + 5] = hi.y;
+            o[8 * c + 6] = hi.z;
+            o[8 * c + 7] = hi.w;
+          }
+          tmem_st32(lane_base + (uint32_t)(2 * C::kAccCols + (cs * C::kNA + a) * C::kACols), o);
+        }
+        // the k-block's B tile into the slot's copy (same 128B-swizzled layout)
+        {
+          const uint4* bsrc = (const uint4*)(smem + stage * C::kStageBytes + C::kNA * C::kAStage);
+          uint4* bdst = (uint4*)(bslots + cs * C::kBBytes);
+          for (int i = (warp - 6) * 32 + lane; i < C::kBBytes / 16; i += 128) bdst[i] = bsrc[i];
+        }
+        fence_proxy_async();  // the B copy is read by the tensor core (async proxy)
+        tmem_wait_st();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) {
+          mbar_arrive(&cready[cs]);
+          mbar_arrive(&empty[stage]);
+        }
+        if (++cs == C::kCvtSlots) {
+          cs = 0;
+          cph ^= 1u;
+        }
+        if (++stage == S) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+    }
   } else {
     // -------------------------------------------------------------- epilogue (warps 2..5)
     const int q = warp & 3;  // TMEM lane quarter this warp may access
@@ -472,11 +639,17 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
       const Unit w = decode_unit<BN>(args, u);
       const int buf = local & 1;
       const uint32_t tph = (uint32_t)((local >> 1) & 1);
-      if (!mbar_wait(&tfull[buf], tph, abort_flag, args.err, 32u, true)) break;
+      if (!warp_wait(&tfull[buf], tph, abort_flag, args.err, 32u)) break;
       tc_fence_after();
       const uint32_t tbase = tmem_base + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * C::kAccCols);
       const int f = w.m0 + row;
       const bool fok = f < args.M;
+      float s0 = 1.0f, s1 = 1.0f;  // fp8 weights: the row scales of the A matrices
+      if (W8 && fok) {
+        const size_t ar = (size_t)w.g * args.a_rows_per_group + f;
+        s0 = args.scale0[ar];
+        if (GATEUP) s1 = args.scale1[ar];
+      }
       for (int c0 = 0; c0 < BN && c0 < w.nrows; c0 += 16) {
         uint32_t g[16], up[16];
         tmem_ld16(tbase + c0, g);
@@ -487,15 +660,16 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
           for (int c = 0; c < 16; ++c) {
             if (c0 + c < w.nrows) {
               const size_t slot = (size_t)(w.slot0 + c0 + c);
+              const float gv = W8 ? __uint_as_float(g[c]) * s0 : __uint_as_float(g[c]);
               if (GATEUP) {
-                const float h = silu_f(__uint_as_float(g[c])) * __uint_as_float(up[c]);
-                ((__nv_bfloat16*)args.out)[slot * args.M + f] = __float2bfloat16_rn(h);
+                const float uv = W8 ? __uint_as_float(up[c]) * s1 : __uint_as_float(up[c]);
+                const float h = silu_f(gv) * uv;
+                if (W8) ((__half*)args.out)[slot * args.M + f] = __float2half_rn(h);
+                else ((__nv_bfloat16*)args.out)[slot * args.M + f] = __float2bfloat16_rn(h);
               } else if (args.out_bf16) {
-                ((__nv_bfloat16*)args.out)[slot * args.M + f] =
-                    __float2bfloat16_rn(__uint_as_float(g[c]));
+                ((__nv_bfloat16*)args.out)[slot * args.M + f] = __float2bfloat16_rn(gv);
               } else {
-                ((float*)args.out)[(size_t)w.split * args.split_stride + slot * args.M + f] =
-                    __uint_as_float(g[c]);
+                ((float*)args.out)[(size_t)w.split * args.split_stride + slot * args.M + f] = gv;
               }
             }
           }
@@ -760,7 +934,7 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
       const Unit w = decode_unit<kPairBN>(args, u);
       const int buf = local & 1;
       const uint32_t tph = (uint32_t)((local >> 1) & 1);
-      if (!mbar_wait(&tfull[buf], tph, abort_flag, args.err, 32u, true)) break;
+      if (!warp_wait(&tfull[buf], tph, abort_flag, args.err, 32u)) break;
       tc_fence_after();
       const uint32_t tbase =
           tmem_base + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * C::kAccCols);
@@ -784,7 +958,7 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(&xb[b]);
-        if (!mbar_wait(&xb[b], (uint32_t)((chunk >> 1) & 1), abort_flag, args.err, 128u, true)) {
+        if (!warp_wait(&xb[b], (uint32_t)((chunk >> 1) & 1), abort_flag, args.err, 128u)) {
           ok = false;
           break;
         }
@@ -818,7 +992,7 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
       const Unit w = decode_unit<kPairBN>(args, u);
       const int buf = local & 1;
       const uint32_t tph = (uint32_t)((local >> 1) & 1);
-      if (!mbar_wait(&tfull[buf], tph, abort_flag, args.err, 32u, true)) break;
+      if (!warp_wait(&tfull[buf], tph, abort_flag, args.err, 32u)) break;
       tc_fence_after();
       const uint32_t tbase =
           tmem_base + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * C::kAccCols);
@@ -856,6 +1030,26 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
   cluster_sync_all();  // neither CTA leaves while the other may still signal it
   tc_fence_after();
   if (warp == 1) tmem_dealloc_pair(tmem_base, C::kTmemCols);
+}
+
+// fp8 layers: the call's hidden states as fp16 (the MMA operand type of those layers), 8 values
+// per thread.
+__global__ void __launch_bounds__(256)
+bf16_to_f16_kernel(const uint4* __restrict__ x, uint4* __restrict__ xh, long long n8) {
+  pdl_wait();
+  pdl_launch_dependents();
+  for (long long i = blockIdx.x * 256LL + threadIdx.x; i < n8; i += (long long)gridDim.x * 256) {
+    const uint4 u = x[i];
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+    uint32_t o[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float2 f = __bfloat1622float2(*(const __nv_bfloat162*)&w[q]);
+      const __half2 h = __floats2half2_rn(f.x, f.y);
+      o[q] = *(const uint32_t*)&h;
+    }
+    xh[i] = make_uint4(o[0], o[1], o[2], o[3]);
+  }
 }
 
 // Xperm[slot] = x[perm_tok[slot]] for every slot of the call (16-byte copies).
@@ -925,8 +1119,23 @@ bool encode_2d(CUtensorMap* m, const void* ptr, long long rows, long long cols, 
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// 2D e4m3 tensor [rows, cols] (one byte per element), box {64 bytes, box_rows}, 64-byte swizzle
+// (16-byte chunk c of row r at c ^ ((r / 2) % 4)): the converter lanes, one row each, then read
+// distinct banks.
+bool encode_2d_u8(CUtensorMap* m, const void* ptr, long long rows, long long cols, int box_rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)cols};
+  cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 struct Maps {
-  CUtensorMap wg, wu, wd, wsg, wsu, wsd;
+  CUtensorMap wg, wu, wd, wsg, wsu, wsd;   // bf16 weights, or e4m3 weights of an fp8 layer
   CUtensorMap wg64, wu64, wsg64, wsu64;  // 64-row boxes for the interleaved gate/up A tile
   CUtensorMap xperm[kNumBN], act[kNumBN], sact[kNumBN];
 };
@@ -937,20 +1146,20 @@ int bn_index(int bn) {
   return kNumBN - 1;
 }
 
-template <int BN, int MODE>
+template <int BN, int MODE, bool W8>
 cudaError_t launch_tc(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& b,
                       const TcArgs& args, int grid, cudaStream_t st) {
-  using C = Cfg<BN, MODE>;
+  using C = Cfg<BN, MODE, W8>;
   static std::once_flag once;
   static cudaError_t attr_err = cudaSuccess;
   std::call_once(once, [] {
-    attr_err = cudaFuncSetAttribute(tc_ffn_kernel<BN, MODE>,
+    attr_err = cudaFuncSetAttribute(tc_ffn_kernel<BN, MODE, W8>,
                                     cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
   });
   if (attr_err != cudaSuccess) return attr_err;
   if (grid <= 0) return cudaSuccess;
-  return launch_pdl(tc_ffn_kernel<BN, MODE>, dim3(grid), dim3(kThreadsTc), C::kSmemBytes, st,
-                    a0, a1, b, args);
+  return launch_pdl(tc_ffn_kernel<BN, MODE, W8>, dim3(grid), dim3(C::kThreads), C::kSmemBytes,
+                    st, a0, a1, b, args);
 }
 
 // SM-pair kernels: one 2-CTA cluster per pair of SMs, at most as many pairs as can be resident.
@@ -990,24 +1199,31 @@ cudaError_t launch_pair(const CUtensorMap& a0, const CUtensorMap& a1, const CUte
                     C::kSmemBytes, st, a0, a1, b, args);
 }
 
-// Single-SM launches: token tiles of 16..128 rows (256-row tiles run on SM pairs).
+// Single-SM launches: token tiles of 16..128 rows (256-row tiles run on SM pairs); W8 for fp8
+// weights.
+template <bool W8>
 cudaError_t launch_up_bn(int bn, const CUtensorMap& a0, const CUtensorMap& a1,
                          const CUtensorMap& b, const TcArgs& args, int grid, cudaStream_t st) {
   switch (bn) {
-    case 16: return launch_tc<16, kModeGateUp>(a0, a1, b, args, grid, st);
-    case 32: return launch_tc<32, kModeGateUp>(a0, a1, b, args, grid, st);
-    case 64: return launch_tc<64, kModeGateUp>(a0, a1, b, args, grid, st);
-    default: return launch_tc<128, kModeGateUp>(a0, a1, b, args, grid, st);
+    case 16: return launch_tc<16, kModeGateUp, W8>(a0, a1, b, args, grid, st);
+    case 32: return launch_tc<32, kModeGateUp, W8>(a0, a1, b, args, grid, st);
+    case 64: return launch_tc<64, kModeGateUp, W8>(a0, a1, b, args, grid, st);
+    default:
+      if constexpr (W8) return cudaErrorInvalidValue;  // fp8 layers use tiles of at most 64
+      else return launch_tc<128, kModeGateUp, W8>(a0, a1, b, args, grid, st);
   }
 }
 
+template <bool W8>
 cudaError_t launch_down_bn(int bn, const CUtensorMap& a0, const CUtensorMap& b,
                            const TcArgs& args, int grid, cudaStream_t st) {
   switch (bn) {
-    case 16: return launch_tc<16, kModeDown>(a0, a0, b, args, grid, st);
-    case 32: return launch_tc<32, kModeDown>(a0, a0, b, args, grid, st);
-    case 64: return launch_tc<64, kModeDown>(a0, a0, b, args, grid, st);
-    default: return launch_tc<128, kModeDown>(a0, a0, b, args, grid, st);
+    case 16: return launch_tc<16, kModeDown, W8>(a0, a0, b, args, grid, st);
+    case 32: return launch_tc<32, kModeDown, W8>(a0, a0, b, args, grid, st);
+    case 64: return launch_tc<64, kModeDown, W8>(a0, a0, b, args, grid, st);
+    default:
+      if constexpr (W8) return cudaErrorInvalidValue;
+      else return launch_tc<128, kModeDown, W8>(a0, a0, b, args, grid, st);
   }
 }
 
@@ -1020,19 +1236,23 @@ cudaError_t launch_down_bn(int bn, const CUtensorMap& a0, const CUtensorMap& b,
 // same shared-memory bytes per flop as two 128-token accumulators and measured slower: OLMoE
 // prefill gate/up 294 -> 316 us.)
 constexpr int kPairMinTokens = 1024;
-int tc_tile_rows(const TcLayer&, int T) {
-  for (int i = 0; i < 4; ++i)
+int tc_tile_rows(const TcLayer& L, int T) {
+  const int top = L.w8 ? 3 : 4;  // fp8 layers: single SMs, tiles of at most 64 tokens
+  for (int i = 0; i < top; ++i)
     if (T <= kBNs[i]) return kBNs[i];
+  if (L.w8) return kBNs[2];
   return T >= kPairMinTokens ? kPairBN : 128;
 }
 // Small calls gather their token rows inside the gate/up kernel (one launch and one HBM round
 // trip fewer); large calls copy them to Xperm first: there the shared-memory-bound gate/up kernel
 // loses more to the warp's cp.async traffic than the separate gather costs.
-bool tc_gathers_in_kernel(const TcLayer&, int T) { return T <= 128; }
+bool tc_gathers_in_kernel(const TcLayer& L, int T) { return T <= 128 && !L.w8; }
 
-int tc_tile_rows_down(const TcLayer&, int T) {
-  for (int i = 0; i < 4; ++i)
+int tc_tile_rows_down(const TcLayer& L, int T) {
+  const int top = L.w8 ? 3 : 4;
+  for (int i = 0; i < top; ++i)
     if (T <= kBNs[i]) return kBNs[i];
+  if (L.w8) return kBNs[2];
   return T >= kPairMinTokens ? kPairBN : 128;
 }
 
@@ -1075,6 +1295,15 @@ int tc_configure(TcLayer& L, const eat_layer_desc& D, int K, int Tmax, const cha
   L.F = D.d_ff;
   L.S = D.n_shared;
   L.Fs = D.n_shared > 0 ? D.d_ff_shared : 0;
+  L.w8 = D.wdtype == EAT_FP8_E4M3;
+  if (L.w8) {
+    L.sg = D.w_gate_scale;
+    L.su = D.w_up_scale;
+    L.sd = D.w_down_scale;
+    L.ssg = D.ws_gate_scale;
+    L.ssu = D.ws_up_scale;
+    L.ssd = D.ws_down_scale;
+  }
   L.K = K;
   L.Tmax = Tmax;
   int dev = 0;
@@ -1101,17 +1330,28 @@ int tc_bind(TcLayer& L, const eat_layer_desc& D, void* xperm, void* act, void* s
   Maps* m = new Maps();
   std::memset(m, 0, sizeof(Maps));
   const long long rows = (long long)L.Tmax * L.K;
-  bool ok = encode_2d(&m->wg, D.w_gate, (long long)L.E * L.F, L.d, kBM) &&
-            encode_2d(&m->wu, D.w_up, (long long)L.E * L.F, L.d, kBM) &&
-            encode_2d(&m->wg64, D.w_gate, (long long)L.E * L.F, L.d, kBM / 2) &&
-            encode_2d(&m->wu64, D.w_up, (long long)L.E * L.F, L.d, kBM / 2) &&
-            encode_2d(&m->wd, D.w_down, (long long)L.E * L.d, L.F, kBM);
-  if (ok && L.S > 0)
-    ok = encode_2d(&m->wsg, D.ws_gate, (long long)L.S * L.Fs, L.d, kBM) &&
-         encode_2d(&m->wsu, D.ws_up, (long long)L.S * L.Fs, L.d, kBM) &&
-         encode_2d(&m->wsg64, D.ws_gate, (long long)L.S * L.Fs, L.d, kBM / 2) &&
-         encode_2d(&m->wsu64, D.ws_up, (long long)L.S * L.Fs, L.d, kBM / 2) &&
-         encode_2d(&m->wsd, D.ws_down, (long long)L.S * L.d, L.Fs, kBM);
+  bool ok;
+  if (L.w8) {
+    ok = encode_2d_u8(&m->wg, D.w_gate, (long long)L.E * L.F, L.d, kBM) &&
+         encode_2d_u8(&m->wu, D.w_up, (long long)L.E * L.F, L.d, kBM) &&
+         encode_2d_u8(&m->wd, D.w_down, (long long)L.E * L.d, L.F, kBM);
+    if (ok && L.S > 0)
+      ok = encode_2d_u8(&m->wsg, D.ws_gate, (long long)L.S * L.Fs, L.d, kBM) &&
+           encode_2d_u8(&m->wsu, D.ws_up, (long long)L.S * L.Fs, L.d, kBM) &&
+           encode_2d_u8(&m->wsd, D.ws_down, (long long)L.S * L.d, L.Fs, kBM);
+  } else {
+    ok = encode_2d(&m->wg, D.w_gate, (long long)L.E * L.F, L.d, kBM) &&
+         encode_2d(&m->wu, D.w_up, (long long)L.E * L.F, L.d, kBM) &&
+         encode_2d(&m->wg64, D.w_gate, (long long)L.E * L.F, L.d, kBM / 2) &&
+         encode_2d(&m->wu64, D.w_up, (long long)L.E * L.F, L.d, kBM / 2) &&
+         encode_2d(&m->wd, D.w_down, (long long)L.E * L.d, L.F, kBM);
+    if (ok && L.S > 0)
+      ok = encode_2d(&m->wsg, D.ws_gate, (long long)L.S * L.Fs, L.d, kBM) &&
+           encode_2d(&m->wsu, D.ws_up, (long long)L.S * L.Fs, L.d, kBM) &&
+           encode_2d(&m->wsg64, D.ws_gate, (long long)L.S * L.Fs, L.d, kBM / 2) &&
+           encode_2d(&m->wsu64, D.ws_up, (long long)L.S * L.Fs, L.d, kBM / 2) &&
+           encode_2d(&m->wsd, D.ws_down, (long long)L.S * L.d, L.Fs, kBM);
+  }
   for (int i = 0; i < kNumBN && ok; ++i) {
     ok = encode_2d(&m->xperm[i], xperm, rows, L.d, kBNs[i]) &&
          encode_2d(&m->act[i], act, rows, L.F, kBNs[i]);
@@ -1140,6 +1380,13 @@ cudaError_t tc_launch_gather(const TcLayer& L, const TcCall& c, cudaStream_t st)
                     (const uint4*)c.x, c.perm_tok, c.offs + L.E, vecs, (uint4*)c.xperm);
 }
 
+cudaError_t tc_launch_to_f16(const TcLayer& L, const void* x, void* xh, int T, cudaStream_t st) {
+  const long long n8 = (long long)T * L.d / 8;
+  const int grid = (int)std::min<long long>((n8 + 255) / 256, 4LL * L.num_sms);
+  return launch_pdl(bf16_to_f16_kernel, dim3(grid), dim3(256), 0, st, (const uint4*)x,
+                    (uint4*)xh, n8);
+}
+
 cudaError_t tc_launch_up(const TcLayer& L, const TcCall& c, bool shared, cudaStream_t st) {
   const Maps* m = (const Maps*)L.maps;
   TcArgs a;
@@ -1154,6 +1401,14 @@ cudaError_t tc_launch_up(const TcLayer& L, const TcCall& c, bool shared, cudaStr
   a.kb_per_split = a.kblocks;
   a.a_rows_per_group = a.M;
   a.err = c.status;
+  if (L.w8) {
+    a.scale0 = shared ? L.ssg : L.sg;
+    a.scale1 = shared ? L.ssu : L.su;
+  }
+  auto up_bn = [&](const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& b, int grid) {
+    return L.w8 ? launch_up_bn<true>(bn, a0, a1, b, a, grid, st)
+                : launch_up_bn<false>(bn, a0, a1, b, a, grid, st);
+  };
   long long max_tiles;
   if (shared) {
     CUtensorMap xm;
@@ -1167,7 +1422,7 @@ cudaError_t tc_launch_up(const TcLayer& L, const TcCall& c, bool shared, cudaStr
     if (pair)
       return launch_pair<kModeGateUpIL>(m->wsg64, m->wsu64, xm, a, units, L.num_sms, st);
     const int grid = (int)std::min<long long>(L.num_sms, units);
-    return launch_up_bn(bn, m->wsg, m->wsu, xm, a, grid, st);
+    return up_bn(m->wsg, m->wsu, xm, grid);
   }
   a.n_groups = L.E;
   a.row_offs = c.offs;
@@ -1180,12 +1435,12 @@ cudaError_t tc_launch_up(const TcLayer& L, const TcCall& c, bool shared, cudaStr
     // small call: the token rows are gathered from x inside the kernel
     a.b_rows = c.perm_tok;
     a.bx = (const __nv_bfloat16*)c.x;
-    return launch_up_bn(bn, m->wg, m->wu, m->wg, a, grid, st);
+    return up_bn(m->wg, m->wu, m->wg, grid);
   }
   if (pair)
     return launch_pair<kModeGateUpIL>(m->wg64, m->wu64, m->xperm[bn_index(kPairRows)], a, units,
                                       L.num_sms, st);
-  return launch_up_bn(bn, m->wg, m->wu, m->xperm[bn_index(bn)], a, grid, st);
+  return up_bn(m->wg, m->wu, m->xperm[bn_index(bn)], grid);
 }
 
 cudaError_t tc_launch_down(const TcLayer& L, const TcCall& c, bool shared, int n_split,
@@ -1204,6 +1459,11 @@ cudaError_t tc_launch_down(const TcLayer& L, const TcCall& c, bool shared, int n
   a.kb_per_split = (a.kblocks + n_split - 1) / n_split;
   a.a_rows_per_group = L.d;
   a.err = c.status;
+  if (L.w8) a.scale0 = shared ? L.ssd : L.sd;
+  auto down_bn = [&](const CUtensorMap& a0, const CUtensorMap& b, int grid) {
+    return L.w8 ? launch_down_bn<true>(bn, a0, b, a, grid, st)
+                : launch_down_bn<false>(bn, a0, b, a, grid, st);
+  };
   long long max_tiles;
   if (shared) {
     a.n_groups = L.S;
@@ -1217,7 +1477,7 @@ cudaError_t tc_launch_down(const TcLayer& L, const TcCall& c, bool shared, int n
       return launch_pair<kModeDown>(m->wsd, m->wsd, m->sact[bn_index(kPairRows)], a, units,
                                     L.num_sms, st);
     const int grid = (int)std::min<long long>(L.num_sms, units);
-    return launch_down_bn(bn, m->wsd, m->sact[bn_index(bn)], a, grid, st);
+    return down_bn(m->wsd, m->sact[bn_index(bn)], grid);
   }
   a.n_groups = L.E;
   a.row_offs = c.offs;
@@ -1231,7 +1491,7 @@ cudaError_t tc_launch_down(const TcLayer& L, const TcCall& c, bool shared, int n
     return launch_pair<kModeDown>(m->wd, m->wd, m->act[bn_index(kPairRows)], a, units, L.num_sms,
                                   st);
   const int grid = (int)std::min<long long>(L.num_sms, units);
-  return launch_down_bn(bn, m->wd, m->act[bn_index(bn)], a, grid, st);
+  return down_bn(m->wd, m->act[bn_index(bn)], grid);
 }
 
 cudaError_t tc_selftest_bounded_wait(unsigned long long limit_ns, unsigned int* dev_status,

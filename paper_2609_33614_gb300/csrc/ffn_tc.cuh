@@ -10,11 +10,14 @@ struct TcLayer {
   bool ready = false;
   int E = 0, d = 0, F = 0, S = 0, Fs = 0, K = 0, Tmax = 0;
   int num_sms = 0;
+  bool w8 = false;  // e4m3 expert weights with per-row fp32 scales (fp16 MMA operands)
+  const float *sg = nullptr, *su = nullptr, *sd = nullptr;     // [E,F], [E,F], [E,d]
+  const float *ssg = nullptr, *ssu = nullptr, *ssd = nullptr;  // shared experts
   void* maps = nullptr;  // host copy of the tensor maps (see ffn_tc.cu)
 };
 
 struct TcCall {
-  const void* x = nullptr;         // [T, d] bf16 hidden states of the call
+  const void* x = nullptr;         // [T, d] hidden states of the call (fp16 for fp8 layers)
   int T = 0;
   int tile_rows = 0;               // BN of the gate/up kernel (token rows per tile)
   int tile_rows_down = 0;          // BN of the down kernel
@@ -23,7 +26,7 @@ struct TcCall {
   const int32_t* tile_offs_down = nullptr;  // tile prefix for tile_rows_down
   const int32_t* perm_tok = nullptr;
   void* xperm = nullptr;           // [Tmax*K, d] gathered rows in slot order
-  void* act = nullptr;             // [Tmax*K, F] bf16
+  void* act = nullptr;             // [Tmax*K, F] bf16 (fp16 for fp8 layers)
   float* opart = nullptr;          // [split][T*K, d] fp32, or [T*K, d] bf16 without split-K
   void* sact = nullptr;            // [S*T, Fs] bf16
   void* sout = nullptr;            // [S*T, d] bf16
@@ -42,6 +45,8 @@ bool tc_gathers_in_kernel(const TcLayer& L, int T);  // gate/up gathers x rows i
 int tc_down_split(const TcLayer& L, int T);  // split-K slices of the routed down projection
 long long tc_opart_rows(const TcLayer& L);   // rows of fp32 partials the workspace must hold
 cudaError_t tc_launch_gather(const TcLayer& L, const TcCall& c, cudaStream_t st);
+// fp8 layers: xh[T, d] fp16 = x[T, d] bf16 (the call's hidden states in the MMA operand type).
+cudaError_t tc_launch_to_f16(const TcLayer& L, const void* x, void* xh, int T, cudaStream_t st);
 cudaError_t tc_launch_up(const TcLayer& L, const TcCall& c, bool shared, cudaStream_t st);
 // Launches one thread waiting on an mbarrier nobody arrives on, bounded by limit_ns (the wait the
 // tensor-core kernels use); the expiry sets bit 64 in *dev_status.

@@ -14,7 +14,7 @@ PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(PKG, "libeat.so")
 
 EAT_OK, EAT_ERR_INVALID_ARG, EAT_ERR_UNSUPPORTED, EAT_ERR_OOM, EAT_ERR_CUDA, EAT_ERR_STATE = range(6)
-EAT_F32, EAT_BF16 = 0, 1
+EAT_F32, EAT_BF16, EAT_FP8_E4M3 = 0, 1, 2
 EAT_C_SUM, EAT_C_RAW = 0, 1
 EAT_ROUTER_EAT, EAT_ROUTER_TOPK, EAT_ROUTER_TOPP = 0, 1, 2
 EAT_SMOOTH_CALL, EAT_SMOOTH_TEMPORAL = 0, 1
@@ -36,7 +36,9 @@ class eat_layer_desc(ctypes.Structure):
     _fields_ = [(n, c_i32) for n in ("d_model", "n_experts", "d_ff", "n_shared", "d_ff_shared",
                                      "max_tokens", "wdtype", "xdtype")] + \
                [(n, c_vp) for n in ("w_router", "b_router", "w_gate", "w_up", "w_down",
-                                    "ws_gate", "ws_up", "ws_down", "opd_scale")]
+                                    "ws_gate", "ws_up", "ws_down", "opd_scale",
+                                    "w_gate_scale", "w_up_scale", "w_down_scale",
+                                    "ws_gate_scale", "ws_up_scale", "ws_down_scale")]
 
 
 class EatError(RuntimeError):
@@ -228,33 +230,43 @@ class EatLayer:
     """Owns an eat_handle for one MoE layer whose weights are CUDA tensors (kept referenced)."""
 
     def __init__(self, w_router, b_router, w_gate, w_up, w_down, max_tokens, params,
-                 ws_gate=None, ws_up=None, ws_down=None, opd_scale=None):
+                 ws_gate=None, ws_up=None, ws_down=None, opd_scale=None, scales=None):
+        """Expert weights fp32, bf16, or torch.float8_e4m3fn with ``scales`` = dict of the fp32
+        per-row scale tensors (w_gate_scale, w_up_scale, w_down_scale and, with shared experts,
+        ws_gate_scale, ws_up_scale, ws_down_scale)."""
         import torch
+        scales = scales or {}
         self._keep = [w_router, b_router, w_gate, w_up, w_down, ws_gate, ws_up, ws_down,
-                      opd_scale]
-        bf16 = w_gate.dtype == torch.bfloat16
+                      opd_scale] + list(scales.values())
+        fp8 = w_gate.dtype == torch.float8_e4m3fn
+        bf16 = w_gate.dtype == torch.bfloat16 or fp8
         E, F, d = w_gate.shape
         S = 0 if ws_gate is None else ws_gate.shape[0]
         Fs = 0 if ws_gate is None else ws_gate.shape[1]
         self.E, self.F, self.d, self.S, self.K = E, F, d, S, params.max_k
-        self.dtype = w_gate.dtype
+        self.dtype = torch.bfloat16 if fp8 else w_gate.dtype  # hidden-state dtype
         self.max_tokens = max_tokens
-        desc = eat_layer_desc(d, E, F, S, Fs, max_tokens, EAT_BF16 if bf16 else EAT_F32,
-                              EAT_BF16 if bf16 else EAT_F32, _ptr(w_router), _ptr(b_router),
-                              _ptr(w_gate), _ptr(w_up), _ptr(w_down), _ptr(ws_gate), _ptr(ws_up),
-                              _ptr(ws_down), _ptr(opd_scale))
+        wdt = EAT_FP8_E4M3 if fp8 else (EAT_BF16 if bf16 else EAT_F32)
+        sc = [_ptr(scales.get(n)) for n in ("w_gate_scale", "w_up_scale", "w_down_scale",
+                                             "ws_gate_scale", "ws_up_scale", "ws_down_scale")]
+        desc = eat_layer_desc(d, E, F, S, Fs, max_tokens, wdt, EAT_BF16 if bf16 else EAT_F32,
+                              _ptr(w_router), _ptr(b_router), _ptr(w_gate), _ptr(w_up),
+                              _ptr(w_down), _ptr(ws_gate), _ptr(ws_up), _ptr(ws_down),
+                              _ptr(opd_scale), *sc)
         self.params = params
         self.h = eat_create(desc, params)
 
     @classmethod
     def from_workload(cls, lw, max_tokens, params=None, device="cuda", opd_scale=None):
-        """Build from a workloads.LayerWeights (moved to ``device`` if needed)."""
+        """Build from a workloads.LayerWeights or workloads.Fp8LayerWeights (moved to
+        ``device`` if needed)."""
         if params is None:
             params = eat_default_params(lw.shape.max_k, temperature=lw.shape.temperature)
         mv = lambda t: None if t is None else t.to(device).contiguous()
+        scales = {n: mv(t) for n, t in getattr(lw, "scales", {}).items()}
         return cls(mv(lw.w_router), mv(lw.b_router), mv(lw.w_gate), mv(lw.w_up), mv(lw.w_down),
                    max_tokens, params, mv(lw.ws_gate), mv(lw.ws_up), mv(lw.ws_down),
-                   mv(opd_scale))
+                   mv(opd_scale), scales=scales)
 
     def close(self):
         if getattr(self, "h", None):

@@ -89,6 +89,48 @@ class LayerWeights:
     ws_down: torch.Tensor | None = None
 
 
+@dataclass
+class Fp8LayerWeights(LayerWeights):
+    """Expert weights as e4m3 with one fp32 scale per row (``scales`` keyed like the C ABI's
+    descriptor fields: w_gate_scale, w_up_scale, w_down_scale, ws_gate_scale, ...)."""
+    scales: dict | None = None
+
+    def dequantized(self) -> LayerWeights:
+        """The weights the fp8 layer computes with: scale[row] * e4m3 value, in fp32."""
+        def dq(q, name):
+            if q is None:
+                return None
+            return q.float() * self.scales[name].unsqueeze(-1).float()
+        return LayerWeights(self.shape, self.w_router, self.b_router,
+                            dq(self.w_gate, "w_gate_scale"), dq(self.w_up, "w_up_scale"),
+                            dq(self.w_down, "w_down_scale"), dq(self.ws_gate, "ws_gate_scale"),
+                            dq(self.ws_up, "ws_up_scale"), dq(self.ws_down, "ws_down_scale"))
+
+
+def quantize_fp8(w: torch.Tensor):
+    """Per-row e4m3 quantization of [..., rows, cols] weights: scale = max |row| / 448 (1 for an
+    all-zero row), q = round-to-nearest e4m3 of w / scale.  Returns (q, scale fp32 [..., rows])."""
+    wf = w.float()
+    amax = wf.abs().amax(dim=-1)
+    scale = torch.where(amax > 0, amax / 448.0, torch.ones_like(amax))
+    q = (wf / scale.unsqueeze(-1)).to(torch.float8_e4m3fn)
+    return q, scale
+
+
+def to_fp8(lw: LayerWeights) -> Fp8LayerWeights:
+    """The layer with its expert weights quantized to e4m3 per row (router unchanged)."""
+    out, scales = {}, {}
+    for name in ("w_gate", "w_up", "w_down", "ws_gate", "ws_up", "ws_down"):
+        t = getattr(lw, name)
+        if t is None:
+            out[name] = None
+            continue
+        out[name], scales[name + "_scale"] = quantize_fp8(t)
+    return Fp8LayerWeights(lw.shape, lw.w_router, lw.b_router, out["w_gate"], out["w_up"],
+                           out["w_down"], out["ws_gate"], out["ws_up"], out["ws_down"],
+                           scales=scales)
+
+
 def make_layer(shape: LayerShape, layer: int = 0, device: str = "cpu") -> LayerWeights:
     """Draw one layer's router and expert weights.  The router (fp32) and its bias are always
     drawn on the CPU generator; the expert weights on ``device``'s generator."""

@@ -45,7 +45,8 @@ def _desc(**kw):
     base = dict(d_model=256, n_experts=8, d_ff=512, n_shared=0, d_ff_shared=0, max_tokens=64,
                 wdtype=eat.EAT_F32, xdtype=eat.EAT_F32, w_router=16, b_router=None,
                 w_gate=4096, w_up=8192, w_down=12288, ws_gate=None, ws_up=None, ws_down=None,
-                opd_scale=None)
+                opd_scale=None, w_gate_scale=None, w_up_scale=None, w_down_scale=None,
+                ws_gate_scale=None, ws_up_scale=None, ws_down_scale=None)
     base.update(kw)
     return eat.eat_layer_desc(*[base[n] for n, _ in eat.eat_layer_desc._fields_])
 
@@ -58,6 +59,11 @@ def _desc(**kw):
     (dict(n_shared=2, d_ff_shared=0), {}, eat.EAT_ERR_UNSUPPORTED),
     (dict(max_tokens=0), {}, eat.EAT_ERR_INVALID_ARG),
     (dict(wdtype=eat.EAT_BF16), {}, eat.EAT_ERR_UNSUPPORTED),
+    (dict(wdtype=eat.EAT_FP8_E4M3), {}, eat.EAT_ERR_UNSUPPORTED),          # fp8 needs bf16 x
+    (dict(wdtype=eat.EAT_FP8_E4M3, xdtype=eat.EAT_BF16), {}, eat.EAT_ERR_INVALID_ARG),  # no scales
+    (dict(wdtype=eat.EAT_FP8_E4M3, xdtype=eat.EAT_BF16, w_gate_scale=64, w_up_scale=64,
+          w_down_scale=64, n_shared=1, d_ff_shared=64, ws_gate=4096, ws_up=4096, ws_down=4096),
+     {}, eat.EAT_ERR_INVALID_ARG),                                                   # shared scales
     (dict(w_gate=None), {}, eat.EAT_ERR_INVALID_ARG),
     (dict(w_up=4100), {}, eat.EAT_ERR_INVALID_ARG),
     (dict(n_shared=1, d_ff_shared=64), {}, eat.EAT_ERR_INVALID_ARG),

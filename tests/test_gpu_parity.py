@@ -202,6 +202,20 @@ def test_sm_pair_one_large_group():
     run_parity(OLMOE_S, lw, [2100])
 
 
+# ------------------------------------------------------------------ fp8 (e4m3) expert weights
+@pytest.mark.parametrize("name,Ts", [("mixtral", [1, 16, 64]), ("olmoe", [32, 300, 1100]),
+                                     ("qwen", [64, 200])])
+def test_fp8_weights(name, Ts):
+    """e4m3 expert weights with per-row scales (the fp8 decode path, also at 300 and 1100 tokens,
+    which stay on single SMs): the oracle runs on the dequantized weights."""
+    shape = {"mixtral": MIX_S, "olmoe": OLMOE_S, "qwen": QWEN_S}[name]
+    lw8 = W.to_fp8(W.make_layer(shape))
+    layer = eat.EatLayer.from_workload(lw8, max(Ts), gpu_params(shape))
+    assert eat.eat_ffn_backend(layer.h) == 1
+    run_parity(shape, lw8.dequantized(), Ts, layer=layer)
+    layer.close()
+
+
 def test_partial_feature_tiles():
     """d = 320 and d_ff = 192: feature tiles of 128 end half-full in both expert GEMMs."""
     sh = W.scaled(W.QWEN, "ragged-d", d_model=320, n_experts=16, d_ff=192, n_shared=1,
