@@ -50,7 +50,8 @@ def workload_spec(name):
                               desc="deepseek-v2-lite-shaped 26-layer MoE stack, prefill 16384"),
         "dsv2l-decode": dict(shape=W.DSV2L, batches=[128], layers=26,
                              desc="deepseek-v2-lite-shaped 26-layer MoE stack, decode batch 128"),
-        # e4m3 expert weights with per-row scales (hidden states bf16, expert GEMMs fp16 x fp16)
+        # e4m3 expert weights with per-row scales (hidden states bf16, e4m3 x e4m3 GEMMs on the
+        # hi/lo split of the other operand)
         "mixtral-decode-fp8": dict(shape=W.MIXTRAL, batches=[1, 16, 64], layers=1, fp8=True,
                                    desc="mixtral-8x7b-shaped MoE layer, e4m3 expert weights, "
                                         "decode, batch 1+16+64 per step"),
@@ -68,7 +69,8 @@ def bench_config(args, spec):
     if args.router == "topp":
         cfg["top_p"] = args.top_p
     if spec.get("fp8"):
-        cfg["expert_weights"] = "e4m3, fp32 scale per row (fp16 x fp16 -> fp32 GEMMs)"
+        cfg["expert_weights"] = ("e4m3, fp32 scale per row (e4m3 x e4m3 -> fp32 GEMMs, other "
+                                 "operand split into e4m3 hi + lo per row)")
     cfg.update({"d_model": shape.d_model, "n_experts": shape.n_experts, "d_ff": shape.d_ff,
                 "n_shared": shape.n_shared, "max_k": shape.max_k, "layers": spec["layers"],
                 "batches": spec["batches"],
@@ -431,7 +433,7 @@ def run_ours(args, world, rank, local):
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": job_ms / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": "f16" if spec.get("fp8") else "bf16",
+        "dtype": "e4m3" if spec.get("fp8") else "bf16",
         "data": "synthetic (seeded N(0,1) hidden states, N(0,0.02^2) weights"
                 + (", quantized to e4m3 per row)" if spec.get("fp8") else ")"),
         "config": bench_config(args, spec),

@@ -106,9 +106,11 @@ eat_status eat_default_params(eat_params* p);
  *   scale[r] * (its e4m3 bytes) (the shared ones NULL when n_shared == 0); ignored otherwise.
  * Supported: 1 <= E <= 256; d, F, Fs multiples of 64; (wdtype, xdtype) both EAT_F32, both
  * EAT_BF16, or EAT_FP8_E4M3 weights with EAT_BF16 hidden states; 1 <= max_tokens <= 65536.  All
- * weight pointers 16-byte aligned.  fp8 layers compute the expert GEMMs in fp16 x fp16 -> fp32
- * (the e4m3 values convert exactly; hidden states and SwiGLU activations round to fp16, so
- * |x| above 65504 overflows) and always use the single-SM kernels. */
+ * weight pointers 16-byte aligned.  fp8 layers feed the e4m3 weights to the tensor cores
+ * unconverted (e4m3 x e4m3 -> fp32 MMAs): each row of a GEMM's other operand (the hidden states,
+ * then the bf16 SwiGLU activations) is scaled by a power of two and split into two e4m3 parts,
+ * hi + lo, which hold a bf16 value exactly down to 2^-10 of its row's largest magnitude; both
+ * parts are multiplied and accumulated in fp32.  fp8 layers always use the single-SM kernels. */
 typedef struct eat_layer_desc {
   int32_t d_model, n_experts, d_ff, n_shared, d_ff_shared, max_tokens;
   int32_t wdtype, xdtype;

@@ -18,7 +18,7 @@ struct eat_handle {
   eat_params prm;
   int E = 0, d = 0, F = 0, S = 0, Fs = 0, Tmax = 0, K = 0;
   bool bf16 = false;  // hidden states and outputs in bf16
-  bool w8 = false;    // e4m3 expert weights (tensor-core kernels with fp16 operands)
+  bool w8 = false;    // e4m3 expert weights (tensor-core kernels, kind::f8f6f4)
   int backend = 0;  // 0 CUDA-core kernels (fp32 layers), 1 tcgen05 kernels (bf16 / fp8 layers)
   size_t elt = 4;
 
@@ -42,7 +42,7 @@ struct eat_handle {
   int nb = 1;                 // column segments per row in the combine kernel
   void* sact = nullptr;   // [S*Tmax, Fs]
   float* sout = nullptr;  // [S*Tmax, d] (fp32; bf16 on the tensor-core path)
-  void* xh = nullptr;     // [Tmax, d] fp16 hidden states of the call (fp8 layers)
+  TcQuant q;              // fp8 layers: e4m3 hi/lo planes and scales of the GEMM B operands
   void* xstage = nullptr; // [Tmax, d]
   void* ystage = nullptr; // [Tmax, d]
   void* xperm = nullptr;  // [Tmax*K, d] gathered token rows (tensor-core path)
@@ -180,12 +180,6 @@ eat_status run_forward(eat_handle* h, const void* x, int T, int ppl_sign, void* 
   if (h->backend == 1) {
     TcCall c;
     c.x = x;
-    if (h->w8) {
-      // fp8 layers multiply in fp16: the call's hidden states once in that type
-      EAT_TRY(launch(h, kGather, st, "hidden states to fp16",
-                     [&] { return tc_launch_to_f16(h->tc, x, h->xh, T, st); }));
-      c.x = h->xh;
-    }
     c.T = T;
     c.tile_rows = tile_rows;
     c.tile_rows_down = tile_rows_down;
@@ -200,15 +194,25 @@ eat_status run_forward(eat_handle* h, const void* x, int T, int ppl_sign, void* 
     c.sout = h->sout;
     c.status = h->status;
     n_split = tc_down_split(h->tc, T);
-    if (!tc_gathers_in_kernel(h->tc, T))
+    // fp8 layers: each GEMM's B operand first becomes e4m3 hi/lo planes (the routed x rows are
+    // gathered into slot order on the way)
+    auto split = [&](TcSplit which, const char* what) {
+      return launch(h, kGather, st, what, [&] { return tc_launch_split(h->tc, c, which, st); });
+    };
+    if (h->w8)
+      EAT_TRY(split(TcSplit::kSlotX, "split x (slots)"));
+    else if (!tc_gathers_in_kernel(h->tc, T))
       EAT_TRY(launch(h, kGather, st, "gather rows",
                      [&] { return tc_launch_gather(h->tc, c, st); }));
     EAT_TRY(launch(h, kUp, st, "tc gate/up", [&] { return tc_launch_up(h->tc, c, false, st); }));
+    if (h->w8) EAT_TRY(split(TcSplit::kAct, "split activations"));
     EAT_TRY(launch(h, kDown, st, "tc down",
                    [&] { return tc_launch_down(h->tc, c, false, n_split, st); }));
     if (h->S > 0) {
+      if (h->w8) EAT_TRY(split(TcSplit::kTokenX, "split x (tokens)"));
       EAT_TRY(launch(h, kSUp, st, "tc shared gate/up",
                      [&] { return tc_launch_up(h->tc, c, true, st); }));
+      if (h->w8) EAT_TRY(split(TcSplit::kSharedAct, "split shared activations"));
       EAT_TRY(launch(h, kSDown, st, "tc shared down",
                      [&] { return tc_launch_down(h->tc, c, true, 1, st); }));
     }
@@ -407,11 +411,22 @@ eat_status eat_create(const eat_layer_desc* desc, const eat_params* params, eat_
     add(&h->sact, h->elt * (size_t)h->S * h->Tmax * h->Fs);
     add(&h->sout, sizeof(float) * (size_t)h->S * h->Tmax * h->d);
   }
-  if (h->backend == 1) {
+  if (h->backend == 1 && !h->w8) {
     add(&h->xperm, h->elt * rows * h->d);
   }
   add(&h->chunk_cnt, sizeof(int32_t) * permute_scratch_ints(h->Tmax, h->E));
-  if (h->w8) add(&h->xh, sizeof(uint16_t) * (size_t)h->Tmax * h->d);
+  if (h->w8) {
+    add(&h->q.xq, 2 * rows * h->d);
+    add(&h->q.xq_s, sizeof(float) * rows);
+    add(&h->q.aq, 2 * rows * h->F);
+    add(&h->q.aq_s, sizeof(float) * rows);
+    if (h->S > 0) {
+      add(&h->q.xqt, 2 * (size_t)h->Tmax * h->d);
+      add(&h->q.xqt_s, sizeof(float) * h->Tmax);
+      add(&h->q.saq, 2 * (size_t)h->S * h->Tmax * h->Fs);
+      add(&h->q.saq_s, sizeof(float) * (size_t)h->S * h->Tmax);
+    }
+  }
   add(&h->xstage, h->elt * (size_t)h->Tmax * h->d);
   add(&h->ystage, h->elt * (size_t)h->Tmax * h->d);
   size_t total = 0;
@@ -437,7 +452,7 @@ eat_status eat_create(const eat_layer_desc* desc, const eat_params* params, eat_
   }
   if (h->backend == 1) {
     const char* msg = nullptr;
-    if (tc_bind(h->tc, D, h->xperm, h->act, h->sact, &msg) != 0) {
+    if (tc_bind(h->tc, D, h->xperm, h->act, h->sact, h->q, &msg) != 0) {
       std::string m = msg ? msg : "tensor map setup failed";
       free_handle(h);
       return fail(nullptr, EAT_ERR_CUDA, m);

@@ -33,6 +33,7 @@ namespace {
 
 constexpr int kBM = 128;                  // weight rows per tile (MMA M)
 constexpr int kBK = 64;                   // 64 bf16 = 128 B: one 128B-swizzle row
+constexpr int kBK8 = 128;                 // 128 e4m3 = 128 B: the same row for fp8 layers
 constexpr int kThreadsTc = 192;           // 6 warps
 constexpr int kNumBN = 4;
 constexpr int kBNs[kNumBN] = {16, 32, 64, 128};  // single-SM token tiles; SM pairs load 128 per CTA
@@ -152,30 +153,15 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
         "=r"(r[14]), "=r"(r[15])
       : "r"(taddr));
 }
-// D[tmem] (+)= A[tmem] . B[smem desc]^T, kind::f16 (A: 128 lanes = rows, K pairs per column).
-__device__ __forceinline__ void mma_f16_ta(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc,
-                                           uint32_t idesc, uint32_t accumulate) {
+// D[tmem] (+)= A[smem desc] . B[smem desc]^T, both K-major, kind::f8f6f4 (e4m3 in, fp32
+// accumulate; K = 32 per instruction, 32 bytes of each 128-byte row like the bf16 form).
+__device__ __forceinline__ void mma_e4m3(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                         uint32_t idesc, uint32_t accumulate) {
   asm volatile(
       "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d_tmem),
-      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      " tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
       : "memory");
-}
-// This lane's 32 consecutive TMEM columns from r[0..31] (the warp's 32 lanes of its quarter).
-__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
-  asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
-      "%11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, "
-      "%29, %30, %31, %32};" ::"r"(taddr),
-      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
-      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
-      "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]),
-      "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]),
-      "r"(r[29]), "r"(r[30]), "r"(r[31])
-      : "memory");
-}
-__device__ __forceinline__ void tmem_wait_st() {
-  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 __device__ __forceinline__ void tmem_wait_ld() {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
@@ -197,23 +183,10 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int n) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) |
          ((uint32_t)(kBM >> 4) << 24);
 }
-// The same with A and B fp16 (fp8 layers: e4m3 weights widened to fp16, fp16 activations).
-__host__ __device__ constexpr uint32_t idesc_f16(int n) {
+// Instruction descriptor, kind::f8f6f4: D fp32, A and B e4m3 (format code 0), both K-major,
+// M = 128, N = n.
+__host__ __device__ constexpr uint32_t idesc_e4m3(int n) {
   return (1u << 4) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
-}
-
-// 16 e4m3 values -> 16 fp16 values (exact: every e4m3 value is an fp16 value).
-__device__ __forceinline__ void e4m3x16_to_f16(const uint4& in, uint4& lo, uint4& hi) {
-  const uint32_t w[4] = {in.x, in.y, in.z, in.w};
-  uint32_t o[8];
-#pragma unroll
-  for (int q = 0; q < 4; ++q)
-    asm("{\n .reg .b16 l, h;\n mov.b32 {l, h}, %2;\n cvt.rn.f16x2.e4m3x2 %0, l;\n"
-        " cvt.rn.f16x2.e4m3x2 %1, h;\n}"
-        : "=r"(o[2 * q]), "=r"(o[2 * q + 1])
-        : "r"(w[q]));
-  lo = make_uint4(o[0], o[1], o[2], o[3]);
-  hi = make_uint4(o[4], o[5], o[6], o[7]);
 }
 
 __host__ __device__ constexpr int tmem_cols_for(int c) {
@@ -232,26 +205,21 @@ struct Cfg {
   static_assert(MODE == kModeDown || MODE == kModeGateUp, "single-SM kernel modes");
   static constexpr bool kGateUp = MODE == kModeGateUp;
   static constexpr int kNA = kGateUp ? 2 : 1;
-  static constexpr int kABytes = kBM * kBK * 2;              // 16-bit A tile the MMA reads
-  static constexpr int kAStage = W8 ? kBM * kBK : kABytes;   // A tile as a stage holds it (e4m3: 8 KB)
-  static constexpr int kBBytes = BN * kBK * 2;
-  static constexpr int kStageBytes = kNA * kAStage + kBBytes;
-  // fp8: widened A tiles live in TMEM (32 columns of fp16 pairs per 64-wide k-block and tile),
-  // as many k-blocks ahead of the MMAs as the columns beside the accumulators hold (at most 8)
-  static constexpr int kACols = 32;
-  static constexpr int kAccCols = kNA * BN;
-  static constexpr int kCvtFit = (512 - 2 * kAccCols) / (kNA * kACols);
-  static constexpr int kCvtSlots = W8 ? (kCvtFit > 8 ? 8 : kCvtFit) : 0;
-  // fp8: each slot also keeps a copy of its k-block's B tile, so a stage is free as soon as the
-  // converters have read it
-  static constexpr int kBSlotsBytes = kCvtSlots * kBBytes;
-  static constexpr int kStagesRaw = (kSmemBudget - 2048 - kBSlotsBytes) / kStageBytes;
+  static constexpr int kNB = W8 ? 2 : 1;         // fp8: the B tile's e4m3 hi and lo parts
+  static constexpr int kKB = W8 ? kBK8 : kBK;    // K elements of a k-block (128 B per row)
+  static constexpr int kABytes = kBM * 128;
+  static constexpr int kBBytes = BN * 128;
+  static constexpr int kStageBytes = kNA * kABytes + kNB * kBBytes;
+  // fp8: the hi and lo B tiles sit back to back in the stage, so one MMA of N = BN + n covers both
+  // (hi in accumulator columns [0, BN), lo in [BN, BN + n)) and reads its A slice once, where the
+  // double-buffered accumulators fit in TMEM (gate/up up to 64 tokens, down up to 128)
+  static constexpr bool kFuse = W8 && 4 * kNA * BN <= 512;
+  static constexpr int kProjCols = kFuse ? 2 * BN : BN;  // accumulator columns per projection
+  static constexpr int kAccCols = kNA * kProjCols;
+  static constexpr int kStagesRaw = (kSmemBudget - 2048) / kStageBytes;
   static constexpr int kStages = kStagesRaw > 12 ? 12 : kStagesRaw;
-  static constexpr int kTmemCols = W8 ? 512 : tmem_cols_for(2 * kAccCols);
-  static constexpr int kSmemBytes = 1024 + kBSlotsBytes + kStages * kStageBytes + 512;
-  static constexpr int kThreads = W8 ? 320 : kThreadsTc;      // + four converter warps (fp8)
-  static_assert(2 * kAccCols + kCvtSlots * kNA * kACols <= 512, "TMEM columns");
-  static_assert(!W8 || BN <= 64, "fp8 layers use token tiles of at most 64");
+  static constexpr int kTmemCols = tmem_cols_for(2 * kAccCols);
+  static constexpr int kSmemBytes = 1024 + kStages * kStageBytes + 512;
   static_assert(kSmemBytes <= 227 * 1024, "shared memory of one CTA");
 };
 
@@ -275,6 +243,8 @@ struct TcArgs {
   const __nv_bfloat16* bx;   // gather mode: token rows [T, row stride kblocks * 64] (16-bit)
   const float* scale0;       // fp8 weights: per-row scales of the A matrix (gate, or down)
   const float* scale1;       // fp8 weights: per-row scales of the up matrix
+  const float* bscale;       // fp8: per-row scales of the B operand, indexed like its rows
+  int b_lo_rows;             // fp8: row offset of the B operand's lo plane in its tensor map
   unsigned int* err;
 };
 
@@ -320,44 +290,37 @@ __device__ __forceinline__ Unit decode_unit(const TcArgs& a, int u) {
 // about -88 the denominator overflows to infinity and the quotient is 0, the function's limit.
 __device__ __forceinline__ float silu_f(float g) { return __fdividef(g, 1.0f + __expf(-g)); }
 
-// W8 (fp8 layers): the stages hold e4m3 A tiles (8 KB, 64B-swizzled); warps 6-9, one per TMEM
-// lane quarter, widen each thread's weight row to fp16 and store it into an A slot in tensor
-// memory (tcgen05.st; cready / cfree barriers) and copy the stage's B tile beside the slot, so the
-// stage is free as soon as the converters are done with it; the MMA takes A from TMEM and B from
-// the slot's copy, and the epilogue applies the per-row weight scales.
+// W8 (fp8 layers): the weights stay e4m3 all the way to the tensor core.  The B operand arrives
+// as two e4m3 planes per row (hi and lo, with hi + lo the row divided by its power-of-two scale,
+// written by split_e4m3_kernel); a stage holds the e4m3 A tiles of a 128-element k-block and the
+// hi and lo B tiles, every k-step issues W . hi and W . lo into the same fp32 accumulator
+// (kind::f8f6f4), and the epilogue multiplies by the weight row's scale and the B row's scale.
 template <int BN, int MODE, bool W8>
-__global__ void __launch_bounds__(Cfg<BN, MODE, W8>::kThreads, 1)
+__global__ void __launch_bounds__(kThreadsTc, 1)
 tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__ CUtensorMap mapA1,
               const __grid_constant__ CUtensorMap mapB, const TcArgs args) {
   using C = Cfg<BN, MODE, W8>;
   constexpr bool GATEUP = C::kGateUp;
   constexpr int S = C::kStages;
   extern __shared__ uint8_t smem_raw[];
-  uint8_t* bslots = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);  // fp8 only
-  uint8_t* smem = bslots + C::kBSlotsBytes;
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint64_t* full = (uint64_t*)(smem + S * C::kStageBytes);
   uint64_t* empty = full + S;
   uint64_t* tfull = empty + S;
   uint64_t* tempty = tfull + 2;
   uint64_t* mma_done = tempty + 2;
-  uint64_t* cready = mma_done + 1;  // [slots] converted A tiles of a slot written (fp8)
-  uint64_t* cfree = cready + 8;     // [slots] the MMAs of a slot completed (fp8)
-  uint32_t* tmem_slot = (uint32_t*)(cfree + 8);
+  uint32_t* tmem_slot = (uint32_t*)(mma_done + 1);
   volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(&full[s], args.b_rows ? 2 : 1);  // + the gathered rows' arrival
-      mbar_init(&empty[s], W8 ? 4 : 1);          // fp8: the four converter warps
+      mbar_init(&empty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tfull[b], 1);
       mbar_init(&tempty[b], 4);
-    }
-    for (int b = 0; b < C::kCvtSlots; ++b) {
-      mbar_init(&cready[b], 4);
-      mbar_init(&cfree[b], 1);
     }
     mbar_init(mma_done, 1);
     *abort_flag = 0;
@@ -377,10 +340,9 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
   pdl_launch_dependents();
 
   // A tiles of one k-block: one 128-row box, or the gate and up boxes of the two accumulators
-  // (e4m3 boxes of 64 bytes x 128 rows for fp8 weights)
   auto load_a = [&](uint8_t* st, uint64_t* bar, int kb, int a_row) {
-    tma_load_2d(st, &mapA0, bar, kb * kBK, a_row);
-    if (GATEUP) tma_load_2d(st + C::kAStage, &mapA1, bar, kb * kBK, a_row);
+    tma_load_2d(st, &mapA0, bar, kb * C::kKB, a_row);
+    if (GATEUP) tma_load_2d(st + C::kABytes, &mapA1, bar, kb * C::kKB, a_row);
   };
 
   const int total_tiles = args.tile_offs
@@ -388,7 +350,7 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
                               : args.n_groups * ((args.uniform_rows + BN - 1) / BN);
   const int units = total_tiles * args.m_tiles * args.n_split;
 
-  if (warp == 0 && args.b_rows) {
+  if (!W8 && warp == 0 && args.b_rows) {
     // ------------------------------------------------------------ producer, gathered tokens:
     // lane 0 issues the weight TMA; all lanes copy the tile's token rows from x with 16-byte
     // cp.async into the 128B-swizzled B tile (lane l: column chunk l % 8 of rows l / 8 + 4 i).
@@ -422,10 +384,10 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
         }
         uint8_t* st = smem + stage * C::kStageBytes;
         if (lane == 0) {
-          mbar_expect_tx(&full[stage], C::kNA * C::kAStage);
+          mbar_expect_tx(&full[stage], C::kNA * C::kABytes);
           load_a(st, &full[stage], kb, a_row);
         }
-        const uint32_t sb = smem_u32(st + C::kNA * C::kAStage);
+        const uint32_t sb = smem_u32(st + C::kNA * C::kABytes);
 #pragma unroll
         for (int i = 0; i < PER; ++i) {
           if (tok[i] >= 0) {
@@ -479,7 +441,9 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
           uint8_t* st = smem + stage * C::kStageBytes;
           mbar_expect_tx(&full[stage], C::kStageBytes);
           load_a(st, &full[stage], kb, a_row);
-          tma_load_2d(st + C::kNA * C::kAStage, &mapB, &full[stage], kb * kBK, b_row);
+          uint8_t* sbt = st + C::kNA * C::kABytes;
+          tma_load_2d(sbt, &mapB, &full[stage], kb * C::kKB, b_row);
+          if (W8) tma_load_2d(sbt + C::kBBytes, &mapB, &full[stage], kb * C::kKB, b_row + args.b_lo_rows);
           ++issued;
           if (++stage == S) {
             stage = 0;
@@ -497,8 +461,6 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
       // ------------------------------------------------------------ MMA issuer
       int stage = 0;
       uint32_t phase = 0;
-      int cs = 0;         // conversion slot (fp8)
-      uint32_t cph = 0;
       int local = 0;
       bool ok = true;
       for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++local) {
@@ -511,50 +473,45 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
         }
         tc_fence_after();
         const uint32_t d0 = tmem_base + (uint32_t)(buf * C::kAccCols);
-        const uint32_t d1 = d0 + BN;
-        // MMA width: the tile's rows rounded up to 16 (a partial tile computes no padding)
+        const uint32_t d1 = d0 + C::kProjCols;
+        // MMA width: the tile's rows rounded up to 16 (a partial tile computes no padding; the
+        // fused fp8 MMA spans the hi tile's BN rows and the lo tile's first n)
         const int n_mma = min(BN, (w.nrows + 15) & ~15);
-        const uint32_t idesc = W8 ? idesc_f16(n_mma) : idesc_bf16(n_mma);
+        const uint32_t idesc = !W8       ? idesc_bf16(n_mma)
+                               : C::kFuse ? idesc_e4m3(BN + n_mma)
+                                          : idesc_e4m3(n_mma);
         for (int kb = w.kb0; kb < w.kb1; ++kb) {
-          // fp8: the slot's converted tiles (the converters waited for the stage's bytes)
-          if (!mbar_wait(W8 ? &cready[cs] : &full[stage], W8 ? cph : phase, abort_flag, args.err,
-                         8u, true)) {
+          if (!mbar_wait(&full[stage], phase, abort_flag, args.err, 8u, true)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t st = smem_u32(smem + stage * C::kStageBytes);
-          const uint32_t sb = W8 ? smem_u32(bslots + cs * C::kBBytes) : st + C::kNA * C::kAStage;
-          if constexpr (W8) {
-            // A from the slot's TMEM columns: 8 columns (16 fp16 of K) per MMA
-            const uint32_t ta = tmem_base + (uint32_t)(2 * C::kAccCols + cs * C::kNA * C::kACols);
+          const uint32_t sa0 = smem_u32(smem + stage * C::kStageBytes);
+          const uint32_t sa1 = sa0 + C::kABytes;
+          const uint32_t sb = sa0 + C::kNA * C::kABytes;
+          // four k-steps of 32 bytes per 128-byte row: 16 bf16 or 32 e4m3 elements each
 #pragma unroll
-            for (int k = 0; k < kBK / 16; ++k) {
-              const uint64_t db = sdesc_k128(sb + k * 32);
-              const uint32_t acc = (kb > w.kb0 || k > 0) ? 1u : 0u;
-              mma_f16_ta(d0, ta + 8 * k, db, idesc, acc);
-              if (C::kNA == 2) mma_f16_ta(d1, ta + C::kACols + 8 * k, db, idesc, acc);
-            }
-          } else {
-            const uint32_t sa0 = st;
-            const uint32_t sa1 = sa0 + C::kABytes;
-#pragma unroll
-            for (int k = 0; k < kBK / 16; ++k) {
-              const uint64_t db = sdesc_k128(sb + k * 32);
-              const uint32_t acc = (kb > w.kb0 || k > 0) ? 1u : 0u;
-              mma_bf16(d0, sdesc_k128(sa0 + k * 32), db, idesc, acc);
+          for (int k = 0; k < 4; ++k) {
+            const uint64_t da0 = sdesc_k128(sa0 + k * 32), db = sdesc_k128(sb + k * 32);
+            const uint32_t acc = (kb > w.kb0 || k > 0) ? 1u : 0u;
+            if constexpr (C::kFuse) {
+              mma_e4m3(d0, da0, db, idesc, acc);
+              if (C::kNA == 2) mma_e4m3(d1, sdesc_k128(sa1 + k * 32), db, idesc, acc);
+            } else if constexpr (W8) {
+              const uint64_t dl = sdesc_k128(sb + C::kBBytes + k * 32);
+              mma_e4m3(d0, da0, db, idesc, acc);
+              mma_e4m3(d0, da0, dl, idesc, 1u);
+              if (C::kNA == 2) {
+                const uint64_t da1 = sdesc_k128(sa1 + k * 32);
+                mma_e4m3(d1, da1, db, idesc, acc);
+                mma_e4m3(d1, da1, dl, idesc, 1u);
+              }
+            } else {
+              mma_bf16(d0, da0, db, idesc, acc);
               if (C::kNA == 2) mma_bf16(d1, sdesc_k128(sa1 + k * 32), db, idesc, acc);
             }
           }
-          if (W8) {
-            mma_commit(&cfree[cs]);  // frees the slot's TMEM columns and B copy
-            if (++cs == C::kCvtSlots) {
-              cs = 0;
-              cph ^= 1u;
-            }
-          } else {
-            mma_commit(&empty[stage]);
-          }
+          mma_commit(&empty[stage]);
           if (++stage == S) {
             stage = 0;
             phase ^= 1u;
@@ -566,69 +523,6 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
       // no MMA may still be running when TMEM is freed
       mma_commit(mma_done);
       mbar_wait(mma_done, 0u, abort_flag, args.err, 16u, false);
-    }
-  } else if (W8 && warp >= 6) {
-    // ------------------------------------------- e4m3 -> fp16 converters (fp8 weights, warps 6-9)
-    // Warp w may store to TMEM lane quarter w % 4: its thread owns weight row 32 (w % 4) + lane of
-    // each A tile, reads the row's 64 e4m3 bytes (64B swizzle: 16-byte chunk c of row r sits at
-    // chunk c ^ ((r / 2) % 4)), widens them to fp16 pairs and stores the 32 columns of the row.
-    const int r = 32 * (warp & 3) + lane;
-    const uint32_t lane_base = tmem_base + ((uint32_t)(32 * (warp & 3)) << 16);
-    int stage = 0, cs = 0;
-    uint32_t phase = 0, cph = 0;
-    bool ok = true;
-    for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
-      const Unit w = decode_unit<BN>(args, u);
-      for (int kb = w.kb0; kb < w.kb1; ++kb) {
-        if (!warp_wait(&full[stage], phase, abort_flag, args.err, 8u) ||
-            !warp_wait(&cfree[cs], cph ^ 1u, abort_flag, args.err, 256u)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-        const uint8_t* src = smem + stage * C::kStageBytes + r * 64;
-#pragma unroll
-        for (int a = 0; a < C::kNA; ++a) {
-          uint32_t o[32];
-#pragma unroll
-          for (int c = 0; c < 4; ++c) {
-            const uint4 v = *(const uint4*)(src + a * C::kAStage + ((c ^ ((r >> 1) & 3)) << 4));
-            uint4 lo, hi;
-            e4m3x16_to_f16(v, lo, hi);
-            o[8 * c + 0] = lo.x;
-            o[8 * c + 1] = lo.y;
-            o[8 * c + 2] = lo.z;
-            o[8 * c + 3] = lo.w;
-            o[8 * c + 4] = hi.x;
-            o[8 * c + 5] = hi.y;
-            o[8 * c + 6] = hi.z;
-            o[8 * c + 7] = hi.w;
-          }
-          tmem_st32(lane_base + (uint32_t)(2 * C::kAccCols + (cs * C::kNA + a) * C::kACols), o);
-        }
-        // the k-block's B tile into the slot's copy (same 128B-swizzled layout)
-        {
-          const uint4* bsrc = (const uint4*)(smem + stage * C::kStageBytes + C::kNA * C::kAStage);
-          uint4* bdst = (uint4*)(bslots + cs * C::kBBytes);
-          for (int i = (warp - 6) * 32 + lane; i < C::kBBytes / 16; i += 128) bdst[i] = bsrc[i];
-        }
-        fence_proxy_async();  // the B copy is read by the tensor core (async proxy)
-        tmem_wait_st();
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) {
-          mbar_arrive(&cready[cs]);
-          mbar_arrive(&empty[stage]);
-        }
-        if (++cs == C::kCvtSlots) {
-          cs = 0;
-          cph ^= 1u;
-        }
-        if (++stage == S) {
-          stage = 0;
-          phase ^= 1u;
-        }
-      }
     }
   } else {
     // -------------------------------------------------------------- epilogue (warps 2..5)
@@ -650,22 +544,33 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
         s0 = args.scale0[ar];
         if (GATEUP) s1 = args.scale1[ar];
       }
+      const float* bsc = W8 ? args.bscale + (w.slot0 - w.g * args.b_shift_per_group) : nullptr;
       for (int c0 = 0; c0 < BN && c0 < w.nrows; c0 += 16) {
         uint32_t g[16], up[16];
         tmem_ld16(tbase + c0, g);
-        if (GATEUP) tmem_ld16(tbase + BN + c0, up);
+        if (GATEUP) tmem_ld16(tbase + C::kProjCols + c0, up);
+        if constexpr (C::kFuse) {  // + the lo parts' columns
+          uint32_t g2[16], up2[16];
+          tmem_ld16(tbase + BN + c0, g2);
+          if (GATEUP) tmem_ld16(tbase + C::kProjCols + BN + c0, up2);
+          tmem_wait_ld();
+#pragma unroll
+          for (int c = 0; c < 16; ++c) {
+            g[c] = __float_as_uint(__uint_as_float(g[c]) + __uint_as_float(g2[c]));
+            if (GATEUP) up[c] = __float_as_uint(__uint_as_float(up[c]) + __uint_as_float(up2[c]));
+          }
+        }
         tmem_wait_ld();
         if (fok) {
 #pragma unroll
           for (int c = 0; c < 16; ++c) {
             if (c0 + c < w.nrows) {
               const size_t slot = (size_t)(w.slot0 + c0 + c);
-              const float gv = W8 ? __uint_as_float(g[c]) * s0 : __uint_as_float(g[c]);
+              const float sc = W8 ? bsc[c0 + c] : 1.0f;
+              const float gv = W8 ? __uint_as_float(g[c]) * (s0 * sc) : __uint_as_float(g[c]);
               if (GATEUP) {
-                const float uv = W8 ? __uint_as_float(up[c]) * s1 : __uint_as_float(up[c]);
-                const float h = silu_f(gv) * uv;
-                if (W8) ((__half*)args.out)[slot * args.M + f] = __float2half_rn(h);
-                else ((__nv_bfloat16*)args.out)[slot * args.M + f] = __float2bfloat16_rn(h);
+                const float uv = W8 ? __uint_as_float(up[c]) * (s1 * sc) : __uint_as_float(up[c]);
+                ((__nv_bfloat16*)args.out)[slot * args.M + f] = __float2bfloat16_rn(silu_f(gv) * uv);
               } else if (args.out_bf16) {
                 ((__nv_bfloat16*)args.out)[slot * args.M + f] = __float2bfloat16_rn(gv);
               } else {
@@ -1032,23 +937,122 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
   if (warp == 1) tmem_dealloc_pair(tmem_base, C::kTmemCols);
 }
 
-// fp8 layers: the call's hidden states as fp16 (the MMA operand type of those layers), 8 values
-// per thread.
+// fp8 layers: the B operand of an expert GEMM as two e4m3 planes.  Output row r (r < *n_dev, or
+// n_host without a count) takes source row map[r] (or r) of a bf16 matrix, picks the power of two
+// s_r that puts the row's largest magnitude in [128, 256) (the e4m3 range ends at 448), and stores
+// hi = e4m3(v / s_r) in plane 0 and lo = e4m3(v / s_r - hi) in plane 1, and s_r in scale[r].  A
+// bf16 value keeps 8 significant bits, hi the leading 4 and the remainder at most 4 more, so
+// hi + lo equals v / s_r exactly down to 2^-10 of the row's largest magnitude (below it the e4m3
+// subnormal step, 2^-9 after scaling, bounds the error).  A row with an infinite or NaN largest
+// magnitude gets a NaN scale, so the outputs it feeds are NaN.
+// Two floats -> two e4m3 bytes, `first` in the low byte (the lower address); the conversion puts
+// its first source operand in the upper byte.
+__device__ __forceinline__ uint16_t e4m3x2_of(float first, float second) {
+  uint16_t r;
+  asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(r) : "f"(second), "f"(first));
+  return r;
+}
+__device__ __forceinline__ float2 f32x2_of_e4m3x2(uint16_t v) {
+  uint32_t h;
+  asm("cvt.rn.f16x2.e4m3x2 %0, %1;" : "=r"(h) : "h"(v));
+  return __half22float2(*(const __half2*)&h);
+}
+
+// 8 bf16 values -> their 8 hi and 8 lo e4m3 bytes (v * inv = hi + lo + remainder).
+__device__ __forceinline__ void split8(const uint4& u, float inv, uint2& hi, uint2& lo) {
+  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+  uint32_t hw[2] = {0u, 0u}, lw[2] = {0u, 0u};
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    // a bf16 is the upper half of the float with the same value
+    const float a = __uint_as_float(w[q] << 16) * inv;  // exact: a power of two
+    const float b = __uint_as_float(w[q] & 0xffff0000u) * inv;
+    const uint16_t h = e4m3x2_of(a, b);
+    const float2 hf = f32x2_of_e4m3x2(h);
+    const uint16_t l = e4m3x2_of(a - hf.x, b - hf.y);  // exact differences
+    hw[q >> 1] |= (uint32_t)h << (16 * (q & 1));
+    lw[q >> 1] |= (uint32_t)l << (16 * (q & 1));
+  }
+  hi = make_uint2(hw[0], hw[1]);
+  lo = make_uint2(lw[0], lw[1]);
+}
+__device__ __forceinline__ float amax8(const uint4& u, float m) {
+  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+  for (int q = 0; q < 4; ++q)
+    m = fmaxf(m, fmaxf(fabsf(__uint_as_float(w[q] << 16)),
+                       fabsf(__uint_as_float(w[q] & 0xffff0000u))));
+  return m;
+}
+
+// One CTA per row; rows of up to 256 x kSplitRegs 16-byte vectors (16384 bf16) are read once and
+// kept in registers, longer ones are read twice.
+constexpr int kSplitRegs = 8;
+
 __global__ void __launch_bounds__(256)
-bf16_to_f16_kernel(const uint4* __restrict__ x, uint4* __restrict__ xh, long long n8) {
+split_e4m3_kernel(const __nv_bfloat16* __restrict__ src, const int32_t* __restrict__ map,
+                  const int32_t* __restrict__ n_dev, int n_host, int cols,
+                  uint8_t* __restrict__ dst, long long plane, float* __restrict__ scale) {
+  __shared__ float red[8];
   pdl_wait();
   pdl_launch_dependents();
-  for (long long i = blockIdx.x * 256LL + threadIdx.x; i < n8; i += (long long)gridDim.x * 256) {
-    const uint4 u = x[i];
-    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
-    uint32_t o[4];
+  const int n = n_dev ? *n_dev : n_host;
+  const int vecs = cols >> 3;
+  const bool in_regs = vecs <= 256 * kSplitRegs;
+  const int tid = threadIdx.x;
+  for (int r = blockIdx.x; r < n; r += gridDim.x) {
+    const int sr = map ? map[r] : r;
+    const uint4* row = (const uint4*)(src + (size_t)sr * cols);
+    uint4 v[kSplitRegs];
+    float m = 0.0f;
+    if (in_regs) {
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const float2 f = __bfloat1622float2(*(const __nv_bfloat162*)&w[q]);
-      const __half2 h = __floats2half2_rn(f.x, f.y);
-      o[q] = *(const uint32_t*)&h;
+      for (int j = 0; j < kSplitRegs; ++j) {
+        const int i = tid + 256 * j;
+        v[j] = i < vecs ? row[i] : make_uint4(0u, 0u, 0u, 0u);
+      }
+#pragma unroll
+      for (int j = 0; j < kSplitRegs; ++j) m = amax8(v[j], m);
+    } else {
+      for (int i = tid; i < vecs; i += 256) m = amax8(row[i], m);
     }
-    xh[i] = make_uint4(o[0], o[1], o[2], o[3]);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+    if ((tid & 31) == 0) red[tid >> 5] = m;
+    __syncthreads();
+    m = red[0];
+#pragma unroll
+    for (int i = 1; i < 8; ++i) m = fmaxf(m, red[i]);
+    __syncthreads();  // red is rewritten for the next row
+    const uint32_t ex = (__float_as_uint(m) >> 23) & 0xffu;  // m in [2^(ex-127), 2^(ex-126))
+    float s = 1.0f, inv = 1.0f;                              // rows below 2^-119: scale 1
+    if (ex == 0xffu) {
+      s = __uint_as_float(0x7fc00000u);
+    } else if (ex >= 8u) {
+      s = __uint_as_float((ex - 7u) << 23);     // 2^(ex - 134)
+      inv = __uint_as_float((261u - ex) << 23);  // 2^(134 - ex)
+    }
+    if (tid == 0) scale[r] = s;
+    uint2* hi_row = (uint2*)(dst + (size_t)r * cols);
+    uint2* lo_row = (uint2*)(dst + plane + (size_t)r * cols);
+    uint2 h, l;
+    if (in_regs) {
+#pragma unroll
+      for (int j = 0; j < kSplitRegs; ++j) {
+        const int i = tid + 256 * j;
+        if (i < vecs) {
+          split8(v[j], inv, h, l);
+          hi_row[i] = h;
+          lo_row[i] = l;
+        }
+      }
+    } else {
+      for (int i = tid; i < vecs; i += 256) {
+        split8(row[i], inv, h, l);
+        hi_row[i] = h;
+        lo_row[i] = l;
+      }
+    }
   }
 }
 
@@ -1119,18 +1123,17 @@ bool encode_2d(CUtensorMap* m, const void* ptr, long long rows, long long cols, 
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// 2D e4m3 tensor [rows, cols] (one byte per element), box {64 bytes, box_rows}, 64-byte swizzle
-// (16-byte chunk c of row r at c ^ ((r / 2) % 4)): the converter lanes, one row each, then read
-// distinct banks.
+// 2D e4m3 tensor [rows, cols] (one byte per element), box {128 bytes, box_rows}, 128B swizzle,
+// OOB -> 0: the fp8 weights and the e4m3 planes of the B operands.
 bool encode_2d_u8(CUtensorMap* m, const void* ptr, long long rows, long long cols, int box_rows) {
   auto fn = encode_fn();
   if (!fn) return false;
   cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
   cuuint64_t strides[1] = {(cuuint64_t)cols};
-  cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)box_rows};
+  cuuint32_t box[2] = {(cuuint32_t)kBK8, (cuuint32_t)box_rows};
   cuuint32_t estr[2] = {1, 1};
   return fn(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(ptr), dims, strides, box, estr,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -1138,6 +1141,9 @@ struct Maps {
   CUtensorMap wg, wu, wd, wsg, wsu, wsd;   // bf16 weights, or e4m3 weights of an fp8 layer
   CUtensorMap wg64, wu64, wsg64, wsu64;  // 64-row boxes for the interleaved gate/up A tile
   CUtensorMap xperm[kNumBN], act[kNumBN], sact[kNumBN];
+  // fp8 layers: the e4m3 hi/lo planes of the B operands (slot rows of x, token rows of x, the
+  // routed and the shared activations)
+  CUtensorMap xq[kNumBN], xqt[kNumBN], aq[kNumBN], saq[kNumBN];
 };
 
 int bn_index(int bn) {
@@ -1158,7 +1164,7 @@ cudaError_t launch_tc(const CUtensorMap& a0, const CUtensorMap& a1, const CUtens
   });
   if (attr_err != cudaSuccess) return attr_err;
   if (grid <= 0) return cudaSuccess;
-  return launch_pdl(tc_ffn_kernel<BN, MODE, W8>, dim3(grid), dim3(C::kThreads), C::kSmemBytes,
+  return launch_pdl(tc_ffn_kernel<BN, MODE, W8>, dim3(grid), dim3(kThreadsTc), C::kSmemBytes,
                     st, a0, a1, b, args);
 }
 
@@ -1200,7 +1206,7 @@ cudaError_t launch_pair(const CUtensorMap& a0, const CUtensorMap& a1, const CUte
 }
 
 // Single-SM launches: token tiles of 16..128 rows (256-row tiles run on SM pairs); W8 for fp8
-// weights.
+// weights (single-SM kernels only, at any call size).
 template <bool W8>
 cudaError_t launch_up_bn(int bn, const CUtensorMap& a0, const CUtensorMap& a1,
                          const CUtensorMap& b, const TcArgs& args, int grid, cudaStream_t st) {
@@ -1208,9 +1214,7 @@ cudaError_t launch_up_bn(int bn, const CUtensorMap& a0, const CUtensorMap& a1,
     case 16: return launch_tc<16, kModeGateUp, W8>(a0, a1, b, args, grid, st);
     case 32: return launch_tc<32, kModeGateUp, W8>(a0, a1, b, args, grid, st);
     case 64: return launch_tc<64, kModeGateUp, W8>(a0, a1, b, args, grid, st);
-    default:
-      if constexpr (W8) return cudaErrorInvalidValue;  // fp8 layers use tiles of at most 64
-      else return launch_tc<128, kModeGateUp, W8>(a0, a1, b, args, grid, st);
+    default: return launch_tc<128, kModeGateUp, W8>(a0, a1, b, args, grid, st);
   }
 }
 
@@ -1221,9 +1225,7 @@ cudaError_t launch_down_bn(int bn, const CUtensorMap& a0, const CUtensorMap& b,
     case 16: return launch_tc<16, kModeDown, W8>(a0, a0, b, args, grid, st);
     case 32: return launch_tc<32, kModeDown, W8>(a0, a0, b, args, grid, st);
     case 64: return launch_tc<64, kModeDown, W8>(a0, a0, b, args, grid, st);
-    default:
-      if constexpr (W8) return cudaErrorInvalidValue;
-      else return launch_tc<128, kModeDown, W8>(a0, a0, b, args, grid, st);
+    default: return launch_tc<128, kModeDown, W8>(a0, a0, b, args, grid, st);
   }
 }
 
@@ -1237,24 +1239,21 @@ cudaError_t launch_down_bn(int bn, const CUtensorMap& a0, const CUtensorMap& b,
 // prefill gate/up 294 -> 316 us.)
 constexpr int kPairMinTokens = 1024;
 int tc_tile_rows(const TcLayer& L, int T) {
-  const int top = L.w8 ? 3 : 4;  // fp8 layers: single SMs, tiles of at most 64 tokens
-  for (int i = 0; i < top; ++i)
+  for (int i = 0; i < kNumBN - 1; ++i)
     if (T <= kBNs[i]) return kBNs[i];
-  if (L.w8) return kBNs[2];
-  return T >= kPairMinTokens ? kPairBN : 128;
+  return T >= kPairMinTokens && !L.w8 ? kPairBN : 128;
 }
 // Small calls gather their token rows inside the gate/up kernel (one launch and one HBM round
 // trip fewer); large calls copy them to Xperm first: there the shared-memory-bound gate/up kernel
-// loses more to the warp's cp.async traffic than the separate gather costs.
+// loses more to the warp's cp.async traffic than the separate gather costs.  fp8 layers always
+// read their B operand from the e4m3 planes that split_e4m3_kernel writes.
 bool tc_gathers_in_kernel(const TcLayer& L, int T) { return T <= 128 && !L.w8; }
 
-int tc_tile_rows_down(const TcLayer& L, int T) {
-  const int top = L.w8 ? 3 : 4;
-  for (int i = 0; i < top; ++i)
-    if (T <= kBNs[i]) return kBNs[i];
-  if (L.w8) return kBNs[2];
-  return T >= kPairMinTokens ? kPairBN : 128;
-}
+int tc_tile_rows_down(const TcLayer& L, int T) { return tc_tile_rows(L, T); }
+
+// k-blocks of a reduction of length n: 64 bf16 or 128 e4m3 elements (128 bytes of each row) per
+// k-block; a ragged last fp8 k-block reads zeros beyond the row (TMA fill).
+static int kblocks_of(const TcLayer& L, int n) { return L.w8 ? (n + kBK8 - 1) / kBK8 : n / kBK; }
 
 // Split-K of the routed down projection: enough work units for ~8 waves of the persistent grid
 // (so the last, partial wave is a small fraction of a memory-bound launch), each K slice at least
@@ -1262,7 +1261,7 @@ int tc_tile_rows_down(const TcLayer& L, int T) {
 // tiles; prefill calls already have plenty and keep one slice.
 static int split_for(const TcLayer& L, int T) {
   const int m_tiles = (L.d + kBM - 1) / kBM;
-  const int kblocks = L.F / kBK;
+  const int kblocks = kblocks_of(L, L.F);
   const int bn = tc_tile_rows_down(L, T);
   const long long rows = (long long)T * L.K;
   const long long est = ((rows + bn - 1) / bn + std::min<long long>(L.E, rows)) * m_tiles;
@@ -1273,7 +1272,7 @@ static int split_for(const TcLayer& L, int T) {
 
 // Split count with no empty K slice: n slices of ceil(kblocks / split) k-blocks each.
 int tc_down_split(const TcLayer& L, int T) {
-  const int kblocks = L.F / kBK;
+  const int kblocks = kblocks_of(L, L.F);
   const int split = split_for(L, T);
   const int per = (kblocks + split - 1) / split;
   return (kblocks + per - 1) / per;
@@ -1326,10 +1325,11 @@ int tc_configure(TcLayer& L, const eat_layer_desc& D, int K, int Tmax, const cha
 }
 
 int tc_bind(TcLayer& L, const eat_layer_desc& D, void* xperm, void* act, void* sact,
-            const char** msg) {
+            const TcQuant& q, const char** msg) {
   Maps* m = new Maps();
   std::memset(m, 0, sizeof(Maps));
   const long long rows = (long long)L.Tmax * L.K;
+  L.q = q;
   bool ok;
   if (L.w8) {
     ok = encode_2d_u8(&m->wg, D.w_gate, (long long)L.E * L.F, L.d, kBM) &&
@@ -1353,6 +1353,15 @@ int tc_bind(TcLayer& L, const eat_layer_desc& D, void* xperm, void* act, void* s
            encode_2d(&m->wsd, D.ws_down, (long long)L.S * L.d, L.Fs, kBM);
   }
   for (int i = 0; i < kNumBN && ok; ++i) {
+    if (L.w8) {
+      // the hi and lo planes of each B operand, one map over both (lo at row offset R)
+      ok = encode_2d_u8(&m->xq[i], q.xq, 2 * rows, L.d, kBNs[i]) &&
+           encode_2d_u8(&m->aq[i], q.aq, 2 * rows, L.F, kBNs[i]);
+      if (ok && L.S > 0)
+        ok = encode_2d_u8(&m->xqt[i], q.xqt, 2LL * L.Tmax, L.d, kBNs[i]) &&
+             encode_2d_u8(&m->saq[i], q.saq, 2LL * L.S * L.Tmax, L.Fs, kBNs[i]);
+      continue;
+    }
     ok = encode_2d(&m->xperm[i], xperm, rows, L.d, kBNs[i]) &&
          encode_2d(&m->act[i], act, rows, L.F, kBNs[i]);
     if (ok && L.S > 0) ok = encode_2d(&m->sact[i], sact, (long long)L.S * L.Tmax, L.Fs, kBNs[i]);
@@ -1380,11 +1389,37 @@ cudaError_t tc_launch_gather(const TcLayer& L, const TcCall& c, cudaStream_t st)
                     (const uint4*)c.x, c.perm_tok, c.offs + L.E, vecs, (uint4*)c.xperm);
 }
 
-cudaError_t tc_launch_to_f16(const TcLayer& L, const void* x, void* xh, int T, cudaStream_t st) {
-  const long long n8 = (long long)T * L.d / 8;
-  const int grid = (int)std::min<long long>((n8 + 255) / 256, 4LL * L.num_sms);
-  return launch_pdl(bf16_to_f16_kernel, dim3(grid), dim3(256), 0, st, (const uint4*)x,
-                    (uint4*)xh, n8);
+cudaError_t tc_launch_split(const TcLayer& L, const TcCall& c, TcSplit which, cudaStream_t st) {
+  const long long rows = (long long)L.Tmax * L.K;
+  const __nv_bfloat16* src = nullptr;
+  const int32_t* map = nullptr;
+  const int32_t* n_dev = nullptr;
+  int n_host = 0, cols = 0;
+  uint8_t* dst = nullptr;
+  float* scale = nullptr;
+  long long plane_rows = 0;
+  switch (which) {
+    case TcSplit::kSlotX:  // routed gate/up: x rows in slot order
+      src = (const __nv_bfloat16*)c.x, map = c.perm_tok, n_dev = c.offs + L.E;
+      n_host = c.T * L.K, cols = L.d, dst = L.q.xq, scale = L.q.xq_s, plane_rows = rows;
+      break;
+    case TcSplit::kTokenX:  // shared gate/up: x rows in token order
+      src = (const __nv_bfloat16*)c.x, n_host = c.T, cols = L.d;
+      dst = L.q.xqt, scale = L.q.xqt_s, plane_rows = L.Tmax;
+      break;
+    case TcSplit::kAct:  // routed down: the gate/up activations of the call's slots
+      src = (const __nv_bfloat16*)c.act, n_dev = c.offs + L.E, n_host = c.T * L.K, cols = L.F;
+      dst = L.q.aq, scale = L.q.aq_s, plane_rows = rows;
+      break;
+    case TcSplit::kSharedAct:  // shared down: rows g * T + t
+      src = (const __nv_bfloat16*)c.sact, n_host = L.S * c.T, cols = L.Fs;
+      dst = L.q.saq, scale = L.q.saq_s, plane_rows = (long long)L.S * L.Tmax;
+      break;
+  }
+  if (n_host <= 0) return cudaSuccess;
+  const int grid = std::min(n_host, 4 * L.num_sms);
+  return launch_pdl(split_e4m3_kernel, dim3(grid), dim3(256), 0, st, src, map, n_dev, n_host,
+                    cols, dst, plane_rows * cols, scale);
 }
 
 cudaError_t tc_launch_up(const TcLayer& L, const TcCall& c, bool shared, cudaStream_t st) {
@@ -1396,7 +1431,7 @@ cudaError_t tc_launch_up(const TcLayer& L, const TcCall& c, bool shared, cudaStr
   a.M = shared ? L.Fs : L.F;
   a.m_tile = kBM;
   a.m_tiles = (a.M + a.m_tile - 1) / a.m_tile;
-  a.kblocks = L.d / kBK;
+  a.kblocks = kblocks_of(L, L.d);
   a.n_split = 1;
   a.kb_per_split = a.kblocks;
   a.a_rows_per_group = a.M;
@@ -1404,6 +1439,8 @@ cudaError_t tc_launch_up(const TcLayer& L, const TcCall& c, bool shared, cudaStr
   if (L.w8) {
     a.scale0 = shared ? L.ssg : L.sg;
     a.scale1 = shared ? L.ssu : L.su;
+    a.bscale = shared ? L.q.xqt_s : L.q.xq_s;
+    a.b_lo_rows = shared ? L.Tmax : L.Tmax * L.K;
   }
   auto up_bn = [&](const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& b, int grid) {
     return L.w8 ? launch_up_bn<true>(bn, a0, a1, b, a, grid, st)
@@ -1412,7 +1449,8 @@ cudaError_t tc_launch_up(const TcLayer& L, const TcCall& c, bool shared, cudaStr
   long long max_tiles;
   if (shared) {
     CUtensorMap xm;
-    if (!encode_2d(&xm, c.x, c.T, L.d, pair ? kPairRows : bn)) return cudaErrorInvalidValue;
+    if (L.w8) xm = m->xqt[bn_index(bn)];
+    else if (!encode_2d(&xm, c.x, c.T, L.d, pair ? kPairRows : bn)) return cudaErrorInvalidValue;
     a.n_groups = L.S;
     a.uniform_rows = c.T;
     a.b_shift_per_group = c.T;
@@ -1440,7 +1478,7 @@ cudaError_t tc_launch_up(const TcLayer& L, const TcCall& c, bool shared, cudaStr
   if (pair)
     return launch_pair<kModeGateUpIL>(m->wg64, m->wu64, m->xperm[bn_index(kPairRows)], a, units,
                                       L.num_sms, st);
-  return up_bn(m->wg, m->wu, m->xperm[bn_index(bn)], grid);
+  return up_bn(m->wg, m->wu, L.w8 ? m->xq[bn_index(bn)] : m->xperm[bn_index(bn)], grid);
 }
 
 cudaError_t tc_launch_down(const TcLayer& L, const TcCall& c, bool shared, int n_split,
@@ -1454,12 +1492,16 @@ cudaError_t tc_launch_down(const TcLayer& L, const TcCall& c, bool shared, int n
   a.M = L.d;
   a.m_tile = pair ? 2 * kBM : kBM;
   a.m_tiles = (L.d + a.m_tile - 1) / a.m_tile;
-  a.kblocks = Kdim / kBK;
+  a.kblocks = kblocks_of(L, Kdim);
   a.n_split = n_split;
   a.kb_per_split = (a.kblocks + n_split - 1) / n_split;
   a.a_rows_per_group = L.d;
   a.err = c.status;
-  if (L.w8) a.scale0 = shared ? L.ssd : L.sd;
+  if (L.w8) {
+    a.scale0 = shared ? L.ssd : L.sd;
+    a.bscale = shared ? L.q.saq_s : L.q.aq_s;
+    a.b_lo_rows = shared ? L.S * L.Tmax : L.Tmax * L.K;
+  }
   auto down_bn = [&](const CUtensorMap& a0, const CUtensorMap& b, int grid) {
     return L.w8 ? launch_down_bn<true>(bn, a0, b, a, grid, st)
                 : launch_down_bn<false>(bn, a0, b, a, grid, st);
@@ -1477,7 +1519,7 @@ cudaError_t tc_launch_down(const TcLayer& L, const TcCall& c, bool shared, int n
       return launch_pair<kModeDown>(m->wsd, m->wsd, m->sact[bn_index(kPairRows)], a, units,
                                     L.num_sms, st);
     const int grid = (int)std::min<long long>(L.num_sms, units);
-    return down_bn(m->wsd, m->sact[bn_index(bn)], grid);
+    return down_bn(m->wsd, L.w8 ? m->saq[bn_index(bn)] : m->sact[bn_index(bn)], grid);
   }
   a.n_groups = L.E;
   a.row_offs = c.offs;
@@ -1491,7 +1533,7 @@ cudaError_t tc_launch_down(const TcLayer& L, const TcCall& c, bool shared, int n
     return launch_pair<kModeDown>(m->wd, m->wd, m->act[bn_index(kPairRows)], a, units, L.num_sms,
                                   st);
   const int grid = (int)std::min<long long>(L.num_sms, units);
-  return down_bn(m->wd, m->act[bn_index(bn)], grid);
+  return down_bn(m->wd, L.w8 ? m->aq[bn_index(bn)] : m->act[bn_index(bn)], grid);
 }
 
 cudaError_t tc_selftest_bounded_wait(unsigned long long limit_ns, unsigned int* dev_status,
