@@ -109,7 +109,7 @@ eat_status eat_default_params(eat_params* p);
  * weight pointers 16-byte aligned.  fp8 layers feed the e4m3 weights to the tensor cores
  * unconverted (e4m3 x e4m3 -> fp32 MMAs): each row of a GEMM's other operand (the hidden states,
  * then the bf16 SwiGLU activations) is scaled by a power of two and split into two e4m3 parts,
- * hi + lo, which hold a bf16 value exactly down to 2^-10 of its row's largest magnitude; both
+ * hi + lo, which hold a bf16 value exactly down to 2^-9 of its row's largest magnitude; both
  * parts are multiplied and accumulated in fp32.  fp8 layers always use the single-SM kernels. */
 typedef struct eat_layer_desc {
   int32_t d_model, n_experts, d_ff, n_shared, d_ff_shared, max_tokens;

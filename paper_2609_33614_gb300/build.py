@@ -48,14 +48,38 @@ def _stamp() -> str:
 FFN_SOURCES = ("ffn_tc.cu", "ffn_tc.cuh")
 
 
+def _strip_comments(src: str) -> str:
+    """C/C++ source without its // and /* */ comments (string and character literals kept)."""
+    out, i, n = [], 0, len(src)
+    while i < n:
+        c = src[i]
+        if c in "\"'":
+            j = i + 1
+            while j < n and src[j] != c:
+                j += 2 if src[j] == "\\" else 1
+            out.append(src[i:j + 1])
+            i = j + 1
+        elif src.startswith("//", i):
+            j = src.find("\n", i)
+            i = n if j < 0 else j
+        elif src.startswith("/*", i):
+            j = src.find("*/", i + 2)
+            i = n if j < 0 else j + 2
+        else:
+            out.append(c)
+            i += 1
+    return "".join(out)
+
+
 def ffn_source_hash() -> str:
-    """Hash of the FFN kernel sources and the compile flags, independent of where the repository
-    lives (the include path enters relative to the repository root)."""
+    """Hash of the FFN kernel sources (comments removed, whitespace runs as one space: edits of
+    comments and layout keep it) and the compile flags, independent of where the repository lives
+    (the include path enters relative to the repository root)."""
     h = hashlib.sha256()
     for name in FFN_SOURCES:
-        with open(os.path.join(CSRC, name), "rb") as fh:
+        with open(os.path.join(CSRC, name), encoding="utf-8") as fh:
             h.update(name.encode())
-            h.update(fh.read())
+            h.update(" ".join(_strip_comments(fh.read()).split()).encode())
     flags = [os.path.relpath(f, ROOT) if os.path.isabs(f) else f for f in ARCH + FLAGS]
     h.update(" ".join(flags).encode())
     return h.hexdigest()

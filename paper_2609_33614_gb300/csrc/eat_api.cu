@@ -42,7 +42,7 @@ struct eat_handle {
   int nb = 1;                 // column segments per row in the combine kernel
   void* sact = nullptr;   // [S*Tmax, Fs]
   float* sout = nullptr;  // [S*Tmax, d] (fp32; bf16 on the tensor-core path)
-  TcQuant q;              // fp8 layers: e4m3 hi/lo planes and scales of the GEMM B operands
+  TcWork q;               // fp8 layers: B-operand planes and scales
   void* xstage = nullptr; // [Tmax, d]
   void* ystage = nullptr; // [Tmax, d]
   void* xperm = nullptr;  // [Tmax*K, d] gathered token rows (tensor-core path)

@@ -245,6 +245,8 @@ struct TcArgs {
   const float* scale1;       // fp8 weights: per-row scales of the up matrix
   const float* bscale;       // fp8: per-row scales of the B operand, indexed like its rows
   int b_lo_rows;             // fp8: row offset of the B operand's lo plane in its tensor map
+  int prefetch_a;            // the group layout was written two or more launches back: issue the
+                             // first stages' weight loads before waiting for the previous kernel
   unsigned int* err;
 };
 
@@ -252,30 +254,49 @@ struct Unit {
   int g, slot0, nrows, m0, kb0, kb1, split;
 };
 
+// The call's group offsets (row_offs, tile_offs), from global memory or a CTA's shared copy.
+struct Offs {
+  const int32_t* row;   // nullptr: uniform groups
+  const int32_t* tile;  // nullptr: uniform groups
+};
+constexpr int kMaxGroups = 256;  // n_experts is at most 256
+
+// All threads of the CTA: the group offsets into shared memory (one round trip instead of the
+// dependent loads of a binary search per unit decode); the caller synchronises before use.  The
+// loads bypass L1 (ld.global.cg): before the CTA's dependency wait, this SM's L1 may still hold
+// the lines of an earlier call's offsets, while L2 holds the permute's completed writes.
+__device__ __forceinline__ Offs stage_offsets(const TcArgs& a, int32_t* s_row, int32_t* s_tile) {
+  for (int i = threadIdx.x; i <= a.n_groups; i += blockDim.x) {
+    if (a.row_offs) s_row[i] = __ldcg(a.row_offs + i);
+    if (a.tile_offs) s_tile[i] = __ldcg(a.tile_offs + i);
+  }
+  return {a.row_offs ? s_row : nullptr, a.tile_offs ? s_tile : nullptr};
+}
+
 template <int BN>
-__device__ __forceinline__ Unit decode_unit(const TcArgs& a, int u) {
+__device__ __forceinline__ Unit decode_unit(const TcArgs& a, int u, Offs o) {
   Unit w;
   w.split = u % a.n_split;
   const int r = u / a.n_split;
   const int mi = r % a.m_tiles;
   const int tl = r / a.m_tiles;
   int g, j;
-  if (a.tile_offs) {
+  if (o.tile) {
     int lo = 0, hi = a.n_groups - 1;
     while (lo < hi) {
       const int mid = (lo + hi + 1) >> 1;
-      if (a.tile_offs[mid] <= tl) lo = mid;
+      if (o.tile[mid] <= tl) lo = mid;
       else hi = mid - 1;
     }
     g = lo;
-    j = tl - a.tile_offs[lo];
+    j = tl - o.tile[lo];
   } else {
     const int tpg = (a.uniform_rows + BN - 1) / BN;
     g = tl / tpg;
     j = tl % tpg;
   }
-  const int beg = a.row_offs ? a.row_offs[g] : g * a.uniform_rows;
-  const int end = a.row_offs ? a.row_offs[g + 1] : (g + 1) * a.uniform_rows;
+  const int beg = o.row ? o.row[g] : g * a.uniform_rows;
+  const int end = o.row ? o.row[g + 1] : (g + 1) * a.uniform_rows;
   w.g = g;
   w.slot0 = beg + j * BN;
   w.nrows = min(BN, end - w.slot0);
@@ -284,6 +305,23 @@ __device__ __forceinline__ Unit decode_unit(const TcArgs& a, int u) {
   w.kb1 = min(a.kblocks, w.kb0 + a.kb_per_split);
   return w;
 }
+
+// A CTA's share of the work: units blockIdx.x, + gridDim.x, ...  (Units are handed out in rounds;
+// an even split of all units' k-blocks over the CTAs, with the split units finished through fp32
+// partials, measured within 1 % on decode calls: the SMs' streaming rates differ by about 10 %,
+// and the CTA finishing a split unit would wait on another CTA of the grid.)
+template <int BN>
+struct UnitIter {
+  int units, u;
+  Offs o;
+  __device__ UnitIter(int units_, Offs o_) : units(units_), u(blockIdx.x), o(o_) {}
+  __device__ bool next(const TcArgs& a, Unit& w) {
+    if (u >= units) return false;
+    w = decode_unit<BN>(a, u, o);
+    u += gridDim.x;
+    return true;
+  }
+};
 
 // silu(g) = g / (1 + e^-g) with the hardware exponential and an approximate division: relative
 // error about 1e-6, far below the bf16 rounding of the activation it feeds (4e-3).  For g below
@@ -335,20 +373,48 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  // everything above is local to the CTA; from here on it reads what earlier kernels wrote
-  pdl_wait();
-  pdl_launch_dependents();
 
   // A tiles of one k-block: one 128-row box, or the gate and up boxes of the two accumulators
   auto load_a = [&](uint8_t* st, uint64_t* bar, int kb, int a_row) {
     tma_load_2d(st, &mapA0, bar, kb * C::kKB, a_row);
     if (GATEUP) tma_load_2d(st + C::kABytes, &mapA1, bar, kb * C::kKB, a_row);
   };
+  __shared__ int32_t s_row[kMaxGroups + 1], s_tile[kMaxGroups + 1];
+  Offs go{nullptr, nullptr};
+  auto count_units = [&]() {
+    const int total_tiles = go.tile ? go.tile[args.n_groups]
+                                    : args.n_groups * ((args.uniform_rows + BN - 1) / BN);
+    return total_tiles * args.m_tiles * args.n_split;
+  };
 
-  const int total_tiles = args.tile_offs
-                              ? args.tile_offs[args.n_groups]
-                              : args.n_groups * ((args.uniform_rows + BN - 1) / BN);
-  const int units = total_tiles * args.m_tiles * args.n_split;
+  // The weights do not depend on the previous kernel, and the group layout (permute output) is at
+  // least two launches old when the host sets prefetch_a (every launch only lets its dependent
+  // start after its own wait): the producer fills the first stages' A tiles while the previous
+  // kernel finishes; the B tiles of those stages follow after the wait.
+  int pre = 0;  // k-blocks whose A tiles are in flight
+  const bool early = args.prefetch_a && !args.b_rows;  // (gathering launches follow the permute)
+  if (early) {
+    go = stage_offsets(args, s_row, s_tile);
+    __syncthreads();
+  }
+  if (early && warp == 0 && lane == 0) {
+    UnitIter<BN> it_p(count_units(), go);
+    for (Unit w; pre < S && it_p.next(args, w);) {
+      const int a_row = w.g * args.a_rows_per_group + w.m0;
+      for (int kb = w.kb0; kb < w.kb1 && pre < S; ++kb, ++pre) {
+        mbar_expect_tx(&full[pre], C::kStageBytes);
+        load_a(smem + pre * C::kStageBytes, &full[pre], kb, a_row);
+      }
+    }
+  }
+  // from here on the CTA reads what the previous kernel wrote
+  pdl_wait();
+  pdl_launch_dependents();
+  if (!early) {
+    go = stage_offsets(args, s_row, s_tile);
+    __syncthreads();
+  }
+  const int units = count_units();
 
   if (!W8 && warp == 0 && args.b_rows) {
     // ------------------------------------------------------------ producer, gathered tokens:
@@ -365,8 +431,8 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
     uint32_t phase = 0;
     long long it = 0, released = 0;
     bool ok = true;
-    for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
-      const Unit w = decode_unit<BN>(args, u);
+    UnitIter<BN> it_u(units, go);
+    for (Unit w; ok && it_u.next(args, w);) {
       const int a_row = w.g * args.a_rows_per_group + w.m0;
       int tok[PER];
 #pragma unroll
@@ -429,18 +495,20 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
       uint32_t phase = 0;
       long long issued = 0;
       bool ok = true;
-      for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
-        const Unit w = decode_unit<BN>(args, u);
+      UnitIter<BN> it_u(units, go);
+      for (Unit w; ok && it_u.next(args, w);) {
         const int a_row = w.g * args.a_rows_per_group + w.m0;
         const int b_row = w.slot0 - w.g * args.b_shift_per_group;
         for (int kb = w.kb0; kb < w.kb1; ++kb) {
-          if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, args.err, 1u, true)) {
-            ok = false;
-            break;
-          }
           uint8_t* st = smem + stage * C::kStageBytes;
-          mbar_expect_tx(&full[stage], C::kStageBytes);
-          load_a(st, &full[stage], kb, a_row);
+          if (issued >= pre) {  // (the first `pre` stages: A already in flight, stage unused)
+            if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, args.err, 1u, true)) {
+              ok = false;
+              break;
+            }
+            mbar_expect_tx(&full[stage], C::kStageBytes);
+            load_a(st, &full[stage], kb, a_row);
+          }
           uint8_t* sbt = st + C::kNA * C::kABytes;
           tma_load_2d(sbt, &mapB, &full[stage], kb * C::kKB, b_row);
           if (W8) tma_load_2d(sbt + C::kBBytes, &mapB, &full[stage], kb * C::kKB, b_row + args.b_lo_rows);
@@ -463,8 +531,8 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
       uint32_t phase = 0;
       int local = 0;
       bool ok = true;
-      for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++local) {
-        const Unit w = decode_unit<BN>(args, u);
+      UnitIter<BN> it_u(units, go);
+      for (Unit w; ok && it_u.next(args, w); ++local) {
         const int buf = local & 1;
         const uint32_t tph = (uint32_t)((local >> 1) & 1);
         if (!mbar_wait(&tempty[buf], tph ^ 1u, abort_flag, args.err, 4u, true)) {
@@ -529,8 +597,8 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
     const int q = warp & 3;  // TMEM lane quarter this warp may access
     const int row = 32 * q + lane;
     int local = 0;
-    for (int u = blockIdx.x; u < units; u += gridDim.x, ++local) {
-      const Unit w = decode_unit<BN>(args, u);
+    UnitIter<BN> it_u(units, go);
+    for (Unit w; it_u.next(args, w); ++local) {
       const int buf = local & 1;
       const uint32_t tph = (uint32_t)((local >> 1) & 1);
       if (!warp_wait(&tfull[buf], tph, abort_flag, args.err, 32u)) break;
@@ -749,7 +817,7 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
       long long issued = 0;
       bool ok = true;
       for (int u = pair; u < units && ok; u += n_pairs) {
-        const Unit w = decode_unit<kPairBN>(args, u);
+        const Unit w = decode_unit<kPairBN>(args, u, Offs{args.row_offs, args.tile_offs});
         const int n = pair_n(w.nrows);
         const int a_row = w.g * args.a_rows_per_group + w.m0 + (int)rank * C::kFeat;
         const int b_row = w.slot0 - w.g * args.b_shift_per_group + (int)rank * (n / 2);
@@ -790,7 +858,7 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
       int local = 0;
       bool ok = true;
       for (int u = pair; u < units && ok; u += n_pairs, ++local) {
-        const Unit w = decode_unit<kPairBN>(args, u);
+        const Unit w = decode_unit<kPairBN>(args, u, Offs{args.row_offs, args.tile_offs});
         const int buf = local & 1;
         const uint32_t tph = (uint32_t)((local >> 1) & 1);
         if (!mbar_wait(&tempty[buf], tph ^ 1u, abort_flag, args.err, 4u, true)) {
@@ -836,7 +904,7 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
     long long chunk = 0;
     bool ok = true;
     for (int u = pair; u < units && ok; u += n_pairs, ++local) {
-      const Unit w = decode_unit<kPairBN>(args, u);
+      const Unit w = decode_unit<kPairBN>(args, u, Offs{args.row_offs, args.tile_offs});
       const int buf = local & 1;
       const uint32_t tph = (uint32_t)((local >> 1) & 1);
       if (!warp_wait(&tfull[buf], tph, abort_flag, args.err, 32u)) break;
@@ -894,7 +962,7 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
     const int q = warp & 3;
     int local = 0;
     for (int u = pair; u < units; u += n_pairs, ++local) {
-      const Unit w = decode_unit<kPairBN>(args, u);
+      const Unit w = decode_unit<kPairBN>(args, u, Offs{args.row_offs, args.tile_offs});
       const int buf = local & 1;
       const uint32_t tph = (uint32_t)((local >> 1) & 1);
       if (!warp_wait(&tfull[buf], tph, abort_flag, args.err, 32u)) break;
@@ -942,8 +1010,9 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
 // s_r that puts the row's largest magnitude in [128, 256) (the e4m3 range ends at 448), and stores
 // hi = e4m3(v / s_r) in plane 0 and lo = e4m3(v / s_r - hi) in plane 1, and s_r in scale[r].  A
 // bf16 value keeps 8 significant bits, hi the leading 4 and the remainder at most 4 more, so
-// hi + lo equals v / s_r exactly down to 2^-10 of the row's largest magnitude (below it the e4m3
-// subnormal step, 2^-9 after scaling, bounds the error).  A row with an infinite or NaN largest
+// hi + lo equals v / s_r exactly where that remainder stays on the e4m3 grid: scaled magnitudes of
+// at least 1/4, i.e. every value within 2^-9 of the row's largest magnitude; below, the error is
+// at most half the e4m3 subnormal step (2^-10 after scaling).  A row with an infinite or NaN largest
 // magnitude gets a NaN scale, so the outputs it feeds are NaN.
 // Two floats -> two e4m3 bytes, `first` in the low byte (the lower address); the conversion puts
 // its first source operand in the upper byte.
@@ -1325,7 +1394,7 @@ int tc_configure(TcLayer& L, const eat_layer_desc& D, int K, int Tmax, const cha
 }
 
 int tc_bind(TcLayer& L, const eat_layer_desc& D, void* xperm, void* act, void* sact,
-            const TcQuant& q, const char** msg) {
+            const TcWork& q, const char** msg) {
   Maps* m = new Maps();
   std::memset(m, 0, sizeof(Maps));
   const long long rows = (long long)L.Tmax * L.K;
@@ -1436,6 +1505,9 @@ cudaError_t tc_launch_up(const TcLayer& L, const TcCall& c, bool shared, cudaStr
   a.kb_per_split = a.kblocks;
   a.a_rows_per_group = a.M;
   a.err = c.status;
+  // the group layout is two or more launches old unless this kernel gathers the rows itself
+  // (then the permute is the previous launch)
+  a.prefetch_a = tc_gathers_in_kernel(L, c.T) && !shared ? 0 : 1;
   if (L.w8) {
     a.scale0 = shared ? L.ssg : L.sg;
     a.scale1 = shared ? L.ssu : L.su;
@@ -1497,6 +1569,7 @@ cudaError_t tc_launch_down(const TcLayer& L, const TcCall& c, bool shared, int n
   a.kb_per_split = (a.kblocks + n_split - 1) / n_split;
   a.a_rows_per_group = L.d;
   a.err = c.status;
+  a.prefetch_a = 1;  // the group layout is the permute's, two or more launches back
   if (L.w8) {
     a.scale0 = shared ? L.ssd : L.sd;
     a.bscale = shared ? L.q.saq_s : L.q.aq_s;

@@ -8,7 +8,7 @@ namespace eat {
 
 // fp8 layers: the workspace's e4m3 hi/lo planes of the GEMMs' B operands ([2][R][cols], the lo
 // plane R rows after the hi plane) and their per-row power-of-two scales [R].
-struct TcQuant {
+struct TcWork {
   uint8_t* xq = nullptr;   // x in slot order, R = Tmax * K, cols = d
   float* xq_s = nullptr;
   uint8_t* xqt = nullptr;  // x in token order (shared experts), R = Tmax, cols = d
@@ -26,7 +26,7 @@ struct TcLayer {
   bool w8 = false;  // e4m3 expert weights with per-row fp32 scales (kind::f8f6f4 MMAs)
   const float *sg = nullptr, *su = nullptr, *sd = nullptr;     // [E,F], [E,F], [E,d]
   const float *ssg = nullptr, *ssu = nullptr, *ssd = nullptr;  // shared experts
-  TcQuant q;             // fp8 layers only
+  TcWork q;
   void* maps = nullptr;  // host copy of the tensor maps (see ffn_tc.cu)
 };
 
@@ -52,9 +52,9 @@ struct TcCall {
 
 // Device checks and the tensor-map encoder; 0 on success, *msg explains a failure.
 int tc_configure(TcLayer& L, const eat_layer_desc& D, int K, int Tmax, const char** msg);
-// Tensor maps over the weights and the handle's workspace buffers (q: fp8 layers only).
+// Tensor maps over the weights and the handle's workspace buffers.
 int tc_bind(TcLayer& L, const eat_layer_desc& D, void* xperm, void* act, void* sact,
-            const TcQuant& q, const char** msg);
+            const TcWork& q, const char** msg);
 void tc_destroy(TcLayer& L);
 int tc_tile_rows(const TcLayer& L, int T);       // gate/up token rows per tile, call of T tokens
 int tc_tile_rows_down(const TcLayer& L, int T);  // down-projection token rows per tile

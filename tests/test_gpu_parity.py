@@ -216,6 +216,38 @@ def test_fp8_weights(name, Ts):
     layer.close()
 
 
+def test_fp8_hidden_state_magnitudes():
+    """fp8 layer, hidden-state rows scaled by 1e-6 ... 1e4 and one all-zero row: each row of the
+    GEMMs' other operand picks its own power-of-two scale before the e4m3 hi/lo split.  The router
+    weights are zero (routing by the bias alone), so the magnitudes reach only the expert GEMMs
+    (logits in the thousands would make the fp32 router, not the split, the limiting error)."""
+    lw = W.make_layer(QWEN_S)
+    lw.w_router = torch.zeros_like(lw.w_router)
+    lw8 = W.to_fp8(lw)
+    x = W.make_tokens(QWEN_S, 48)
+    x = (x.float() * torch.logspace(-6, 4, 48).view(48, 1)).to(x.dtype)
+    x[17] = 0
+    layer = eat.EatLayer.from_workload(lw8, 48, gpu_params(QWEN_S))
+    run_parity(QWEN_S, lw8.dequantized(), [48], layer=layer, inputs=[x])
+    layer.close()
+
+
+@pytest.mark.parametrize("fp8", [False, True])
+def test_many_short_gate_up_units(fp8):
+    """d_ff = 4096 over d_model = 256: 32 feature tiles per expert, so calls of 16 or more tokens
+    hand every CTA several gate/up units of only 4 (bf16) or 2 (e4m3) k-blocks, and the weight
+    prefetch of the down kernel spans units."""
+    sh = W.scaled(W.MIXTRAL, "short-k", d_model=256, d_ff=4096)
+    lw = W.make_layer(sh)
+    if fp8:
+        lw8 = W.to_fp8(lw)
+        layer = eat.EatLayer.from_workload(lw8, 100, gpu_params(sh))
+        run_parity(sh, lw8.dequantized(), [16, 64, 100, 1, 37], layer=layer)
+        layer.close()
+    else:
+        run_parity(sh, lw, [16, 64, 100, 1, 37])
+
+
 def test_partial_feature_tiles():
     """d = 320 and d_ff = 192: feature tiles of 128 end half-full in both expert GEMMs."""
     sh = W.scaled(W.QWEN, "ragged-d", d_model=320, n_experts=16, d_ff=192, n_shared=1,
@@ -416,6 +448,17 @@ def test_full_mixtral_decode_batches():
     for B in (1, 16, 64):
         layer = eat.EatLayer.from_workload(lw, 64, gpu_params(W.MIXTRAL))
         run_parity(W.MIXTRAL, lw, [B] * 3, layer=layer, L=L, sample=8, x_device="cuda")
+        layer.close()
+
+
+def test_full_mixtral_decode_fp8():
+    """The same layer with e4m3 expert weights (the fp8 decode configuration)."""
+    lw8 = W.to_fp8(_big(W.MIXTRAL))
+    dq = lw8.dequantized()
+    L = oracle_layer_lazy(dq)
+    for B in (1, 16, 64):
+        layer = eat.EatLayer.from_workload(lw8, 64, gpu_params(W.MIXTRAL))
+        run_parity(W.MIXTRAL, dq, [B] * 2, layer=layer, L=L, sample=8, x_device="cuda")
         layer.close()
 
 
