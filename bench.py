@@ -413,13 +413,16 @@ def run_ours(args, world, rank, local):
     xd = {B: torch.empty(B, shape.d_model, dtype=shape.xdtype, device=dev) for B in batches}
 
     def step_host(s):
+        # every call copies its x in and its y out inside the step; the step ends when the host
+        # holds all of the step's outputs
         for bi, B in enumerate(batches):
             if n_layers == 1:
-                eat.eat_moe_forward_host(handles[0][bi].h, xh[B][s % len(xh[B])], B, 0, yh[B])
+                eat.eat_moe_forward_host_async(handles[0][bi].h, xh[B][s % len(xh[B])], B, 0,
+                                               yh[B], stream)
             else:
                 xd[B].copy_(xh[B][s % len(xh[B])], non_blocking=True)
                 yh[B].copy_(layers_fwd(bi, B, xd[B]), non_blocking=True)
-                torch.cuda.current_stream().synchronize()
+        stream.synchronize()
 
     e2e_ms, _, _, _ = timed(step_host)
     e2e_ms = max_over_ranks(e2e_ms, world)

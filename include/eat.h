@@ -165,6 +165,16 @@ eat_status eat_moe_forward(eat_handle* h, const void* x, int32_t T, int32_t ppl_
 eat_status eat_moe_forward_host(eat_handle* h, const void* x_host, int32_t T, int32_t ppl_sign,
                                 void* y_host, void* stream);
 
+/* eat_moe_forward_host without the final synchronisation: enqueues the host-to-device copy of
+ * x_host, the layer and the device-to-host copy of y_host on `stream`, and returns.  The caller
+ * keeps both host buffers alive, and x_host unchanged, until the stream has passed this call
+ * (cudaStreamSynchronize or an event) and reads y_host only after that.  With page-locked host
+ * buffers (cudaHostAlloc / cudaHostRegister) the copies are asynchronous and consecutive calls
+ * queue back to back on the GPU; with pageable buffers the runtime may block.  Calls on one handle
+ * share its staging buffers, which stream order makes safe. */
+eat_status eat_moe_forward_host_async(eat_handle* h, const void* x_host, int32_t T,
+                                      int32_t ppl_sign, void* y_host, void* stream);
+
 /* Size of the fixed device scratch eat_route_noalloc uses (1 MiB = 131072 fp64 router scores). */
 #define EAT_NOALLOC_SCRATCH_BYTES (1u << 20)
 

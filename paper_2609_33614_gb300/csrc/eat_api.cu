@@ -491,8 +491,8 @@ eat_status eat_moe_forward(eat_handle* h, const void* x, int32_t T, int32_t ppl_
   return run_forward(h, x, T, ppl_sign, y, idx_opt, w_opt, k_opt, (cudaStream_t)stream);
 }
 
-eat_status eat_moe_forward_host(eat_handle* h, const void* x_host, int32_t T, int32_t ppl_sign,
-                                void* y_host, void* stream) {
+static eat_status forward_host(eat_handle* h, const void* x_host, int32_t T, int32_t ppl_sign,
+                               void* y_host, void* stream, bool sync) {
   EAT_TRY(check_call(h, x_host, T, ppl_sign));
   if (!y_host) return fail(h, EAT_ERR_INVALID_ARG, "y_host is NULL");
   cudaStream_t st = (cudaStream_t)stream;
@@ -501,9 +501,19 @@ eat_status eat_moe_forward_host(eat_handle* h, const void* x_host, int32_t T, in
   if (e != cudaSuccess) return cuda_fail(h, e, "x host-to-device copy");
   EAT_TRY(run_forward(h, h->xstage, T, ppl_sign, h->ystage, nullptr, nullptr, nullptr, st));
   e = cudaMemcpyAsync(y_host, h->ystage, bytes, cudaMemcpyDeviceToHost, st);
-  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  if (e == cudaSuccess && sync) e = cudaStreamSynchronize(st);
   if (e != cudaSuccess) return cuda_fail(h, e, "y device-to-host copy");
   return EAT_OK;
+}
+
+eat_status eat_moe_forward_host(eat_handle* h, const void* x_host, int32_t T, int32_t ppl_sign,
+                                void* y_host, void* stream) {
+  return forward_host(h, x_host, T, ppl_sign, y_host, stream, true);
+}
+
+eat_status eat_moe_forward_host_async(eat_handle* h, const void* x_host, int32_t T,
+                                      int32_t ppl_sign, void* y_host, void* stream) {
+  return forward_host(h, x_host, T, ppl_sign, y_host, stream, false);
 }
 
 eat_status eat_set_tau_state(eat_handle* h, float* tau_state) {

@@ -58,6 +58,7 @@ _SIGS = {
     "eat_route": (c_i32, [c_vp, c_vp, c_i32, c_i32, c_vp, c_vp, c_vp, c_vp]),
     "eat_moe_forward": (c_i32, [c_vp, c_vp, c_i32, c_i32, c_vp, c_vp, c_vp, c_vp, c_vp]),
     "eat_moe_forward_host": (c_i32, [c_vp, c_vp, c_i32, c_i32, c_vp, c_vp]),
+    "eat_moe_forward_host_async": (c_i32, [c_vp, c_vp, c_i32, c_i32, c_vp, c_vp]),
     "eat_route_noalloc": (c_i32, [c_vp, c_i32, c_i32, c_i32, c_i32, c_vp, c_vp, c_vp, c_vp, c_vp,
                                   ctypes.POINTER(eat_params), c_i32, c_vp, c_vp, c_vp, c_vp]),
     "eat_set_tau_state": (c_i32, [c_vp, c_vp]),
@@ -143,6 +144,12 @@ def eat_moe_forward(h, x, T, ppl_sign, y, idx=None, w=None, k=None, stream=None)
 def eat_moe_forward_host(h, x_host, T, ppl_sign, y_host, stream=None):
     _check(lib().eat_moe_forward_host(h, _ptr(x_host), T, ppl_sign, _ptr(y_host),
                                       _stream(stream)), h)
+
+
+def eat_moe_forward_host_async(h, x_host, T, ppl_sign, y_host, stream=None):
+    """Enqueue-only variant (see include/eat.h): synchronise the stream before reading y_host."""
+    _check(lib().eat_moe_forward_host_async(h, _ptr(x_host), T, ppl_sign, _ptr(y_host),
+                                            _stream(stream)), h)
 
 
 def eat_route_noalloc(x, T, d_model, n_experts, xdtype, w_router, b_router, N, P, C, params,

@@ -90,6 +90,7 @@ def test_null_handle_calls(lib):
     assert lib.eat_route(None, 1, 1, 0, 1, 1, 1, None) == eat.EAT_ERR_INVALID_ARG
     assert lib.eat_moe_forward(None, 1, 1, 0, 1, None, None, None, None) == eat.EAT_ERR_INVALID_ARG
     assert lib.eat_moe_forward_host(None, 1, 1, 0, 1, None) == eat.EAT_ERR_INVALID_ARG
+    assert lib.eat_moe_forward_host_async(None, 1, 1, 0, 1, None) == eat.EAT_ERR_INVALID_ARG
     assert lib.eat_reset_accounts(None, None) == eat.EAT_ERR_INVALID_ARG
     assert lib.eat_destroy(None) == eat.EAT_OK
     assert lib.eat_ffn_backend(None) == -1

@@ -321,6 +321,18 @@ def test_max_tokens_bound_and_host_path():
     yh = torch.empty_like(xh).pin_memory()
     eat.eat_moe_forward_host(layer.h, xh, 40, 0, yh)
     assert torch.equal(yh, y_dev.cpu())
+    # the enqueue-only variant: two calls queued back to back, one synchronisation; the second
+    # call routes with the accounts the first one updated
+    layer.set_accounts(*acc)
+    layer.forward(x[:40].contiguous(), 0)
+    y_dev2 = layer.forward(x[:40].contiguous(), 0)
+    layer.set_accounts(*acc)
+    yh1, yh2 = torch.empty_like(yh).pin_memory(), torch.empty_like(yh).pin_memory()
+    s = torch.cuda.current_stream()
+    eat.eat_moe_forward_host_async(layer.h, xh, 40, 0, yh1, s)
+    eat.eat_moe_forward_host_async(layer.h, xh, 40, 0, yh2, s)
+    s.synchronize()
+    assert torch.equal(yh1, y_dev.cpu()) and torch.equal(yh2, y_dev2.cpu())
     layer.close()
 
 
