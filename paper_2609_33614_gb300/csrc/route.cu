@@ -132,7 +132,10 @@ router_logits_small_kernel(const TX* __restrict__ x, const float* __restrict__ w
   const int beg = s * d_per_split;
   const int end = min(d, beg + d_per_split);
   const TX* xr = x + (size_t)t * d;
-  for (int e = warp; e < E; e += kLogitThreads / 32) {
+  // one expert per warp: blockIdx.z picks the group of kLogitThreads / 32 experts
+  {
+    const int e = blockIdx.z * (kLogitThreads / 32) + warp;
+    if (e >= E) return;
     const float* wrow = wr + (size_t)e * d;
     float hi = 0.f, lo = 0.f;
     float acc = 0.f;
@@ -304,7 +307,10 @@ constexpr int kSelectThreads = 256;
 // C_i / sum C, c_mode 1 the raw C_i.  sum N is exact (int64), sum C a compensated fp32 sum of the
 // fp32-rounded C_i; the three ratios are fp32 divisions (relative error ~3e-7, far inside the
 // 1e-5 margin at which a token's selection counts as decided).  No fp64 arithmetic: it would run
-// on GB300's narrow fp64 pipe in every block.
+// on GB300's narrow fp64 pipe in every block.  The selection kernel runs this before its
+// dependency wait: the accounts are at least two launches old (the router-score kernel comes
+// between), and every kernel lets its dependent start only after its own wait.  The loads bypass
+// L1 (ld.global.cg), which may still hold an earlier call's lines before the wait.
 __device__ void history_score_block(const int64_t* accN, const double* accP, const double* accC,
                                     int E, const RouteParams& rp, float* s_h) {
   __shared__ long long red_n[kSelectThreads / 32];
@@ -313,8 +319,8 @@ __device__ void history_score_block(const int64_t* accN, const double* accP, con
   long long n_sum = 0;
   float c_hi = 0.f, c_lo = 0.f;
   for (int e = tid; e < E; e += blockDim.x) {
-    n_sum += (long long)accN[e];
-    df_add(c_hi, c_lo, (float)accC[e]);
+    n_sum += (long long)__ldcg(accN + e);
+    df_add(c_hi, c_lo, (float)__ldcg(accC + e));
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
@@ -343,13 +349,14 @@ __device__ void history_score_block(const int64_t* accN, const double* accP, con
   const float total_n = (float)red_n[0];
   const float total_c = red_c[0][0];
   for (int e = tid; e < E; e += blockDim.x) {
-    const long long ni = accN[e];
+    const long long ni = __ldcg(accN + e);
     const float n = (float)ni;
     const float a = ni > 0 ? n / total_n : 0.f;
-    const float b = ni > 0 ? (float)accP[e] / n : 0.f;
+    const float b = ni > 0 ? (float)__ldcg(accP + e) / n : 0.f;
+    const float ce = (float)__ldcg(accC + e);
     float c;
-    if (rp.c_mode == EAT_C_RAW) c = (float)accC[e];
-    else c = total_c > 0.f ? (float)accC[e] / total_c : 0.f;
+    if (rp.c_mode == EAT_C_RAW) c = ce;
+    else c = total_c > 0.f ? ce / total_c : 0.f;
     s_h[e] = rp.w1 * a + rp.w2 * b + rp.w3 * c;
   }
   __syncthreads();
@@ -374,9 +381,9 @@ route_select_kernel(const float2* __restrict__ part, int n_split, const float* _
                     float* __restrict__ out_w, int32_t* __restrict__ out_k,
                     float* __restrict__ out_p) {
   __shared__ float s_h[kMaxExperts];
+  history_score_block(accN, accP, accC, E, rp, s_h);
   pdl_wait();
   pdl_launch_dependents();
-  history_score_block(accN, accP, accC, E, rp, s_h);
 
   const int lane = threadIdx.x & 31;
   const int warps = blockDim.x >> 5;
@@ -395,6 +402,7 @@ route_select_kernel(const float2* __restrict__ part, int n_split, const float* _
     float z = -INFINITY;
     if (valid[i]) {
       float hi = 0.f, lo = 0.f;
+#pragma unroll 8
       for (int sp = 0; sp < n_split; ++sp) {
         const float2 v = part[((size_t)sp * T + t) * E + e];
         df_add(hi, lo, v.x, v.y);
@@ -624,7 +632,7 @@ cudaError_t launch_router_logits(const void* x, int x_bf16, const float* w_route
   if (T <= kSmallT && vec_ok) {
     int per = (d + n_split - 1) / n_split;
     per = (per + 127) / 128 * 128;
-    dim3 grid(T, n_split);
+    dim3 grid(T, n_split, (E + kLogitThreads / 32 - 1) / (kLogitThreads / 32));
     if (x_bf16)
       return launch_pdl(router_logits_small_kernel<__nv_bfloat16>, grid, dim3(kLogitThreads), 0,
                         st, (const __nv_bfloat16*)x, w_router, T, d, E, per, part);
