@@ -47,9 +47,11 @@ def workload_spec(name):
         "qwen-prefill": dict(shape=W.QWEN, batches=[8192], layers=1,
                              desc="qwen1.5-moe-shaped layer (60 routed + 4 shared), prefill 8192"),
         "dsv2l-prefill": dict(shape=W.DSV2L, batches=[16384], layers=26,
-                              desc="deepseek-v2-lite-shaped 26-layer MoE stack, prefill 16384"),
+                              desc="deepseek-v2-lite-shaped 26-layer MoE stack (pre-norm residual "
+                                   "blocks), prefill 16384"),
         "dsv2l-decode": dict(shape=W.DSV2L, batches=[128], layers=26,
-                             desc="deepseek-v2-lite-shaped 26-layer MoE stack, decode batch 128"),
+                             desc="deepseek-v2-lite-shaped 26-layer MoE stack (pre-norm residual "
+                                  "blocks), decode batch 128"),
         # e4m3 expert weights with per-row scales (hidden states bf16, e4m3 x e4m3 GEMMs on the
         # hi/lo split of the other operand)
         "mixtral-decode-fp8": dict(shape=W.MIXTRAL, batches=[1, 16, 64], layers=1, fp8=True,
@@ -278,14 +280,24 @@ def run_ours(args, world, rank, local):
     ys = {B: torch.empty(B, shape.d_model, dtype=shape.xdtype, device=dev) for B in batches}
     tokens_per_step = sum(batches)
 
-    # residual stream buffers for stacks: x_{l+1} = x_l + y_l (the transformer block's residual
-    # add, outside the MoE layer)
+    # stacks run pre-norm blocks: the MoE layer reads RMSNorm(x_l) (unit gain) and the residual
+    # stream takes x_{l+1} = x_l + y_l, both outside the MoE layer.  (Without the norm the residual
+    # of the random-weight SwiGLU stack grows layer by layer until it overflows.)
     xr = {B: [torch.empty(B, shape.d_model, dtype=shape.xdtype, device=dev) for _ in range(2)]
           for B in batches}
 
-    def layers_fwd(bi, B, x):
+    def rms_norm(x):
+        return torch.nn.functional.rms_norm(x, (shape.d_model,), eps=1e-6)
+
+    def layers_fwd(bi, B, x, routing=None):
         for l in range(n_layers):
-            eat.eat_moe_forward(handles[l][bi].h, x, B, 0, ys[B])
+            h = rms_norm(x) if n_layers > 1 else x
+            if routing is None:
+                eat.eat_moe_forward(handles[l][bi].h, h, B, 0, ys[B])
+            else:  # also write the routing (idx, w, k) and count the tokens per k
+                idx, w, k, hist = routing
+                eat.eat_moe_forward(handles[l][bi].h, h, B, 0, ys[B], idx[B], w[B], k[B])
+                hist += torch.bincount(k[B].long(), minlength=hist.numel())
             if l + 1 < n_layers:
                 nxt = xr[B][l % 2]
                 torch.add(x, ys[B], out=nxt)
@@ -367,6 +379,22 @@ def run_ours(args, world, rank, local):
 
     # second pass with per-kernel CUDA events (roofline of the dominant kernel)
     ms_p, p0, p1, prof = timed(step_direct, profile=True)
+
+    # tokens per number of selected experts over the timed steps: an untimed replay from the same
+    # reset state with the routing written out (the routing is deterministic, so it is the timed
+    # run's)
+    reset_all()
+    kmax = shape.max_k
+    r_idx = {B: torch.empty(B, kmax, dtype=torch.int32, device=dev) for B in batches}
+    r_w = {B: torch.empty(B, kmax, dtype=torch.float32, device=dev) for B in batches}
+    r_k = {B: torch.empty(B, dtype=torch.int32, device=dev) for B in batches}
+    k_hist = torch.zeros(kmax + 1, dtype=torch.int64, device=dev)
+    scratch = torch.zeros_like(k_hist)
+    for s in range(n_steps_total):
+        for bi, B in enumerate(batches):
+            layers_fwd(bi, B, xs[B][s % len(xs[B])],
+                       (r_idx, r_w, r_k, k_hist if s >= args.warmup else scratch))
+    k_hist = {str(i): int(c) for i, c in enumerate(k_hist.cpu().tolist())}
     kinds = {}
     for l in range(n_layers):
         for bi, B in enumerate(batches):
@@ -443,6 +471,7 @@ def run_ours(args, world, rank, local):
         "roofline": roof,
         "experts_per_token": acts / max(1, sum(B * args.steps for B in batches) * n_layers),
         "union_per_call": unions,
+        "k_histogram": k_hist,
         "kernels_ms_per_step": {k: v["ms"] / args.steps for k, v in kinds.items()},
         "gpu_launches": launches,
         "clocks": clocks,

@@ -150,7 +150,9 @@ eat_status eat_reset_accounts(eat_handle* h, void* stream);
 eat_status eat_route(eat_handle* h, const void* x, int32_t T, int32_t ppl_sign,
                      int32_t* idx, float* w, int32_t* k, void* stream);
 
-/* One layer call = one EMA timestep of §3.2: routing as eat_route from the pre-call accounts,
+/* One layer call = one EMA timestep of §3.2 over T tokens, 1 <= T <= max_tokens (an empty call has
+ * no batch mean to fold into the accounts and is rejected with EAT_ERR_INVALID_ARG): routing as
+ * eat_route from the pre-call accounts,
  * y [T, d] (xdtype) = sum over selected e of g_norm,e * E_e(x_t) + sum of shared experts, then
  * the account update: N_e += n_e, P_total,e += sum of p over e's activations,
  * C_e <- (1 - alpha) C_e + alpha * mean ||E_e(x_t)||_2 when n_e > 0.

@@ -314,6 +314,18 @@ def test_max_tokens_bound_and_host_path():
     with pytest.raises(eat.EatError) as ei:
         eat.eat_moe_forward(layer.h, x, 41, 0, y)
     assert ei.value.status == eat.EAT_ERR_INVALID_ARG
+    # an empty call is rejected, by the layer call and by routing alone, and changes nothing
+    acc0 = layer.accounts()
+    idx = torch.empty(1, MIX_S.max_k, dtype=torch.int32, device="cuda")
+    w = torch.empty(1, MIX_S.max_k, dtype=torch.float32, device="cuda")
+    k = torch.empty(1, dtype=torch.int32, device="cuda")
+    for call in (lambda: eat.eat_moe_forward(layer.h, x, 0, 0, y),
+                 lambda: eat.eat_route(layer.h, x, 0, 0, idx, w, k)):
+        with pytest.raises(eat.EatError) as ei:
+            call()
+        assert ei.value.status == eat.EAT_ERR_INVALID_ARG
+    for u, v in zip(acc0, layer.accounts()):
+        assert torch.equal(u, v)
     acc = layer.accounts()
     y_dev = layer.forward(x[:40].contiguous(), 0)
     layer.set_accounts(*acc)
