@@ -38,6 +38,9 @@ Readings taken where the paper is silent or ambiguous (each is also listed in th
   R11 P_total accumulates the raw probability p of each activation.
   R12 C_s takes one EMA step per call with the batch mean of the unweighted expert-output L2
       norms of that expert's activations; experts with no activation keep C_s.
+  R15 a token whose routing probabilities are not all numbers (NaN: a non-finite hidden state
+      or router weight) selects no expert, in every router mode; its output row is NaN and it
+      adds nothing to the accounts.
   SwiGLU experts: E_e(x) = W_down (silu(W_gate x) * (W_up x)), silu(z) = z / (1 + exp(-z)).
 
 Parity pins (tests/test_oracle_pins.py): hand-worked examples of Eq. 1-8 (tests/golden),
@@ -307,7 +310,9 @@ def route(x: np.ndarray, layer: Layer, acc: Accounts, prm: Params, ppl_sign: int
     g_norm = np.zeros_like(p)
     for t in range(p.shape[0]):
         th = threshold(p[t], prm, ppl_sign, None if tau_prev is None else float(tau_prev[t]))
-        if prm.router == "eat":
+        if np.isnan(p[t]).any():
+            sel = []  # reading R15
+        elif prm.router == "eat":
             sel = select(I[t], th.tau_final, prm.max_k)
         elif prm.router == "topk":
             sel = topk_select(p[t], prm.max_k)
@@ -392,6 +397,9 @@ def moe_forward(x: np.ndarray, layer: Layer, acc: Accounts, prm: Params,
             y[t] += r.g_norm[t, e] * out[row]
             norms[(t, e)] = float(np.sqrt((out[row] ** 2).sum()))
     y += shared_output(x, layer)
+    for t in range(T):
+        if not r.selected[t]:
+            y[t] = np.nan  # reading R15
     new_acc = account_update(acc, r.selected, r.p, norms, prm.alpha)
     return ForwardResult(y, r, norms, new_acc)
 
@@ -407,6 +415,8 @@ def token_output(x_t: np.ndarray, layer: Layer, routing: Routing, t: int) -> tup
         y += routing.g_norm[t, e] * out
         norms[e] = float(np.sqrt((out ** 2).sum()))
     y += shared_output(x_t, layer)[0]
+    if not routing.selected[t]:
+        y[:] = np.nan  # reading R15
     return y, norms
 
 

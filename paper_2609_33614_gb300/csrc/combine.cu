@@ -85,7 +85,8 @@ __device__ __forceinline__ float warp_sum_many(float (&v)[N], int lane) {
 
 // Expert outputs are bf16 rows (OB, no split-K) or fp32 split-K partials; the shared experts'
 // outputs bf16 (s_bf16) or fp32.  Slots past k_t are -1 with gate 0.  All of a token's slot rows
-// are loaded before any use.
+// are loaded before any use.  A token with no selected expert (k_t = 0, which only a NaN routing
+// probability produces) gets a NaN row.
 template <typename TY, int KM, bool OB>
 __global__ void __launch_bounds__(kCombThreads)
 combine_kernel(const void* __restrict__ opart, int n_split, size_t split_stride,
@@ -169,6 +170,10 @@ combine_kernel(const void* __restrict__ opart, int n_split, size_t split_stride,
       const V8 q = load8(sout, s_bf16, ((size_t)s * T + t) * d + c);
 #pragma unroll
       for (int i = 0; i < 8; ++i) acc[i] += q.v[i];
+    }
+    if (slots[0] < 0) {  // no expert selected: the token's routing was not finite (NaN row)
+#pragma unroll
+      for (int i = 0; i < 8; ++i) acc[i] = __int_as_float(0x7fc00000);
     }
     store8(y + (size_t)t * d + c, acc);
   }

@@ -444,6 +444,13 @@ route_select_kernel(const float2* __restrict__ part, int n_split, const float* _
       psum += p[i];
     }
   }
+  // A NaN probability (non-finite hidden state or router weights) loses every comparison, which
+  // would select every expert in the rank-based modes: such a token selects none (reading R15 of
+  // the oracle), its output row is NaN and it adds nothing to the accounts.
+  bool nan_p = false;
+#pragma unroll
+  for (int i = 0; i < EPL; ++i) nan_p |= valid[i] && isnan(p[i]);
+  const bool bad = __any_sync(full, nan_p);
   // Eq. 3-4: mean and population standard deviation of g = p
   const float mu = warp_sum(psum) * inv_e;
   float dev = 0.f;
@@ -581,6 +588,10 @@ route_select_kernel(const float2* __restrict__ part, int n_split, const float* _
     for (int i = 0; i < EPL; ++i) sel[i] = cand[i] && r[i] < K;
   }
 
+  if (bad) {
+#pragma unroll
+    for (int i = 0; i < EPL; ++i) sel[i] = false;
+  }
   // Eq. 7-8: renormalised gates over the selected experts, g = p
   float gs = 0.f;
 #pragma unroll

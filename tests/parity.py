@@ -115,6 +115,9 @@ def check_routing(routing: orc.Routing, sel_gpu: list, w_gpu: np.ndarray, K: int
     for t, sel in enumerate(sel_gpu):
         I, tau = routing.I[t], routing.tau_final[t]
         assert sel == sorted(sel), f"token {t}: idx not ascending {sel}"
+        if np.isnan(routing.p[t]).any():  # reading R15: no expert, zero gates
+            assert sel == [] and np.all(w_gpu[t] == 0.0), f"token {t}: NaN p selected {sel}"
+            continue
         if mode != "eat":
             if ambiguous_baseline(routing.p[t], K, mode, top_p):
                 amb.append(t)
@@ -164,6 +167,9 @@ def oracle_outputs(x64: np.ndarray, layer: orc.Layer, routing: orc.Routing, sel:
         sh = orc.shared_output(x64[idx], layer)
         for r, t in enumerate(idx):
             y[t] = y[t] + sh[r]
+    for t in toks:
+        if not sel[t]:
+            y[t] = np.full(x64.shape[1], np.nan)  # reading R15
     return y, norms
 
 
@@ -182,13 +188,24 @@ def oracle_outputs_batched(x64, layer, routing, sel, eps):
             y[t] += g * o[r]
             norms[(t, e)] = float(np.sqrt((o[r] ** 2).sum()))
     y += orc.shared_output(x64, layer)
+    for t in range(T):
+        if not sel[t]:
+            y[t] = np.nan  # reading R15
     return y, norms
 
 
 def rel_err_rows(y_gpu: np.ndarray, y_ref: np.ndarray) -> np.ndarray:
-    den = np.abs(y_ref).max(axis=1)
+    """Per row: max |gpu - ref| / max |ref|; a NaN reference row (reading R15) matches only an
+    all-NaN GPU row (error 0, else inf)."""
+    nan_ref = np.isnan(y_ref).all(axis=1)
+    yr = np.where(nan_ref[:, None], 0.0, y_ref)
+    yg = np.where(nan_ref[:, None], 0.0, y_gpu)
+    den = np.abs(yr).max(axis=1)
     den[den == 0] = 1.0
-    return np.abs(y_gpu - y_ref).max(axis=1) / den
+    err = np.abs(yg - yr).max(axis=1) / den
+    err[nan_ref] = np.where(np.isnan(y_gpu[nan_ref]).all(axis=1), 0.0, np.inf)
+    err[np.isnan(err)] = np.inf
+    return err
 
 
 def check_accounts(acc_before: orc.Accounts, acc_gpu_after, stats_gpu, routing, sel, norms_ref,

@@ -216,6 +216,25 @@ def test_fp8_weights(name, Ts):
     layer.close()
 
 
+@pytest.mark.parametrize("mode", ["eat", "topk", "topp"])
+def test_nonfinite_tokens_select_nothing(mode):
+    """Tokens with a NaN or an infinite hidden-state element (reading R15): in every router mode
+    they select no expert (k = 0, the rank-based modes included), their output rows are NaN, and
+    the other tokens and the accounts follow the oracle."""
+    kw = {"eat": {}, "topk": {"router_mode": eat.EAT_ROUTER_TOPK},
+          "topp": {"router_mode": eat.EAT_ROUTER_TOPP, "top_p": 0.6}}[mode]
+    lw = W.make_layer(QWEN_S)
+    x = W.make_tokens(QWEN_S, 40)
+    x[5, 3] = float("nan")
+    x[9, 100] = float("inf")
+    x[39] = float("nan")
+    outs = run_parity(QWEN_S, lw, [40], prm_kw=kw, inputs=[x])
+    y = outs[0]
+    for t in (5, 9, 39):
+        assert torch.isnan(y[t]).all()
+    assert not torch.isnan(y[[0, 1, 2, 10, 38]]).any()
+
+
 def test_fp8_hidden_state_magnitudes():
     """fp8 layer, hidden-state rows scaled by 1e-6 ... 1e4 and one all-zero row: each row of the
     GEMMs' other operand picks its own power-of-two scale before the e4m3 hi/lo split.  The router

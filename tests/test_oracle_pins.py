@@ -546,3 +546,33 @@ def test_temporal_equals_call_when_prev_is_tau():
         a = orc.threshold(p, P0, 1)
         b = orc.threshold(p, P0.with_(smoothing="temporal"), 1, a.tau)
         assert close(a.tau_final, b.tau_final)
+
+
+def test_nan_token_selects_nothing_and_leaves_accounts():
+    """Reading R15: a token with a non-finite hidden state has NaN routing probabilities; in every
+    router mode it selects no expert, its output row is NaN, and the other tokens' outputs and the
+    account update equal those of the same call without it."""
+    import oracle.eat_oracle as orc
+    rng = np.random.default_rng(13)
+    E, d, F, T = 6, 16, 12, 9
+    layer = orc.Layer(rng.normal(0, 0.3, (E, d)), rng.normal(0, 0.5, E),
+                      rng.normal(0, 0.2, (E, F, d)), rng.normal(0, 0.2, (E, F, d)),
+                      rng.normal(0, 0.2, (E, d, F)))
+    x = rng.normal(0, 1, (T, d))
+    x[2, 5] = np.nan
+    x[6, 0] = np.inf
+    keep = [t for t in range(T) if t not in (2, 6)]
+    acc = orc.Accounts(np.array([3, 0, 5, 1, 2, 4], np.int64), rng.uniform(0, 2, E),
+                       rng.uniform(0, 1, E))
+    for router in ("eat", "topk", "topp"):
+        prm = orc.Params(max_k=2, router=router)
+        full = orc.moe_forward(x, layer, acc, prm)
+        part = orc.moe_forward(x[keep], layer, acc, prm)
+        assert full.routing.selected[2] == [] and full.routing.selected[6] == []
+        assert np.isnan(full.y[2]).all() and np.isnan(full.y[6]).all()
+        assert np.allclose(full.y[keep], part.y, rtol=1e-12, atol=1e-14)
+        assert np.array_equal(full.accounts_after.N, part.accounts_after.N)
+        assert np.allclose(full.accounts_after.P, part.accounts_after.P, rtol=1e-13)
+        assert np.allclose(full.accounts_after.C, part.accounts_after.C, rtol=1e-13)
+        assert np.array_equal(full.accounts_after.N, acc.N + np.bincount(
+            [e for t in keep for e in full.routing.selected[t]], minlength=E))
