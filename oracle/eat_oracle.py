@@ -18,7 +18,7 @@ Paper: "EAT: Expert Account Tracker for Efficient MoE Inference" (arxiv 2609.336
   * §4.1  Top-P comparison router (P = 0.6 / 0.2 / 0.4) and the vanilla fixed Top-K router
 
 Readings taken where the paper is silent or ambiguous (each is also listed in the design notes):
-  R1  the "raw router gating score g" of §3.3 is the softmax probability p of §3.2 (g == p).
+  R1  the raw gating score g that §3.3 thresholds is the softmax probability p of §3.2 (g == p).
   R2  empty-history terms of Eq. 1 are 0 (N_i/sum N with sum N = 0, P_i/N_i with N_i = 0).
   R3  c_mode "sum" (default): the C_s term of Eq. 1 enters as the share C_i / sum_j C_j;
       c_mode "raw": the literal C_i.

@@ -1,7 +1,7 @@
-// Tensor-core expert FFN kernels for bf16 layers (the dominant cost of the EAT MoE layer): grouped
-// SwiGLU expert GEMMs over the activated experts only (§3.4: "only activated experts ...
-// participate"), written for sm_103a with tcgen05.mma (accumulators in TMEM), TMA tile loads into
-// 128B-swizzled shared memory and mbarrier pipelines.
+// Tensor-core expert FFN kernels for bf16 and e4m3-weight layers (the dominant cost of the EAT MoE
+// layer): grouped SwiGLU expert GEMMs over the activated experts only (§3.4: an expert runs only
+// on the tokens that selected it), written for sm_103a with tcgen05.mma (accumulators in TMEM),
+// TMA tile loads into 128B-swizzled shared memory and mbarrier pipelines.
 //
 // Orientation ("swap AB"): a tile is 128 weight rows (output features of one expert) x BN tokens
 // (16..128 rows of that expert's slot list), so decode calls with a handful of tokens still issue

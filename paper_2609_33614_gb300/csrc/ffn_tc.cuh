@@ -1,5 +1,5 @@
-// Tensor-core (tcgen05 + TMEM + TMA) expert FFN kernels for bf16 layers: interface used by the
-// host runtime.
+// Tensor-core (tcgen05 + TMEM + TMA) expert FFN kernels for bf16 and e4m3-weight layers:
+// interface used by the host runtime.
 #pragma once
 
 #include "eat_internal.cuh"

@@ -1,5 +1,5 @@
 // Permute by expert: groups the selected (token, expert) pairs of one call by expert so that the
-// expert FFNs read contiguous row lists ("only activated experts participate", §3.4).
+// expert FFNs read contiguous row lists (§3.4: an expert runs only on the tokens that selected it).
 //
 // Every pair gets a STABLE slot (tokens ascending inside each expert), so every later per-expert
 // sum (P_total, the EMA norm mean) runs in a fixed order.  Inside a CTA each warp builds, per
