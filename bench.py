@@ -60,6 +60,9 @@ def workload_spec(name):
         "olmoe-decode-fp8": dict(shape=W.OLMOE, batches=[32], layers=1, fp8=True,
                                  desc="olmoe-shaped MoE layer, e4m3 expert weights, decode "
                                       "batch 32 per step"),
+        "olmoe-prefill-fp8": dict(shape=W.OLMOE, batches=[4096], layers=1, fp8=True,
+                                  desc="olmoe-shaped MoE layer, e4m3 expert weights, prefill "
+                                       "4096 tokens per step"),
     }
     return specs[name]
 

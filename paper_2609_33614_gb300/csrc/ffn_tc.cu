@@ -1054,8 +1054,67 @@ __device__ __forceinline__ float amax8(const uint4& u, float m) {
   return m;
 }
 
-// One CTA per row; rows of up to 256 x kSplitRegs 16-byte vectors (16384 bf16) are read once and
-// kept in registers, longer ones are read twice.
+// The row's power-of-two scale from its largest magnitude m: s with m / s in [128, 256), its
+// inverse, and a NaN scale for a non-finite m (rows below 2^-119 keep scale 1).
+__device__ __forceinline__ void split_scale(float m, float& s, float& inv) {
+  const uint32_t ex = (__float_as_uint(m) >> 23) & 0xffu;  // m in [2^(ex-127), 2^(ex-126))
+  s = 1.0f;
+  inv = 1.0f;
+  if (ex == 0xffu) {
+    s = __uint_as_float(0x7fc00000u);
+  } else if (ex >= 8u) {
+    s = __uint_as_float((ex - 7u) << 23);     // 2^(ex - 134)
+    inv = __uint_as_float((261u - ex) << 23);  // 2^(134 - ex)
+  }
+}
+
+// Rows of at most 32 x VPL 16-byte vectors (256 bf16 per VPL): one warp per row, the row held in
+// registers and reduced with shuffles, eight rows per 256-thread CTA and no block barrier, so a
+// prefill call keeps thousands of rows in flight.
+template <int VPL>
+__global__ void __launch_bounds__(256)
+split_e4m3_warp_kernel(const __nv_bfloat16* __restrict__ src, const int32_t* __restrict__ map,
+                       const int32_t* __restrict__ n_dev, int n_host, int cols,
+                       uint8_t* __restrict__ dst, long long plane, float* __restrict__ scale) {
+  pdl_wait();
+  pdl_launch_dependents();
+  const int n = n_dev ? *n_dev : n_host;
+  const int lane = threadIdx.x & 31;
+  const int r = blockIdx.x * 8 + (threadIdx.x >> 5);
+  if (r >= n) return;
+  const int vecs = cols >> 3;
+  const int sr = map ? map[r] : r;
+  const uint4* row = (const uint4*)(src + (size_t)sr * cols);
+  uint4 v[VPL];
+  float m = 0.0f;
+#pragma unroll
+  for (int j = 0; j < VPL; ++j) {
+    const int i = lane + 32 * j;
+    v[j] = i < vecs ? row[i] : make_uint4(0u, 0u, 0u, 0u);
+  }
+#pragma unroll
+  for (int j = 0; j < VPL; ++j) m = amax8(v[j], m);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+  float s, inv;
+  split_scale(m, s, inv);
+  if (lane == 0) scale[r] = s;
+  uint2* hi_row = (uint2*)(dst + (size_t)r * cols);
+  uint2* lo_row = (uint2*)(dst + plane + (size_t)r * cols);
+#pragma unroll
+  for (int j = 0; j < VPL; ++j) {
+    const int i = lane + 32 * j;
+    if (i < vecs) {
+      uint2 h, l;
+      split8(v[j], inv, h, l);
+      hi_row[i] = h;
+      lo_row[i] = l;
+    }
+  }
+}
+
+// Longer rows: one CTA per row; rows of up to 256 x kSplitRegs 16-byte vectors (16384 bf16) are
+// read once and kept in registers, longer ones are read twice.
 constexpr int kSplitRegs = 8;
 
 __global__ void __launch_bounds__(256)
@@ -1093,14 +1152,8 @@ split_e4m3_kernel(const __nv_bfloat16* __restrict__ src, const int32_t* __restri
 #pragma unroll
     for (int i = 1; i < 8; ++i) m = fmaxf(m, red[i]);
     __syncthreads();  // red is rewritten for the next row
-    const uint32_t ex = (__float_as_uint(m) >> 23) & 0xffu;  // m in [2^(ex-127), 2^(ex-126))
-    float s = 1.0f, inv = 1.0f;                              // rows below 2^-119: scale 1
-    if (ex == 0xffu) {
-      s = __uint_as_float(0x7fc00000u);
-    } else if (ex >= 8u) {
-      s = __uint_as_float((ex - 7u) << 23);     // 2^(ex - 134)
-      inv = __uint_as_float((261u - ex) << 23);  // 2^(134 - ex)
-    }
+    float s, inv;
+    split_scale(m, s, inv);
     if (tid == 0) scale[r] = s;
     uint2* hi_row = (uint2*)(dst + (size_t)r * cols);
     uint2* lo_row = (uint2*)(dst + plane + (size_t)r * cols);
@@ -1486,6 +1539,14 @@ cudaError_t tc_launch_split(const TcLayer& L, const TcCall& c, TcSplit which, cu
       break;
   }
   if (n_host <= 0) return cudaSuccess;
+  const int vecs = cols / 8;
+  const dim3 wgrid((n_host + 7) / 8);
+  if (vecs <= 32 * 8)
+    return launch_pdl(split_e4m3_warp_kernel<8>, wgrid, dim3(256), 0, st, src, map, n_dev, n_host,
+                      cols, dst, plane_rows * cols, scale);
+  if (vecs <= 32 * 16)
+    return launch_pdl(split_e4m3_warp_kernel<16>, wgrid, dim3(256), 0, st, src, map, n_dev,
+                      n_host, cols, dst, plane_rows * cols, scale);
   const int grid = std::min(n_host, 4 * L.num_sms);
   return launch_pdl(split_e4m3_kernel, dim3(grid), dim3(256), 0, st, src, map, n_dev, n_host,
                     cols, dst, plane_rows * cols, scale);
