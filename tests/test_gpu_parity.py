@@ -202,12 +202,34 @@ def test_sm_pair_one_large_group():
     run_parity(OLMOE_S, lw, [2100])
 
 
+@pytest.mark.parametrize("E,K,T", [(256, 8, 1500), (64, 2, 1100)])
+def test_fp8_large_calls_small_groups(E, K, T):
+    """e4m3 weights at call sizes where bf16 layers switch to the SM-pair kernels (fp8 layers keep
+    the single-SM kernels, 128-token tiles): mostly partial tiles."""
+    sh = W.scaled(W.OLMOE, f"pair8-{E}", d_model=256, n_experts=E, d_ff=384, max_k=K)
+    lw8 = W.to_fp8(W.make_layer(sh))
+    layer = eat.EatLayer.from_workload(lw8, T, gpu_params(sh))
+    run_parity(sh, lw8.dequantized(), [T, T], layer=layer)
+    layer.close()
+
+
+def test_fp8_large_call_one_group():
+    """e4m3 weights, one expert takes all 2100 tokens: 16 full 128-token tiles and a partial one."""
+    lw = W.make_layer(OLMOE_S)
+    lw.b_router = torch.full_like(lw.b_router, -30.0)
+    lw.b_router[7] = 30.0
+    lw8 = W.to_fp8(lw)
+    layer = eat.EatLayer.from_workload(lw8, 2100, gpu_params(OLMOE_S))
+    run_parity(OLMOE_S, lw8.dequantized(), [2100], layer=layer)
+    layer.close()
+
+
 # ------------------------------------------------------------------ fp8 (e4m3) expert weights
 @pytest.mark.parametrize("name,Ts", [("mixtral", [1, 16, 64]), ("olmoe", [32, 300, 1100]),
-                                     ("qwen", [64, 200])])
+                                     ("qwen", [64, 200, 1500])])
 def test_fp8_weights(name, Ts):
-    """e4m3 expert weights with per-row scales (the fp8 decode path, also at 300 and 1100 tokens,
-    which stay on single SMs): the oracle runs on the dequantized weights."""
+    """e4m3 expert weights with per-row scales, decode sizes and calls of 1100 / 1500 tokens
+    (qwen: routed and shared experts); the oracle runs on the dequantized weights."""
     shape = {"mixtral": MIX_S, "olmoe": OLMOE_S, "qwen": QWEN_S}[name]
     lw8 = W.to_fp8(W.make_layer(shape))
     layer = eat.EatLayer.from_workload(lw8, max(Ts), gpu_params(shape))
