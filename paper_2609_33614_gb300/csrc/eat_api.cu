@@ -1,6 +1,10 @@
 // extern "C" boundary of libeat.so (declared in include/eat.h): handle, argument validation,
 // workspace, and the stream-ordered launch sequence of one EAT MoE layer call.
 #include "eat_internal.cuh"
+#if __has_include(<nvtx3/nvToolsExt.h>)
+#include <nvtx3/nvToolsExt.h>
+#define EAT_HAVE_NVTX 1
+#endif
 #include "ffn_tc.cuh"
 
 #include <algorithm>
@@ -82,11 +86,26 @@ enum Kind {
 };
 
 // Run one launch, optionally bracketed by CUDA events for the per-kernel profile.
+inline void nvtx_push(const char* what) {
+#ifdef EAT_HAVE_NVTX
+  nvtxRangePushA(what);
+#else
+  (void)what;
+#endif
+}
+inline void nvtx_pop() {
+#ifdef EAT_HAVE_NVTX
+  nvtxRangePop();
+#endif
+}
+
 template <typename Fn>
 eat_status launch(eat_handle* h, int kind, cudaStream_t st, const char* what, Fn&& fn) {
   const bool rec = h->prof && h->prof_n < h->prof_cap;
   if (rec) cudaEventRecord(h->ev[2 * h->prof_n], st);
+  nvtx_push(what);  // a named range per launch for timeline tools (no-op without one attached)
   const cudaError_t e = fn();
+  nvtx_pop();
   ++h->launches;
   if (rec) {
     cudaEventRecord(h->ev[2 * h->prof_n + 1], st);
@@ -433,6 +452,7 @@ eat_status eat_create(const eat_layer_desc* desc, const eat_params* params, eat_
   for (auto& p : parts) total = align_up(total, 256) + align_up(p.bytes, 256);
   cudaError_t e = cudaMalloc(&h->mem, total);
   if (e != cudaSuccess) {
+    cudaGetLastError();  // a failed allocation leaves the context usable: clear its error
     free_handle(h);
     return fail(nullptr, EAT_ERR_OOM,
                 "cudaMalloc of " + std::to_string(total) + " bytes failed: " +

@@ -6,6 +6,8 @@ selections and k bit-exact on non-ambiguous tokens, gates within 1e-5, n_e and N
 and the C_s update rule within 1e-6 relative, C_s against the oracle's norms within 1e-6 (fp32)
 or 2e-2 (bf16), layer outputs within 1e-5 (fp32) or 2e-2 (bf16) max relative error per token.
 """
+import ctypes
+
 import numpy as np
 import pytest
 import torch
@@ -255,6 +257,93 @@ def test_nonfinite_tokens_select_nothing(mode):
     for t in (5, 9, 39):
         assert torch.isnan(y[t]).all()
     assert not torch.isnan(y[[0, 1, 2, 10, 38]]).any()
+
+
+def test_toy_free_running_first_divergence():
+    """The toy configuration run free for 16 steps: the GPU and the oracle each evolve their own
+    accounts (no teacher forcing).  Selections must agree token for token until the first step
+    that holds a near-tie token (the only legitimate source of a difference, which then feeds
+    different accounts into every later step); the step reached is printed."""
+    sh = W.TOY
+    lw = W.make_layer(sh)
+    layer = eat.EatLayer.from_workload(lw, 64, gpu_params(sh))
+    L = oracle_layer(lw)
+    prm = oracle_params(sh)
+    acc = orc.Accounts.zeros(sh.n_experts)
+    first = None
+    for step in range(16):
+        x = W.make_tokens(sh, 64, step=step)
+        _, idx, w, k = layer.forward(x.cuda(), 0, with_routing=True)
+        res = orc.moe_forward(np64(x), L, acc, prm)
+        sel_gpu = par.gpu_selection(idx, k)
+        near = [t for t in range(64)
+                if par.ambiguous(res.routing.I[t], res.routing.tau_final[t], sh.max_k)]
+        diff = [t for t in range(64) if sel_gpu[t] != res.routing.selected[t]]
+        if diff:
+            assert set(diff) <= set(near), f"step {step}: tokens {diff} differ without a near-tie"
+            first = step
+            break
+        if near:  # a near-tie agreed this time; later accounts may still drift apart
+            first = step
+            break
+        N, P, C = (t.cpu().numpy() for t in layer.accounts())
+        assert np.array_equal(N, res.accounts_after.N)
+        assert np.allclose(P, res.accounts_after.P, rtol=1e-6)
+        assert np.allclose(C, res.accounts_after.C, rtol=1e-5, atol=1e-12)
+        acc = res.accounts_after
+    print(f"free-running toy: identical through step {15 if first is None else first - 1}")
+    layer.close()
+
+
+def test_two_handles_on_two_streams_interleaved():
+    """Two handles (one layer each) driven from two CUDA streams with their calls interleaved give
+    the results of running each alone: a handle's workspace and accounts are its own."""
+    lw = W.make_layer(OLMOE_S)
+    xs = [W.make_tokens(OLMOE_S, 48, step=s).cuda() for s in range(4)]
+    ref = []
+    solo = eat.EatLayer.from_workload(lw, 48, gpu_params(OLMOE_S))
+    for x in xs:
+        ref.append(solo.forward(x, 0).clone())
+    solo.close()
+    a = eat.EatLayer.from_workload(lw, 48, gpu_params(OLMOE_S))
+    b = eat.EatLayer.from_workload(lw, 48, gpu_params(OLMOE_S))
+    sa, sb = torch.cuda.Stream(), torch.cuda.Stream()
+    ya = [torch.empty_like(x) for x in xs]
+    yb = [torch.empty_like(x) for x in xs]
+    torch.cuda.synchronize()
+    for i, x in enumerate(xs):
+        eat.eat_moe_forward(a.h, x, 48, 0, ya[i], stream=sa)
+        eat.eat_moe_forward(b.h, x, 48, 0, yb[i], stream=sb)
+    torch.cuda.synchronize()
+    for i in range(4):
+        assert torch.equal(ya[i], ref[i]) and torch.equal(yb[i], ref[i])
+    a.close()
+    b.close()
+
+
+def test_workspace_allocation_failure_and_new_handle():
+    """A layer whose workspace cannot be allocated (65536 tokens x 16 experts of d_ff 262144:
+    over 500 GB of activations) fails with EAT_ERR_OOM, leaves no handle and no pending CUDA
+    error; the context stays usable, and a handle created after another was destroyed works."""
+    fields = dict(d_model=64, n_experts=16, d_ff=262144, n_shared=0, d_ff_shared=0,
+                  max_tokens=65536, wdtype=eat.EAT_BF16, xdtype=eat.EAT_BF16, w_router=1 << 20,
+                  b_router=None, w_gate=1 << 21, w_up=1 << 22, w_down=1 << 23, ws_gate=None,
+                  ws_up=None, ws_down=None, opd_scale=None, w_gate_scale=None, w_up_scale=None,
+                  w_down_scale=None, ws_gate_scale=None, ws_up_scale=None, ws_down_scale=None)
+    big = eat.eat_layer_desc(*[fields[n] for n, _ in eat.eat_layer_desc._fields_])
+    prm = eat.eat_default_params(16)
+    h = ctypes.c_void_p()
+    r = eat.lib().eat_create(ctypes.byref(big), ctypes.byref(prm), ctypes.byref(h))
+    assert r == eat.EAT_ERR_OOM and h.value is None
+    assert b"cudaMalloc" in eat.lib().eat_last_error(None)
+    torch.cuda.synchronize()
+    assert torch.cuda.is_available() and (torch.ones(4, device="cuda") * 2).sum().item() == 8
+    lw = W.make_layer(MIX_S)
+    layer0 = eat.EatLayer.from_workload(lw, 8, gpu_params(MIX_S))
+    layer0.close()
+    layer1 = eat.EatLayer.from_workload(lw, 8, gpu_params(MIX_S))
+    run_parity(MIX_S, lw, [8], layer=layer1)
+    layer1.close()
 
 
 def test_fp8_hidden_state_magnitudes():
