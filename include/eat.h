@@ -163,7 +163,10 @@ eat_status eat_moe_forward(eat_handle* h, const void* x, int32_t T, int32_t ppl_
 
 /* eat_moe_forward with HOST buffers: copies x_host [T, d] to the device, runs the layer, copies
  * y back into y_host [T, d] and synchronises the stream before returning.  Pinned host memory
- * gives asynchronous copies; pageable memory works but is staged by the driver. */
+ * gives asynchronous copies; pageable memory works but is staged by the driver.  The input copy
+ * runs on a stream of the handle (created on the first host-buffer call) into one of two staging
+ * buffers used in turn, so it overlaps the kernels of the handle's previous call; the layer's
+ * kernels on `stream` wait for it. */
 eat_status eat_moe_forward_host(eat_handle* h, const void* x_host, int32_t T, int32_t ppl_sign,
                                 void* y_host, void* stream);
 

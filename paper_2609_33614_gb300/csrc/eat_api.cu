@@ -47,8 +47,14 @@ struct eat_handle {
   void* sact = nullptr;   // [S*Tmax, Fs]
   float* sout = nullptr;  // [S*Tmax, d] (fp32; bf16 on the tensor-core path)
   TcWork q;               // fp8 layers: B-operand planes and scales
-  void* xstage = nullptr; // [Tmax, d]
+  void* xstage = nullptr; // [2][Tmax, d] inputs of host-buffer calls, used in turn
   void* ystage = nullptr; // [Tmax, d]
+  // host-buffer calls copy their input on their own stream, into the staging buffer the call
+  // before last used, so the copy overlaps the previous call's kernels (created on first use)
+  cudaStream_t copy_st = nullptr;
+  cudaEvent_t ev_copied[2] = {nullptr, nullptr};  // input copy i done (copy stream)
+  cudaEvent_t ev_done[2] = {nullptr, nullptr};    // the call that read buffer i done (its stream)
+  int stage_i = 0;
   void* xperm = nullptr;  // [Tmax*K, d] gathered token rows (tensor-core path)
   unsigned int* status = nullptr;  // device status word: bounded waits that expired
   int32_t* chunk_cnt = nullptr;    // permute scratch: ticket word, then [chunks][E] counts
@@ -283,6 +289,11 @@ eat_status run_forward(eat_handle* h, const void* x, int T, int ppl_sign, void* 
 void free_handle(eat_handle* h) {
   if (!h) return;
   for (cudaEvent_t e : h->ev) cudaEventDestroy(e);
+  for (int i = 0; i < 2; ++i) {
+    if (h->ev_copied[i]) cudaEventDestroy(h->ev_copied[i]);
+    if (h->ev_done[i]) cudaEventDestroy(h->ev_done[i]);
+  }
+  if (h->copy_st) cudaStreamDestroy(h->copy_st);
   tc_destroy(h->tc);
   if (h->mem) cudaFree(h->mem);
   delete h;
@@ -446,7 +457,7 @@ eat_status eat_create(const eat_layer_desc* desc, const eat_params* params, eat_
       add(&h->q.saq_s, sizeof(float) * (size_t)h->S * h->Tmax);
     }
   }
-  add(&h->xstage, h->elt * (size_t)h->Tmax * h->d);
+  add(&h->xstage, 2 * h->elt * (size_t)h->Tmax * h->d);
   add(&h->ystage, h->elt * (size_t)h->Tmax * h->d);
   size_t total = 0;
   for (auto& p : parts) total = align_up(total, 256) + align_up(p.bytes, 256);
@@ -517,10 +528,28 @@ static eat_status forward_host(eat_handle* h, const void* x_host, int32_t T, int
   if (!y_host) return fail(h, EAT_ERR_INVALID_ARG, "y_host is NULL");
   cudaStream_t st = (cudaStream_t)stream;
   const size_t bytes = h->elt * (size_t)T * h->d;
-  cudaError_t e = cudaMemcpyAsync(h->xstage, x_host, bytes, cudaMemcpyHostToDevice, st);
+  cudaError_t e = cudaSuccess;
+  if (!h->copy_st) {
+    e = cudaStreamCreateWithFlags(&h->copy_st, cudaStreamNonBlocking);
+    for (int i = 0; i < 2 && e == cudaSuccess; ++i) {
+      e = cudaEventCreateWithFlags(&h->ev_copied[i], cudaEventDisableTiming);
+      if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_done[i], cudaEventDisableTiming);
+    }
+    if (e != cudaSuccess) return cuda_fail(h, e, "copy stream setup");
+  }
+  const int i = h->stage_i;
+  h->stage_i ^= 1;
+  void* xs = (char*)h->xstage + (size_t)i * h->elt * h->Tmax * h->d;
+  // the copy waits for the call that last read this buffer (an event never recorded counts as
+  // complete), and this call's kernels wait for the copy
+  e = cudaStreamWaitEvent(h->copy_st, h->ev_done[i], 0);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(xs, x_host, bytes, cudaMemcpyHostToDevice, h->copy_st);
+  if (e == cudaSuccess) e = cudaEventRecord(h->ev_copied[i], h->copy_st);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(st, h->ev_copied[i], 0);
   if (e != cudaSuccess) return cuda_fail(h, e, "x host-to-device copy");
-  EAT_TRY(run_forward(h, h->xstage, T, ppl_sign, h->ystage, nullptr, nullptr, nullptr, st));
-  e = cudaMemcpyAsync(y_host, h->ystage, bytes, cudaMemcpyDeviceToHost, st);
+  EAT_TRY(run_forward(h, xs, T, ppl_sign, h->ystage, nullptr, nullptr, nullptr, st));
+  e = cudaEventRecord(h->ev_done[i], st);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(y_host, h->ystage, bytes, cudaMemcpyDeviceToHost, st);
   if (e == cudaSuccess && sync) e = cudaStreamSynchronize(st);
   if (e != cudaSuccess) return cuda_fail(h, e, "y device-to-host copy");
   return EAT_OK;
