@@ -362,14 +362,66 @@ __device__ void history_score_block(const int64_t* accN, const double* accP, con
   __syncthreads();
 }
 
-// Value of rank r (0-based ascending, ties by index) among the token's probabilities.
+// Warp-wide bitonic sort of the 32 x EPL (key, index) pairs a warp holds (element j * 32 + lane
+// in register j of that lane), ascending by key and, for equal keys, by index: the order the
+// selection's rank rules use.  The network is fixed (no data-dependent branches on the warp's
+// control flow); strides below 32 exchange across lanes, larger ones between a lane's registers.
 template <int EPL>
-__device__ __forceinline__ float order_stat(const float (&p)[EPL], const int (&rank)[EPL],
-                                            const bool (&valid)[EPL], int r) {
-  float v = 0.f;
+__device__ __forceinline__ void warp_sort_pairs(float (&k)[EPL], int (&x)[EPL], int lane) {
+  const unsigned full = 0xffffffffu;
 #pragma unroll
-  for (int i = 0; i < EPL; ++i) v += (valid[i] && rank[i] == r) ? p[i] : 0.f;
-  return warp_sum(v);  // exactly one lane-element matches: the sum is that value
+  for (int size = 2; size <= 32 * EPL; size <<= 1) {
+#pragma unroll
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      if (stride >= 32) {
+        const int js = stride >> 5;
+#pragma unroll
+        for (int j = 0; j < EPL; ++j) {
+          if ((j & js) == 0) {
+            const int jp = j | js;
+            const bool up = ((j * 32 + lane) & size) == 0;
+            const bool gt = k[j] > k[jp] || (k[j] == k[jp] && x[j] > x[jp]);
+            if (gt == up) {
+              const float tk = k[j];
+              k[j] = k[jp];
+              k[jp] = tk;
+              const int tx = x[j];
+              x[j] = x[jp];
+              x[jp] = tx;
+            }
+          }
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < EPL; ++j) {
+          const float ok = __shfl_xor_sync(full, k[j], stride);
+          const int ox = __shfl_xor_sync(full, x[j], stride);
+          const bool up = ((j * 32 + lane) & size) == 0;
+          const bool keep_min = up == ((lane & stride) == 0);
+          const bool other_less = ok < k[j] || (ok == k[j] && ox < x[j]);
+          if (keep_min == other_less) {
+            k[j] = ok;
+            x[j] = ox;
+          }
+        }
+      }
+    }
+  }
+}
+// Element r (0-based) of the sorted pairs, broadcast to the warp.
+template <int EPL>
+__device__ __forceinline__ void sorted_at(const float (&k)[EPL], const int (&x)[EPL], int r,
+                                          float& kr, int& xr) {
+  float kv = 0.f;
+  int xv = 0;
+#pragma unroll
+  for (int j = 0; j < EPL; ++j)
+    if (j == (r >> 5)) {
+      kv = k[j];
+      xv = x[j];
+    }
+  kr = __shfl_sync(0xffffffffu, kv, r & 31);
+  xr = __shfl_sync(0xffffffffu, xv, r & 31);
 }
 
 template <int EPL>
@@ -394,21 +446,39 @@ route_select_kernel(const float2* __restrict__ part, int n_split, const float* _
 
   float p[EPL], I[EPL];
   bool valid[EPL];
-  float lmax = -INFINITY;
+  float hi[EPL], lo[EPL], bv[EPL];
 #pragma unroll
   for (int i = 0; i < EPL; ++i) {
     const int e = lane + 32 * i;
     valid[i] = e < E;
+    hi[i] = 0.f;
+    lo[i] = 0.f;
+    bv[i] = bias && valid[i] ? bias[e] : 0.f;
+  }
+  // the score partials in slice order, a chunk of slices' loads in flight before their sums
+  constexpr int kChunk = EPL <= 2 ? 4 : (EPL <= 4 ? 2 : 1);
+  for (int sp0 = 0; sp0 < n_split; sp0 += kChunk) {
+    float2 v[kChunk][EPL];
+#pragma unroll
+    for (int c = 0; c < kChunk; ++c)
+#pragma unroll
+      for (int i = 0; i < EPL; ++i)
+        v[c][i] = sp0 + c < n_split && valid[i]
+                      ? part[((size_t)(sp0 + c) * T + t) * E + lane + 32 * i]
+                      : make_float2(0.f, 0.f);
+#pragma unroll
+    for (int c = 0; c < kChunk; ++c)
+#pragma unroll
+      for (int i = 0; i < EPL; ++i)
+        if (sp0 + c < n_split && valid[i]) df_add(hi[i], lo[i], v[c][i].x, v[c][i].y);
+  }
+  float lmax = -INFINITY;
+#pragma unroll
+  for (int i = 0; i < EPL; ++i) {
     float z = -INFINITY;
     if (valid[i]) {
-      float hi = 0.f, lo = 0.f;
-#pragma unroll 8
-      for (int sp = 0; sp < n_split; ++sp) {
-        const float2 v = part[((size_t)sp * T + t) * E + e];
-        df_add(hi, lo, v.x, v.y);
-      }
-      if (bias) df_add(hi, lo, bias[e]);
-      z = (hi + lo) * inv_temp;
+      if (bias) df_add(hi[i], lo[i], bv[i]);
+      z = (hi[i] + lo[i]) * inv_temp;
     }
     p[i] = z;
     lmax = fmaxf(lmax, z);
@@ -469,33 +539,26 @@ route_select_kernel(const float2* __restrict__ part, int n_split, const float* _
   }
   float tau_f = rp.kappa1 * (rp.ppl_factor * tau) + rp.kappa2 * second;
 
-  int rank[EPL];
-#pragma unroll
-  for (int i = 0; i < EPL; ++i) rank[i] = 0;
   if (rp.clamp) {
-    // rank of each p among all E (ascending, ties by index): sort-free order statistics
+    // order statistics of p (ascending, ties by index; padding lanes sort last)
+    float sk[EPL];
+    int sx[EPL];
 #pragma unroll
-    for (int jb = 0; jb < EPL; ++jb) {
-      for (int jl = 0; jl < 32; ++jl) {
-        const int ej = jb * 32 + jl;
-        const float pj = __shfl_sync(full, p[jb], jl);
-        if (ej < E) {
-#pragma unroll
-          for (int i = 0; i < EPL; ++i) {
-            const int ei = lane + 32 * i;
-            rank[i] += (pj < p[i] || (pj == p[i] && ej < ei)) ? 1 : 0;
-          }
-        }
-      }
+    for (int i = 0; i < EPL; ++i) {
+      sk[i] = valid[i] ? p[i] : INFINITY;
+      sx[i] = lane + 32 * i;
     }
+    warp_sort_pairs<EPL>(sk, sx, lane);
     const float h_lo = (float)(E - 1) * rp.q_lo;
     const float h_hi = (float)(E - 1) * rp.q_hi;
     const int lo0 = (int)floorf(h_lo), hi0 = (int)floorf(h_hi);
     const int lo1 = min(lo0 + 1, E - 1), hi1 = min(hi0 + 1, E - 1);
-    const float v_lo0 = order_stat<EPL>(p, rank, valid, lo0);
-    const float v_lo1 = order_stat<EPL>(p, rank, valid, lo1);
-    const float v_hi0 = order_stat<EPL>(p, rank, valid, hi0);
-    const float v_hi1 = order_stat<EPL>(p, rank, valid, hi1);
+    float v_lo0, v_lo1, v_hi0, v_hi1;
+    int unused;
+    sorted_at<EPL>(sk, sx, lo0, v_lo0, unused);
+    sorted_at<EPL>(sk, sx, lo1, v_lo1, unused);
+    sorted_at<EPL>(sk, sx, hi0, v_hi0, unused);
+    sorted_at<EPL>(sk, sx, hi1, v_hi1, unused);
     const float q_lo = v_lo0 + (h_lo - (float)lo0) * (v_lo1 - v_lo0);
     const float q_hi = v_hi0 + (h_hi - (float)hi0) * (v_hi1 - v_hi0);
     tau_f = fminf(fmaxf(tau_f, q_lo), q_hi);
@@ -565,27 +628,25 @@ route_select_kernel(const float2* __restrict__ part, int n_split, const float* _
 #pragma unroll
     for (int i = 0; i < EPL; ++i) sel[i] = cand[i];
   } else {
-    // keep the K largest candidates by (I desc, index asc)
-    int r[EPL];
+    // keep the K largest candidates by (I desc, index asc): sort (-I, index) ascending with the
+    // non-candidates last and keep what does not come after the K-th pair
+    float sk[EPL];
+    int sx[EPL];
 #pragma unroll
-    for (int i = 0; i < EPL; ++i) r[i] = 0;
-#pragma unroll
-    for (int jb = 0; jb < EPL; ++jb) {
-      for (int jl = 0; jl < 32; ++jl) {
-        const int ej = jb * 32 + jl;
-        const float Ij = __shfl_sync(full, I[jb], jl);
-        const bool cj = __shfl_sync(full, cand[jb] ? 1 : 0, jl) != 0;
-        if (cj) {
-#pragma unroll
-          for (int i = 0; i < EPL; ++i) {
-            const int ei = lane + 32 * i;
-            r[i] += (Ij > I[i] || (Ij == I[i] && ej < ei)) ? 1 : 0;
-          }
-        }
-      }
+    for (int i = 0; i < EPL; ++i) {
+      sk[i] = cand[i] ? -I[i] : INFINITY;
+      sx[i] = lane + 32 * i;
     }
+    warp_sort_pairs<EPL>(sk, sx, lane);
+    float kk;
+    int kx;
+    sorted_at<EPL>(sk, sx, K - 1, kk, kx);
 #pragma unroll
-    for (int i = 0; i < EPL; ++i) sel[i] = cand[i] && r[i] < K;
+    for (int i = 0; i < EPL; ++i) {
+      const float key = -I[i];
+      const int ei = lane + 32 * i;
+      sel[i] = cand[i] && (key < kk || (key == kk && ei <= kx));
+    }
   }
 
   if (bad) {
