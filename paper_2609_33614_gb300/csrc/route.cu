@@ -9,8 +9,9 @@
 //  route_select_kernel: one warp per token.  Each lane owns experts lane, lane+32, ...; the warp
 //      does the softmax (§3.2), importance (Eq. 2), mean / population std (Eq. 3-4), tau (Eq. 5),
 //      PPL factor and smoothing (§3.3), the clamp to the type-7 q_lo / q_hi quantiles of p
-//      (order statistics by in-warp rank counting, no sort), the candidate set and K cap
-//      (Eq. 6, ties to the lower index) and the renormalised gates (Eq. 7-8), with shuffles only.
+//      (order statistics from a warp-wide bitonic sort of (value, index) pairs), the candidate
+//      set and K cap (Eq. 6, ties to the lower index; the K-th pair of the same sort) and the
+//      renormalised gates (Eq. 7-8), with shuffles only.
 //      The history score S_h (Eq. 1) is computed once per block from the accounts.
 #include "eat_internal.cuh"
 
