@@ -679,10 +679,15 @@ struct PairCfg {
   static constexpr bool kIL = MODE == kModeGateUpIL;
   static constexpr int kABytes = kBM * kBK * 2;
   static constexpr int kBBytes = kPairRows * kBK * 2;
-  static constexpr int kStageBytes = kABytes + kBBytes;
+  // k-blocks per pipeline stage: each stage completes on one barrier phase, and a phase costs
+  // ~0.6 µs however few bytes it carries, so a stage carries two k-blocks' A and B tiles (64 KB
+  // per CTA)
+  static constexpr int kKPS = 2;
+  static constexpr int kSubBytes = kABytes + kBBytes;  // one k-block's A and B tiles
+  static constexpr int kStageBytes = kKPS * kSubBytes;
   static constexpr int kXchgFloats = kIL ? 2 * 2 * 2 * 16 * 32 : 0;
   // the whole 227 KB a CTA may hold: 1 KB of alignment slack and 256 B of barriers besides the
-  // stages (seven for the down projection, six beside the gate/up exchange buffers)
+  // stages (three, beside the gate/up exchange buffers too)
   static constexpr int kStagesRaw = (227 * 1024 - 1024 - 256 - kXchgFloats * 4) / kStageBytes;
   static constexpr int kStages = kStagesRaw > 8 ? 8 : kStagesRaw;
   static constexpr int kAccCols = kPairBN;
@@ -821,21 +826,29 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
         const int n = pair_n(w.nrows);
         const int a_row = w.g * args.a_rows_per_group + w.m0 + (int)rank * C::kFeat;
         const int b_row = w.slot0 - w.g * args.b_shift_per_group + (int)rank * (n / 2);
-        for (int kb = w.kb0; kb < w.kb1; ++kb) {
+        for (int kb = w.kb0; kb < w.kb1; kb += C::kKPS) {
+          const int nk = min(C::kKPS, w.kb1 - kb);  // k-blocks of this stage
           if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, args.err, 1u, true)) {
             ok = false;
             break;
           }
           uint8_t* st = smem + stage * C::kStageBytes;
           const uint32_t fb = full0 + 8u * (uint32_t)stage;
-          if (leader) mbar_expect_tx(&full[stage], 2 * C::kStageBytes);
-          if (IL) {
-            tma_load_2d_pair(st, &mapA0, fb, kb * kBK, a_row);
-            tma_load_2d_pair(st + C::kABytes / 2, &mapA1, fb, kb * kBK, a_row);
-          } else {
-            tma_load_2d_pair(st, &mapA0, fb, kb * kBK, a_row);
+          if (leader) mbar_expect_tx(&full[stage], 2 * nk * C::kSubBytes);
+#pragma unroll
+          for (int j = 0; j < C::kKPS; ++j) {
+            if (j < nk) {
+              uint8_t* sj = st + j * C::kSubBytes;
+              const int kx = (kb + j) * kBK;
+              if (IL) {
+                tma_load_2d_pair(sj, &mapA0, fb, kx, a_row);
+                tma_load_2d_pair(sj + C::kABytes / 2, &mapA1, fb, kx, a_row);
+              } else {
+                tma_load_2d_pair(sj, &mapA0, fb, kx, a_row);
+              }
+              tma_load_2d_pair(sj + C::kABytes, &mapB, fb, kx, b_row);
+            }
           }
-          tma_load_2d_pair(st + C::kABytes, &mapB, fb, kb * kBK, b_row);
           ++issued;
           if (++stage == S) {
             stage = 0;
@@ -868,18 +881,24 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
         tc_fence_after();
         const uint32_t d0 = tmem_base + (uint32_t)(buf * C::kAccCols);
         const uint32_t idesc = idesc_bf16_pair(pair_n(w.nrows));
-        for (int kb = w.kb0; kb < w.kb1; ++kb) {
+        for (int kb = w.kb0; kb < w.kb1; kb += C::kKPS) {
+          const int nk = min(C::kKPS, w.kb1 - kb);
           if (!mbar_wait(&full[stage], phase, abort_flag, args.err, 8u, true)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t sa = smem_u32(smem + stage * C::kStageBytes);
-          const uint32_t sb = sa + C::kABytes;
 #pragma unroll
-          for (int k = 0; k < kBK / 16; ++k)
-            mma_bf16_pair(d0, sdesc_k128(sa + k * 32), sdesc_k128(sb + k * 32), idesc,
-                          (kb > w.kb0 || k > 0) ? 1u : 0u);
+          for (int j = 0; j < C::kKPS; ++j) {
+            if (j < nk) {
+              const uint32_t sa = smem_u32(smem + stage * C::kStageBytes + j * C::kSubBytes);
+              const uint32_t sb = sa + C::kABytes;
+#pragma unroll
+              for (int k = 0; k < kBK / 16; ++k)
+                mma_bf16_pair(d0, sdesc_k128(sa + k * 32), sdesc_k128(sb + k * 32), idesc,
+                              (kb > w.kb0 || j > 0 || k > 0) ? 1u : 0u);
+            }
+          }
           mma_commit_pair(&empty[stage]);
           if (++stage == S) {
             stage = 0;
