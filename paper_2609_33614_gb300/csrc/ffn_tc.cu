@@ -209,7 +209,11 @@ struct Cfg {
   static constexpr int kKB = W8 ? kBK8 : kBK;    // K elements of a k-block (128 B per row)
   static constexpr int kABytes = kBM * 128;
   static constexpr int kBBytes = BN * 128;
-  static constexpr int kStageBytes = kNA * kABytes + kNB * kBBytes;
+  // k-blocks per pipeline stage: a stage completes on one barrier phase, which costs ~0.6 µs
+  // however few bytes it carries, so the bf16 down projection's one-box stages carry two k-blocks
+  static constexpr int kKPS = (!kGateUp && !W8) ? 2 : 1;
+  static constexpr int kSubBytes = kNA * kABytes + kNB * kBBytes;  // one k-block's tiles
+  static constexpr int kStageBytes = kKPS * kSubBytes;
   // fp8: the hi and lo B tiles sit back to back in the stage, so one MMA of N = BN + n covers both
   // (hi in accumulator columns [0, BN), lo in [BN, BN + n)) and reads its A slice once, where the
   // double-buffered accumulators fit in TMEM (gate/up up to 64 tokens, down up to 128)
@@ -391,7 +395,7 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
   // least two launches old when the host sets prefetch_a (every launch only lets its dependent
   // start after its own wait): the producer fills the first stages' A tiles while the previous
   // kernel finishes; the B tiles of those stages follow after the wait.
-  int pre = 0;  // k-blocks whose A tiles are in flight
+  int pre = 0;  // stages whose A tiles are in flight
   const bool early = args.prefetch_a && !args.b_rows;  // (gathering launches follow the permute)
   if (early) {
     go = stage_offsets(args, s_row, s_tile);
@@ -401,9 +405,11 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
     UnitIter<BN> it_p(count_units(), go);
     for (Unit w; pre < S && it_p.next(args, w);) {
       const int a_row = w.g * args.a_rows_per_group + w.m0;
-      for (int kb = w.kb0; kb < w.kb1 && pre < S; ++kb, ++pre) {
-        mbar_expect_tx(&full[pre], C::kStageBytes);
-        load_a(smem + pre * C::kStageBytes, &full[pre], kb, a_row);
+      for (int kb = w.kb0; kb < w.kb1 && pre < S; kb += C::kKPS, ++pre) {
+        const int nk = min(C::kKPS, w.kb1 - kb);  // k-blocks of this stage
+        mbar_expect_tx(&full[pre], nk * C::kSubBytes);
+        for (int j = 0; j < nk; ++j)
+          load_a(smem + pre * C::kStageBytes + j * C::kSubBytes, &full[pre], kb + j, a_row);
       }
     }
   }
@@ -416,7 +422,7 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
   }
   const int units = count_units();
 
-  if (!W8 && warp == 0 && args.b_rows) {
+  if (C::kKPS == 1 && !W8 && warp == 0 && args.b_rows) {
     // ------------------------------------------------------------ producer, gathered tokens:
     // lane 0 issues the weight TMA; all lanes copy the tile's token rows from x with 16-byte
     // cp.async into the 128B-swizzled B tile (lane l: column chunk l % 8 of rows l / 8 + 4 i).
@@ -499,19 +505,23 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
       for (Unit w; ok && it_u.next(args, w);) {
         const int a_row = w.g * args.a_rows_per_group + w.m0;
         const int b_row = w.slot0 - w.g * args.b_shift_per_group;
-        for (int kb = w.kb0; kb < w.kb1; ++kb) {
+        for (int kb = w.kb0; kb < w.kb1; kb += C::kKPS) {
+          const int nk = min(C::kKPS, w.kb1 - kb);
           uint8_t* st = smem + stage * C::kStageBytes;
           if (issued >= pre) {  // (the first `pre` stages: A already in flight, stage unused)
             if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, args.err, 1u, true)) {
               ok = false;
               break;
             }
-            mbar_expect_tx(&full[stage], C::kStageBytes);
-            load_a(st, &full[stage], kb, a_row);
+            mbar_expect_tx(&full[stage], nk * C::kSubBytes);
+            for (int j = 0; j < nk; ++j) load_a(st + j * C::kSubBytes, &full[stage], kb + j, a_row);
           }
-          uint8_t* sbt = st + C::kNA * C::kABytes;
-          tma_load_2d(sbt, &mapB, &full[stage], kb * C::kKB, b_row);
-          if (W8) tma_load_2d(sbt + C::kBBytes, &mapB, &full[stage], kb * C::kKB, b_row + args.b_lo_rows);
+          for (int j = 0; j < nk; ++j) {
+            uint8_t* sbt = st + j * C::kSubBytes + C::kNA * C::kABytes;
+            const int kx = (kb + j) * C::kKB;
+            tma_load_2d(sbt, &mapB, &full[stage], kx, b_row);
+            if (W8) tma_load_2d(sbt + C::kBBytes, &mapB, &full[stage], kx, b_row + args.b_lo_rows);
+          }
           ++issued;
           if (++stage == S) {
             stage = 0;
@@ -548,35 +558,40 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
         const uint32_t idesc = !W8       ? idesc_bf16(n_mma)
                                : C::kFuse ? idesc_e4m3(BN + n_mma)
                                           : idesc_e4m3(n_mma);
-        for (int kb = w.kb0; kb < w.kb1; ++kb) {
+        for (int kb = w.kb0; kb < w.kb1; kb += C::kKPS) {
+          const int nk = min(C::kKPS, w.kb1 - kb);
           if (!mbar_wait(&full[stage], phase, abort_flag, args.err, 8u, true)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t sa0 = smem_u32(smem + stage * C::kStageBytes);
-          const uint32_t sa1 = sa0 + C::kABytes;
-          const uint32_t sb = sa0 + C::kNA * C::kABytes;
-          // four k-steps of 32 bytes per 128-byte row: 16 bf16 or 32 e4m3 elements each
 #pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            const uint64_t da0 = sdesc_k128(sa0 + k * 32), db = sdesc_k128(sb + k * 32);
-            const uint32_t acc = (kb > w.kb0 || k > 0) ? 1u : 0u;
-            if constexpr (C::kFuse) {
-              mma_e4m3(d0, da0, db, idesc, acc);
-              if (C::kNA == 2) mma_e4m3(d1, sdesc_k128(sa1 + k * 32), db, idesc, acc);
-            } else if constexpr (W8) {
-              const uint64_t dl = sdesc_k128(sb + C::kBBytes + k * 32);
-              mma_e4m3(d0, da0, db, idesc, acc);
-              mma_e4m3(d0, da0, dl, idesc, 1u);
-              if (C::kNA == 2) {
-                const uint64_t da1 = sdesc_k128(sa1 + k * 32);
-                mma_e4m3(d1, da1, db, idesc, acc);
-                mma_e4m3(d1, da1, dl, idesc, 1u);
+          for (int j = 0; j < C::kKPS; ++j) {
+            if (j >= nk) break;
+            const uint32_t sa0 = smem_u32(smem + stage * C::kStageBytes + j * C::kSubBytes);
+            const uint32_t sa1 = sa0 + C::kABytes;
+            const uint32_t sb = sa0 + C::kNA * C::kABytes;
+            // four k-steps of 32 bytes per 128-byte row: 16 bf16 or 32 e4m3 elements each
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              const uint64_t da0 = sdesc_k128(sa0 + k * 32), db = sdesc_k128(sb + k * 32);
+              const uint32_t acc = (kb > w.kb0 || j > 0 || k > 0) ? 1u : 0u;
+              if constexpr (C::kFuse) {
+                mma_e4m3(d0, da0, db, idesc, acc);
+                if (C::kNA == 2) mma_e4m3(d1, sdesc_k128(sa1 + k * 32), db, idesc, acc);
+              } else if constexpr (W8) {
+                const uint64_t dl = sdesc_k128(sb + C::kBBytes + k * 32);
+                mma_e4m3(d0, da0, db, idesc, acc);
+                mma_e4m3(d0, da0, dl, idesc, 1u);
+                if (C::kNA == 2) {
+                  const uint64_t da1 = sdesc_k128(sa1 + k * 32);
+                  mma_e4m3(d1, da1, db, idesc, acc);
+                  mma_e4m3(d1, da1, dl, idesc, 1u);
+                }
+              } else {
+                mma_bf16(d0, da0, db, idesc, acc);
+                if (C::kNA == 2) mma_bf16(d1, sdesc_k128(sa1 + k * 32), db, idesc, acc);
               }
-            } else {
-              mma_bf16(d0, da0, db, idesc, acc);
-              if (C::kNA == 2) mma_bf16(d1, sdesc_k128(sa1 + k * 32), db, idesc, acc);
             }
           }
           mma_commit(&empty[stage]);
