@@ -209,10 +209,12 @@ struct Cfg {
   static constexpr int kKB = W8 ? kBK8 : kBK;    // K elements of a k-block (128 B per row)
   static constexpr int kABytes = kBM * 128;
   static constexpr int kBBytes = BN * 128;
-  // k-blocks per pipeline stage: a stage completes on one barrier phase, which costs ~0.6 µs
-  // however few bytes it carries, so the bf16 down projection's one-box stages carry two k-blocks
-  static constexpr int kKPS = (!kGateUp && !W8) ? 2 : 1;
   static constexpr int kSubBytes = kNA * kABytes + kNB * kBBytes;  // one k-block's tiles
+  // k-blocks per pipeline stage: a stage completes on one barrier phase, which costs ~0.6 µs
+  // however few bytes it carries, so a stage carries two k-blocks wherever three such stages fit
+  // (not in the bf16 gate/up kernel, whose gathering producer copies one k-block per stage)
+  static constexpr int kKPS =
+      (kGateUp && !W8) ? 1 : (6 * kSubBytes <= kSmemBudget - 2048 ? 2 : 1);
   static constexpr int kStageBytes = kKPS * kSubBytes;
   // fp8: the hi and lo B tiles sit back to back in the stage, so one MMA of N = BN + n covers both
   // (hi in accumulator columns [0, BN), lo in [BN, BN + n)) and reads its A slice once, where the
