@@ -336,8 +336,8 @@ __device__ __forceinline__ float silu_f(float g) { return __fdividef(g, 1.0f + _
 
 // W8 (fp8 layers): the weights stay e4m3 all the way to the tensor core.  The B operand arrives
 // as two e4m3 planes per row (hi and lo, with hi + lo the row divided by its power-of-two scale,
-// written by split_e4m3_kernel); a stage holds the e4m3 A tiles of a 128-element k-block and the
-// hi and lo B tiles, every k-step issues W . hi and W . lo into the same fp32 accumulator
+// written by split_e4m3_kernel); a k-block holds the e4m3 A tiles of 128 elements and the hi and
+// lo B tiles, every k-step issues W . hi and W . lo into the same fp32 accumulator
 // (kind::f8f6f4), and the epilogue multiplies by the weight row's scale and the B row's scale.
 template <int BN, int MODE, bool W8>
 __global__ void __launch_bounds__(kThreadsTc, 1)
@@ -678,9 +678,9 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
 
 // ------------------------------------------------------------ SM-pair kernels (cta_group::2)
 // Large calls run on pairs of SMs (2-CTA clusters).  The pair issues M = 256 x N = 256 MMAs: each
-// CTA holds 128 rows of A (weight rows) and 128 of the tile's 256 token rows of B, so a stage is
-// 32 KB per SM for the flops the single-SM kernel stages in 48 KB, and six stages are in flight
-// (the single-SM kernels, with four, wait on TMA latency about half the time).  Rank 0 of the pair
+// CTA holds 128 rows of A (weight rows) and 128 of the tile's 256 token rows of B, so a k-block is
+// 32 KB per SM for the flops the single-SM kernel stages in 48 KB; a pipeline stage holds two
+// k-blocks and three stages are in flight.  Rank 0 of the pair
 // issues the MMAs (tcgen05.mma.cta_group::2) and commits them to the barriers of both CTAs; both
 // CTAs load their halves with TMA completing on rank 0's full barrier (rank 0 expects the bytes
 // of both); each CTA drains its own TMEM rows, and rank 0 reuses an accumulator buffer once the
