@@ -386,6 +386,22 @@ def test_partial_feature_tiles():
     run_parity(sh, lw, [97, 3000, 5])
 
 
+@pytest.mark.parametrize("fp8", [False, True])
+def test_odd_k_block_counts(fp8):
+    """d = 192 and d_ff = 320: 3 and 5 k-blocks of 64 bf16 elements (2 and 3 ragged k-blocks of 128
+    e4m3 ones), so the kernels whose pipeline stages hold two k-blocks end every unit on a stage
+    with one; batch 1, 50 and 1200 run the 16- and 64-token single-SM kernels and the SM pairs."""
+    sh = W.scaled(W.MIXTRAL, "odd-kb", d_model=192, n_experts=8, d_ff=320, max_k=2)
+    lw = W.make_layer(sh)
+    if not fp8:
+        run_parity(sh, lw, [1, 50, 1200])
+        return
+    lw8 = W.to_fp8(lw)
+    layer = eat.EatLayer.from_workload(lw8, 1200, gpu_params(sh))
+    run_parity(sh, lw8.dequantized(), [1, 50, 1200], layer=layer)
+    layer.close()
+
+
 def test_degenerate_fixed_topk_on_gpu():
     """beta = 0, alpha1 = 0, alpha2 huge, no clamp: vanilla Top-K by p (index tie-break)."""
     kw = {"beta": 0.0, "alpha1": 0.0, "alpha2": 1e30, "clamp_enabled": 0}
