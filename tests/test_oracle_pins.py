@@ -433,6 +433,17 @@ MUTANTS = {
                          lambda orig: lambda acc, sel, p, n, a: orig(acc, sel, p, n, 1.0 - a)),
     "importance_beta_swapped": ("importance",
                                 lambda orig: lambda p, s, b: orig(p, s, 1.0 - b)),
+    "drop_w1_term": ("history_score",
+                     lambda orig: lambda acc, prm: orig(acc, prm.with_(w1=0.0))),
+    "renorm_over_all_experts": ("renormalize",
+                                lambda orig: lambda g, sel, eps: (np.asarray(g, np.float64) *
+                                                                  orig(g, sel, eps).astype(bool)) /
+                                (np.asarray(g, np.float64).sum() + eps)),
+    "ppl_factor_sign_flipped": ("ppl_factor",
+                                lambda orig: lambda sign, prm: orig(-sign, prm)),
+    "norm_squared_in_account": ("account_update",
+                                lambda orig: lambda acc, sel, p, n, a:
+                                orig(acc, sel, p, {k: v * v for k, v in n.items()}, a)),
 }
 
 
