@@ -52,6 +52,9 @@ struct eat_handle {
   // host-buffer calls copy their input on their own stream, into the staging buffer the call
   // before last used, so the copy overlaps the previous call's kernels (created on first use)
   cudaStream_t copy_st = nullptr;
+  // shared experts run on a stream of the handle, forked from the call's stream before routing
+  cudaStream_t side_st = nullptr;
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
   cudaEvent_t ev_copied[2] = {nullptr, nullptr};  // input copy i done (copy stream)
   cudaEvent_t ev_done[2] = {nullptr, nullptr};    // the call that read buffer i done (its stream)
   int stage_i = 0;
@@ -191,11 +194,73 @@ eat_status run_route(eat_handle* h, const void* x, int T, int ppl_sign, int32_t*
   return EAT_OK;
 }
 
+// The always-on shared experts of §3.1 (weight 1).  They read only x, so a small call runs them on
+// the handle's side stream while the routing kernels, which leave most SMs idle, run on its own.
+eat_status run_shared(eat_handle* h, const TcCall& c, const void* x, int T, cudaStream_t ss) {
+  if (h->backend == 1) {
+    auto split = [&](TcSplit which, const char* what) {
+      return launch(h, kGather, ss, what, [&] { return tc_launch_split(h->tc, c, which, ss); });
+    };
+    if (h->w8) EAT_TRY(split(TcSplit::kTokenX, "split x (tokens)"));
+    EAT_TRY(launch(h, kSUp, ss, "tc shared gate/up",
+                   [&] { return tc_launch_up(h->tc, c, true, ss); }));
+    if (h->w8) EAT_TRY(split(TcSplit::kSharedAct, "split shared activations"));
+    return launch(h, kSDown, ss, "tc shared down",
+                  [&] { return tc_launch_down(h->tc, c, true, 1, ss); });
+  }
+  const int tpg = (T + kSimtTileRows - 1) / kSimtTileRows;
+  GroupMap gs{nullptr, nullptr, nullptr, kRowIdentity, h->S, T, tpg * h->S};
+  EAT_TRY(launch(h, kSUp, ss, "shared gate/up", [&] {
+    return launch_ffn_gateup_simt(h->bf16, x, h->desc.ws_gate, h->desc.ws_up, h->Fs, h->d, gs,
+                                  h->sact, ss);
+  }));
+  return launch(h, kSDown, ss, "shared down", [&] {
+    return launch_ffn_down_simt(h->bf16, h->sact, h->desc.ws_down, h->d, h->Fs, gs,
+                                (float*)h->sout, ss);
+  });
+}
+
+// Small calls, whose shared-expert GEMMs have fewer work units than the GPU has SMs, run those
+// GEMMs on the side stream next to the routing kernels; larger calls fill the GPU with them alone
+// and keep them in the call's stream after the routed experts.
+bool shared_on_side_stream(const eat_handle* h, int T, int tile_rows) {
+  if (h->S == 0 || h->backend != 1) return false;
+  const long long units =
+      (long long)h->S * ((h->Fs + 127) / 128) * ((T + tile_rows - 1) / tile_rows);
+  return units < h->tc.num_sms;
+}
+
 eat_status run_forward(eat_handle* h, const void* x, int T, int ppl_sign, void* y,
                        int32_t* idx_opt, float* w_opt, int32_t* k_opt, cudaStream_t st) {
-  EAT_TRY(run_route(h, x, T, ppl_sign, h->idx, h->w, h->k, h->psel, true, st));
   const int tile_rows = h->backend == 1 ? tc_tile_rows(h->tc, T) : kSimtTileRows;
   const int tile_rows_down = h->backend == 1 ? tc_tile_rows_down(h->tc, T) : kSimtTileRows;
+  TcCall c;
+  c.x = x;
+  c.T = T;
+  c.tile_rows = tile_rows;
+  c.tile_rows_down = tile_rows_down;
+  c.offs = h->perm.offs;
+  c.tile_offs = h->perm.tile_offs;
+  c.tile_offs_down = h->perm.tile_offs2;
+  c.perm_tok = h->perm.perm_tok;
+  c.xperm = h->xperm;
+  c.act = h->act;
+  c.opart = h->opart;
+  c.sact = h->sact;
+  c.sout = h->sout;
+  c.status = h->status;
+  const bool side = shared_on_side_stream(h, T, tile_rows);
+  if (side) {
+    // fork: the side stream starts after everything enqueued on st so far (x written, the
+    // previous call's combine done with the shared outputs)
+    cudaError_t e = cudaEventRecord(h->ev_fork, st);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(h->side_st, h->ev_fork, 0);
+    if (e != cudaSuccess) return cuda_fail(h, e, "shared-expert stream fork");
+    EAT_TRY(run_shared(h, c, x, T, h->side_st));
+    e = cudaEventRecord(h->ev_join, h->side_st);
+    if (e != cudaSuccess) return cuda_fail(h, e, "shared-expert stream join");
+  }
+  EAT_TRY(run_route(h, x, T, ppl_sign, h->idx, h->w, h->k, h->psel, true, st));
   EAT_TRY(launch(h, kPermute, st, "permute", [&] {
     return launch_permute(h->idx, h->k, h->psel, T, h->K, h->E, tile_rows, tile_rows_down,
                           h->perm, h->chunk_cnt, st);
@@ -203,21 +268,6 @@ eat_status run_forward(eat_handle* h, const void* x, int T, int ppl_sign, void* 
   const int rows = T * h->K;
   int n_split = 1;
   if (h->backend == 1) {
-    TcCall c;
-    c.x = x;
-    c.T = T;
-    c.tile_rows = tile_rows;
-    c.tile_rows_down = tile_rows_down;
-    c.offs = h->perm.offs;
-    c.tile_offs = h->perm.tile_offs;
-    c.tile_offs_down = h->perm.tile_offs2;
-    c.perm_tok = h->perm.perm_tok;
-    c.xperm = h->xperm;
-    c.act = h->act;
-    c.opart = h->opart;
-    c.sact = h->sact;
-    c.sout = h->sout;
-    c.status = h->status;
     n_split = tc_down_split(h->tc, T);
     // fp8 layers: each GEMM's B operand first becomes e4m3 hi/lo planes (the routed x rows are
     // gathered into slot order on the way)
@@ -233,14 +283,6 @@ eat_status run_forward(eat_handle* h, const void* x, int T, int ppl_sign, void* 
     if (h->w8) EAT_TRY(split(TcSplit::kAct, "split activations"));
     EAT_TRY(launch(h, kDown, st, "tc down",
                    [&] { return tc_launch_down(h->tc, c, false, n_split, st); }));
-    if (h->S > 0) {
-      if (h->w8) EAT_TRY(split(TcSplit::kTokenX, "split x (tokens)"));
-      EAT_TRY(launch(h, kSUp, st, "tc shared gate/up",
-                     [&] { return tc_launch_up(h->tc, c, true, st); }));
-      if (h->w8) EAT_TRY(split(TcSplit::kSharedAct, "split shared activations"));
-      EAT_TRY(launch(h, kSDown, st, "tc shared down",
-                     [&] { return tc_launch_down(h->tc, c, true, 1, st); }));
-    }
   } else {
     GroupMap gm{h->perm.offs, h->perm.tile_offs, h->perm.perm_tok, kRowGather, h->E, 0,
                 (rows + kSimtTileRows - 1) / kSimtTileRows + h->E};
@@ -251,18 +293,12 @@ eat_status run_forward(eat_handle* h, const void* x, int T, int ppl_sign, void* 
     EAT_TRY(launch(h, kDown, st, "ffn down", [&] {
       return launch_ffn_down_simt(h->bf16, h->act, h->desc.w_down, h->d, h->F, gm, h->opart, st);
     }));
-    if (h->S > 0) {
-      const int tpg = (T + kSimtTileRows - 1) / kSimtTileRows;
-      GroupMap gs{nullptr, nullptr, nullptr, kRowIdentity, h->S, T, tpg * h->S};
-      EAT_TRY(launch(h, kSUp, st, "shared gate/up", [&] {
-        return launch_ffn_gateup_simt(h->bf16, x, h->desc.ws_gate, h->desc.ws_up, h->Fs, h->d,
-                                      gs, h->sact, st);
-      }));
-      EAT_TRY(launch(h, kSDown, st, "shared down", [&] {
-        return launch_ffn_down_simt(h->bf16, h->sact, h->desc.ws_down, h->d, h->Fs, gs,
-                                    (float*)h->sout, st);
-      }));
-    }
+  }
+  if (side) {
+    const cudaError_t e = cudaStreamWaitEvent(st, h->ev_join, 0);  // join before the combine
+    if (e != cudaSuccess) return cuda_fail(h, e, "shared-expert stream join");
+  } else if (h->S > 0) {
+    EAT_TRY(run_shared(h, c, x, T, st));
   }
   EAT_TRY(launch(h, kCombine, st, "combine", [&] {
     const int tc = h->backend == 1;
@@ -294,6 +330,9 @@ void free_handle(eat_handle* h) {
     if (h->ev_done[i]) cudaEventDestroy(h->ev_done[i]);
   }
   if (h->copy_st) cudaStreamDestroy(h->copy_st);
+  if (h->ev_fork) cudaEventDestroy(h->ev_fork);
+  if (h->ev_join) cudaEventDestroy(h->ev_join);
+  if (h->side_st) cudaStreamDestroy(h->side_st);
   tc_destroy(h->tc);
   if (h->mem) cudaFree(h->mem);
   delete h;
@@ -487,6 +526,15 @@ eat_status eat_create(const eat_layer_desc* desc, const eat_params* params, eat_
       std::string m = msg ? msg : "tensor map setup failed";
       free_handle(h);
       return fail(nullptr, EAT_ERR_CUDA, m);
+    }
+  }
+  if (h->S > 0) {  // created here, not on first use, so that a call may be stream-captured
+    e = cudaStreamCreateWithFlags(&h->side_st, cudaStreamNonBlocking);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming);
+    if (e != cudaSuccess) {
+      free_handle(h);
+      return fail(nullptr, EAT_ERR_CUDA, std::string("side stream: ") + cudaGetErrorString(e));
     }
   }
   *out = h;
