@@ -157,7 +157,10 @@ eat_status eat_route(eat_handle* h, const void* x, int32_t T, int32_t ppl_sign,
  * the account update: N_e += n_e, P_total,e += sum of p over e's activations,
  * C_e <- (1 - alpha) C_e + alpha * mean ||E_e(x_t)||_2 when n_e > 0.
  * idx_opt / w_opt / k_opt may be NULL; when given they receive the routing as in eat_route.
- * y must not alias x; x and y must be 16-byte aligned. */
+ * y must not alias x; x and y must be 16-byte aligned.  A layer with shared experts may run them,
+ * for a small call, on a stream of the handle that forks from `stream` at the start of the call
+ * and joins it again before the outputs are combined (events recorded on `stream`), so the call
+ * stays ordered on `stream` and can be stream-captured into a CUDA graph. */
 eat_status eat_moe_forward(eat_handle* h, const void* x, int32_t T, int32_t ppl_sign, void* y,
                            int32_t* idx_opt, float* w_opt, int32_t* k_opt, void* stream);
 
