@@ -295,18 +295,21 @@ def test_toy_free_running_first_divergence():
     layer.close()
 
 
-def test_two_handles_on_two_streams_interleaved():
+@pytest.mark.parametrize("shape", ["olmoe", "qwen"])
+def test_two_handles_on_two_streams_interleaved(shape):
     """Two handles (one layer each) driven from two CUDA streams with their calls interleaved give
-    the results of running each alone: a handle's workspace and accounts are its own."""
-    lw = W.make_layer(OLMOE_S)
-    xs = [W.make_tokens(OLMOE_S, 48, step=s).cuda() for s in range(4)]
+    the results of running each alone: a handle's workspace and accounts are its own (with shared
+    experts, so are the stream and events their small calls fork onto)."""
+    sh = OLMOE_S if shape == "olmoe" else QWEN_S
+    lw = W.make_layer(sh)
+    xs = [W.make_tokens(sh, 48, step=s).cuda() for s in range(4)]
     ref = []
-    solo = eat.EatLayer.from_workload(lw, 48, gpu_params(OLMOE_S))
+    solo = eat.EatLayer.from_workload(lw, 48, gpu_params(sh))
     for x in xs:
         ref.append(solo.forward(x, 0).clone())
     solo.close()
-    a = eat.EatLayer.from_workload(lw, 48, gpu_params(OLMOE_S))
-    b = eat.EatLayer.from_workload(lw, 48, gpu_params(OLMOE_S))
+    a = eat.EatLayer.from_workload(lw, 48, gpu_params(sh))
+    b = eat.EatLayer.from_workload(lw, 48, gpu_params(sh))
     sa, sb = torch.cuda.Stream(), torch.cuda.Stream()
     ya = [torch.empty_like(x) for x in xs]
     yb = [torch.empty_like(x) for x in xs]
@@ -577,14 +580,17 @@ def test_bounded_wait_expires_and_context_survives():
 
 
 # ------------------------------------------------------------------ CUDA graph capture
-def test_forward_replays_as_cuda_graph():
+@pytest.mark.parametrize("shape", ["mixtral", "qwen"])
+def test_forward_replays_as_cuda_graph(shape):
     """A layer call has no host synchronisation and decides its expert schedule on the device, so
     it can be captured once and replayed: the replays must match direct calls bit for bit, accounts
-    included (two handles on the same weights, same inputs)."""
-    lw = W.make_layer(MIX_S)
-    a = eat.EatLayer.from_workload(lw, 64, gpu_params(MIX_S))
-    b = eat.EatLayer.from_workload(lw, 64, gpu_params(MIX_S))
-    x = W.make_tokens(MIX_S, 64).cuda()
+    included (two handles on the same weights, same inputs).  The qwen-shaped layer's 64-token call
+    runs its shared experts on the handle's second stream, forked and joined inside the capture."""
+    sh = MIX_S if shape == "mixtral" else QWEN_S
+    lw = W.make_layer(sh)
+    a = eat.EatLayer.from_workload(lw, 64, gpu_params(sh))
+    b = eat.EatLayer.from_workload(lw, 64, gpu_params(sh))
+    x = W.make_tokens(sh, 64).cuda()
     y_graph = torch.empty_like(x)
     stream = torch.cuda.Stream()
     g = torch.cuda.CUDAGraph()
