@@ -702,7 +702,7 @@ struct PairCfg {
   static constexpr int kKPS = 2;
   static constexpr int kSubBytes = kABytes + kBBytes;  // one k-block's A and B tiles
   static constexpr int kStageBytes = kKPS * kSubBytes;
-  static constexpr int kXchgFloats = kIL ? 2 * 2 * 2 * 16 * 32 : 0;
+  static constexpr int kXchgFloats = kIL ? 2 * 2 * 2 * 32 * 32 : 0;
   // the whole 227 KB a CTA may hold: 1 KB of alignment slack and 256 B of barriers besides the
   // stages (three, beside the gate/up exchange buffers too)
   static constexpr int kStagesRaw = (227 * 1024 - 1024 - 256 - kXchgFloats * 4) / kStageBytes;
@@ -934,7 +934,7 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
     const int q = warp & 3;
     const int half = q & 1;
     const bool is_gate = q < 2;
-    float* xh = xchg + half * (2 * 2 * 16 * 32);
+    float* xh = xchg + half * (2 * 2 * 32 * 32);
     uint64_t* xb = xbar + half * 2;
     int local = 0;
     long long chunk = 0;
@@ -950,20 +950,30 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
       const int f = w.m0 + (int)rank * C::kFeat + 32 * half + lane;
       const bool fok = f < args.M;
       const int keep = is_gate ? 0 : 16;
-      for (int c0 = 0; c0 < kPairBN && c0 < w.nrows; c0 += 32, ++chunk) {
-        uint32_t v0[16], v1[16];
+      for (int c0 = 0; c0 < kPairBN && c0 < w.nrows; c0 += 64, ++chunk) {
+        // 64 columns per exchange: the gate warp computes columns c0 + [0, 16) and c0 + [32, 48),
+        // the up warp c0 + [16, 32) and c0 + [48, 64); each sends the other its other 32
+        uint32_t v0[16], v1[16], v2[16], v3[16];
         tmem_ld16(tbase + c0, v0);
         tmem_ld16(tbase + c0 + 16, v1);
+        tmem_ld16(tbase + c0 + 32, v2);
+        tmem_ld16(tbase + c0 + 48, v3);
         tmem_wait_ld();
         const int b = (int)(chunk & 1);
-        float* mine_out = xh + (b * 2 + (is_gate ? 0 : 1)) * 512;
-        const float* theirs = xh + (b * 2 + (is_gate ? 1 : 0)) * 512;
+        float* mine_out = xh + (b * 2 + (is_gate ? 0 : 1)) * 1024;
+        const float* theirs = xh + (b * 2 + (is_gate ? 1 : 0)) * 1024;
         if (is_gate) {
 #pragma unroll
-          for (int j = 0; j < 16; ++j) mine_out[j * 32 + lane] = __uint_as_float(v1[j]);
+          for (int j = 0; j < 16; ++j) {
+            mine_out[j * 32 + lane] = __uint_as_float(v1[j]);
+            mine_out[(16 + j) * 32 + lane] = __uint_as_float(v3[j]);
+          }
         } else {
 #pragma unroll
-          for (int j = 0; j < 16; ++j) mine_out[j * 32 + lane] = __uint_as_float(v0[j]);
+          for (int j = 0; j < 16; ++j) {
+            mine_out[j * 32 + lane] = __uint_as_float(v0[j]);
+            mine_out[(16 + j) * 32 + lane] = __uint_as_float(v2[j]);
+          }
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(&xb[b]);
@@ -973,11 +983,12 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
         }
         if (fok) {
 #pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            const int col = c0 + keep + j;
+          for (int j = 0; j < 32; ++j) {
+            const int col = c0 + keep + (j < 16 ? j : 16 + j);
             if (col < w.nrows) {
               const float o = theirs[j * 32 + lane];
-              const float m = __uint_as_float(is_gate ? v0[j] : v1[j]);
+              const uint32_t mv = j < 16 ? (is_gate ? v0[j] : v1[j]) : (is_gate ? v2[j - 16] : v3[j - 16]);
+              const float m = __uint_as_float(mv);
               const float h = is_gate ? silu_f(m) * o : silu_f(o) * m;
               ((__nv_bfloat16*)args.out)[(size_t)(w.slot0 + col) * args.M + f] =
                   __float2bfloat16_rn(h);
