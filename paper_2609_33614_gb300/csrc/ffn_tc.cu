@@ -702,7 +702,13 @@ struct PairCfg {
   static constexpr int kKPS = 2;
   static constexpr int kSubBytes = kABytes + kBBytes;  // one k-block's A and B tiles
   static constexpr int kStageBytes = kKPS * kSubBytes;
-  static constexpr int kXchgFloats = kIL ? 2 * 2 * 2 * 32 * 32 : 0;
+  // the interleaved gate/up kernel drains TMEM with two warps per lane quarter (one per half of the
+  // 256 token columns): 10 warps; the down kernel with one (6 warps)
+  static constexpr int kEpiWarps = kIL ? 8 : 4;
+  static constexpr int kThreads = 64 + 32 * kEpiWarps;
+  // exchange buffers of the 4 (feature half, column half) warp pairs: 2 buffers x gate and up x
+  // 16 columns x 32 lanes
+  static constexpr int kXchgFloats = kIL ? 4 * 2 * 2 * 16 * 32 : 0;
   // the whole 227 KB a CTA may hold: 1 KB of alignment slack and 256 B of barriers besides the
   // stages (three, beside the gate/up exchange buffers too)
   static constexpr int kStagesRaw = (227 * 1024 - 1024 - 256 - kXchgFloats * 4) / kStageBytes;
@@ -776,7 +782,7 @@ __host__ __device__ constexpr uint32_t idesc_bf16_pair(int n) {
 __device__ __forceinline__ int pair_n(int nrows) { return min(kPairBN, (nrows + 31) & ~31); }
 
 template <int MODE>
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreadsTc, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg<MODE>::kThreads, 1)
 tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__ CUtensorMap mapA1,
                const __grid_constant__ CUtensorMap mapB, const TcArgs args) {
   using C = PairCfg<MODE>;
@@ -791,7 +797,7 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
   uint64_t* tempty = tfull + 2;
   uint64_t* mma_done = tempty + 2;
   uint64_t* xbar = mma_done + 1;
-  uint32_t* tmem_slot = (uint32_t*)(xbar + 4);
+  uint32_t* tmem_slot = (uint32_t*)(xbar + 8);
   volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
 
   const uint32_t rank = cluster_rank();
@@ -804,10 +810,10 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tfull[b], 1);
-      mbar_init(&tempty[b], 8);  // the epilogue warps of both CTAs (rank 0's barrier is used)
+      mbar_init(&tempty[b], 2 * C::kEpiWarps);  // the epilogue warps of both CTAs (rank 0's)
     }
     mbar_init(mma_done, 1);
-    for (int i = 0; i < 4; ++i) mbar_init(&xbar[i], 2);
+    for (int i = 0; i < 8; ++i) mbar_init(&xbar[i], 2);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -930,12 +936,17 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
     }
     if (lane == 0) mbar_wait(mma_done, 0u, abort_flag, args.err, 16u, false);
   } else if (IL) {
-    // ---------------------------------------- epilogue, interleaved gate/up (warps 2..5)
+    // ---------------------------------------- epilogue, interleaved gate/up (warps 2..9)
+    // Warp w drains TMEM lane quarter w % 4 (gate rows in quarters 0-1, up rows in 2-3) for the
+    // token columns [128 ch, 128 ch + 128), ch = (w - 2) / 4; a gate warp and the up warp of the
+    // same features and columns exchange halves through shared memory, 32 columns at a time.
     const int q = warp & 3;
     const int half = q & 1;
     const bool is_gate = q < 2;
-    float* xh = xchg + half * (2 * 2 * 32 * 32);
-    uint64_t* xb = xbar + half * 2;
+    const int ch = (warp - 2) >> 2;
+    const int xp = half * 2 + ch;  // the warp pair's exchange buffers and barriers
+    float* xh = xchg + xp * (2 * 2 * 16 * 32);
+    uint64_t* xb = xbar + xp * 2;
     int local = 0;
     long long chunk = 0;
     bool ok = true;
@@ -950,31 +961,18 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
       const int f = w.m0 + (int)rank * C::kFeat + 32 * half + lane;
       const bool fok = f < args.M;
       const int keep = is_gate ? 0 : 16;
-      for (int c0 = 0; c0 < kPairBN && c0 < w.nrows; c0 += 64, ++chunk) {
-        // 64 columns per exchange: the gate warp computes columns c0 + [0, 16) and c0 + [32, 48),
-        // the up warp c0 + [16, 32) and c0 + [48, 64); each sends the other its other 32
-        uint32_t v0[16], v1[16], v2[16], v3[16];
+      const int c_end = min(128 * ch + 128, w.nrows);
+      for (int c0 = 128 * ch; c0 < c_end; c0 += 32, ++chunk) {
+        uint32_t v0[16], v1[16];
         tmem_ld16(tbase + c0, v0);
         tmem_ld16(tbase + c0 + 16, v1);
-        tmem_ld16(tbase + c0 + 32, v2);
-        tmem_ld16(tbase + c0 + 48, v3);
         tmem_wait_ld();
         const int b = (int)(chunk & 1);
-        float* mine_out = xh + (b * 2 + (is_gate ? 0 : 1)) * 1024;
-        const float* theirs = xh + (b * 2 + (is_gate ? 1 : 0)) * 1024;
-        if (is_gate) {
+        float* mine_out = xh + (b * 2 + (is_gate ? 0 : 1)) * 512;
+        const float* theirs = xh + (b * 2 + (is_gate ? 1 : 0)) * 512;
 #pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            mine_out[j * 32 + lane] = __uint_as_float(v1[j]);
-            mine_out[(16 + j) * 32 + lane] = __uint_as_float(v3[j]);
-          }
-        } else {
-#pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            mine_out[j * 32 + lane] = __uint_as_float(v0[j]);
-            mine_out[(16 + j) * 32 + lane] = __uint_as_float(v2[j]);
-          }
-        }
+        for (int j = 0; j < 16; ++j)
+          mine_out[j * 32 + lane] = __uint_as_float(is_gate ? v1[j] : v0[j]);
         __syncwarp();
         if (lane == 0) mbar_arrive(&xb[b]);
         if (!warp_wait(&xb[b], (uint32_t)((chunk >> 1) & 1), abort_flag, args.err, 128u)) {
@@ -983,12 +981,11 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
         }
         if (fok) {
 #pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            const int col = c0 + keep + (j < 16 ? j : 16 + j);
+          for (int j = 0; j < 16; ++j) {
+            const int col = c0 + keep + j;
             if (col < w.nrows) {
               const float o = theirs[j * 32 + lane];
-              const uint32_t mv = j < 16 ? (is_gate ? v0[j] : v1[j]) : (is_gate ? v2[j - 16] : v3[j - 16]);
-              const float m = __uint_as_float(mv);
+              const float m = __uint_as_float(is_gate ? v0[j] : v1[j]);
               const float h = is_gate ? silu_f(m) * o : silu_f(o) * m;
               ((__nv_bfloat16*)args.out)[(size_t)(w.slot0 + col) * args.M + f] =
                   __float2bfloat16_rn(h);
@@ -1178,7 +1175,7 @@ cudaError_t launch_pair(const CUtensorMap& a0, const CUtensorMap& a1, const CUte
     if (attr_err != cudaSuccess) return;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(num_sms & ~1);
-    cfg.blockDim = dim3(kThreadsTc);
+    cfg.blockDim = dim3(C::kThreads);
     cfg.dynamicSmemBytes = C::kSmemBytes;
     cudaLaunchAttribute at[1];
     at[0].id = cudaLaunchAttributeClusterDimension;
@@ -1197,7 +1194,7 @@ cudaError_t launch_pair(const CUtensorMap& a0, const CUtensorMap& a1, const CUte
   if (attr_err != cudaSuccess) return attr_err;
   const long long pairs = std::min<long long>(max_pairs, units);
   if (pairs <= 0) return cudaSuccess;
-  return launch_pdl(tc_pair_kernel<MODE>, dim3((unsigned)(2 * pairs)), dim3(kThreadsTc),
+  return launch_pdl(tc_pair_kernel<MODE>, dim3((unsigned)(2 * pairs)), dim3(C::kThreads),
                     C::kSmemBytes, st, a0, a1, b, args);
 }
 
