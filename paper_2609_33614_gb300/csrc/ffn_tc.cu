@@ -702,9 +702,9 @@ struct PairCfg {
   static constexpr int kKPS = 2;
   static constexpr int kSubBytes = kABytes + kBBytes;  // one k-block's A and B tiles
   static constexpr int kStageBytes = kKPS * kSubBytes;
-  // the interleaved gate/up kernel drains TMEM with two warps per lane quarter (one per half of the
-  // 256 token columns): 10 warps; the down kernel with one (6 warps)
-  static constexpr int kEpiWarps = kIL ? 8 : 4;
+  // TMEM is drained by two warps per lane quarter, one per half of the 256 token columns: the
+  // accumulator buffer goes back to the MMA issuer in half the time (10 warps in all)
+  static constexpr int kEpiWarps = 8;
   static constexpr int kThreads = 64 + 32 * kEpiWarps;
   // exchange buffers of the 4 (feature half, column half) warp pairs: 2 buffers x gate and up x
   // 16 columns x 32 lanes
@@ -1002,8 +1002,10 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
       }
     }
   } else {
-    // ---------------------------------------------------- epilogue, down projection (warps 2..5)
+    // ------------------------------------------- epilogue, down projection (warps 2..9)
+    // warp w drains TMEM lane quarter w % 4 for the token columns [128 ch, 128 ch + 128)
     const int q = warp & 3;
+    const int ch = (warp - 2) >> 2;
     int local = 0;
     for (int u = pair; u < units; u += n_pairs, ++local) {
       const Unit w = decode_unit<kPairBN>(args, u, Offs{args.row_offs, args.tile_offs});
@@ -1015,7 +1017,8 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
           tmem_base + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * C::kAccCols);
       const int f = w.m0 + (int)rank * C::kFeat + 32 * q + lane;
       const bool fok = f < args.M;
-      for (int c0 = 0; c0 < kPairBN && c0 < w.nrows; c0 += 16) {
+      const int c_end = min(128 * ch + 128, w.nrows);
+      for (int c0 = 128 * ch; c0 < c_end; c0 += 16) {
         uint32_t g[16];
         tmem_ld16(tbase + c0, g);
         tmem_wait_ld();
