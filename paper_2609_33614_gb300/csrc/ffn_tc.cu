@@ -14,8 +14,9 @@
 //       it, bf16 rows O[slot][c].
 // Persistent CTAs (one per SM) walk the work units (token tile, feature tile, K slice) of all
 // groups; the group sizes live on the device (written by the permute kernel), so no host sync.
-// Warp roles: warp 0 lane 0 issues TMA; warp 1 owns TMEM and lane 0 issues MMAs; warps 2-5 drain
-// TMEM (double-buffered accumulators, so the epilogue of tile i overlaps the MMAs of tile i + 1).
+// Warp roles: warp 0 lane 0 issues TMA; warp 1 owns TMEM and lane 0 issues MMAs; warps 2-5 (and
+// 6-9 for e4m3 tiles of 64 or more tokens, each warp half of the tile's columns) drain TMEM
+// (double-buffered accumulators, so the epilogue of tile i overlaps the MMAs of tile i + 1).
 // Every mbarrier wait is bounded (2 s); on expiry the kernel records an error in the device status
 // word, lets in-flight copies and MMAs finish, frees its TMEM and returns.
 #include "ffn_tc.cuh"
@@ -34,7 +35,6 @@ namespace {
 constexpr int kBM = 128;                  // weight rows per tile (MMA M)
 constexpr int kBK = 64;                   // 64 bf16 = 128 B: one 128B-swizzle row
 constexpr int kBK8 = 128;                 // 128 e4m3 = 128 B: the same row for fp8 layers
-constexpr int kThreadsTc = 192;           // 6 warps
 constexpr int kNumBN = 4;
 constexpr int kBNs[kNumBN] = {16, 32, 64, 128};  // single-SM token tiles; SM pairs load 128 per CTA
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;
@@ -215,6 +215,11 @@ struct Cfg {
   // (not in the bf16 gate/up kernel, whose gathering producer copies one k-block per stage)
   static constexpr int kKPS =
       (kGateUp && !W8) ? 1 : (6 * kSubBytes <= kSmemBudget - 2048 ? 2 : 1);
+  // e4m3 tiles of 64 or more tokens are drained by two warps per TMEM lane quarter (one per half
+  // of the tile's columns), so an accumulator buffer returns to the MMA issuer sooner (e4m3
+  // prefill +20 %; the bf16 gathering gate/up at 128-token tiles was slower with eight)
+  static constexpr int kEpiWarps = (W8 && BN >= 64) ? 8 : 4;
+  static constexpr int kThreads = 64 + 32 * kEpiWarps;
   static constexpr int kStageBytes = kKPS * kSubBytes;
   // fp8: the hi and lo B tiles sit back to back in the stage, so one MMA of N = BN + n covers both
   // (hi in accumulator columns [0, BN), lo in [BN, BN + n)) and reads its A slice once, where the
@@ -340,7 +345,7 @@ __device__ __forceinline__ float silu_f(float g) { return __fdividef(g, 1.0f + _
 // lo B tiles, every k-step issues W . hi and W . lo into the same fp32 accumulator
 // (kind::f8f6f4), and the epilogue multiplies by the weight row's scale and the B row's scale.
 template <int BN, int MODE, bool W8>
-__global__ void __launch_bounds__(kThreadsTc, 1)
+__global__ void __launch_bounds__(Cfg<BN, MODE, W8>::kThreads, 1)
 tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__ CUtensorMap mapA1,
               const __grid_constant__ CUtensorMap mapB, const TcArgs args) {
   using C = Cfg<BN, MODE, W8>;
@@ -364,7 +369,7 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tfull[b], 1);
-      mbar_init(&tempty[b], 4);
+      mbar_init(&tempty[b], C::kEpiWarps);
     }
     mbar_init(mma_done, 1);
     *abort_flag = 0;
@@ -610,9 +615,11 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
       mbar_wait(mma_done, 0u, abort_flag, args.err, 16u, false);
     }
   } else {
-    // -------------------------------------------------------------- epilogue (warps 2..5)
+    // ------------------------------------------------- epilogue (warps 2 .. 2 + kEpiWarps - 1)
     const int q = warp & 3;  // TMEM lane quarter this warp may access
     const int row = 32 * q + lane;
+    constexpr int kCols = BN / (C::kEpiWarps / 4);  // the tile columns of one warp
+    const int cbeg = ((warp - 2) >> 2) * kCols;
     int local = 0;
     UnitIter<BN> it_u(units, go);
     for (Unit w; it_u.next(args, w); ++local) {
@@ -630,7 +637,8 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
         if (GATEUP) s1 = args.scale1[ar];
       }
       const float* bsc = W8 ? args.bscale + (w.slot0 - w.g * args.b_shift_per_group) : nullptr;
-      for (int c0 = 0; c0 < BN && c0 < w.nrows; c0 += 16) {
+      const int cend = min(cbeg + kCols, w.nrows);
+      for (int c0 = cbeg; c0 < cend; c0 += 16) {
         uint32_t g[16], up[16];
         tmem_ld16(tbase + c0, g);
         if (GATEUP) tmem_ld16(tbase + C::kProjCols + c0, up);
@@ -1160,7 +1168,7 @@ cudaError_t launch_tc(const CUtensorMap& a0, const CUtensorMap& a1, const CUtens
   });
   if (attr_err != cudaSuccess) return attr_err;
   if (grid <= 0) return cudaSuccess;
-  return launch_pdl(tc_ffn_kernel<BN, MODE, W8>, dim3(grid), dim3(kThreadsTc), C::kSmemBytes,
+  return launch_pdl(tc_ffn_kernel<BN, MODE, W8>, dim3(grid), dim3(C::kThreads), C::kSmemBytes,
                     st, a0, a1, b, args);
 }
 
