@@ -230,12 +230,38 @@ def kernel_flops(kind, shape, acts, T):
     raise KeyError(kind)
 
 
-def traffic_for(kind, workload, experts_per_launch):
+def roofline(dk, decode, fp8, peaks):
+    """The dominant kernel against its roofline.  dk: the kernel's event-timed total ms, launch
+    count and algorithmic bytes and flops summed over its launches; decode calls are bound by HBM
+    (bytes of the activated experts' weights and the activation rows), prefill calls by the
+    tensor pipe (flops).  peaks: (HBM GB/s, bf16 burst TFLOP/s, bf16 sustained TFLOP/s, source)."""
+    hbm, _bf16_burst, bf16_sus, peak_src = peaks
+    avg_launch_s = dk["ms"] / 1e3 / max(1, dk["launches"])
+    if decode:
+        achieved = dk["bytes"] / max(1, dk["launches"]) / avg_launch_s / 1e9
+        return {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
+                "frac": achieved / hbm, "peak_source": peak_src}
+    achieved = dk["flops"] / max(1, dk["launches"]) / avg_launch_s / 1e12
+    if fp8:
+        # an e4m3 contraction: the measured bf16 peak x the nominal e4m3 / bf16 ratio (4.5 /
+        # 2.25 PFLOP/s dense); the kernels issue two e4m3 MMAs (hi and lo parts of the other
+        # operand) per algorithmic product, so they cannot pass half of it
+        peak, src = 2.0 * bf16_sus, peak_src + " sustained bf16 x 2 (nominal e4m3 / bf16)"
+    else:
+        peak, src = bf16_sus, peak_src + " sustained"
+    roof = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+            "frac": achieved / peak, "peak_source": src}
+    if fp8:
+        roof["mma_flops_per_algorithmic_flop"] = 2
+    return roof
+
+
+def traffic_for(kind, workload, experts_per_launch, path=None):
     """DRAM bytes per launch from the committed ncu summary (profiles/traffic.json), if it was
     taken on the current FFN kernel sources (its source hash equals build.ffn_source_hash());
     else None.  Decode captures are stored per activated expert and scaled by this run's mean
     activated experts per launch."""
-    path = os.path.join(ROOT, "profiles", "traffic.json")
+    path = path or os.path.join(ROOT, "profiles", "traffic.json")
     try:
         from paper_2609_33614_gb300 import build
         with open(path) as fh:
@@ -419,29 +445,10 @@ def run_ours(args, world, rank, local):
     total_kernel_ms = sum(k["ms"] for k in kinds.values())
     dom = max((k for k in kinds if k.startswith("ffn") or k.startswith("shared")),
               key=lambda k: kinds[k]["ms"])
-    hbm, bf16_burst, bf16_sus, peak_src = load_peaks()
     dk = kinds[dom]
     avg_launch_s = dk["ms"] / 1e3 / max(1, dk["launches"])
-    decode = max(batches) <= 256
-    if decode:
-        achieved = dk["bytes"] / max(1, dk["launches"]) / avg_launch_s / 1e9
-        roof = {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
-                "frac": achieved / hbm, "peak_source": peak_src,
-                "traffic": traffic_for(dom, args.workload, dk["union"] / max(1, dk["launches"]))}
-    else:
-        achieved = dk["flops"] / max(1, dk["launches"]) / avg_launch_s / 1e12
-        if spec.get("fp8"):
-            # an e4m3 contraction: the measured bf16 peak x the nominal e4m3 / bf16 ratio (4.5 /
-            # 2.25 PFLOP/s dense); the kernels issue two e4m3 MMAs (hi and lo parts of the other
-            # operand) per algorithmic product, so they cannot pass half of it
-            peak, src = 2.0 * bf16_sus, peak_src + " sustained bf16 x 2 (nominal e4m3 / bf16)"
-        else:
-            peak, src = bf16_sus, peak_src + " sustained"
-        roof = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                "frac": achieved / peak, "peak_source": src,
-                "traffic": traffic_for(dom, args.workload, dk["union"] / max(1, dk["launches"]))}
-        if spec.get("fp8"):
-            roof["mma_flops_per_algorithmic_flop"] = 2
+    roof = roofline(dk, max(batches) <= 256, bool(spec.get("fp8")), load_peaks())
+    roof["traffic"] = traffic_for(dom, args.workload, dk["union"] / max(1, dk["launches"]))
     roof.update({"kernel": dom, "kernel_share": dk["ms"] / total_kernel_ms,
                  "avg_launch_us": avg_launch_s * 1e6,
                  "algorithmic_bytes_per_launch": dk["bytes"] / max(1, dk["launches"])})

@@ -47,3 +47,38 @@ def test_kernel_bytes_formula():
     b = bench.kernel_bytes("ffn_up", sh, 2, 2, 1)
     assert b == 2 * 2 * 14336 * 4096 * 2 + 2 * 4096 * 2 + 2 * 14336 * 2
     assert bench.kernel_flops("ffn_down", sh, 2, 1) == 2 * 2 * 4096 * 14336
+
+
+def test_roofline_units_and_peaks():
+    """Decode lines are HBM-bound (GB/s of algorithmic bytes per event-timed launch), prefill lines
+    tensor-bound against the sustained bf16 peak, and e4m3 contractions against twice it (the
+    nominal e4m3 / bf16 ratio)."""
+    sys.path.insert(0, ROOT)
+    import bench
+    peaks = (6800.0, 1900.0, 1700.0, "measured")
+    dk = {"ms": 2.0, "launches": 4, "bytes": 4 * 3.4e9, "flops": 4 * 8.5e11}  # 0.5 ms each
+    hbm = bench.roofline(dk, True, False, peaks)
+    assert hbm["bound"] == "hbm" and hbm["unit"] == "GB/s"
+    assert abs(hbm["achieved"] - 6800.0) < 1e-6 and abs(hbm["frac"] - 1.0) < 1e-12
+    ten = bench.roofline(dk, False, False, peaks)
+    assert ten["unit"] == "TFLOP/s" and abs(ten["achieved"] - 1700.0) < 1e-6
+    assert ten["peak"] == 1700.0 and abs(ten["frac"] - 1.0) < 1e-12
+    f8 = bench.roofline(dk, False, True, peaks)
+    assert f8["peak"] == 3400.0 and abs(f8["frac"] - 0.5) < 1e-12
+    assert f8["mma_flops_per_algorithmic_flop"] == 2
+
+
+def test_traffic_needs_the_current_kernel_sources(tmp_path):
+    """A recorded DRAM capture counts only while the FFN kernel sources hash to the recorded value;
+    decode captures scale per activated expert."""
+    sys.path.insert(0, ROOT)
+    import bench
+    from paper_2609_33614_gb300 import build
+    cur = build.ffn_source_hash()
+    rec = {"w": {"ffn_up": {"dram_bytes_per_expert": 2.0e8, "source_hash": cur},
+                 "ffn_down": {"dram_bytes_per_launch": 5.0e8, "source_hash": "0" * 64}}}
+    path = tmp_path / "traffic.json"
+    path.write_text(json.dumps(rec))
+    assert bench.traffic_for("ffn_up", "w", 3.5, path=str(path)) == 7.0e8
+    assert bench.traffic_for("ffn_down", "w", 1.0, path=str(path)) is None
+    assert bench.traffic_for("ffn_up", "other", 1.0, path=str(path)) is None
