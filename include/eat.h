@@ -237,7 +237,11 @@ eat_status eat_get_call_stats(eat_handle* h, int32_t* n_e, double* sum_p, double
  *   out[0] forward calls, out[1] sum over calls of the number of distinct activated experts,
  *   out[2] sum over calls of the activations (sum_t k_t), out[3] kernel launches issued by this
  *   handle (all entry points), out[4] the device status word: 0, or the bits of kernel waits that
- *   expired (a kernel that gives up on a wait returns early and its outputs are invalid). */
+ *   expired (a kernel that gives up on a wait returns early and its outputs are invalid):
+ *   1 the TMA producer waiting for a free pipeline stage, 2 copies still in flight at exit,
+ *   4 the MMA issuer waiting for a free accumulator, 8 the MMA issuer waiting for a stage's data,
+ *   16 MMAs still running before TMEM is freed, 32 the epilogue waiting for an accumulator,
+ *   64 eat_selftest_bounded_wait, 128 the gate/up epilogue's exchange between warps. */
 eat_status eat_get_counters(eat_handle* h, int64_t* out, int32_t n);
 
 /* Per-kernel device timing.  eat_profile_begin(h, capacity) makes every later launch of this
