@@ -11,7 +11,8 @@ fp32 are widened to float64 exactly; nothing is rounded in between.
 Paper: "EAT: Expert Account Tracker for Efficient MoE Inference" (arxiv 2609.33614).
   * §3.1  vanilla MoE layer: router -> selected experts -> renormalised weighted sum
   * §3.2  expert account (N, P_total, C_s), history score S_h (Eq. 1), importance I (Eq. 2)
-  * §3.3  threshold tau (Eq. 3-5), PPL adjustment, boundedness, smoothing
+  * §3.3  threshold tau (Eq. 3-5), PPL adjustment (and the perplexity it reads), boundedness,
+          smoothing
   * §3.4  candidate set / K cap (Eq. 6), mask and renormalisation (Eq. 7-8)
   * Table 1  hyper-parameter defaults
   * §3.5  OPD inference reweighting of the routing probabilities (scales supplied by the caller)
@@ -206,6 +207,23 @@ def ppl_factor(ppl_sign: int, prm: Params) -> float:
     if ppl_sign < 0:
         return prm.ppl_down
     return 1.0
+
+
+def perplexity(nll: np.ndarray) -> float:
+    """The model perplexity §3.3 calibrates tau with: PPL = exp of the mean token negative
+    log-likelihood over the tokens of the current window (at least one)."""
+    nll = np.asarray(nll, F64)
+    return float(math.exp(nll.sum() / nll.shape[0]))
+
+
+def ppl_sign_update(ppl_prev: float, nll: np.ndarray) -> tuple[int, float]:
+    """The sign the §3.3 adjustment reads: +1 when PPL_curr - PPL_prev > 0 (a drop in
+    performance), -1 otherwise; 0 when there is no previous perplexity (NaN) or the current one is
+    not a number.  Returns (sign, PPL_curr); PPL_curr is the next window's PPL_prev."""
+    curr = perplexity(nll)
+    if math.isnan(ppl_prev) or math.isnan(curr):
+        return 0, curr
+    return (1 if curr - ppl_prev > 0 else -1), curr
 
 
 @dataclass

@@ -404,7 +404,7 @@ def _pins(m):
     """Run every pin against module m; returns the names that fail."""
     failed = []
     for name, fn in (("w1", check_w1), ("w2", check_w2), ("w3", check_w3), ("w4", check_w4),
-                     ("swiglu", check_swiglu)):
+                     ("swiglu", check_swiglu), ("w6", check_w6)):
         try:
             fn(m)
         except AssertionError:
@@ -441,6 +441,8 @@ MUTANTS = {
                                 (np.asarray(g, np.float64).sum() + eps)),
     "ppl_factor_sign_flipped": ("ppl_factor",
                                 lambda orig: lambda sign, prm: orig(-sign, prm)),
+    "perplexity_of_summed_nll": ("perplexity",
+                                 lambda orig: lambda nll: float(math.exp(np.sum(nll)))),
     "norm_squared_in_account": ("account_update",
                                 lambda orig: lambda acc, sel, p, n, a:
                                 orig(acc, sel, p, {k: v * v for k, v in n.items()}, a)),
@@ -548,6 +550,33 @@ def check_w5(m):
 
 def test_w5_temporal_smoothing():
     check_w5(orc)
+
+
+def check_w6(m):
+    prev = float("nan")
+    for win in GOLD["W6"]["windows"]:
+        sign, curr = m.ppl_sign_update(prev, np.array(win["nll"]))
+        assert sign == win["sign"] and close(curr, win["ppl"])
+        prev = curr
+
+
+def test_w6_ppl_sign_from_likelihoods():
+    check_w6(orc)
+
+
+def test_perplexity_closed_forms():
+    """PPL of a constant likelihood c is e^c; the sign follows the mean NLL (exp is monotone), a
+    window no worse than the last gives -1 ('otherwise'), and a NaN likelihood gives no signal."""
+    rng = np.random.default_rng(21)
+    for c in (0.0, 0.3, 2.5, 7.0):
+        assert close(orc.perplexity(np.full(5, c)), math.exp(c))
+    for _ in range(50):
+        a, b = rng.uniform(0, 5, 7), rng.uniform(0, 5, 3)
+        s, _ = orc.ppl_sign_update(orc.perplexity(a), b)
+        assert s == (1 if b.mean() > a.mean() else -1)
+    assert orc.ppl_sign_update(math.exp(1.0), np.array([1.0]))[0] == -1
+    assert orc.ppl_sign_update(1.0, np.array([np.nan, 1.0]))[0] == 0
+    assert orc.ppl_sign_update(float("nan"), np.array([1.0])) == (0, math.e)
 
 
 def test_temporal_equals_call_when_prev_is_tau():
