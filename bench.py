@@ -101,16 +101,17 @@ class ClockSampler:
          "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
          "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
-    def __init__(self, gpu_index):
+    def __init__(self, gpu_index, interval_ms=20):
         self.gpu = gpu_index
+        self.interval_ms = interval_ms
         self.proc = None
-        self.lines = []
+        self.lines = []  # (host time, csv line)
 
     def __enter__(self):
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.Q}",
-                 "--format=csv,noheader,nounits", "-lms", "50"],
+                 "--format=csv,noheader,nounits", "-lms", str(self.interval_ms)],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.t = threading.Thread(target=self._read, daemon=True)
             self.t.start()
@@ -120,7 +121,7 @@ class ClockSampler:
 
     def _read(self):
         for line in self.proc.stdout:
-            self.lines.append(line.strip())
+            self.lines.append((time.time(), line.strip()))
 
     def __exit__(self, *a):
         if self.proc:
@@ -130,10 +131,14 @@ class ClockSampler:
             except Exception:
                 self.proc.kill()
 
-    def summary(self):
+    def summary(self, window=None):
+        """Median SM clock, max clock and throttle reasons over the samples (those read inside
+        the host-time window (t0, t1) only, when given)."""
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         sm, mx, reasons = [], [], set()
-        for ln in self.lines:
+        for ts, ln in self.lines:
+            if window is not None and not window[0] <= ts <= window[1]:
+                continue
             f = [x.strip() for x in ln.split(",")]
             if len(f) < 9:
                 continue
@@ -234,8 +239,11 @@ def roofline(dk, decode, fp8, peaks):
     """The dominant kernel against its roofline.  dk: the kernel's event-timed total ms, launch
     count and algorithmic bytes and flops summed over its launches; decode calls are bound by HBM
     (bytes of the activated experts' weights and the activation rows), prefill calls by the
-    tensor pipe (flops).  peaks: (HBM GB/s, bf16 burst TFLOP/s, bf16 sustained TFLOP/s, source)."""
-    hbm, _bf16_burst, bf16_sus, peak_src = peaks
+    tensor pipe (flops).  peaks: (HBM GB/s, bf16 burst TFLOP/s, bf16 sustained TFLOP/s, source).
+    A contraction's launches are event-timed one by one inside sub-millisecond steps, a burst
+    regime, so the burst peak is the denominator; the fraction of the sustained figure is kept
+    beside it as a labelled note."""
+    hbm, bf16_burst, bf16_sus, peak_src = peaks
     avg_launch_s = dk["ms"] / 1e3 / max(1, dk["launches"])
     if decode:
         achieved = dk["bytes"] / max(1, dk["launches"]) / avg_launch_s / 1e9
@@ -246,11 +254,13 @@ def roofline(dk, decode, fp8, peaks):
         # an e4m3 contraction: the measured bf16 peak x the nominal e4m3 / bf16 ratio (4.5 /
         # 2.25 PFLOP/s dense); the kernels issue two e4m3 MMAs (hi and lo parts of the other
         # operand) per algorithmic product, so they cannot pass half of it
-        peak, src = 2.0 * bf16_sus, peak_src + " sustained bf16 x 2 (nominal e4m3 / bf16)"
+        peak, sus = 2.0 * bf16_burst, 2.0 * bf16_sus
+        src = peak_src + " burst bf16 x 2 (nominal e4m3 / bf16)"
     else:
-        peak, src = bf16_sus, peak_src + " sustained"
+        peak, sus, src = bf16_burst, bf16_sus, peak_src + " burst"
     roof = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-            "frac": achieved / peak, "peak_source": src}
+            "frac": achieved / peak, "peak_source": src,
+            "note": {"frac_of_sustained": achieved / sus, "sustained_peak": sus}}
     if fp8:
         roof["mma_flops_per_algorithmic_flop"] = 2
     return roof
@@ -277,17 +287,23 @@ def traffic_for(kind, workload, experts_per_launch, path=None):
 
 
 # ------------------------------------------------------------------------------- our arm
-def run_ours(args, world, rank, local):
+def run_ours(args, world, rank, local, workload, clk, soak_s=1.0, with_cpu_baseline=True):
+    """Measure one workload on this rank's GPU: the timed pass (CUDA events on the launching
+    stream), a pass with per-launch events (dominant kernel and its roofline), an untimed routing
+    replay (k histogram), the end-to-end pass through the host-buffer entry point, for single-layer
+    prefill workloads the cold and warm prefill passes, and a soak of the same steps that gives the
+    clock sampler `clk` samples under this load.  Returns the result fields of the JSON line."""
     import torch
     from paper_2609_33614_gb300 import eat, workloads as W
 
-    spec = workload_spec(args.workload)
+    spec = workload_spec(workload)
     shape = spec["shape"]
     batches = spec["batches"]
     n_layers = spec["layers"]
     dev = torch.device("cuda", torch.cuda.current_device())
     stream = torch.cuda.current_stream()
     n_steps_total = args.warmup + args.steps
+    t_start = time.time()
 
     # layers (weights drawn on the GPU generator) and one handle per (layer, batch)
     layer_w = [W.make_layer(shape, l, device="cuda") for l in range(n_layers)]
@@ -363,9 +379,11 @@ def run_ours(args, world, rank, local):
             for h in row:
                 h.reset()
 
-    def timed(fn, profile=False):
+    def timed(fn, profile=False, window=None, before_step=None):
         reset_all()
         for s in range(args.warmup):
+            if before_step:
+                before_step()
             fn(s)
         if profile:
             for row in handles:
@@ -374,13 +392,18 @@ def run_ours(args, world, rank, local):
         before = [[eat.eat_get_counters(h.h) for h in row] for row in handles]
         barrier(world)
         torch.cuda.synchronize()
+        t0 = time.time()
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
         e0.record(stream)
         for s in range(args.warmup, n_steps_total):
+            if before_step:
+                before_step()
             fn(s)
         e1.record(stream)
         torch.cuda.synchronize()
+        if window is not None:
+            window[:] = [t0, time.time()]
         barrier(world)
         ms = e0.elapsed_time(e1)
         after = [[eat.eat_get_counters(h.h) for h in row] for row in handles]
@@ -389,17 +412,14 @@ def run_ours(args, world, rank, local):
             prof = [[eat.eat_profile_end(h.h) for h in row] for row in handles]
         return ms, before, after, prof
 
-    with ClockSampler(local) as clk:
-        ms, c0, c1, _ = timed(step)
-    clocks = clk.summary()
+    timed_window = [0.0, 0.0]
+    ms, c0, c1, _ = timed(step, window=timed_window)
     job_ms = max_over_ranks(ms, world)
     total_tokens = sum_over_ranks(tokens_per_step * args.steps, world)
     value = total_tokens / (job_ms / 1e3)
 
     launches = sum(c1[l][b]["launches"] - c0[l][b]["launches"]
                    for l in range(n_layers) for b in range(len(batches)))
-    calls = sum(c1[l][b]["calls"] - c0[l][b]["calls"]
-                for l in range(n_layers) for b in range(len(batches)))
     acts = sum(c1[l][b]["activations"] - c0[l][b]["activations"]
                for l in range(n_layers) for b in range(len(batches)))
     unions = {B: (sum(c1[l][bi]["union_sum"] - c0[l][bi]["union_sum"] for l in range(n_layers)) /
@@ -448,10 +468,11 @@ def run_ours(args, world, rank, local):
     dk = kinds[dom]
     avg_launch_s = dk["ms"] / 1e3 / max(1, dk["launches"])
     roof = roofline(dk, max(batches) <= 256, bool(spec.get("fp8")), load_peaks())
-    roof["traffic"] = traffic_for(dom, args.workload, dk["union"] / max(1, dk["launches"]))
+    roof["traffic"] = traffic_for(dom, workload, dk["union"] / max(1, dk["launches"]))
     roof.update({"kernel": dom, "kernel_share": dk["ms"] / total_kernel_ms,
                  "avg_launch_us": avg_launch_s * 1e6,
-                 "algorithmic_bytes_per_launch": dk["bytes"] / max(1, dk["launches"])})
+                 "algorithmic_bytes_per_launch": dk["bytes"] / max(1, dk["launches"]),
+                 "algorithmic_flops_per_launch": dk["flops"] / max(1, dk["launches"])})
 
     # end to end through the public host-buffer entry point (copies inside the timed region)
     xh = {B: [x.cpu().pin_memory() for x in xs[B]] for B in batches}
@@ -479,13 +500,55 @@ def run_ours(args, world, rank, local):
            "h2d_bytes_per_step": tokens_per_step * shape.d_model * elt,
            "d2h_bytes_per_step": tokens_per_step * shape.d_model * elt}
 
+    # cold and warm prefill: every timed call starts from the same account state, the empty history
+    # of a reset (cold) or the state left by 8 calls of 256 tokens (warm), restored in stream order
+    # before each call (three small device copies inside the timed region)
+    prefill_states = None
+    if n_layers == 1 and len(batches) == 1 and batches[0] > 256:
+        E = shape.n_experts
+        h0 = handles[0][0]
+        zero = (torch.zeros(E, dtype=torch.int64, device=dev),
+                torch.zeros(E, dtype=torch.float64, device=dev),
+                torch.zeros(E, dtype=torch.float64, device=dev))
+        h0.reset()
+        for s in range(8):
+            h0.forward(xs[batches[0]][s % len(xs[batches[0]])][:256].contiguous(), 0)
+        warm = tuple(t.clone() for t in h0.accounts())
+        prefill_states = {}
+        for name, snap in (("cold", zero), ("warm", warm)):
+            st_ms, q0, q1, _ = timed(step, before_step=lambda snap=snap: h0.set_accounts(*snap))
+            st_ms = max_over_ranks(st_ms, world)
+            dC = q1[0][0]["calls"] - q0[0][0]["calls"]
+            prefill_states[name] = {
+                "value": sum_over_ranks(tokens_per_step * args.steps, world) / (st_ms / 1e3),
+                "unit": "tokens/s", "ms_per_step": st_ms / args.steps,
+                "union_per_call": (q1[0][0]["union_sum"] - q0[0][0]["union_sum"]) / max(1, dC),
+                "experts_per_token": (q1[0][0]["activations"] - q0[0][0]["activations"]) /
+                max(1, dC * batches[0])}
+        prefill_states["warm"]["state"] = "accounts after 8 calls of 256 tokens from a reset"
+
+    # soak: the same steps, untimed, so that the clock sampler sees this load for soak_s seconds
+    t_soak = time.time()
+    s = 0
+    while time.time() - t_soak < soak_s:
+        step(s)
+        s += 1
+        if s % 8 == 0:
+            torch.cuda.synchronize()
+    torch.cuda.synchronize()
+    t_end = time.time()
+
+    clocks = clk.summary((t_start, t_end))
+    clocks["timed_region"] = clk.summary(tuple(timed_window))
+    clocks["sampled"] = "nvidia-smi every 20 ms over this workload's timed, per-launch, e2e " \
+                        f"passes and a {soak_s:.1f} s soak of the same steps"
+    if clocks.get("sm_mhz"):
+        roof["avg_launch_us_x_sm_mhz"] = avg_launch_s * 1e6 * clocks["sm_mhz"]
+
     result = {
-        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+        "value": value, "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": job_ms / args.steps,
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "e4m3" if spec.get("fp8") else "bf16",
-        "data": "synthetic (seeded N(0,1) hidden states, N(0,0.02^2) weights"
-                + (", quantized to e4m3 per row)" if spec.get("fp8") else ")"),
         "config": bench_config(args, spec),
         "roofline": roof,
         "experts_per_token": acts / max(1, sum(B * args.steps for B in batches) * n_layers),
@@ -496,12 +559,18 @@ def run_ours(args, world, rank, local):
         "clocks": clocks,
         "e2e": e2e,
     }
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        result["cpu_baseline"] = oracle_sample(args.workload, layer_w[0], handles[0][0],
+    if prefill_states is not None:
+        result["prefill_states"] = prefill_states
+    if rank == 0 and world == 1 and with_cpu_baseline and not args.no_cpu_baseline:
+        result["cpu_baseline"] = oracle_sample(workload, layer_w[0], handles[0][0],
                                                min_seconds=10.0)
+        result["cpu_baseline"]["single_thread"] = oracle_sample_single_thread(
+            workload, layer_w[0], handles[0][0], min_seconds=5.0)
     for row in handles:
         for h in row:
             h.close()
+    del layer_w, handles
+    torch.cuda.empty_cache()
     return result
 
 
@@ -551,6 +620,49 @@ def oracle_sample(workload, lw, handle=None, min_seconds=10.0, max_steps=None, b
             "kind": "oracle",
             "sample": f"{calls} oracle layer calls cycling batches {bs} ({toks} tokens, "
                       f"{el:.1f} s), fp64 numpy, weights widened to fp64 before timing"}
+
+
+def _blas_thread_setter():
+    """openblas_set_num_threads (under any of its exported names) of the BLAS library numpy
+    loaded into this process, found through /proc/self/maps; None when there is none."""
+    import ctypes
+    import numpy  # noqa: F401  (loads the BLAS library)
+    paths = set()
+    try:
+        with open("/proc/self/maps") as fh:
+            for ln in fh:
+                f = ln.split()
+                if len(f) >= 6 and "blas" in f[-1].lower() and ".so" in f[-1]:
+                    paths.add(f[-1])
+    except OSError:
+        return None
+    for path in sorted(paths):
+        try:
+            lib = ctypes.CDLL(path)
+        except OSError:
+            continue
+        for name in ("openblas_set_num_threads", "scipy_openblas_set_num_threads64_",
+                     "scipy_openblas_set_num_threads", "openblas_set_num_threads64_"):
+            fn = getattr(lib, name, None)
+            if fn is not None:
+                fn.argtypes = [ctypes.c_int]
+                fn.restype = None
+                return fn
+    return None
+
+
+def oracle_sample_single_thread(workload, lw, handle=None, min_seconds=5.0):
+    """The same oracle sample with its BLAS library limited to one thread (restored after)."""
+    setter = _blas_thread_setter()
+    if setter is None:
+        return {"unavailable": "no openblas_set_num_threads in the BLAS library numpy loaded"}
+    setter(1)
+    try:
+        r = oracle_sample(workload, lw, handle, min_seconds=min_seconds)
+    finally:
+        setter(int(os.environ["OPENBLAS_NUM_THREADS"]))
+    r["cores"] = 1
+    return r
 
 
 def run_reference(args, world, rank):
@@ -605,6 +717,8 @@ def main(argv=None):
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="mixtral-decode")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-prefill-record", action="store_true",
+                    help="default workload only: skip the OLMoE prefill sub-record")
     ap.add_argument("--router", default="eat", choices=["eat", "topk", "topp"],
                     help="selection rule: EAT (default) or the paper's Top-K / Top-P baselines")
     ap.add_argument("--top-p", type=float, default=0.6)
@@ -621,7 +735,21 @@ def main(argv=None):
         if rank == 0:
             build.build()
         barrier(world)
-        res = run_ours(args, world, rank, local)
+        with ClockSampler(local) as clk:
+            res = run_ours(args, world, rank, local, args.workload, clk)
+            if args.workload == "mixtral-decode" and not args.no_prefill_record:
+                # the prefill half of the metric, measured in the same run: one OLMoE-shaped
+                # prefill layer (4096 tokens per call)
+                pre = run_ours(args, world, rank, local, "olmoe-prefill", clk, soak_s=0.5,
+                               with_cpu_baseline=False)
+                pre.pop("n_gpus")
+                pre["workload"] = "olmoe-prefill"
+                res["prefill"] = pre
+        res = {"metric": METRIC, **res, "higher_is_better": True, "scaling": "weak",
+               "vs_baseline": None,
+               "data": "synthetic (seeded N(0,1) hidden states, N(0,0.02^2) weights" +
+                       (", quantized to e4m3 per row)" if workload_spec(args.workload).get("fp8")
+                        else ")")}
     if rank == 0 and res is not None:
         print(json.dumps(res))
     if world > 1:

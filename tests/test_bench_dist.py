@@ -51,7 +51,8 @@ def test_kernel_bytes_formula():
 
 def test_roofline_units_and_peaks():
     """Decode lines are HBM-bound (GB/s of algorithmic bytes per event-timed launch), prefill lines
-    tensor-bound against the sustained bf16 peak, and e4m3 contractions against twice it (the
+    tensor-bound against the burst bf16 peak (launches event-timed one by one), with the fraction
+    of the sustained peak as a note, and e4m3 contractions against twice the bf16 figures (the
     nominal e4m3 / bf16 ratio)."""
     sys.path.insert(0, ROOT)
     import bench
@@ -62,9 +63,11 @@ def test_roofline_units_and_peaks():
     assert abs(hbm["achieved"] - 6800.0) < 1e-6 and abs(hbm["frac"] - 1.0) < 1e-12
     ten = bench.roofline(dk, False, False, peaks)
     assert ten["unit"] == "TFLOP/s" and abs(ten["achieved"] - 1700.0) < 1e-6
-    assert ten["peak"] == 1700.0 and abs(ten["frac"] - 1.0) < 1e-12
+    assert ten["peak"] == 1900.0 and abs(ten["frac"] - 1700.0 / 1900.0) < 1e-12
+    assert abs(ten["note"]["frac_of_sustained"] - 1.0) < 1e-12
     f8 = bench.roofline(dk, False, True, peaks)
-    assert f8["peak"] == 3400.0 and abs(f8["frac"] - 0.5) < 1e-12
+    assert f8["peak"] == 3800.0 and abs(f8["frac"] - 1700.0 / 3800.0) < 1e-12
+    assert abs(f8["note"]["frac_of_sustained"] - 0.5) < 1e-12
     assert f8["mma_flops_per_algorithmic_flop"] == 2
 
 
@@ -82,3 +85,14 @@ def test_traffic_needs_the_current_kernel_sources(tmp_path):
     assert bench.traffic_for("ffn_up", "w", 3.5, path=str(path)) == 7.0e8
     assert bench.traffic_for("ffn_down", "w", 1.0, path=str(path)) is None
     assert bench.traffic_for("ffn_up", "other", 1.0, path=str(path)) is None
+
+
+def test_blas_thread_setter_found_or_none():
+    """The single-thread oracle timing finds the BLAS library's thread setter, or reports that it
+    cannot (then the line says so instead of timing all cores as one)."""
+    sys.path.insert(0, ROOT)
+    import bench
+    fn = bench._blas_thread_setter()
+    if fn is not None:
+        fn(1)
+        fn(os.cpu_count() or 1)
