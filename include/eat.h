@@ -39,7 +39,8 @@ typedef enum eat_status {
   EAT_ERR_UNSUPPORTED = 2,  /* valid request outside what this build implements */
   EAT_ERR_OOM = 3,          /* device allocation failed in eat_create */
   EAT_ERR_CUDA = 4,         /* a CUDA runtime call or kernel launch failed */
-  EAT_ERR_STATE = 5         /* handle not usable (e.g. device-side status word set) */
+  EAT_ERR_STATE = 5         /* handle not usable: a kernel of an earlier call gave up on a bounded
+                               wait (device status word set); cleared by eat_reset_accounts */
 } eat_status;
 
 /* EAT_FP8_E4M3 is an expert-weight type only (wdtype, with xdtype EAT_BF16): OCP e4m3 bytes with
@@ -138,7 +139,9 @@ typedef struct eat_handle eat_handle;
  * receives the handle; on failure *out is set to NULL and nothing stays allocated. */
 eat_status eat_create(const eat_layer_desc* desc, const eat_params* params, eat_handle** out);
 
-/* Zero the accounts N, P_total, C_s (§3.2: an expert with no history) and the counters. */
+/* Zero the accounts N, P_total, C_s (§3.2: an expert with no history), the counters and the
+ * device status word, and return the handle to service after EAT_ERR_STATE.  Synchronises
+ * `stream` (every earlier call on it has finished when it returns). */
 eat_status eat_reset_accounts(eat_handle* h, void* stream);
 
 /* Routing only (§3.2-§3.4, Eq. 1-8) for T tokens x [T, d] (xdtype), 1 <= T <= max_tokens,
@@ -149,6 +152,15 @@ eat_status eat_reset_accounts(eat_handle* h, void* stream);
  * w [T, K] fp32 renormalised gates g_norm (Eq. 7), 0 after the k-th; k [T] int32 count. */
 eat_status eat_route(eat_handle* h, const void* x, int32_t T, int32_t ppl_sign,
                      int32_t* idx, float* w, int32_t* k, void* stream);
+
+/* Failure state (every entry point that runs the layer or routes): the expert kernels never trap;
+ * a wait that expires after its 2 s bound sets a bit in the handle's device status word and the
+ * kernel returns early.  The combine kernel of that call then writes NaN rows to y and the account
+ * update leaves N, P_total and C_s unchanged; the call's last kernel copies the word to host-mapped
+ * memory.  The next eat_route / eat_moe_forward / eat_moe_forward_host(_async) on the handle that
+ * finds the copy set returns EAT_ERR_STATE, and so does every later one until
+ * eat_reset_accounts; eat_moe_forward_host, which synchronises, returns EAT_ERR_STATE for the
+ * failing call itself. */
 
 /* One layer call = one EMA timestep of §3.2 over T tokens, 1 <= T <= max_tokens (an empty call has
  * no batch mean to fold into the accounts and is rejected with EAT_ERR_INVALID_ARG): routing as
@@ -183,7 +195,8 @@ eat_status eat_moe_forward_host(eat_handle* h, const void* x_host, int32_t T, in
 eat_status eat_moe_forward_host_async(eat_handle* h, const void* x_host, int32_t T,
                                       int32_t ppl_sign, void* y_host, void* stream);
 
-/* Size of the fixed device scratch eat_route_noalloc uses (1 MiB = 131072 fp64 router scores). */
+/* Size of the fixed device scratch eat_route_noalloc uses: 1 MiB = 131072 partial router scores,
+ * each a compensated fp32 pair (hi, lo) of 8 bytes. */
 #define EAT_NOALLOC_SCRATCH_BYTES (1u << 20)
 
 /* Routing for callers that cannot allocate device memory.  The paper has no counterpart: this is a
@@ -198,7 +211,9 @@ eat_status eat_moe_forward_host_async(eat_handle* h, const void* x_host, int32_t
  *  - T * n_experts must be <= 131072 (EAT_NOALLOC_SCRATCH_BYTES / 8), else EAT_ERR_INVALID_ARG;
  *    larger batches are routed in several calls.
  *  - The first call on each device looks up the scratch's device address (a one-time set-up per
- *    device, done with that device current); make that first call before any stream capture.
+ *    device, done with that device current), and so does the first call after the device's
+ *    current context changed (e.g. after cudaDeviceReset); make that first call before any
+ *    stream capture.
  *  - Calls share the scratch: two calls that may overlap on the GPU (different streams or host
  *    threads) race on it and must be serialised by the caller.
  *  - There is no per-stream threshold state without a handle: EAT_SMOOTH_TEMPORAL is routed as
@@ -216,6 +231,31 @@ eat_status eat_route_noalloc(const void* x, int32_t T, int32_t d_model, int32_t 
  * NaN entries mean "no previous call" (the same-call blend is used).  NULL detaches the state
  * (temporal mode then behaves as EAT_SMOOTH_CALL).  The array must stay alive while attached. */
 eat_status eat_set_tau_state(eat_handle* h, float* tau_state);
+
+/* The perplexity signal of §3.3's performance-based adjustment, for a model loop on the device.
+ * nll: device [n] fp32 negative log-likelihoods of the n >= 1 tokens of the current window (e.g.
+ * the tokens generated since the last call); ppl_state: a caller-owned device fp64 scalar holding
+ * the previous window's perplexity (set it to NaN before the first window: no previous value);
+ * sign: device int32 output.  One kernel on `stream` computes PPL_curr = exp(mean nll) (fp64 sum
+ * in a fixed order), writes *sign = +1 when PPL_curr - PPL_prev > 0 (a drop in performance), -1
+ * otherwise, 0 when there is no previous value or PPL_curr is NaN, and stores PPL_curr into
+ * *ppl_state.  Errors through eat_last_error(NULL). */
+eat_status eat_ppl_update(const float* nll, int32_t n, double* ppl_state, int32_t* sign,
+                          void* stream);
+
+/* Attach a device PPL sign (the `sign` of eat_ppl_update, caller-owned, alive while attached) to
+ * the handle: eat_route / eat_moe_forward then read the sign from device memory when their
+ * selection kernel runs, stream-ordered after the eat_ppl_update that wrote it, and ignore their
+ * ppl_sign argument (which is still validated).  NULL detaches it. */
+eat_status eat_set_ppl_sign_source(eat_handle* h, const int32_t* sign);
+
+/* Layer-wise routing policy after §5.2 (experts in lower layers matter less than in higher ones:
+ * the paper keeps 1.3-1.5 experts per token in layers 0-23 of a 32-layer stack and the full K
+ * above).  Adjusts *p for layer `layer` of an n_layers stack: in the lower three quarters, max_k
+ * becomes max(1, max_k / 3) and alpha1 (the threshold floor of Eq. 5) doubles; the upper quarter
+ * keeps *p.  Call it on each layer's params before eat_create.  EAT_ERR_INVALID_ARG unless
+ * 0 <= layer < n_layers and p is non-NULL. */
+eat_status eat_layer_policy(int32_t layer, int32_t n_layers, eat_params* p);
 
 /* Free everything the handle owns.  Synchronises the device first.  NULL is accepted. */
 eat_status eat_destroy(eat_handle* h);
@@ -241,7 +281,8 @@ eat_status eat_get_call_stats(eat_handle* h, int32_t* n_e, double* sum_p, double
  *   1 the TMA producer waiting for a free pipeline stage, 2 copies still in flight at exit,
  *   4 the MMA issuer waiting for a free accumulator, 8 the MMA issuer waiting for a stage's data,
  *   16 MMAs still running before TMEM is freed, 32 the epilogue waiting for an accumulator,
- *   64 eat_selftest_bounded_wait, 128 the gate/up epilogue's exchange between warps. */
+ *   64 eat_selftest_bounded_wait / eat_selftest_expire_wait, 128 the gate/up epilogue's exchange
+ *   between warps. */
 eat_status eat_get_counters(eat_handle* h, int64_t* out, int32_t n);
 
 /* Per-kernel device timing.  eat_profile_begin(h, capacity) makes every later launch of this
@@ -262,6 +303,13 @@ int32_t eat_ffn_backend(const eat_handle* h);
  * gives up, sets bit 64 in a device status word and the kernel returns; *status_out receives the
  * word (64 when the bound works) and the context stays usable.  Synchronous; allocates 4 bytes. */
 eat_status eat_selftest_bounded_wait(int64_t limit_ns, uint32_t* status_out);
+
+/* Diagnostic of the failure state: enqueues on `stream` the same bounded wait on a barrier nothing
+ * arrives on, writing the handle's device status word.  After limit_ns (1 us .. 1 s) it gives up
+ * and sets bit 64, exactly as an expert kernel whose wait expired would set its bit: the next
+ * layer call on `stream` writes NaN outputs, leaves the accounts unchanged, and later calls return
+ * EAT_ERR_STATE until eat_reset_accounts.  No fault, trap or hang is involved. */
+eat_status eat_selftest_expire_wait(eat_handle* h, int64_t limit_ns, void* stream);
 
 /* Last error on the handle (never NULL), or a generic text for a NULL handle. */
 const char* eat_last_error(const eat_handle* h);

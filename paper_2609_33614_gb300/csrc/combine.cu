@@ -13,6 +13,11 @@
 //      N += n_e, P_total += sum p, C_s <- (1 - alpha) C_s + alpha * mean ||o||_2 when n_e > 0.
 //      Per-slot work stays off GB300's narrow fp64 pipe: an fp64 square root per slot made the
 //      block of a heavily used expert the longest of the step.
+//  Both read the device status word: when an earlier kernel of the call gave up on a bounded wait
+//  (its outputs are then invalid), the combine writes NaN rows and the account update leaves N,
+//  P_total and C_s as they were, so one expired wait cannot feed invalid norms into the accounts
+//  that every later call routes by.  Block 0 of the account kernel copies the word to a
+//  host-mapped mirror, which the entry points read without synchronising.
 #include "eat_internal.cuh"
 
 namespace eat {
@@ -92,7 +97,8 @@ __global__ void __launch_bounds__(kCombThreads)
 combine_kernel(const void* __restrict__ opart, int n_split, size_t split_stride,
                const int32_t* __restrict__ slot_of, const float* __restrict__ w,
                const void* __restrict__ sout, int s_bf16, int S, int T, int K, int d, int nseg,
-               TY* __restrict__ y, float* __restrict__ nrm_part) {
+               TY* __restrict__ y, float* __restrict__ nrm_part,
+               const unsigned int* __restrict__ status) {
   pdl_wait();
   pdl_launch_dependents();
   const unsigned full = 0xffffffffu;
@@ -171,7 +177,9 @@ combine_kernel(const void* __restrict__ opart, int n_split, size_t split_stride,
 #pragma unroll
       for (int i = 0; i < 8; ++i) acc[i] += q.v[i];
     }
-    if (slots[0] < 0) {  // no expert selected: the token's routing was not finite (NaN row)
+    // no expert selected (the token's routing was not finite), or an expert kernel of this call
+    // gave up on a wait (its outputs are invalid): a NaN row
+    if (slots[0] < 0 || __ldcg(status) != 0u) {
 #pragma unroll
       for (int i = 0; i < 8; ++i) acc[i] = __int_as_float(0x7fc00000);
     }
@@ -188,7 +196,8 @@ account_kernel(const int32_t* __restrict__ offs, const float* __restrict__ perm_
                const float* __restrict__ nrm_part, int nb, double alpha, int64_t* __restrict__ N,
                double* __restrict__ P, double* __restrict__ C, int32_t* __restrict__ st_n,
                double* __restrict__ st_p, double* __restrict__ st_norm,
-               unsigned long long* __restrict__ counters) {
+               unsigned long long* __restrict__ counters, const unsigned int* __restrict__ status,
+               unsigned int* __restrict__ status_mirror) {
   __shared__ float red[4][kAccThreads / 32];
   pdl_wait();
   pdl_launch_dependents();
@@ -253,15 +262,19 @@ account_kernel(const int32_t* __restrict__ offs, const float* __restrict__ perm_
     }
     const double a = (double)ah + (double)al, b = (double)bh + (double)bl;
     const int n = end - beg;
-    N[e] += n;
-    P[e] += a;
-    if (n > 0) C[e] = (1.0 - alpha) * C[e] + alpha * (b / (double)n);
+    const unsigned int sw = __ldcg(status);
+    if (sw == 0u) {  // every kernel of the call completed its work
+      N[e] += n;
+      P[e] += a;
+      if (n > 0) C[e] = (1.0 - alpha) * C[e] + alpha * (b / (double)n);
+      if (n > 0) atomicAdd(&counters[1], 1ull);
+      atomicAdd(&counters[2], (unsigned long long)n);
+      if (e == 0) atomicAdd(&counters[0], 1ull);
+    }
     st_n[e] = n;
     st_p[e] = a;
     st_norm[e] = b;
-    if (n > 0) atomicAdd(&counters[1], 1ull);
-    atomicAdd(&counters[2], (unsigned long long)n);
-    if (e == 0) atomicAdd(&counters[0], 1ull);
+    if (e == 0 && status_mirror) *(volatile unsigned int*)status_mirror = sw;
   }
 }
 
@@ -275,27 +288,27 @@ template <typename TY, int KM>
 cudaError_t launch_combine_t(int o_bf16, cudaStream_t st, const void* opart, int n_split,
                              size_t stride, const int32_t* slot_of, const float* w,
                              const void* sout, int s_bf16, int S, int T, int K, int d, void* y,
-                             float* nrm_part) {
+                             float* nrm_part, const unsigned int* status) {
   const int nseg = combine_col_blocks(d);
   const long long tasks = (long long)T * nseg;
   const dim3 grid((unsigned)((tasks + kCombThreads / 32 - 1) / (kCombThreads / 32)));
   if (o_bf16)
     return launch_pdl(combine_kernel<TY, KM, true>, grid, dim3(kCombThreads), 0, st, opart,
                       n_split, stride, slot_of, w, sout, s_bf16, S, T, K, d, nseg, (TY*)y,
-                      nrm_part);
+                      nrm_part, status);
   return launch_pdl(combine_kernel<TY, KM, false>, grid, dim3(kCombThreads), 0, st, opart,
                     n_split, stride, slot_of, w, sout, s_bf16, S, T, K, d, nseg, (TY*)y,
-                    nrm_part);
+                    nrm_part, status);
 }
 
 template <typename TY>
 cudaError_t launch_combine_k(int o_bf16, cudaStream_t st, const void* opart, int n_split,
                              size_t stride, const int32_t* slot_of, const float* w,
                              const void* sout, int s_bf16, int S, int T, int K, int d, void* y,
-                             float* nrm_part) {
+                             float* nrm_part, const unsigned int* status) {
 #define EAT_COMB(KM)                                                                           \
   launch_combine_t<TY, KM>(o_bf16, st, opart, n_split, stride, slot_of, w, sout, s_bf16, S, T, \
-                           K, d, y, nrm_part)
+                           K, d, y, nrm_part, status)
   if (K <= 2) return EAT_COMB(2);
   if (K <= 4) return EAT_COMB(4);
   if (K <= 8) return EAT_COMB(8);
@@ -308,20 +321,23 @@ cudaError_t launch_combine_k(int o_bf16, cudaStream_t st, const void* opart, int
 cudaError_t launch_combine(int y_bf16, const void* opart, int o_bf16, int n_split,
                            int split_stride_rows, const int32_t* slot_of, const float* w,
                            const void* sout, int s_bf16, int S, int T, int K, int d, void* y,
-                           float* nrm_part, cudaStream_t st) {
+                           float* nrm_part, const unsigned int* status, cudaStream_t st) {
   const size_t stride = (size_t)split_stride_rows * d;
   if (y_bf16)
     return launch_combine_k<__nv_bfloat16>(o_bf16, st, opart, n_split, stride, slot_of, w, sout,
-                                           s_bf16, S, T, K, d, y, nrm_part);
+                                           s_bf16, S, T, K, d, y, nrm_part, status);
   return launch_combine_k<float>(o_bf16, st, opart, n_split, stride, slot_of, w, sout, s_bf16, S,
-                                 T, K, d, y, nrm_part);
+                                 T, K, d, y, nrm_part, status);
 }
 
 cudaError_t launch_account(const int32_t* offs, const float* perm_p, const float* nrm_part, int nb,
                            int E, double alpha, int64_t* N, double* P, double* C, int32_t* st_n,
-                           double* st_p, double* st_norm, long long* counters, cudaStream_t st) {
+                           double* st_p, double* st_norm, long long* counters,
+                           const unsigned int* status, unsigned int* status_mirror,
+                           cudaStream_t st) {
   return launch_pdl(account_kernel, dim3(E), dim3(kAccThreads), 0, st, offs, perm_p, nrm_part,
-                    nb, alpha, N, P, C, st_n, st_p, st_norm, (unsigned long long*)counters);
+                    nb, alpha, N, P, C, st_n, st_p, st_norm, (unsigned long long*)counters, status,
+                    status_mirror);
 }
 
 }  // namespace eat

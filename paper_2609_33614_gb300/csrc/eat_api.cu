@@ -60,9 +60,15 @@ struct eat_handle {
   int stage_i = 0;
   void* xperm = nullptr;  // [Tmax*K, d] gathered token rows (tensor-core path)
   unsigned int* status = nullptr;  // device status word: bounded waits that expired
+  // host-mapped copy of the status word, written by the account kernel of every forward call
+  // (the host pointer is read by the entry points without a synchronisation)
+  unsigned int* mirror_host = nullptr;
+  unsigned int* mirror_dev = nullptr;
+  bool failed = false;  // a call saw the status word set: calls fail until eat_reset_accounts
   int32_t* chunk_cnt = nullptr;    // permute scratch: ticket word, then [chunks][E] counts
   long long opart_rows = 0;
   float* tau_state = nullptr;  // caller-owned [Tmax] previous tau_final per stream, or null
+  const int32_t* ppl_sign_src = nullptr;  // caller-owned device PPL sign (eat_ppl_update), or null
 
   TcLayer tc{};
 
@@ -154,10 +160,28 @@ RouteParams route_params(const eat_params& p, int ppl_sign) {
   r.opd_scale = nullptr;
   r.tau_in = nullptr;
   r.tau_out = nullptr;
+  r.ppl_sign_dev = nullptr;
+  r.ppl_up = (float)p.ppl_up;
+  r.ppl_down = (float)p.ppl_down;
   return r;
 }
 
 size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+// A kernel of an earlier call gave up on a bounded wait (the status word is set): that call's
+// outputs were NaN and the accounts stayed as they were; the handle refuses further calls until
+// eat_reset_accounts.
+eat_status check_state(eat_handle* h) {
+  const unsigned int sw = h->mirror_host ? *(volatile unsigned int*)h->mirror_host : 0u;
+  if (!h->failed && sw == 0u) return EAT_OK;
+  h->failed = true;
+  char msg[200];
+  snprintf(msg, sizeof msg,
+           "a kernel of an earlier call gave up on a bounded wait (status word 0x%x): its outputs "
+           "were NaN and the accounts were left unchanged; eat_reset_accounts clears the state",
+           sw);
+  return fail(h, EAT_ERR_STATE, msg);
+}
 
 eat_status check_call(eat_handle* h, const void* x, int32_t T, int32_t ppl_sign) {
   if (!h) return fail(nullptr, EAT_ERR_INVALID_ARG, "null handle");
@@ -170,7 +194,7 @@ eat_status check_call(eat_handle* h, const void* x, int32_t T, int32_t ppl_sign)
     return fail(h, EAT_ERR_INVALID_ARG, "ppl_sign must be -1, 0 or +1");
   if (((uintptr_t)x & 15) != 0)
     return fail(h, EAT_ERR_INVALID_ARG, "x must be 16-byte aligned");
-  return EAT_OK;
+  return check_state(h);
 }
 
 // Router + selection into (idx, w, k, psel).
@@ -178,6 +202,7 @@ eat_status run_route(eat_handle* h, const void* x, int T, int ppl_sign, int32_t*
                      int32_t* k, float* psel, bool write_tau, cudaStream_t st) {
   RouteParams rp = route_params(h->prm, ppl_sign);
   rp.opd_scale = h->desc.opd_scale;
+  rp.ppl_sign_dev = h->ppl_sign_src;
   if (h->prm.smoothing_mode == EAT_SMOOTH_TEMPORAL && h->tau_state) {
     rp.tau_in = h->tau_state;
     rp.tau_out = write_tau ? h->tau_state : nullptr;
@@ -303,11 +328,12 @@ eat_status run_forward(eat_handle* h, const void* x, int T, int ppl_sign, void* 
   EAT_TRY(launch(h, kCombine, st, "combine", [&] {
     const int tc = h->backend == 1;
     return launch_combine(h->bf16, h->opart, tc && n_split == 1, n_split, rows, h->perm.slot_of,
-                          h->w, h->sout, tc, h->S, T, h->K, h->d, y, h->nrm_part, st);
+                          h->w, h->sout, tc, h->S, T, h->K, h->d, y, h->nrm_part, h->status, st);
   }));
   EAT_TRY(launch(h, kAccount, st, "account update", [&] {
     return launch_account(h->perm.offs, h->perm.perm_p, h->nrm_part, h->nb, h->E, h->prm.alpha,
-                          h->N, h->P, h->C, h->st_n, h->st_p, h->st_norm, h->counters, st);
+                          h->N, h->P, h->C, h->st_n, h->st_p, h->st_norm, h->counters, h->status,
+                          h->mirror_dev, st);
   }));
   if (idx_opt || w_opt || k_opt) {
     cudaError_t e = cudaSuccess;
@@ -334,6 +360,7 @@ void free_handle(eat_handle* h) {
   if (h->ev_join) cudaEventDestroy(h->ev_join);
   if (h->side_st) cudaStreamDestroy(h->side_st);
   tc_destroy(h->tc);
+  if (h->mirror_host) cudaFreeHost(h->mirror_host);
   if (h->mem) cudaFree(h->mem);
   delete h;
 }
@@ -528,6 +555,17 @@ eat_status eat_create(const eat_layer_desc* desc, const eat_params* params, eat_
       return fail(nullptr, EAT_ERR_CUDA, m);
     }
   }
+  e = cudaHostAlloc((void**)&h->mirror_host, 16, cudaHostAllocMapped);
+  if (e == cudaSuccess) {
+    std::memset(h->mirror_host, 0, 16);
+    e = cudaHostGetDevicePointer((void**)&h->mirror_dev, h->mirror_host, 0);
+  }
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    free_handle(h);
+    return fail(nullptr, EAT_ERR_OOM,
+                std::string("mapped host status word: ") + cudaGetErrorString(e));
+  }
   if (h->S > 0) {  // created here, not on first use, so that a call may be stream-captured
     e = cudaStreamCreateWithFlags(&h->side_st, cudaStreamNonBlocking);
     if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming);
@@ -549,7 +587,11 @@ eat_status eat_reset_accounts(eat_handle* h, void* stream) {
   if (e == cudaSuccess) e = cudaMemsetAsync(h->C, 0, sizeof(double) * h->E, st);
   if (e == cudaSuccess) e = cudaMemsetAsync(h->counters, 0, sizeof(long long) * 4, st);
   if (e == cudaSuccess) e = cudaMemsetAsync(h->status, 0, sizeof(unsigned int) * 4, st);
+  // every earlier call has written its copy of the status word before the copy is cleared
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
   if (e != cudaSuccess) return cuda_fail(h, e, "reset accounts");
+  *(volatile unsigned int*)h->mirror_host = 0u;
+  h->failed = false;
   h->launches = 0;
   return EAT_OK;
 }
@@ -600,6 +642,7 @@ static eat_status forward_host(eat_handle* h, const void* x_host, int32_t T, int
   if (e == cudaSuccess) e = cudaMemcpyAsync(y_host, h->ystage, bytes, cudaMemcpyDeviceToHost, st);
   if (e == cudaSuccess && sync) e = cudaStreamSynchronize(st);
   if (e != cudaSuccess) return cuda_fail(h, e, "y device-to-host copy");
+  if (sync) return check_state(h);  // this call's own kernels, now complete
   return EAT_OK;
 }
 
@@ -618,6 +661,14 @@ eat_status eat_set_tau_state(eat_handle* h, float* tau_state) {
   if (((uintptr_t)tau_state & 3) != 0)
     return fail(h, EAT_ERR_INVALID_ARG, "tau_state must be 4-byte aligned");
   h->tau_state = tau_state;
+  return EAT_OK;
+}
+
+eat_status eat_set_ppl_sign_source(eat_handle* h, const int32_t* sign) {
+  if (!h) return fail(nullptr, EAT_ERR_INVALID_ARG, "null handle");
+  if (((uintptr_t)sign & 3) != 0)
+    return fail(h, EAT_ERR_INVALID_ARG, "sign must be 4-byte aligned");
+  h->ppl_sign_src = sign;
   return EAT_OK;
 }
 
@@ -740,6 +791,17 @@ eat_status eat_selftest_bounded_wait(int64_t limit_ns, uint32_t* status_out) {
   if (e != cudaSuccess) return fail(nullptr, EAT_ERR_CUDA, std::string("self-test: ") +
                                                               cudaGetErrorString(e));
   *status_out = v;
+  return EAT_OK;
+}
+
+eat_status eat_selftest_expire_wait(eat_handle* h, int64_t limit_ns, void* stream) {
+  if (!h) return fail(nullptr, EAT_ERR_INVALID_ARG, "null handle");
+  if (limit_ns < 1000 || limit_ns > 1000000000LL)
+    return fail(h, EAT_ERR_INVALID_ARG, "need 1 us <= limit_ns <= 1 s");
+  ++h->launches;
+  const cudaError_t e =
+      tc_selftest_bounded_wait((unsigned long long)limit_ns, h->status, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(h, e, "self-test launch");
   return EAT_OK;
 }
 

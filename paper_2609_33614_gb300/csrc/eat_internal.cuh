@@ -85,6 +85,10 @@ struct RouteParams {
   const float* opd_scale;  // [E] or nullptr
   const float* tau_in;     // [T] previous tau_final per token stream (temporal smoothing) or null
   float* tau_out;          // [T] tau_final written back (temporal smoothing, forward calls) or null
+  // device-side PPL sign (eat_ppl_update's output) read by the selection kernel instead of the
+  // host-side ppl_factor, or null; its factors
+  const int32_t* ppl_sign_dev;
+  float ppl_up, ppl_down;
 };
 
 // Partial router logits: part[s][t][e] = sum over the s-th slice of d of x[t,j] Wr[e,j], as an
@@ -155,10 +159,19 @@ int combine_col_blocks(int d);  // column segments per token row (norm partials 
 cudaError_t launch_combine(int y_bf16, const void* opart, int o_bf16, int n_split,
                            int split_stride_rows, const int32_t* slot_of, const float* w,
                            const void* sout, int s_bf16, int S, int T, int K, int d, void* y,
-                           float* nrm_part, cudaStream_t st);
+                           float* nrm_part, const unsigned int* status, cudaStream_t st);
+// status: the device status word (nonzero: an expert kernel of the call gave up on a bounded wait;
+// the update is then skipped); status_mirror: device address of a host-mapped copy of the word
+// that block 0 writes, or null.
 cudaError_t launch_account(const int32_t* offs, const float* perm_p, const float* nrm_part, int nb,
                            int E, double alpha, int64_t* N, double* P, double* C, int32_t* st_n,
-                           double* st_p, double* st_norm, long long* counters, cudaStream_t st);
+                           double* st_p, double* st_norm, long long* counters,
+                           const unsigned int* status, unsigned int* status_mirror,
+                           cudaStream_t st);
+
+// §3.3 perplexity of a window of token negative log-likelihoods and the sign of its change.
+cudaError_t launch_ppl_update(const float* nll, int n, double* state, int32_t* sign,
+                              cudaStream_t st);
 
 // Records msg as the text eat_last_error(NULL) returns on this thread (entry points without a
 // handle).

@@ -538,7 +538,12 @@ route_select_kernel(const float2* __restrict__ part, int n_split, const float* _
     const float prev = rp.tau_in[t];
     if (!isnan(prev)) second = prev;
   }
-  float tau_f = rp.kappa1 * (rp.ppl_factor * tau) + rp.kappa2 * second;
+  float ppl_f = rp.ppl_factor;
+  if (rp.ppl_sign_dev) {  // the sign eat_ppl_update wrote on the device (read after the wait)
+    const int sg = __ldcg(rp.ppl_sign_dev);
+    ppl_f = sg > 0 ? rp.ppl_up : (sg < 0 ? rp.ppl_down : 1.0f);
+  }
+  float tau_f = rp.kappa1 * (ppl_f * tau) + rp.kappa2 * second;
 
   if (rp.clamp) {
     // order statistics of p (ascending, ties by index; padding lanes sort last)

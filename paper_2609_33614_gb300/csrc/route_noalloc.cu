@@ -7,28 +7,62 @@
 // or a host framework whose rules route every device allocation through its own allocator.  They
 // cannot create an eat_handle (eat_create allocates the accounts and the workspace).  This entry
 // point takes every input and output from the caller and keeps its only scratch -- the partial
-// router scores -- in a fixed array compiled into the library below.
+// router scores, as compensated fp32 pairs -- in a fixed array compiled into the library below.
 #include "eat_internal.cuh"
+
+#include <cuda.h>
+#include <cudaTypedefs.h>
 
 #include <mutex>
 #include <string>
 
 namespace {
 
-// Scratch of the partial router scores, [split][T][E] fp32 pairs (8 bytes each).  Every GPU that loads the library
-// holds these 1 MiB until the process exits.  Calls share the array and it keeps the previous
-// call's contents; nothing in it needs to start at zero (the scores kernel writes every entry it
-// later reads).  Two calls that overlap on the GPU (different streams, or threads) race on it.
+// Scratch of the partial router scores: [split][T][E] compensated fp32 pairs (hi, lo) of 8 bytes
+// each, 131072 pairs in all.  Every GPU that loads the library holds these 1 MiB until the process
+// exits.  Calls share the array and it keeps the previous call's contents; nothing in it needs to
+// start at zero (the scores kernel writes every entry it later reads).  Two calls that overlap on
+// the GPU (different streams, or threads) race on it.
 constexpr size_t kScratchScores = EAT_NOALLOC_SCRATCH_BYTES / sizeof(float2);
 static __device__ __align__(256) float2 g_route_scratch[kScratchScores];
 
 constexpr int kMaxDevices = 64;
 std::mutex g_mu;
-void* g_scratch_ptr[kMaxDevices] = {};
+// Per device: the scratch's device address and the unique id of the context it was looked up in.
+struct Cached {
+  unsigned long long ctx_id = 0;
+  void* ptr = nullptr;
+};
+Cached g_scratch[kMaxDevices];
 
-// Device address of the scratch on the current device, looked up once per device.  In host code
+// Unique id of the context current on this thread (driver entry points fetched through the
+// runtime, so the library needs no link against the driver library); false if there is none or
+// the driver cannot tell.
+bool current_context_id(unsigned long long* id) {
+  static PFN_cuCtxGetCurrent_v4000 get_cur = nullptr;
+  static PFN_cuCtxGetId_v12000 get_id = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 4000, cudaEnableDefault, &q) ==
+            cudaSuccess && q == cudaDriverEntryPointSuccess)
+      get_cur = (PFN_cuCtxGetCurrent_v4000)p;
+    p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess && q == cudaDriverEntryPointSuccess)
+      get_id = (PFN_cuCtxGetId_v12000)p;
+  });
+  CUcontext c = nullptr;
+  if (!get_cur || !get_id || get_cur(&c) != CUDA_SUCCESS || !c) return false;
+  return get_id(c, id) == CUDA_SUCCESS;
+}
+
+// Device address of the scratch in the current device's current context.  In host code
 // g_route_scratch names a host-side stand-in, not device memory, so only this address may be
-// handed to a kernel.
+// handed to a kernel.  It is looked up once per device, with that device current, and again
+// whenever the device's current context is another one than at the last look-up (after
+// cudaDeviceReset the module is loaded anew and the array may move).
 eat_status scratch_address(float2** out) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -41,17 +75,23 @@ eat_status scratch_address(float2** out) {
     return EAT_ERR_UNSUPPORTED;
   }
   std::lock_guard<std::mutex> lock(g_mu);
-  if (!g_scratch_ptr[dev]) {
-    void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_route_scratch);
-    if (e != cudaSuccess || !p) {
-      eat::set_thread_error((std::string("cudaGetSymbolAddress of the routing scratch: ") +
-                             cudaGetErrorString(e)).c_str());
-      return EAT_ERR_CUDA;
-    }
-    g_scratch_ptr[dev] = p;
+  unsigned long long id = 0;
+  if (g_scratch[dev].ptr && current_context_id(&id) && id == g_scratch[dev].ctx_id) {
+    *out = (float2*)g_scratch[dev].ptr;
+    return EAT_OK;
   }
-  *out = (float2*)g_scratch_ptr[dev];
+  void* p = nullptr;
+  e = cudaGetSymbolAddress(&p, g_route_scratch);
+  if (e != cudaSuccess || !p) {
+    eat::set_thread_error((std::string("cudaGetSymbolAddress of the routing scratch: ") +
+                           cudaGetErrorString(e)).c_str());
+    return EAT_ERR_CUDA;
+  }
+  // the look-up made the device's primary context current if none was; a context the driver
+  // cannot identify is not cached (then every call looks the address up)
+  if (current_context_id(&id)) g_scratch[dev] = {id, p};
+  else g_scratch[dev] = {};
+  *out = (float2*)p;
   return EAT_OK;
 }
 
@@ -119,6 +159,9 @@ extern "C" eat_status eat_route_noalloc(const void* x, int32_t T, int32_t d_mode
   rp.opd_scale = nullptr;
   rp.tau_in = nullptr;
   rp.tau_out = nullptr;
+  rp.ppl_sign_dev = nullptr;
+  rp.ppl_up = (float)p.ppl_up;
+  rp.ppl_down = (float)p.ppl_down;
 
   cudaStream_t st = (cudaStream_t)stream;
   cudaError_t e = eat::launch_router_logits(x, xdtype == EAT_BF16, w_router, T, d_model,

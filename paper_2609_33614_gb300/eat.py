@@ -62,6 +62,9 @@ _SIGS = {
     "eat_route_noalloc": (c_i32, [c_vp, c_i32, c_i32, c_i32, c_i32, c_vp, c_vp, c_vp, c_vp, c_vp,
                                   ctypes.POINTER(eat_params), c_i32, c_vp, c_vp, c_vp, c_vp]),
     "eat_set_tau_state": (c_i32, [c_vp, c_vp]),
+    "eat_ppl_update": (c_i32, [c_vp, c_i32, c_vp, c_vp, c_vp]),
+    "eat_set_ppl_sign_source": (c_i32, [c_vp, c_vp]),
+    "eat_layer_policy": (c_i32, [c_i32, c_i32, ctypes.POINTER(eat_params)]),
     "eat_destroy": (c_i32, [c_vp]),
     "eat_get_accounts": (c_i32, [c_vp, c_vp, c_vp, c_vp, c_vp]),
     "eat_set_accounts": (c_i32, [c_vp, c_vp, c_vp, c_vp, c_vp]),
@@ -71,6 +74,7 @@ _SIGS = {
     "eat_profile_end": (c_i32, [c_vp, ctypes.POINTER(c_dbl), ctypes.POINTER(c_i64), c_i32]),
     "eat_ffn_backend": (c_i32, [c_vp]),
     "eat_selftest_bounded_wait": (c_i32, [c_i64, ctypes.POINTER(ctypes.c_uint32)]),
+    "eat_selftest_expire_wait": (c_i32, [c_vp, c_i64, c_vp]),
     "eat_last_error": (ctypes.c_char_p, [c_vp]),
     "eat_status_string": (ctypes.c_char_p, [c_i32]),
 }
@@ -165,23 +169,26 @@ def eat_set_tau_state(h, tau_state):
     _check(lib().eat_set_tau_state(h, _ptr(tau_state)), h)
 
 
-def ppl_sign(ppl_prev: float, ppl_curr: float) -> int:
-    """The sign eat_route / eat_moe_forward take for the §3.3 adjustment from two perplexities of
-    the model (e.g. exp of the mean token negative log-likelihood over the last two windows):
-    +1 if PPL rose, -1 otherwise; 0 when no previous value exists."""
-    if ppl_prev is None:
-        return 0
-    return 1 if ppl_curr - ppl_prev > 0 else -1
+def eat_ppl_update(nll, n, ppl_state, sign, stream=None):
+    """Perplexity of a window of token NLLs and the sign of its change (see include/eat.h)."""
+    _check(lib().eat_ppl_update(_ptr(nll), n, _ptr(ppl_state), _ptr(sign), _stream(stream)))
+
+
+def eat_set_ppl_sign_source(h, sign):
+    _check(lib().eat_set_ppl_sign_source(h, _ptr(sign)), h)
+
+
+def eat_layer_policy(layer: int, n_layers: int, params: eat_params) -> eat_params:
+    """The §5.2 layer-wise adjustment of ``params`` (in place, also returned)."""
+    _check(lib().eat_layer_policy(layer, n_layers, ctypes.byref(params)))
+    return params
 
 
 def layer_policy(layer: int, n_layers: int, max_k: int) -> dict:
-    """Per-layer EAT settings after §5.2 (lower layers tolerate far fewer experts, the top ~quarter
-    of the stack needs close to the full K): the lower three quarters route with at most
-    max(1, max_k // 3) experts and a doubled threshold floor, the upper layers use the defaults.
-    Returns eat_params overrides."""
-    if layer < (3 * n_layers) // 4:
-        return {"max_k": max(1, max_k // 3), "alpha1": 1.0}
-    return {"max_k": max_k}
+    """eat_layer_policy applied to the defaults with K = max_k, as eat_params overrides."""
+    p = eat_layer_policy(layer, n_layers, eat_default_params(max_k))
+    d = eat_default_params(max_k)
+    return {"max_k": p.max_k, **({"alpha1": p.alpha1} if p.alpha1 != d.alpha1 else {})}
 
 
 def eat_destroy(h):
@@ -228,6 +235,10 @@ def eat_selftest_bounded_wait(limit_ns: int) -> int:
     out = ctypes.c_uint32(0)
     _check(lib().eat_selftest_bounded_wait(limit_ns, ctypes.byref(out)))
     return out.value
+
+
+def eat_selftest_expire_wait(h, limit_ns: int, stream=None):
+    _check(lib().eat_selftest_expire_wait(h, limit_ns, _stream(stream)), h)
 
 
 # ------------------------------------------------------------------------------------------------

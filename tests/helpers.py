@@ -42,7 +42,8 @@ class LazyExperts:
     def __getitem__(self, e):
         e = int(e)
         if e not in self.cache:
-            self.cache[e] = np64(self.t[e])
+            # widened to float64 on the device (exact) and copied once
+            self.cache[e] = self.t[e].detach().to(torch.float64).cpu().numpy()
         return self.cache[e]
 
 

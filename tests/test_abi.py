@@ -99,6 +99,7 @@ def test_null_handle_calls(lib):
     out = ctypes.c_uint32(7)
     assert lib.eat_selftest_bounded_wait(10, ctypes.byref(out)) == eat.EAT_ERR_INVALID_ARG
     assert lib.eat_selftest_bounded_wait(10**6, None) == eat.EAT_ERR_INVALID_ARG
+    assert lib.eat_selftest_expire_wait(None, 10**6, None) == eat.EAT_ERR_INVALID_ARG
 
 
 def test_binding_raises_with_message(lib):
@@ -106,3 +107,26 @@ def test_binding_raises_with_message(lib):
         eat._check(lib.eat_route(None, 1, 1, 0, 1, 1, 1, None))
     assert ei.value.status == eat.EAT_ERR_INVALID_ARG
     assert "null handle" in str(ei.value)
+
+
+def test_layer_policy_and_ppl_argument_checks(lib):
+    """eat_layer_policy is host arithmetic on the params (§5.2: the lower three quarters of a
+    stack sparser, the upper quarter unchanged); eat_ppl_update rejects bad arguments before any
+    launch."""
+    for n_layers, K in ((32, 2), (26, 6), (4, 8)):
+        for layer in range(n_layers):
+            p = eat.eat_layer_policy(layer, n_layers, eat.eat_default_params(K))
+            low = layer < (3 * n_layers) // 4
+            assert p.max_k == (max(1, K // 3) if low else K)
+            assert p.alpha1 == (1.0 if low else 0.5)
+            assert (p.beta, p.alpha2, p.kappa1) == (0.6, 1.0, 0.7)
+    p = eat.eat_default_params(2)
+    assert lib.eat_layer_policy(3, 3, ctypes.byref(p)) == eat.EAT_ERR_INVALID_ARG
+    assert lib.eat_layer_policy(-1, 3, ctypes.byref(p)) == eat.EAT_ERR_INVALID_ARG
+    assert lib.eat_layer_policy(0, 3, None) == eat.EAT_ERR_INVALID_ARG
+    assert lib.eat_ppl_update(None, 4, 64, 64, None) == eat.EAT_ERR_INVALID_ARG
+    assert lib.eat_ppl_update(64, 0, 64, 64, None) == eat.EAT_ERR_INVALID_ARG
+    assert b"n >= 1" in lib.eat_last_error(None)
+    assert lib.eat_ppl_update(64, 4, 68, 64, None) == eat.EAT_ERR_INVALID_ARG
+    assert lib.eat_set_ppl_sign_source(None, None) == eat.EAT_ERR_INVALID_ARG
+

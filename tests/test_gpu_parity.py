@@ -56,10 +56,12 @@ def _acc(layer):
 
 
 def run_parity(shape, lw, Ts, signs=None, prm_kw=None, layer=None, L=None, sample=None,
-               x_device="cpu", max_tokens=None, inputs=None, opd_scale=None, tau_state=None):
+               x_device="cpu", max_tokens=None, inputs=None, opd_scale=None, tau_state=None,
+               report=None):
     """Run len(Ts) steps and check each one.  sample: number of tokens whose outputs are checked
-    (None: all).  inputs: optional list of x tensors replacing the seeded draws.  Returns the
-    list of GPU outputs."""
+    (None: all).  inputs: optional list of x tensors replacing the seeded draws.  report: a label;
+    when given, each step's worst output error and near-tie count are printed.  Returns the list of
+    GPU outputs."""
     prm_kw = prm_kw or {}
     own = layer is None
     if own:
@@ -108,6 +110,9 @@ def run_parity(shape, lw, Ts, signs=None, prm_kw=None, layer=None, L=None, sampl
             norms_ref = None
         assert err.max() <= Y_TOL[shape.xdtype], \
             f"step {step}: output rel err {err.max():.3g} (token {toks[int(err.argmax())]})"
+        if report is not None:
+            print(f"parity {shape.name} {report} step {step}: T={T} checked {len(toks)} rows, "
+                  f"max rel err {err.max():.3g}, near-tie tokens {len(amb)}")
         par.check_accounts(acc0, (N1, P1, C1), (n_e, s_p, s_n), routing, sel, norms_ref,
                            prm.alpha, C_TOL[shape.xdtype])
         outs.append(y)
@@ -549,6 +554,47 @@ def test_reversed_ppl_factors():
     run_parity(MIX_S, lw, [64] * 4, signs=[1, -1, 1, 1], prm_kw={"ppl_up": 0.8, "ppl_down": 1.1})
 
 
+def test_ppl_feed_on_device():
+    """§3.3 fed from token likelihoods on the device: eat_ppl_update turns each window's NLLs into
+    the perplexity and the sign of its change (against the oracle: the hand-worked windows of the
+    golden example W6, then random windows), and a handle attached to that sign routes exactly as
+    the same handle given the oracle's sign on the host."""
+    import json
+    import math
+    import os
+    gold = json.load(open(os.path.join(os.path.dirname(__file__), "golden",
+                                       "worked_examples.json")))["W6"]["windows"]
+    g = torch.Generator().manual_seed(5)
+    windows = [w["nll"] for w in gold] + \
+        [(torch.rand(n, generator=g) * 4).tolist() for n in (1, 7, 300, 5000)]
+    state = torch.full((1,), float("nan"), dtype=torch.float64, device="cuda")
+    sign = torch.zeros(1, dtype=torch.int32, device="cuda")
+    lw = W.make_layer(MIX_S)
+    a = eat.EatLayer.from_workload(lw, 64, gpu_params(MIX_S))
+    b = eat.EatLayer.from_workload(lw, 64, gpu_params(MIX_S))
+    eat.eat_set_ppl_sign_source(a.h, sign)
+    prev = float("nan")
+    for i, win in enumerate(windows):
+        nll = torch.tensor(win, dtype=torch.float32)
+        eat.eat_ppl_update(nll.cuda(), len(win), state, sign)
+        x = W.make_tokens(MIX_S, 64, step=i).cuda()
+        ya = a.forward(x, 0)  # the sign comes from the device
+        torch.cuda.synchronize()
+        ref_sign, curr = orc.ppl_sign_update(prev, nll.double().numpy())
+        if i < len(gold):
+            assert ref_sign == gold[i]["sign"]
+        assert int(sign.item()) == ref_sign, f"window {i}"
+        assert math.isclose(float(state.item()), curr, rel_tol=1e-13)
+        yb = b.forward(x, ref_sign)
+        assert torch.equal(ya, yb)
+        prev = curr
+    for u, v in zip(a.accounts(), b.accounts()):
+        assert torch.equal(u, v)
+    eat.eat_set_ppl_sign_source(a.h, None)
+    a.close()
+    b.close()
+
+
 def test_layer_policy_stack():
     """Per-layer parameters on a stack (§5.2: lower layers sparser, upper layers up to full K)."""
     from paper_2609_33614_gb300.eat import layer_policy
@@ -576,6 +622,55 @@ def test_bounded_wait_expires_and_context_survives():
     layer = eat.EatLayer.from_workload(lw, 16, gpu_params(MIX_S))
     layer.forward(W.make_tokens(MIX_S, 16).cuda(), 0)
     assert eat.eat_get_counters(layer.h)["status"] == 0
+    layer.close()
+
+
+def test_expired_wait_leaves_accounts_and_fails_later_calls():
+    """A wait that runs out on the handle's status word (the 20 ms bounded wait an expert kernel
+    uses, on a barrier nothing arrives on): the next layer call writes NaN rows and leaves N,
+    P_total and C_s unchanged; every later call returns EAT_ERR_STATE (the host-buffer call too)
+    until eat_reset_accounts, after which the handle follows the oracle again.  No fault, trap or
+    hang is involved."""
+    lw = W.make_layer(MIX_S)
+    layer = eat.EatLayer.from_workload(lw, 32, gpu_params(MIX_S))
+    for s in range(2):
+        layer.forward(W.make_tokens(MIX_S, 32, step=s).cuda(), 0)
+    torch.cuda.synchronize()
+    acc0 = [t.clone() for t in layer.accounts()]
+    c0 = eat.eat_get_counters(layer.h)
+    eat.eat_selftest_expire_wait(layer.h, 20_000_000)
+    x = W.make_tokens(MIX_S, 32, step=5).cuda()
+    y = layer.forward(x, 0)  # enqueued behind the expiring wait: accepted, then invalid
+    torch.cuda.synchronize()
+    assert torch.isnan(y.float()).all()
+    for u, v in zip(acc0, layer.accounts()):
+        assert torch.equal(u, v)
+    c1 = eat.eat_get_counters(layer.h)
+    assert c1["status"] == 64 and c1["calls"] == c0["calls"]
+    idx = torch.empty(32, MIX_S.max_k, dtype=torch.int32, device="cuda")
+    w = torch.empty(32, MIX_S.max_k, dtype=torch.float32, device="cuda")
+    k = torch.empty(32, dtype=torch.int32, device="cuda")
+    xh = x.cpu().pin_memory()
+    yh = torch.empty_like(xh).pin_memory()
+    for call in (lambda: layer.forward(x, 0), lambda: eat.eat_route(layer.h, x, 32, 0, idx, w, k),
+                 lambda: eat.eat_moe_forward_host(layer.h, xh, 32, 0, yh),
+                 lambda: eat.eat_moe_forward_host_async(layer.h, xh, 32, 0, yh)):
+        with pytest.raises(eat.EatError) as ei:
+            call()
+        assert ei.value.status == eat.EAT_ERR_STATE
+        assert "bounded wait" in str(ei.value)
+    for u, v in zip(acc0, layer.accounts()):
+        assert torch.equal(u, v)
+    layer.reset()
+    assert eat.eat_get_counters(layer.h)["status"] == 0
+    run_parity(MIX_S, lw, [32, 7], layer=layer)
+    # a host-buffer call that is itself the failing call reports it after its synchronisation
+    eat.eat_selftest_expire_wait(layer.h, 20_000_000)
+    with pytest.raises(eat.EatError) as ei:
+        eat.eat_moe_forward_host(layer.h, xh, 32, 0, yh)
+    assert ei.value.status == eat.EAT_ERR_STATE
+    assert torch.isnan(yh.float()).all()
+    layer.reset()
     layer.close()
 
 
@@ -612,7 +707,10 @@ def test_forward_replays_as_cuda_graph(shape):
     b.close()
 
 
-# ------------------------------------------------------------------ full-size layers (sampled)
+# ------------------------------------------------------------------ full-size layers, every token
+# Every output row and every account of the call is checked against the oracle at the
+# configurations' own sizes (C_s against the oracle's own norms as well as the update rule); the
+# worst output error of each configuration is printed.
 def _big(shape, layer_id=0):
     return W.make_layer(shape, layer_id, device="cuda")
 
@@ -623,7 +721,7 @@ def test_full_mixtral_decode_batches():
     L = oracle_layer_lazy(lw)
     for B in (1, 16, 64):
         layer = eat.EatLayer.from_workload(lw, 64, gpu_params(W.MIXTRAL))
-        run_parity(W.MIXTRAL, lw, [B] * 3, layer=layer, L=L, sample=8, x_device="cuda")
+        run_parity(W.MIXTRAL, lw, [B] * 3, layer=layer, L=L, x_device="cuda", report=f"B{B}")
         layer.close()
 
 
@@ -634,7 +732,7 @@ def test_full_mixtral_decode_fp8():
     L = oracle_layer_lazy(dq)
     for B in (1, 16, 64):
         layer = eat.EatLayer.from_workload(lw8, 64, gpu_params(W.MIXTRAL))
-        run_parity(W.MIXTRAL, dq, [B] * 2, layer=layer, L=L, sample=8, x_device="cuda")
+        run_parity(W.MIXTRAL, dq, [B] * 2, layer=layer, L=L, x_device="cuda", report=f"fp8 B{B}")
         layer.close()
 
 
@@ -642,7 +740,7 @@ def test_full_olmoe_prefill_then_decode():
     lw = _big(W.OLMOE)
     L = oracle_layer_lazy(lw)
     layer = eat.EatLayer.from_workload(lw, 4096, gpu_params(W.OLMOE))
-    run_parity(W.OLMOE, lw, [4096, 32, 32], layer=layer, L=L, sample=12, x_device="cuda")
+    run_parity(W.OLMOE, lw, [4096, 32, 32], layer=layer, L=L, x_device="cuda", report="")
     layer.close()
 
 
@@ -650,13 +748,39 @@ def test_full_qwen_prefill():
     lw = _big(W.QWEN)
     L = oracle_layer_lazy(lw)
     layer = eat.EatLayer.from_workload(lw, 8192, gpu_params(W.QWEN))
-    run_parity(W.QWEN, lw, [8192], layer=layer, L=L, sample=8, x_device="cuda")
+    run_parity(W.QWEN, lw, [8192, 64], layer=layer, L=L, x_device="cuda", report="")
     layer.close()
 
 
-def test_full_dsv2l_layer_prefill_then_decode():
-    lw = _big(W.DSV2L, 25)
+@pytest.mark.parametrize("layer_id", [0, 12, 25])
+def test_full_dsv2l_layer_prefill_then_decode(layer_id):
+    """One DeepSeek-V2-Lite-shaped layer at full width: prefill of 16384 tokens, then a decode
+    call of 128 routed by the accounts the prefill left.  Layer 0 has the flattest routing (bias
+    scale 0.2: the most near-ties), layer 25 the most skewed (1.0)."""
+    lw = _big(W.DSV2L, layer_id)
     L = oracle_layer_lazy(lw)
     layer = eat.EatLayer.from_workload(lw, 16384, gpu_params(W.DSV2L))
-    run_parity(W.DSV2L, lw, [16384, 128], layer=layer, L=L, sample=8, x_device="cuda")
+    run_parity(W.DSV2L, lw, [16384, 128], layer=layer, L=L, x_device="cuda",
+               report=f"layer {layer_id}")
     layer.close()
+
+
+def test_full_dsv2l_decode_stack_26_layers():
+    """The 26-layer DeepSeek-V2-Lite-shaped stack in decode at batch 128, two steps, through the
+    pre-norm residual chain the benchmark runs (reading R13): layer l reads h_l = RMSNorm(x_l)
+    and x_{l+1} = x_l + y_l, with every layer's own accounts.  Each layer is checked on every
+    token from the GPU's own h_l (teacher forcing).  Layer-major order: step s of layer l needs
+    only layer l's earlier steps and layer l - 1's output of step s."""
+    B, steps = 128, 2
+    xs = [W.make_tokens(W.DSV2L, B, step=s, device="cuda") for s in range(steps)]
+    for l in range(W.DSV2L.n_layers):
+        lw = _big(W.DSV2L, l)
+        L = oracle_layer_lazy(lw)
+        layer = eat.EatLayer.from_workload(lw, B, gpu_params(W.DSV2L))
+        hs = [torch.nn.functional.rms_norm(x, (W.DSV2L.d_model,), eps=1e-6) for x in xs]
+        outs = run_parity(W.DSV2L, lw, [B] * steps, layer=layer, L=L, inputs=hs,
+                          report=f"stack layer {l}")
+        layer.close()
+        xs = [x + y for x, y in zip(xs, outs)]
+        del lw, L
+    assert all(bool(torch.isfinite(x.float()).all()) for x in xs)
