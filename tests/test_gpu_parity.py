@@ -386,6 +386,16 @@ def test_many_short_gate_up_units(fp8):
         run_parity(sh, lw, [16, 64, 100, 1, 37])
 
 
+@pytest.mark.parametrize("d,F,E,K", [(1024, 320, 64, 8), (2048, 192, 16, 4), (512, 4096, 8, 2)])
+def test_decode_calls_ragged_shapes(d, F, E, K):
+    """Decode-sized calls (1 to 32 tokens: token tiles of 16 and 32, split-K down projections)
+    on layers with ragged feature tiles (d_ff 320, 192), odd down k-block counts and many feature
+    tiles per expert (d_ff 4096), with PPL signs of both kinds."""
+    sh = W.scaled(W.OLMOE, f"fused-{d}-{F}", d_model=d, n_experts=E, d_ff=F, max_k=K)
+    lw = W.make_layer(sh)
+    run_parity(sh, lw, [32, 1, 7, 16, 32, 25], signs=[0, 1, -1, 0, 1, -1])
+
+
 def test_partial_feature_tiles():
     """d = 320 and d_ff = 192: feature tiles of 128 end half-full in both expert GEMMs."""
     sh = W.scaled(W.QWEN, "ragged-d", d_model=320, n_experts=16, d_ff=192, n_shared=1,
