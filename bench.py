@@ -479,6 +479,10 @@ def run_ours(args, world, rank, local, workload, clk, soak_s=1.0, with_cpu_basel
     yh = {B: torch.empty(B, shape.d_model, dtype=shape.xdtype).pin_memory() for B in batches}
 
     xd = {B: torch.empty(B, shape.d_model, dtype=shape.xdtype, device=dev) for B in batches}
+    for B in batches:  # every pinned input has been copied once before the timed steps
+        for x in xh[B]:
+            xd[B].copy_(x, non_blocking=True)
+    torch.cuda.synchronize()
 
     def step_host(s):
         # every call copies its x in and its y out inside the step; the step ends when the host
@@ -562,10 +566,10 @@ def run_ours(args, world, rank, local, workload, clk, soak_s=1.0, with_cpu_basel
     if prefill_states is not None:
         result["prefill_states"] = prefill_states
     if rank == 0 and world == 1 and with_cpu_baseline and not args.no_cpu_baseline:
-        result["cpu_baseline"] = oracle_sample(workload, layer_w[0], handles[0][0],
-                                               min_seconds=10.0)
-        result["cpu_baseline"]["single_thread"] = oracle_sample_single_thread(
-            workload, layer_w[0], handles[0][0], min_seconds=5.0)
+        # the oracle runs after every GPU measurement of the process (its BLAS threads would
+        # compete with the host thread that issues the end-to-end copies): keep what it needs
+        N, P, C = handles[0][0].accounts()
+        result["_oracle_inputs"] = (workload, layer_w[0], (N.cpu(), P.cpu(), C.cpu()))
     for row in handles:
         for h in row:
             h.close()
@@ -586,11 +590,12 @@ def _oracle_layer(lw):
                      f(lw.ws_gate), f(lw.ws_up), f(lw.ws_down))
 
 
-def oracle_sample(workload, lw, handle=None, min_seconds=10.0, max_steps=None, batches=None):
+def oracle_sample(workload, lw, accounts=None, min_seconds=10.0, max_steps=None, batches=None):
     """Time the fp64 oracle, as it stands, on a bounded sample of the workload: successive layer
     calls cycling through the workload's batch sizes (prefill workloads: the first 256 tokens of
-    the prefill batch), from the GPU handle's current accounts if given, until min_seconds of CPU
-    time have run (or max_steps calls)."""
+    the prefill batch), from the given accounts (N, P, C tensors, e.g. a GPU handle's after its
+    timed steps) or the empty history, until min_seconds of CPU time have run (or max_steps
+    calls)."""
     import numpy as np
     import torch
     import oracle.eat_oracle as orc
@@ -601,9 +606,8 @@ def oracle_sample(workload, lw, handle=None, min_seconds=10.0, max_steps=None, b
     bs = batches or [min(B, 256) for B in spec["batches"]]
     L = _oracle_layer(lw)
     prm = orc.Params(max_k=shape.max_k, temperature=shape.temperature)
-    if handle is not None:
-        N, P, C = handle.accounts()
-        acc = orc.Accounts(N.cpu().numpy(), P.cpu().numpy(), C.cpu().numpy())
+    if accounts is not None:
+        acc = orc.Accounts(*(t.cpu().numpy() for t in accounts))
     else:
         acc = orc.Accounts.zeros(shape.n_experts)
     toks, calls, el = 0, 0, 0.0
@@ -651,14 +655,14 @@ def _blas_thread_setter():
     return None
 
 
-def oracle_sample_single_thread(workload, lw, handle=None, min_seconds=5.0):
+def oracle_sample_single_thread(workload, lw, accounts=None, min_seconds=5.0):
     """The same oracle sample with its BLAS library limited to one thread (restored after)."""
     setter = _blas_thread_setter()
     if setter is None:
         return {"unavailable": "no openblas_set_num_threads in the BLAS library numpy loaded"}
     setter(1)
     try:
-        r = oracle_sample(workload, lw, handle, min_seconds=min_seconds)
+        r = oracle_sample(workload, lw, accounts, min_seconds=min_seconds)
     finally:
         setter(int(os.environ["OPENBLAS_NUM_THREADS"]))
     r["cores"] = 1
@@ -745,6 +749,13 @@ def main(argv=None):
                 pre.pop("n_gpus")
                 pre["workload"] = "olmoe-prefill"
                 res["prefill"] = pre
+            ctx = res.pop("_oracle_inputs", None)
+            if ctx is not None:
+                wl, lw, acc = ctx
+                res["cpu_baseline"] = oracle_sample(wl, lw, acc, min_seconds=10.0)
+                res["cpu_baseline"]["single_thread"] = oracle_sample_single_thread(
+                    wl, lw, acc, min_seconds=5.0)
+                del lw
         res = {"metric": METRIC, **res, "higher_is_better": True, "scaling": "weak",
                "vs_baseline": None,
                "data": "synthetic (seeded N(0,1) hidden states, N(0,0.02^2) weights" +
