@@ -462,6 +462,13 @@ def run_ours(args, world, rank, local, workload, clk, soak_s=1.0, with_cpu_basel
                     k["bytes"] += n * kernel_bytes(kind, shape, dU / max(1, dC), dA / max(1, dC), B,
                                                    fp8=bool(spec.get("fp8")))
                     k["flops"] += n * kernel_flops(kind, shape, dA / max(1, dC), B)
+                    folded = shape.n_shared and prof[l][bi]["shared_up"][1] == 0
+                    if folded and kind in ("ffn_up", "ffn_down"):
+                        # large calls run the shared experts inside the routed launches
+                        sk = "shared_up" if kind == "ffn_up" else "shared_down"
+                        k["bytes"] += n * kernel_bytes(sk, shape, 0, 0, B,
+                                                       fp8=bool(spec.get("fp8")))
+                        k["flops"] += n * kernel_flops(sk, shape, 0, B)
     total_kernel_ms = sum(k["ms"] for k in kinds.values())
     dom = max((k for k in kinds if k.startswith("ffn") or k.startswith("shared")),
               key=lambda k: kinds[k]["ms"])

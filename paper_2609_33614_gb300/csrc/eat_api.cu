@@ -275,6 +275,8 @@ eat_status run_forward(eat_handle* h, const void* x, int T, int ppl_sign, void* 
   c.sout = h->sout;
   c.status = h->status;
   const bool side = shared_on_side_stream(h, T, tile_rows);
+  // large calls on SM pairs: the shared experts' units follow the routed ones in the same launches
+  c.fold_shared = !side && h->backend == 1 && tc_folds_shared(h->tc, T);
   if (side) {
     // fork: the side stream starts after everything enqueued on st so far (x written, the
     // previous call's combine done with the shared outputs)
@@ -322,7 +324,7 @@ eat_status run_forward(eat_handle* h, const void* x, int T, int ppl_sign, void* 
   if (side) {
     const cudaError_t e = cudaStreamWaitEvent(st, h->ev_join, 0);  // join before the combine
     if (e != cudaSuccess) return cuda_fail(h, e, "shared-expert stream join");
-  } else if (h->S > 0) {
+  } else if (h->S > 0 && !c.fold_shared) {
     EAT_TRY(run_shared(h, c, x, T, st));
   }
   EAT_TRY(launch(h, kCombine, st, "combine", [&] {

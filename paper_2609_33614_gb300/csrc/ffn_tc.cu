@@ -789,10 +789,15 @@ __host__ __device__ constexpr uint32_t idesc_bf16_pair(int n) {
 // MMA width of a pair unit: token rows rounded up to 32 (16 per CTA), at most 256.
 __device__ __forceinline__ int pair_n(int nrows) { return min(kPairBN, (nrows + 31) & ~31); }
 
-template <int MODE>
+// With FOLD a launch carries two unit sets: the routed experts (args, mapA0/A1/B) and, after them,
+// the always-on shared experts of the same call (args_s, mapA0s/A1s/Bs), so a large call's
+// projection pays one ramp and one tail for both.  Without FOLD the second set is ignored.
+template <int MODE, bool FOLD>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg<MODE>::kThreads, 1)
 tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__ CUtensorMap mapA1,
-               const __grid_constant__ CUtensorMap mapB, const TcArgs args) {
+               const __grid_constant__ CUtensorMap mapB, const TcArgs args,
+               const __grid_constant__ CUtensorMap mapA0s, const __grid_constant__ CUtensorMap mapA1s,
+               const __grid_constant__ CUtensorMap mapBs, const TcArgs args_s) {
   using C = PairCfg<MODE>;
   constexpr bool IL = C::kIL;
   constexpr int S = C::kStages;
@@ -829,6 +834,10 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
   if (threadIdx.x == 32) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(&mapA0) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(&mapB) : "memory");
+    if (FOLD) {
+      asm volatile("prefetch.tensormap [%0];" ::"l"(&mapA0s) : "memory");
+      asm volatile("prefetch.tensormap [%0];" ::"l"(&mapBs) : "memory");
+    }
   }
   tc_fence_before();
   cluster_sync_all();  // both CTAs' barriers exist before either signals the other
@@ -841,7 +850,20 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
   const int total_tiles = args.tile_offs
                               ? args.tile_offs[args.n_groups]
                               : args.n_groups * ((args.uniform_rows + kPairBN - 1) / kPairBN);
-  const int units = total_tiles * args.m_tiles * args.n_split;
+  const int units_r = total_tiles * args.m_tiles * args.n_split;
+  const int units = units_r + (FOLD ? args_s.n_groups *
+                                            ((args_s.uniform_rows + kPairBN - 1) / kPairBN) *
+                                            args_s.m_tiles * args_s.n_split
+                                      : 0);
+  // unit u of the launch: the routed set first, then the shared one (true)
+  auto unit_at = [&](int u, Unit& w) -> bool {
+    if (!FOLD || u < units_r) {
+      w = decode_unit<kPairBN>(args, u, Offs{args.row_offs, args.tile_offs});
+      return false;
+    }
+    w = decode_unit<kPairBN>(args_s, u - units_r, Offs{nullptr, nullptr});
+    return true;
+  };
   const uint32_t full0 = map_rank(smem_u32(full), 0);      // rank 0's full[0]
   const uint32_t tempty0 = map_rank(smem_u32(tempty), 0);  // rank 0's tempty[0]
 
@@ -853,10 +875,16 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
       long long issued = 0;
       bool ok = true;
       for (int u = pair; u < units && ok; u += n_pairs) {
-        const Unit w = decode_unit<kPairBN>(args, u, Offs{args.row_offs, args.tile_offs});
+        Unit w;
+        const bool sh = unit_at(u, w);
+        const CUtensorMap* mA0 = sh ? &mapA0s : &mapA0;
+        const CUtensorMap* mA1 = sh ? &mapA1s : &mapA1;
+        const CUtensorMap* mB = sh ? &mapBs : &mapB;
         const int n = pair_n(w.nrows);
-        const int a_row = w.g * args.a_rows_per_group + w.m0 + (int)rank * C::kFeat;
-        const int b_row = w.slot0 - w.g * args.b_shift_per_group + (int)rank * (n / 2);
+        const int a_rows = sh ? args_s.a_rows_per_group : args.a_rows_per_group;
+        const int b_shift = sh ? args_s.b_shift_per_group : args.b_shift_per_group;
+        const int a_row = w.g * a_rows + w.m0 + (int)rank * C::kFeat;
+        const int b_row = w.slot0 - w.g * b_shift + (int)rank * (n / 2);
         for (int kb = w.kb0; kb < w.kb1; kb += C::kKPS) {
           const int nk = min(C::kKPS, w.kb1 - kb);  // k-blocks of this stage
           if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, args.err, 1u, true)) {
@@ -872,12 +900,12 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
               uint8_t* sj = st + j * C::kSubBytes;
               const int kx = (kb + j) * kBK;
               if (IL) {
-                tma_load_2d_pair(sj, &mapA0, fb, kx, a_row);
-                tma_load_2d_pair(sj + C::kABytes / 2, &mapA1, fb, kx, a_row);
+                tma_load_2d_pair(sj, mA0, fb, kx, a_row);
+                tma_load_2d_pair(sj + C::kABytes / 2, mA1, fb, kx, a_row);
               } else {
-                tma_load_2d_pair(sj, &mapA0, fb, kx, a_row);
+                tma_load_2d_pair(sj, mA0, fb, kx, a_row);
               }
-              tma_load_2d_pair(sj + C::kABytes, &mapB, fb, kx, b_row);
+              tma_load_2d_pair(sj + C::kABytes, mB, fb, kx, b_row);
             }
           }
           ++issued;
@@ -902,7 +930,8 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
       int local = 0;
       bool ok = true;
       for (int u = pair; u < units && ok; u += n_pairs, ++local) {
-        const Unit w = decode_unit<kPairBN>(args, u, Offs{args.row_offs, args.tile_offs});
+        Unit w;
+        unit_at(u, w);
         const int buf = local & 1;
         const uint32_t tph = (uint32_t)((local >> 1) & 1);
         if (!mbar_wait(&tempty[buf], tph ^ 1u, abort_flag, args.err, 4u, true)) {
@@ -959,7 +988,12 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
     long long chunk = 0;
     bool ok = true;
     for (int u = pair; u < units && ok; u += n_pairs, ++local) {
-      const Unit w = decode_unit<kPairBN>(args, u, Offs{args.row_offs, args.tile_offs});
+      Unit w;
+      // the unit set's output and width as scalars (a reference to either parameter struct
+      // would let the stores below alias it and reload its fields every element)
+      const bool sh = unit_at(u, w);
+      __nv_bfloat16* const out = (__nv_bfloat16*)(sh ? args_s.out : args.out);
+      const int M = sh ? args_s.M : args.M;
       const int buf = local & 1;
       const uint32_t tph = (uint32_t)((local >> 1) & 1);
       if (!warp_wait(&tfull[buf], tph, abort_flag, args.err, 32u)) break;
@@ -967,7 +1001,7 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
       const uint32_t tbase =
           tmem_base + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * C::kAccCols);
       const int f = w.m0 + (int)rank * C::kFeat + 32 * half + lane;
-      const bool fok = f < args.M;
+      const bool fok = f < M;
       const int keep = is_gate ? 0 : 16;
       const int c_end = min(128 * ch + 128, w.nrows);
       for (int c0 = 128 * ch; c0 < c_end; c0 += 32, ++chunk) {
@@ -995,8 +1029,7 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
               const float o = theirs[j * 32 + lane];
               const float m = __uint_as_float(is_gate ? v0[j] : v1[j]);
               const float h = is_gate ? silu_f(m) * o : silu_f(o) * m;
-              ((__nv_bfloat16*)args.out)[(size_t)(w.slot0 + col) * args.M + f] =
-                  __float2bfloat16_rn(h);
+              out[(size_t)(w.slot0 + col) * M + f] = __float2bfloat16_rn(h);
             }
           }
         }
@@ -1016,7 +1049,12 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
     const int ch = (warp - 2) >> 2;
     int local = 0;
     for (int u = pair; u < units; u += n_pairs, ++local) {
-      const Unit w = decode_unit<kPairBN>(args, u, Offs{args.row_offs, args.tile_offs});
+      Unit w;
+      const bool sh = unit_at(u, w);  // (scalars, as in the gate/up epilogue)
+      void* const out = sh ? args_s.out : args.out;
+      const int M = sh ? args_s.M : args.M;
+      const int out_bf16 = sh ? args_s.out_bf16 : args.out_bf16;
+      const long long sstride = sh ? args_s.split_stride : args.split_stride;
       const int buf = local & 1;
       const uint32_t tph = (uint32_t)((local >> 1) & 1);
       if (!warp_wait(&tfull[buf], tph, abort_flag, args.err, 32u)) break;
@@ -1024,7 +1062,7 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
       const uint32_t tbase =
           tmem_base + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * C::kAccCols);
       const int f = w.m0 + (int)rank * C::kFeat + 32 * q + lane;
-      const bool fok = f < args.M;
+      const bool fok = f < M;
       const int c_end = min(128 * ch + 128, w.nrows);
       for (int c0 = 128 * ch; c0 < c_end; c0 += 16) {
         uint32_t g[16];
@@ -1035,12 +1073,10 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
           for (int c = 0; c < 16; ++c) {
             if (c0 + c < w.nrows) {
               const size_t slot = (size_t)(w.slot0 + c0 + c);
-              if (args.out_bf16)
-                ((__nv_bfloat16*)args.out)[slot * args.M + f] =
-                    __float2bfloat16_rn(__uint_as_float(g[c]));
+              if (out_bf16)
+                ((__nv_bfloat16*)out)[slot * M + f] = __float2bfloat16_rn(__uint_as_float(g[c]));
               else
-                ((float*)args.out)[(size_t)w.split * args.split_stride + slot * args.M + f] =
-                    __uint_as_float(g[c]);
+                ((float*)out)[(size_t)w.split * sstride + slot * M + f] = __uint_as_float(g[c]);
             }
           }
         }
@@ -1173,15 +1209,19 @@ cudaError_t launch_tc(const CUtensorMap& a0, const CUtensorMap& a1, const CUtens
 }
 
 // SM-pair kernels: one 2-CTA cluster per pair of SMs, at most as many pairs as can be resident.
-template <int MODE>
-cudaError_t launch_pair(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& b,
-                        const TcArgs& args, long long units, int num_sms, cudaStream_t st) {
+// The routed set (a0, a1, b, args) and, when sargs is given, the shared set of the same call in
+// the same launch; units counts both.
+template <int MODE, bool FOLD>
+cudaError_t launch_pair_t(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& b,
+                          const TcArgs& args, long long units, int num_sms, cudaStream_t st,
+                          const CUtensorMap* sa0, const CUtensorMap* sa1, const CUtensorMap* sb,
+                          const TcArgs* sargs) {
   using C = PairCfg<MODE>;
   static std::once_flag once;
   static cudaError_t attr_err = cudaSuccess;
   static int max_pairs = 0;
   std::call_once(once, [num_sms] {
-    attr_err = cudaFuncSetAttribute(tc_pair_kernel<MODE>,
+    attr_err = cudaFuncSetAttribute(tc_pair_kernel<MODE, FOLD>,
                                     cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
     if (attr_err != cudaSuccess) return;
     cudaLaunchConfig_t cfg = {};
@@ -1196,7 +1236,7 @@ cudaError_t launch_pair(const CUtensorMap& a0, const CUtensorMap& a1, const CUte
     cfg.attrs = at;
     cfg.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, tc_pair_kernel<MODE>, &cfg) != cudaSuccess || n <= 0) {
+    if (cudaOccupancyMaxActiveClusters(&n, tc_pair_kernel<MODE, FOLD>, &cfg) != cudaSuccess || n <= 0) {
       cudaGetLastError();
       n = num_sms / 2;
     }
@@ -1205,8 +1245,21 @@ cudaError_t launch_pair(const CUtensorMap& a0, const CUtensorMap& a1, const CUte
   if (attr_err != cudaSuccess) return attr_err;
   const long long pairs = std::min<long long>(max_pairs, units);
   if (pairs <= 0) return cudaSuccess;
-  return launch_pdl(tc_pair_kernel<MODE>, dim3((unsigned)(2 * pairs)), dim3(C::kThreads),
-                    C::kSmemBytes, st, a0, a1, b, args);
+  TcArgs none;
+  std::memset(&none, 0, sizeof(none));
+  return launch_pdl(tc_pair_kernel<MODE, FOLD>, dim3((unsigned)(2 * pairs)), dim3(C::kThreads),
+                    C::kSmemBytes, st, a0, a1, b, args, sa0 ? *sa0 : a0, sa1 ? *sa1 : a1,
+                    sb ? *sb : b, sargs ? *sargs : none);
+}
+template <int MODE>
+cudaError_t launch_pair(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& b,
+                        const TcArgs& args, long long units, int num_sms, cudaStream_t st,
+                        const CUtensorMap* sa0 = nullptr, const CUtensorMap* sa1 = nullptr,
+                        const CUtensorMap* sb = nullptr, const TcArgs* sargs = nullptr) {
+  if (sargs)
+    return launch_pair_t<MODE, true>(a0, a1, b, args, units, num_sms, st, sa0, sa1, sb, sargs);
+  return launch_pair_t<MODE, false>(a0, a1, b, args, units, num_sms, st, nullptr, nullptr,
+                                    nullptr, nullptr);
 }
 
 // Single-SM launches: token tiles of 16..128 rows (256-row tiles run on SM pairs); W8 for fp8
@@ -1252,6 +1305,10 @@ int tc_tile_rows(const TcLayer& L, int T) {
 // loses more to the warp's cp.async traffic than the separate gather costs.  fp8 layers always
 // read their B operand from the e4m3 planes that split_e4m3_kernel writes.
 bool tc_gathers_in_kernel(const TcLayer& L, int T) { return T <= 128 && !L.w8; }
+
+bool tc_folds_shared(const TcLayer& L, int T) {
+  return L.S > 0 && !L.w8 && tc_tile_rows(L, T) == kPairBN;
+}
 
 int tc_tile_rows_down(const TcLayer& L, int T) { return tc_tile_rows(L, T); }
 
@@ -1421,14 +1478,31 @@ cudaError_t tc_launch_up(const TcLayer& L, const TcCall& c, bool shared, cudaStr
                 : launch_up_bn<false>(bn, a0, a1, b, a, grid, st);
   };
   long long max_tiles;
+  // the shared experts' unit set: every token of the call in order, weight 1 (reading R9)
+  auto shared_args = [&](TcArgs& s) {
+    s = a;
+    s.M = L.Fs;
+    s.m_tiles = (s.M + s.m_tile - 1) / s.m_tile;
+    s.a_rows_per_group = s.M;
+    s.prefetch_a = 1;
+    if (L.w8) {
+      s.scale0 = L.ssg;
+      s.scale1 = L.ssu;
+      s.bscale = L.q.xqt_s;
+      s.b_lo_rows = L.Tmax;
+    }
+    s.n_groups = L.S;
+    s.row_offs = nullptr;
+    s.tile_offs = nullptr;
+    s.uniform_rows = c.T;
+    s.b_shift_per_group = c.T;
+    s.out = c.sact;
+  };
   if (shared) {
     CUtensorMap xm;
     if (L.w8) xm = m->xqt[bn_index(bn)];
     else if (!encode_2d(&xm, c.x, c.T, L.d, pair ? kPairRows : bn)) return cudaErrorInvalidValue;
-    a.n_groups = L.S;
-    a.uniform_rows = c.T;
-    a.b_shift_per_group = c.T;
-    a.out = c.sact;
+    shared_args(a);
     max_tiles = (long long)L.S * ((c.T + bn - 1) / bn);
     const long long units = max_tiles * a.m_tiles;
     if (pair)
@@ -1448,6 +1522,16 @@ cudaError_t tc_launch_up(const TcLayer& L, const TcCall& c, bool shared, cudaStr
     a.b_rows = c.perm_tok;
     a.bx = (const __nv_bfloat16*)c.x;
     return up_bn(m->wg, m->wu, m->wg, grid);
+  }
+  if (pair && c.fold_shared && L.S > 0) {  // the shared experts in the same launch
+    TcArgs sa;
+    shared_args(sa);
+    CUtensorMap xm;
+    if (!encode_2d(&xm, c.x, c.T, L.d, kPairRows)) return cudaErrorInvalidValue;
+    const long long s_units = (long long)L.S * ((c.T + bn - 1) / bn) * sa.m_tiles;
+    return launch_pair<kModeGateUpIL>(m->wg64, m->wu64, m->xperm[bn_index(kPairRows)], a,
+                                      units + s_units, L.num_sms, st, &m->wsg64, &m->wsu64, &xm,
+                                      &sa);
   }
   if (pair)
     return launch_pair<kModeGateUpIL>(m->wg64, m->wu64, m->xperm[bn_index(kPairRows)], a, units,
@@ -1482,12 +1566,28 @@ cudaError_t tc_launch_down(const TcLayer& L, const TcCall& c, bool shared, int n
                 : launch_down_bn<false>(bn, a0, b, a, grid, st);
   };
   long long max_tiles;
+  auto shared_args = [&](TcArgs& s) {
+    s = a;
+    s.kblocks = kblocks_of(L, L.Fs);
+    s.n_split = 1;
+    s.kb_per_split = s.kblocks;
+    if (L.w8) {
+      s.scale0 = L.ssd;
+      s.bscale = L.q.saq_s;
+      s.b_lo_rows = L.S * L.Tmax;
+    }
+    s.n_groups = L.S;
+    s.row_offs = nullptr;
+    s.tile_offs = nullptr;
+    s.uniform_rows = c.T;
+    s.out = c.sout;
+    s.out_bf16 = 1;
+    s.split_stride = 0;
+  };
   if (shared) {
-    a.n_groups = L.S;
-    a.uniform_rows = c.T;
-    a.out = c.sout;
-    a.out_bf16 = 1;
-    a.split_stride = 0;
+    shared_args(a);
+    a.n_split = n_split;
+    a.kb_per_split = (a.kblocks + n_split - 1) / n_split;
     max_tiles = (long long)L.S * ((c.T + bn - 1) / bn);
     const long long units = max_tiles * a.m_tiles;
     if (pair)
@@ -1504,6 +1604,14 @@ cudaError_t tc_launch_down(const TcLayer& L, const TcCall& c, bool shared, int n
   a.split_stride = (long long)c.T * L.K * L.d;
   max_tiles = (long long)(c.T * L.K + bn - 1) / bn + L.E;
   const long long units = max_tiles * a.m_tiles * n_split;
+  if (pair && c.fold_shared && L.S > 0) {  // the shared experts in the same launch
+    TcArgs sa;
+    shared_args(sa);
+    const long long s_units = (long long)L.S * ((c.T + bn - 1) / bn) * sa.m_tiles;
+    return launch_pair<kModeDown>(m->wd, m->wd, m->act[bn_index(kPairRows)], a, units + s_units,
+                                  L.num_sms, st, &m->wsd, &m->wsd,
+                                  &m->sact[bn_index(kPairRows)], &sa);
+  }
   if (pair)
     return launch_pair<kModeDown>(m->wd, m->wd, m->act[bn_index(kPairRows)], a, units, L.num_sms,
                                   st);

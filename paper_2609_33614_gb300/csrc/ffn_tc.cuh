@@ -48,6 +48,7 @@ struct TcCall {
   void* sact = nullptr;            // [S*T, Fs] bf16
   void* sout = nullptr;            // [S*T, d] bf16
   unsigned int* status = nullptr;  // device status word (bounded-wait failures)
+  bool fold_shared = false;        // the routed launches also run the shared experts (SM pairs)
 };
 
 // Device checks and the tensor-map encoder; 0 on success, *msg explains a failure.
@@ -59,6 +60,9 @@ void tc_destroy(TcLayer& L);
 int tc_tile_rows(const TcLayer& L, int T);       // gate/up token rows per tile, call of T tokens
 int tc_tile_rows_down(const TcLayer& L, int T);  // down-projection token rows per tile
 bool tc_gathers_in_kernel(const TcLayer& L, int T);  // gate/up gathers x rows itself (no Xperm)
+// A call of T tokens runs its shared experts inside the routed SM-pair launches (TcCall's
+// fold_shared): one unit set after the other, one ramp and one tail per projection.
+bool tc_folds_shared(const TcLayer& L, int T);
 int tc_down_split(const TcLayer& L, int T);  // split-K slices of the routed down projection
 long long tc_opart_rows(const TcLayer& L);   // rows of fp32 partials the workspace must hold
 cudaError_t tc_launch_gather(const TcLayer& L, const TcCall& c, cudaStream_t st);

@@ -160,6 +160,14 @@ def test_qwen_shaped_shared_experts():
     run_parity(QWEN_S, lw, [300, 17, 1])
 
 
+def test_shared_experts_in_the_routed_sm_pair_launches():
+    """Calls of 1024 tokens or more run the always-on shared experts' units after the routed ones
+    in the same SM-pair launches: full and ragged 256-token shared tiles (1024, 2100), shared
+    d_ff (192) unlike the routed one (128), then a small call on the single-SM kernels."""
+    lw = W.make_layer(QWEN_S)
+    run_parity(QWEN_S, lw, [1024, 2100, 40])
+
+
 def test_dsv2l_shaped_residual_chain():
     """Three layers, independent accounts, x_{l+1} = bf16(x_l + y_l) with the GPU's x_l."""
     T = 96
