@@ -783,6 +783,38 @@ def test_full_dsv2l_layer_prefill_then_decode(layer_id):
     layer.close()
 
 
+@pytest.mark.parametrize("mode,top_p", [("topk", None), ("topp", 0.4)])
+def test_full_olmoe_prefill_baseline_routers(mode, top_p):
+    """The §4.1 baseline routers at full size: OLMoE-shaped prefill of 4096 tokens (SM pairs) and a
+    decode call of 32, every token and account checked."""
+    kw = {"router_mode": eat.EAT_ROUTER_TOPK} if mode == "topk" else \
+        {"router_mode": eat.EAT_ROUTER_TOPP, "top_p": top_p}
+    lw = _big(W.OLMOE)
+    L = oracle_layer_lazy(lw)
+    layer = eat.EatLayer.from_workload(lw, 4096, gpu_params(W.OLMOE, **kw))
+    run_parity(W.OLMOE, lw, [4096, 32], layer=layer, L=L, x_device="cuda", prm_kw=kw,
+               report=mode)
+    layer.close()
+
+
+def test_temporal_smoothing_large_calls():
+    """EMA of tau_final over calls (temporal reading) with calls on the SM-pair path: 2048 token
+    streams, three calls with PPL signs of both kinds."""
+    lw = W.make_layer(OLMOE_S)
+    state = torch.full((2048,), float("nan"), device="cuda")
+    run_parity(OLMOE_S, lw, [2048, 2048, 1500], signs=[1, -1, 0], max_tokens=2048,
+               prm_kw={"smoothing_mode": eat.EAT_SMOOTH_TEMPORAL}, tau_state=state)
+
+
+def test_maximum_call_size():
+    """The largest call a handle takes (max_tokens = 65536) on a small layer with shared experts:
+    one 65536-token call on the SM pairs (routed and shared experts in the same launches, about
+    4400 token tiles), then a decode call routed by the accounts it left."""
+    sh = W.scaled(W.QWEN, "qwen-max", d_model=128, n_experts=60, d_ff=128, d_ff_shared=128)
+    lw = W.make_layer(sh)
+    run_parity(sh, lw, [65536, 8], max_tokens=65536)
+
+
 def test_full_dsv2l_decode_stack_26_layers():
     """The 26-layer DeepSeek-V2-Lite-shaped stack in decode at batch 128, two steps, through the
     pre-norm residual chain the benchmark runs (reading R13): layer l reads h_l = RMSNorm(x_l)
