@@ -7,16 +7,20 @@
 //      accumulates g_norm * o into y in the order j = 0..k_t-1, adds the always-on shared experts
 //      with weight 1, and writes the segment's sum of squares of every slot (||o||_2 of the
 //      unweighted expert output feeds C_s) to nrm_part[slot][segment].
-//  account_kernel: one block per expert.  Finishes ||o||_2 of each slot from its segment sums
-//      (fp32, fixed order), sums p and ||o||_2 over the expert's slots with compensated fp32
-//      additions (a fixed tree; about fp64 accuracy) and applies, in fp64 on one thread,
-//      N += n_e, P_total += sum p, C_s <- (1 - alpha) C_s + alpha * mean ||o||_2 when n_e > 0.
-//      Per-slot work stays off GB300's narrow fp64 pipe: an fp64 square root per slot made the
-//      block of a heavily used expert the longest of the step.
+//  account_kernel: blocks (e, c) over each expert's slots in chunks of 1024.  Finishes ||o||_2 of
+//      each slot from its segment sums (fp32, fixed order), sums p and ||o||_2 over the chunk with
+//      compensated fp32 additions (a fixed tree; about fp64 accuracy); an expert of one chunk is
+//      finished by its block, a larger one by the last of its blocks to arrive (a ticket per
+//      expert, reset by that block), which adds the chunks' compensated sums in chunk order.  The
+//      finishing block applies, in fp64 on one thread, N += n_e, P_total += sum p and
+//      C_s <- (1 - alpha) C_s + alpha * mean ||o||_2 when n_e > 0.  Per-slot work stays off
+//      GB300's narrow fp64 pipe, and no block walks more than one chunk: one block per expert
+//      left the most popular expert's block (~4000 slots at a 4096-token call) the longest of
+//      the step.
 //  Both read the device status word: when an earlier kernel of the call gave up on a bounded wait
 //  (its outputs are then invalid), the combine writes NaN rows and the account update leaves N,
 //  P_total and C_s as they were, so one expired wait cannot feed invalid norms into the accounts
-//  that every later call routes by.  Block 0 of the account kernel copies the word to a
+//  that every later call routes by.  The block that finishes expert 0 copies the word to a
 //  host-mapped mirror, which the entry points read without synchronising.
 #include "eat_internal.cuh"
 
@@ -27,6 +31,7 @@ namespace {
 constexpr int kCombThreads = 256;  // 8 warps: 8 (token, segment) tasks per block
 constexpr int kSegCols = 256;      // columns per warp task, 8 per lane
 constexpr int kAccThreads = 256;
+constexpr int kAccChunk = 4 * kAccThreads;  // slots of one account block
 
 // 8 consecutive values as fp32, from fp32 (two 16-byte loads) or bf16 (one 16-byte load).
 struct V8 {
@@ -196,18 +201,23 @@ account_kernel(const int32_t* __restrict__ offs, const float* __restrict__ perm_
                const float* __restrict__ nrm_part, int nb, double alpha, int64_t* __restrict__ N,
                double* __restrict__ P, double* __restrict__ C, int32_t* __restrict__ st_n,
                double* __restrict__ st_p, double* __restrict__ st_norm,
-               unsigned long long* __restrict__ counters, const unsigned int* __restrict__ status,
+               unsigned long long* __restrict__ counters, float4* __restrict__ chunk_sums,
+               unsigned int* __restrict__ tickets, const unsigned int* __restrict__ status,
                unsigned int* __restrict__ status_mirror) {
   __shared__ float red[4][kAccThreads / 32];
   pdl_wait();
   pdl_launch_dependents();
-  const int e = blockIdx.x;
+  const int e = blockIdx.x, c = blockIdx.y;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int beg = offs[e], end = offs[e + 1];
+  const int n = end - beg;
+  const int n_chunks = n > 0 ? (n + kAccChunk - 1) / kAccChunk : 1;
+  if (c >= n_chunks) return;
   const bool vec = (nb & 3) == 0;
   float p_hi = 0.f, p_lo = 0.f, n_hi = 0.f, n_lo = 0.f;
-  // four slots per thread per pass, all loads issued before the sums
-  for (int i0 = beg + tid; i0 < end; i0 += 4 * kAccThreads) {
+  {
+    // four slots per thread, all loads issued before the sums
+    const int i0 = beg + c * kAccChunk + tid;
     float pv[4], nv[4];
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
@@ -242,10 +252,10 @@ account_kernel(const int32_t* __restrict__ offs, const float* __restrict__ perm_
   for (int o = 16; o > 0; o >>= 1) {
     const float a = __shfl_xor_sync(0xffffffffu, p_hi, o);
     const float b = __shfl_xor_sync(0xffffffffu, p_lo, o);
-    const float c = __shfl_xor_sync(0xffffffffu, n_hi, o);
+    const float cc = __shfl_xor_sync(0xffffffffu, n_hi, o);
     const float dd = __shfl_xor_sync(0xffffffffu, n_lo, o);
     df_add(p_hi, p_lo, a, b);
-    df_add(n_hi, n_lo, c, dd);
+    df_add(n_hi, n_lo, cc, dd);
   }
   if (lane == 0) {
     red[0][warp] = p_hi;
@@ -254,28 +264,41 @@ account_kernel(const int32_t* __restrict__ offs, const float* __restrict__ perm_
     red[3][warp] = n_lo;
   }
   __syncthreads();
-  if (tid == 0) {
-    float ah = 0.f, al = 0.f, bh = 0.f, bl = 0.f;
-    for (int wi = 0; wi < kAccThreads / 32; ++wi) {
-      df_add(ah, al, red[0][wi], red[1][wi]);
-      df_add(bh, bl, red[2][wi], red[3][wi]);
-    }
-    const double a = (double)ah + (double)al, b = (double)bh + (double)bl;
-    const int n = end - beg;
-    const unsigned int sw = __ldcg(status);
-    if (sw == 0u) {  // every kernel of the call completed its work
-      N[e] += n;
-      P[e] += a;
-      if (n > 0) C[e] = (1.0 - alpha) * C[e] + alpha * (b / (double)n);
-      if (n > 0) atomicAdd(&counters[1], 1ull);
-      atomicAdd(&counters[2], (unsigned long long)n);
-      if (e == 0) atomicAdd(&counters[0], 1ull);
-    }
-    st_n[e] = n;
-    st_p[e] = a;
-    st_norm[e] = b;
-    if (e == 0 && status_mirror) *(volatile unsigned int*)status_mirror = sw;
+  if (tid != 0) return;
+  float ah = 0.f, al = 0.f, bh = 0.f, bl = 0.f;
+  for (int wi = 0; wi < kAccThreads / 32; ++wi) {
+    df_add(ah, al, red[0][wi], red[1][wi]);
+    df_add(bh, bl, red[2][wi], red[3][wi]);
   }
+  if (n_chunks > 1) {
+    // publish this chunk's sums; the last block of the expert to arrive adds all chunks in order
+    float4* cs = chunk_sums + (size_t)e * gridDim.y;
+    cs[c] = make_float4(ah, al, bh, bl);
+    __threadfence();
+    if (atomicAdd(&tickets[e], 1u) != (unsigned)(n_chunks - 1)) return;
+    __threadfence();
+    tickets[e] = 0u;  // for the next call (which starts after this kernel has completed)
+    ah = al = bh = bl = 0.f;
+    for (int ci = 0; ci < n_chunks; ++ci) {
+      const float4 v = __ldcg(cs + ci);
+      df_add(ah, al, v.x, v.y);
+      df_add(bh, bl, v.z, v.w);
+    }
+  }
+  const double a = (double)ah + (double)al, b = (double)bh + (double)bl;
+  const unsigned int sw = __ldcg(status);
+  if (sw == 0u) {  // every kernel of the call completed its work
+    N[e] += n;
+    P[e] += a;
+    if (n > 0) C[e] = (1.0 - alpha) * C[e] + alpha * (b / (double)n);
+    if (n > 0) atomicAdd(&counters[1], 1ull);
+    atomicAdd(&counters[2], (unsigned long long)n);
+    if (e == 0) atomicAdd(&counters[0], 1ull);
+  }
+  st_n[e] = n;
+  st_p[e] = a;
+  st_norm[e] = b;
+  if (e == 0 && status_mirror) *(volatile unsigned int*)status_mirror = sw;
 }
 
 }  // namespace
@@ -330,14 +353,18 @@ cudaError_t launch_combine(int y_bf16, const void* opart, int o_bf16, int n_spli
                                  T, K, d, y, nrm_part, status);
 }
 
+int account_chunks(long long rows) {
+  return rows > kAccChunk ? (int)((rows + kAccChunk - 1) / kAccChunk) : 1;
+}
+
 cudaError_t launch_account(const int32_t* offs, const float* perm_p, const float* nrm_part, int nb,
-                           int E, double alpha, int64_t* N, double* P, double* C, int32_t* st_n,
-                           double* st_p, double* st_norm, long long* counters,
-                           const unsigned int* status, unsigned int* status_mirror,
-                           cudaStream_t st) {
-  return launch_pdl(account_kernel, dim3(E), dim3(kAccThreads), 0, st, offs, perm_p, nrm_part,
-                    nb, alpha, N, P, C, st_n, st_p, st_norm, (unsigned long long*)counters, status,
-                    status_mirror);
+                           int E, long long rows, double alpha, int64_t* N, double* P, double* C,
+                           int32_t* st_n, double* st_p, double* st_norm, long long* counters,
+                           float4* chunk_sums, unsigned int* tickets, const unsigned int* status,
+                           unsigned int* status_mirror, cudaStream_t st) {
+  return launch_pdl(account_kernel, dim3(E, account_chunks(rows)), dim3(kAccThreads), 0, st, offs,
+                    perm_p, nrm_part, nb, alpha, N, P, C, st_n, st_p, st_norm,
+                    (unsigned long long*)counters, chunk_sums, tickets, status, status_mirror);
 }
 
 }  // namespace eat

@@ -66,6 +66,8 @@ struct eat_handle {
   unsigned int* mirror_dev = nullptr;
   bool failed = false;  // a call saw the status word set: calls fail until eat_reset_accounts
   int32_t* chunk_cnt = nullptr;    // permute scratch: ticket word, then [chunks][E] counts
+  float4* acc_sums = nullptr;        // account scratch: [E][chunks] compensated chunk sums
+  unsigned int* acc_tickets = nullptr;  // [E] account tickets (zero between calls)
   long long opart_rows = 0;
   float* tau_state = nullptr;  // caller-owned [Tmax] previous tau_final per stream, or null
   const int32_t* ppl_sign_src = nullptr;  // caller-owned device PPL sign (eat_ppl_update), or null
@@ -333,9 +335,9 @@ eat_status run_forward(eat_handle* h, const void* x, int T, int ppl_sign, void* 
                           h->w, h->sout, tc, h->S, T, h->K, h->d, y, h->nrm_part, h->status, st);
   }));
   EAT_TRY(launch(h, kAccount, st, "account update", [&] {
-    return launch_account(h->perm.offs, h->perm.perm_p, h->nrm_part, h->nb, h->E, h->prm.alpha,
-                          h->N, h->P, h->C, h->st_n, h->st_p, h->st_norm, h->counters, h->status,
-                          h->mirror_dev, st);
+    return launch_account(h->perm.offs, h->perm.perm_p, h->nrm_part, h->nb, h->E, rows,
+                          h->prm.alpha, h->N, h->P, h->C, h->st_n, h->st_p, h->st_norm,
+                          h->counters, h->acc_sums, h->acc_tickets, h->status, h->mirror_dev, st);
   }));
   if (idx_opt || w_opt || k_opt) {
     cudaError_t e = cudaSuccess;
@@ -513,6 +515,8 @@ eat_status eat_create(const eat_layer_desc* desc, const eat_params* params, eat_
     add(&h->xperm, h->elt * rows * h->d);
   }
   add(&h->chunk_cnt, sizeof(int32_t) * permute_scratch_ints(h->Tmax, h->E));
+  add(&h->acc_sums, sizeof(float4) * (size_t)h->E * account_chunks((long long)rows));
+  add(&h->acc_tickets, sizeof(unsigned int) * h->E);
   if (h->w8) {
     add(&h->q.xq, 2 * rows * h->d);
     add(&h->q.xq_s, sizeof(float) * rows);

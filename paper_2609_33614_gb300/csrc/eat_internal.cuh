@@ -160,14 +160,17 @@ cudaError_t launch_combine(int y_bf16, const void* opart, int o_bf16, int n_spli
                            int split_stride_rows, const int32_t* slot_of, const float* w,
                            const void* sout, int s_bf16, int S, int T, int K, int d, void* y,
                            float* nrm_part, const unsigned int* status, cudaStream_t st);
-// status: the device status word (nonzero: an expert kernel of the call gave up on a bounded wait;
-// the update is then skipped); status_mirror: device address of a host-mapped copy of the word
-// that block 0 writes, or null.
+// rows: the call's T * K selection slots (bounds the blocks per expert); chunk_sums:
+// [E][account_chunks(rows)] scratch; tickets: [E] words, zero between calls (the kernel leaves
+// them zero).  status: the device status word (nonzero: an expert kernel of the call gave up on a
+// bounded wait; the update is then skipped); status_mirror: device address of a host-mapped copy
+// of the word, written by the block that finishes expert 0, or null.
+int account_chunks(long long rows);
 cudaError_t launch_account(const int32_t* offs, const float* perm_p, const float* nrm_part, int nb,
-                           int E, double alpha, int64_t* N, double* P, double* C, int32_t* st_n,
-                           double* st_p, double* st_norm, long long* counters,
-                           const unsigned int* status, unsigned int* status_mirror,
-                           cudaStream_t st);
+                           int E, long long rows, double alpha, int64_t* N, double* P, double* C,
+                           int32_t* st_n, double* st_p, double* st_norm, long long* counters,
+                           float4* chunk_sums, unsigned int* tickets, const unsigned int* status,
+                           unsigned int* status_mirror, cudaStream_t st);
 
 // §3.3 perplexity of a window of token negative log-likelihoods and the sign of its change.
 cudaError_t launch_ppl_update(const float* nll, int n, double* state, int32_t* sign,

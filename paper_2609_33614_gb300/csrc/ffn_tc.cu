@@ -212,9 +212,7 @@ struct Cfg {
   static constexpr int kSubBytes = kNA * kABytes + kNB * kBBytes;  // one k-block's tiles
   // k-blocks per pipeline stage: a stage completes on one barrier phase, which costs ~0.6 µs
   // however few bytes it carries, so a stage carries two k-blocks wherever three such stages fit
-  // (not in the bf16 gate/up kernel, whose gathering producer copies one k-block per stage)
-  static constexpr int kKPS =
-      (kGateUp && !W8) ? 1 : (6 * kSubBytes <= kSmemBudget - 2048 ? 2 : 1);
+  static constexpr int kKPS = 6 * kSubBytes <= kSmemBudget - 2048 ? 2 : 1;
   // e4m3 tiles of 64 or more tokens are drained by two warps per TMEM lane quarter (one per half
   // of the tile's columns), so an accumulator buffer returns to the MMA issuer sooner (e4m3
   // prefill +20 %; the bf16 gathering gate/up at 128-token tiles was slower with eight)
@@ -429,12 +427,13 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
   }
   const int units = count_units();
 
-  if (C::kKPS == 1 && !W8 && warp == 0 && args.b_rows) {
+  if (GATEUP && !W8 && warp == 0 && args.b_rows) {
     // ------------------------------------------------------------ producer, gathered tokens:
     // lane 0 issues the weight TMA; all lanes copy the tile's token rows from x with 16-byte
-    // cp.async into the 128B-swizzled B tile (lane l: column chunk l % 8 of rows l / 8 + 4 i).
-    // A stage's rows are released LAG stages later: wait for the lane's own copies, fence the
-    // async proxy, and one arrive per warp on the stage's full barrier.
+    // cp.async into the 128B-swizzled B tile of each k-block of the stage (lane l: column chunk
+    // l % 8 of rows l / 8 + 4 i).  A stage's rows are released LAG stages later: wait for the
+    // lane's own copies, fence the async proxy, and one arrive per warp on the stage's full
+    // barrier.
     constexpr int PER = BN / 4;
     constexpr int LAG = S > 2 ? S - 2 : 1;
     const unsigned fullmask = 0xffffffffu;
@@ -453,7 +452,8 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
         const int r = r0 + 4 * i;
         tok[i] = r < w.nrows ? args.b_rows[w.slot0 + r] : -1;
       }
-      for (int kb = w.kb0; kb < w.kb1; ++kb) {
+      for (int kb = w.kb0; kb < w.kb1; kb += C::kKPS) {
+        const int nk = C::kKPS == 1 ? 1 : min(C::kKPS, w.kb1 - kb);  // k-blocks of this stage
         bool okw = true;
         if (lane == 0) okw = mbar_wait(&empty[stage], phase ^ 1u, abort_flag, args.err, 1u, true);
         okw = __shfl_sync(fullmask, okw ? 1 : 0, 0) != 0;
@@ -463,16 +463,22 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
         }
         uint8_t* st = smem + stage * C::kStageBytes;
         if (lane == 0) {
-          mbar_expect_tx(&full[stage], C::kNA * C::kABytes);
-          load_a(st, &full[stage], kb, a_row);
-        }
-        const uint32_t sb = smem_u32(st + C::kNA * C::kABytes);
+          mbar_expect_tx(&full[stage], nk * C::kNA * C::kABytes);
 #pragma unroll
-        for (int i = 0; i < PER; ++i) {
-          if (tok[i] >= 0) {
-            const int r = r0 + 4 * i;
-            cp_async16(sb + r * 128 + ((cc ^ (r & 7)) << 4),
-                       args.bx + (size_t)tok[i] * ld + kb * kBK + cc * 8);
+          for (int j = 0; j < C::kKPS; ++j)
+            if (j < nk) load_a(st + j * C::kSubBytes, &full[stage], kb + j, a_row);
+        }
+#pragma unroll
+        for (int j = 0; j < C::kKPS; ++j) {
+          if (j >= nk) break;
+          const uint32_t sb = smem_u32(st + j * C::kSubBytes + C::kNA * C::kABytes);
+#pragma unroll
+          for (int i = 0; i < PER; ++i) {
+            if (tok[i] >= 0) {
+              const int r = r0 + 4 * i;
+              cp_async16(sb + r * 128 + ((cc ^ (r & 7)) << 4),
+                         args.bx + (size_t)tok[i] * ld + (kb + j) * kBK + cc * 8);
+            }
           }
         }
         cp_async_commit();

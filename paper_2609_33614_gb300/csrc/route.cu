@@ -1,8 +1,9 @@
 // Router and EAT selection (§3.1-§3.4 of the EAT paper, Eq. 1-8).
 //
-//  router_logits_small_kernel (T <= 128, decode) / router_logits_tile_kernel (bf16 x, prefill) /
-//      router_logits_kernel (other prefill calls; both tiled through shared memory): partial
-//      router scores x . w_r over slices of d: fp32 FMA inside 16- or 32-wide chunks, chunk sums accumulated in fp64 or Kahan-compensated fp32, so the
+//  router_logits_small_kernel (T <= 128, decode) / router_logits_sk_kernel (bf16 x, larger calls;
+//      stream-K over tiles and chunks of d) / router_logits_kernel (other large calls; both tiled
+//      through shared memory): partial router scores x . w_r over slices of d: fp32 FMA inside
+//      16- or 32-wide chunks, chunk sums accumulated in Kahan-compensated fp32, so the
 //      logits carry ~1e-7 absolute error (the selection compares I against tau at 1e-5 and P_total
 //      sums p at 1e-6 relative).  The scores stay off the tensor cores: their fp32 accumulation
 //      biased the scores enough to move P_total by ~1e-6 relative.
@@ -16,6 +17,9 @@
 #include "eat_internal.cuh"
 
 #include <math.h>
+
+#include <algorithm>
+#include <atomic>
 
 namespace eat {
 
@@ -165,15 +169,34 @@ router_logits_small_kernel(const TX* __restrict__ x, const float* __restrict__ w
   }
 }
 
-// Router scores for large T with bf16 x (d a multiple of 32, 16-byte aligned x and W_r): CTA tile
-// of 64 tokens x 64 experts over one slice of d, 256 threads with 4 tokens x 4 experts each (the
-// experts tx, tx + 16, tx + 32, tx + 48, so a warp's weight reads cover 16 consecutive rows and
-// hit distinct bank groups).  Both operands sit row-major in shared memory as fp32 (row stride 36
-// floats), double-buffered by 32-column chunk: W_r rows arrive by cp.async, x rows are loaded
-// into registers one chunk ahead and converted when stored.  Each output takes 32 fp32 FMAs per
-// chunk and the chunk sums are added with Kahan compensation, as in router_logits_kernel.  With
-// 4 x 4 outputs a thread needs about 100 registers, so two CTAs (16 warps) share an SM.
-constexpr int kRT = 64, kRE = 64, kRS = kChunkK + 4;
+// Router scores for large T with bf16 x (d a multiple of 32, 16-byte aligned x and W_r).  The
+// work is the units (64-token x 64-expert tile, 32-column chunk of d), numbered tile-major, and a
+// persistent grid of G CTAs (as many as fit on the SMs, each at least kSKMinUnits units) takes
+// contiguous, equal runs of them (stream-K): no tail wave, and a CTA's run may start or end inside
+// a tile.  Each thread keeps TM tokens x 4 experts (experts tx, tx + 16, tx + 32, tx + 48, so a
+// warp's weight reads cover 16 consecutive rows and hit distinct bank groups) and adds each
+// chunk's 32 fp32 FMAs into a Kahan-compensated fp32 sum, as the other router-score kernels do.
+// Where its run leaves a tile, a CTA writes the tile's compensated sums to split slice
+// seg = (its index) - (index of the CTA that starts the tile); the CTA that ends a tile also
+// writes zero pairs to the slices after its own, up to n_split, so the selection kernel adds a
+// fixed number of slices for every tile.  x and W_r go through a three-stage shared-memory ring
+// as fp32 (row stride 36 floats): W_r by cp.async, x through registers (converted when stored),
+// two units ahead; one block barrier per unit.
+constexpr int kSKT = 64, kSKE = 64, kSKS = kChunkK + 4, kSKStages = 3;
+constexpr int kSKTM = 4;        // tokens per thread: 256 threads, two CTAs per SM
+constexpr int kSKMinUnits = 8;  // 256 columns of d per CTA at least
+constexpr size_t kSKSmem = (size_t)kSKStages * (kSKT + kSKE) * kSKS * sizeof(float);
+template <int TM>
+struct SkCfg {
+  static constexpr int kThreads = kSKT * kSKE / (4 * TM);
+  static constexpr int kWPieces = kSKE * kChunkK / 4 / kThreads;  // 16-byte pieces per thread
+  static constexpr int kXPieces = kSKT * kChunkK / 8 / kThreads;
+};
+
+// the CTA whose run [g U / G, (g + 1) U / G) holds unit u
+__host__ __device__ __forceinline__ int sk_owner(long long u, long long U, int G) {
+  return (int)(((u + 1) * (long long)G - 1) / U);
+}
 
 __device__ __forceinline__ void bf16x8_to_f32(const uint4& u, float (&v)[8]) {
   const uint32_t w[4] = {u.x, u.y, u.z, u.w};
@@ -185,109 +208,156 @@ __device__ __forceinline__ void bf16x8_to_f32(const uint4& u, float (&v)[8]) {
   }
 }
 
-__global__ void __launch_bounds__(kLogitThreads, 2)
-router_logits_tile_kernel(const __nv_bfloat16* __restrict__ x, const float* __restrict__ wr,
-                          int T, int d, int E, int d_per_split, float2* __restrict__ part) {
-  __shared__ __align__(16) float xs[2][kRT][kRS];
-  __shared__ __align__(16) float ws[2][kRE][kRS];
+// A unit's place: token tile, expert tile and chunk, advanced one unit at a time (no division in
+// the loop).
+struct SkCursor {
+  int tt, et, ch;
+  __device__ __forceinline__ void next(int etiles, int nc) {
+    if (++ch == nc) {
+      ch = 0;
+      if (++et == etiles) {
+        et = 0;
+        ++tt;
+      }
+    }
+  }
+};
+
+template <int TM>
+__global__ void __launch_bounds__(SkCfg<TM>::kThreads, 2)
+router_logits_sk_kernel(const __nv_bfloat16* __restrict__ x, const float* __restrict__ wr, int T,
+                        int d, int E, int n_split, float2* __restrict__ part) {
+  using C = SkCfg<TM>;
+  extern __shared__ __align__(16) float sk_smem[];
+  float* xs = sk_smem;                              // [stage][64 tokens][kSKS]
+  float* ws = sk_smem + kSKStages * kSKT * kSKS;    // [stage][64 experts][kSKS]
   pdl_wait();
   pdl_launch_dependents();
-  const int tid = threadIdx.x;
-  const int tx = tid & 15, ty = tid >> 4;
-  const int t0 = blockIdx.x * kRT, e0 = blockIdx.y * kRE;
-  const int dbeg = blockIdx.z * d_per_split;
-  const int dend = min(d, dbeg + d_per_split);
-  const int n_chunks = dend > dbeg ? (dend - dbeg) / kChunkK : 0;
-  // x loader: row tid / 4, 8 columns at (tid % 4) * 8
-  const int xr = tid >> 2, xc = (tid & 3) * 8;
-  const bool x_ok = t0 + xr < T;
-  const __nv_bfloat16* xsrc = x + (size_t)(x_ok ? t0 + xr : 0) * d + xc;
-  uint4 xraw = make_uint4(0u, 0u, 0u, 0u);
-  auto load_x = [&](int k0) {
-    if (x_ok) xraw = *(const uint4*)(xsrc + k0);
-  };
-  auto store_x = [&](int b) {
-    float v[8];
-    bf16x8_to_f32(xraw, v);
-    *(float4*)&xs[b][xr][xc] = make_float4(v[0], v[1], v[2], v[3]);
-    *(float4*)&xs[b][xr][xc + 4] = make_float4(v[4], v[5], v[6], v[7]);
-  };
-  // W_r loader: pieces tid and tid + 256 -- row q / 8, 4 columns at (q % 8) * 4
-  auto load_w = [&](int k0, int b) {
+  const int nc = d / kChunkK;
+  const int etiles = (E + kSKE - 1) / kSKE;
+  const int U = ((T + kSKT - 1) / kSKT) * etiles * nc;
+  const int G = gridDim.x, g = blockIdx.x;
+  const int u0 = (int)((long long)g * U / G), u1 = (int)((long long)(g + 1) * U / G);
+  const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+  SkCursor ld, cu;  // the next unit to load, the unit being computed
+  {
+    const int tile = u0 / nc;
+    ld.tt = tile / etiles;
+    ld.et = tile - ld.tt * etiles;
+    ld.ch = u0 - tile * nc;
+    cu = ld;
+  }
+
+  // W_r: 64 rows x 32 floats in 16-byte pieces q = tid + kThreads r: row q / 8, columns (q % 8) * 4
+  // x: 64 rows x 32 bf16 in 16-byte pieces q = tid + kThreads r: row q / 4, columns (q % 4) * 8
+  uint4 xr[C::kXPieces];
+  // the next unit's W_r pieces (cp.async) and x pieces (registers), then advance the cursor
+  auto issue = [&](bool live, int stage) {
+    if (live) {
+      const int t0 = ld.tt * kSKT, e0 = ld.et * kSKE, k0 = ld.ch * kChunkK;
+      float* wsb = ws + stage * kSKE * kSKS;
 #pragma unroll
-    for (int r = 0; r < 2; ++r) {
-      const int q = tid + r * kLogitThreads;
-      const int row = q >> 3, c4 = (q & 7) * 4;
-      const int e = e0 + row;
-      if (e < E)
-        cp_async16((uint32_t)__cvta_generic_to_shared(&ws[b][row][c4]),
-                   wr + (size_t)e * d + k0 + c4);
-      else
-        *(float4*)&ws[b][row][c4] = make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int r = 0; r < C::kWPieces; ++r) {
+        const int q = tid + r * C::kThreads, row = q >> 3, c4 = (q & 7) * 4;
+        if (e0 + row < E)
+          cp_async16((uint32_t)__cvta_generic_to_shared(&wsb[row * kSKS + c4]),
+                     wr + (size_t)(e0 + row) * d + k0 + c4);
+        else
+          *(float4*)&wsb[row * kSKS + c4] = make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+#pragma unroll
+      for (int r = 0; r < C::kXPieces; ++r) {
+        const int q = tid + r * C::kThreads, row = q >> 2, c8 = (q & 3) * 8;
+        xr[r] = t0 + row < T ? *(const uint4*)(x + (size_t)(t0 + row) * d + k0 + c8)
+                             : make_uint4(0u, 0u, 0u, 0u);
+      }
+      ld.next(etiles, nc);
     }
-    cp_async_commit();
+    cp_async_commit();  // (an empty group past the run keeps the group count uniform)
   };
-  float sum[4][4], comp[4][4];
+  auto store_x = [&](bool live, int stage) {
+    if (live) {
+      float* xsb = xs + stage * kSKT * kSKS;
 #pragma unroll
-  for (int i = 0; i < 4; ++i)
+      for (int r = 0; r < C::kXPieces; ++r) {
+        const int q = tid + r * C::kThreads, row = q >> 2, c8 = (q & 3) * 8;
+        float v[8];
+        bf16x8_to_f32(xr[r], v);
+        *(float4*)&xsb[row * kSKS + c8] = make_float4(v[0], v[1], v[2], v[3]);
+        *(float4*)&xsb[row * kSKS + c8 + 4] = make_float4(v[4], v[5], v[6], v[7]);
+      }
+    }
+  };
+
+  float sum[TM][4], comp[TM][4];
+#pragma unroll
+  for (int i = 0; i < TM; ++i)
 #pragma unroll
     for (int j = 0; j < 4; ++j) sum[i][j] = comp[i][j] = 0.f;
 
-  if (n_chunks > 0) {
-    load_w(dbeg, 0);
-    load_x(dbeg);
-    store_x(0);
-  }
-  for (int c = 0; c < n_chunks; ++c) {
-    const int cur = c & 1;
-    const bool more = c + 1 < n_chunks;
-    __syncthreads();  // chunk c - 1 consumed: buffer cur ^ 1 is free; xs[cur] is complete
-    if (more) {
-      load_w(dbeg + (c + 1) * kChunkK, cur ^ 1);
-      load_x(dbeg + (c + 1) * kChunkK);
-      cp_async_wait<1>();
-    } else {
-      cp_async_wait<0>();
-    }
-    __syncthreads();  // every thread's W_r pieces of chunk c have landed
-    float acc[4][4];
+  issue(true, 0);
+  store_x(true, 0);
+  issue(u0 + 1 < u1, 1);
+  store_x(u0 + 1 < u1, 1);
+  int stage = 0;
+  for (int u = u0; u < u1; ++u) {
+    cp_async_wait<1>();  // this thread's W_r pieces of unit u have landed
+    __syncthreads();     // everyone's pieces of unit u are visible; unit u - 1's stage is free
+    const int ahead = stage == 0 ? kSKStages - 1 : stage - 1;  // the stage of unit u + 2
+    const bool live2 = u + 2 < u1;
+    issue(live2, ahead);
+    const float* xsb = xs + stage * kSKT * kSKS;
+    const float* wsb = ws + stage * kSKE * kSKS;
+    float acc[TM][4];
 #pragma unroll
-    for (int i = 0; i < 4; ++i)
+    for (int i = 0; i < TM; ++i)
 #pragma unroll
       for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
 #pragma unroll
     for (int kk = 0; kk < kChunkK; kk += 4) {
-      float4 a[4], b[4];
+      float4 b[4];
 #pragma unroll
-      for (int i = 0; i < 4; ++i) a[i] = *(const float4*)&xs[cur][ty * 4 + i][kk];
+      for (int j = 0; j < 4; ++j) b[j] = *(const float4*)&wsb[(tx + 16 * j) * kSKS + kk];
 #pragma unroll
-      for (int j = 0; j < 4; ++j) b[j] = *(const float4*)&ws[cur][tx + 16 * j][kk];
-#pragma unroll
-      for (int i = 0; i < 4; ++i)
+      for (int i = 0; i < TM; ++i) {
+        const float4 a = *(const float4*)&xsb[(ty * TM + i) * kSKS + kk];
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-          acc[i][j] = fmaf(a[i].x, b[j].x, acc[i][j]);
-          acc[i][j] = fmaf(a[i].y, b[j].y, acc[i][j]);
-          acc[i][j] = fmaf(a[i].z, b[j].z, acc[i][j]);
-          acc[i][j] = fmaf(a[i].w, b[j].w, acc[i][j]);
+          acc[i][j] = fmaf(a.x, b[j].x, acc[i][j]);
+          acc[i][j] = fmaf(a.y, b[j].y, acc[i][j]);
+          acc[i][j] = fmaf(a.z, b[j].z, acc[i][j]);
+          acc[i][j] = fmaf(a.w, b[j].w, acc[i][j]);
         }
+      }
     }
 #pragma unroll
-    for (int i = 0; i < 4; ++i)
+    for (int i = 0; i < TM; ++i)
 #pragma unroll
       for (int j = 0; j < 4; ++j) kahan_add(sum[i][j], comp[i][j], acc[i][j]);
-    if (more) store_x(cur ^ 1);
-  }
+    store_x(live2, ahead);
+    const bool tile_end = cu.ch == nc - 1;
+    if (tile_end || u + 1 == u1) {
+      const long long tile = (long long)cu.tt * etiles + cu.et;
+      const int seg = g - sk_owner(tile * nc, U, G);  // < n_split (the host's bound)
+      const int t0 = cu.tt * kSKT, e0 = cu.et * kSKE;
+      const int zend = tile_end ? n_split : seg + 1;
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int t = t0 + ty * 4 + i;
-    if (t >= T) continue;
+      for (int i = 0; i < TM; ++i) {
+        const int t = t0 + ty * TM + i;
+        if (t >= T) continue;
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const int e = e0 + tx + 16 * j;
-      if (e < E)
-        part[((size_t)blockIdx.z * T + t) * E + e] = make_float2(sum[i][j], -comp[i][j]);
+        for (int j = 0; j < 4; ++j) {
+          const int e = e0 + tx + 16 * j;
+          if (e >= E || seg >= n_split) continue;
+          part[((size_t)seg * T + t) * E + e] = make_float2(sum[i][j], -comp[i][j]);
+          for (int z = seg + 1; z < zend; ++z)
+            part[((size_t)z * T + t) * E + e] = make_float2(0.f, 0.f);
+          sum[i][j] = comp[i][j] = 0.f;
+        }
+      }
     }
+    cu.next(etiles, nc);
+    stage = stage == kSKStages - 1 ? 0 : stage + 1;
   }
 }
 
@@ -688,14 +758,80 @@ route_select_kernel(const float2* __restrict__ part, int n_split, const float* _
 
 }  // namespace
 
+namespace {
+
+// CTAs of router_logits_sk_kernel resident per SM, and the SM count, of the current device (both
+// queried once per device; concurrent first calls compute the same values)
+struct SkDevice {
+  std::atomic<int> ready{0};
+  int sms = 0, per_sm = 0;
+};
+SkDevice g_sk_dev[64];
+
+bool sk_device(int& sms, int& per_sm) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
+  SkDevice& D = g_sk_dev[dev];
+  if (!D.ready.load(std::memory_order_acquire)) {
+    int n = 0, b = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        cudaFuncSetAttribute(router_logits_sk_kernel<kSKTM>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSKSmem) != cudaSuccess ||
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, router_logits_sk_kernel<kSKTM>,
+                                                      SkCfg<kSKTM>::kThreads, kSKSmem) != cudaSuccess ||
+        n < 1 || b < 1)
+      return false;
+    D.sms = n;
+    D.per_sm = b;
+    D.ready.store(1, std::memory_order_release);
+  }
+  sms = D.sms;
+  per_sm = D.per_sm;
+  return true;
+}
+
+// Grid and split slices of the stream-K router for a call; cap > 0 bounds the slices (a caller
+// with fixed scratch).  A tile of nc units meets at most 1 + ceil((nc - 1) / m) CTA runs when every
+// run holds at least m units; n_split is that bound (slices a tile does not use are zero pairs).
+struct SkPlan {
+  int grid = 0, n_split = 0;
+};
+bool sk_plan(int T, int d, int E, int cap, SkPlan& out) {
+  int sms = 0, per_sm = 0;
+  if (!sk_device(sms, per_sm)) return false;
+  const long long nc = d / kChunkK;
+  const long long tiles = (long long)((T + kSKT - 1) / kSKT) * ((E + kSKE - 1) / kSKE);
+  const long long U = tiles * nc;
+  long long G = std::min<long long>((long long)sms * per_sm, U / kSKMinUnits);
+  G = std::max<long long>(1, std::min(G, U));
+  auto bound = [&](long long g) {
+    const long long m = U / g;
+    return g == tiles && U % g == 0 ? 1LL : std::min(nc, 1 + (nc - 1 + m - 1) / m);
+  };
+  long long n = bound(G);
+  if (cap > 0 && n > cap) {
+    if (cap == 1) {
+      G = tiles;  // every CTA one whole tile
+    } else {
+      const long long m_req = (nc - 1 + cap - 2) / (cap - 1);
+      G = std::max<long long>(1, U / m_req);
+    }
+    n = bound(G);
+  }
+  out.grid = (int)G;
+  out.n_split = (int)n;
+  return true;
+}
+
+bool sk_eligible(int T, int d) { return T > kSmallT && d % kChunkK == 0; }
+
+}  // namespace
+
 int router_split(int T, int d, int E) {
   if (T <= kSmallT) return (d + kSmallSlice - 1) / kSmallSlice;
-  if (d % kChunkK == 0) {
-    // tile kernel (two 256-thread CTAs per SM): up to two waves, slices of at least 256 columns
-    const long long tiles = (long long)((T + kRT - 1) / kRT) * ((E + kRE - 1) / kRE);
-    int split = 1;
-    while (tiles * split * 2 <= 4 * 152 && d / (split * 2) >= 256 && split < 64) split *= 2;
-    return split;
+  if (sk_eligible(T, d)) {
+    SkPlan pl;
+    if (sk_plan(T, d, E, 0, pl)) return pl.n_split;
   }
   // enough CTAs for two waves, each slice at least 256 columns of d
   const long long tiles = (long long)((T + kTileT - 1) / kTileT) * ((E + kTileE - 1) / kTileE);
@@ -717,13 +853,16 @@ cudaError_t launch_router_logits(const void* x, int x_bf16, const float* w_route
     return launch_pdl(router_logits_small_kernel<float>, grid, dim3(kLogitThreads), 0, st,
                       (const float*)x, w_router, T, d, E, per, part);
   }
+  if (x_bf16 && sk_eligible(T, d) && vec_ok) {
+    SkPlan pl;
+    if (!sk_plan(T, d, E, n_split, pl)) return cudaErrorInvalidDevice;
+    if (pl.n_split > n_split) return cudaErrorInvalidValue;
+    return launch_pdl(router_logits_sk_kernel<kSKTM>, dim3(pl.grid), dim3(SkCfg<kSKTM>::kThreads),
+                      kSKSmem, st,
+                      (const __nv_bfloat16*)x, w_router, T, d, E, n_split, part);
+  }
   int per = (d + n_split - 1) / n_split;
   per = (per + kChunkK - 1) / kChunkK * kChunkK;
-  if (x_bf16 && d % kChunkK == 0 && vec_ok) {
-    dim3 grid((T + kRT - 1) / kRT, (E + kRE - 1) / kRE, n_split);
-    return launch_pdl(router_logits_tile_kernel, grid, dim3(kLogitThreads), 0, st,
-                      (const __nv_bfloat16*)x, w_router, T, d, E, per, part);
-  }
   dim3 grid((T + kTileT - 1) / kTileT, (E + kTileE - 1) / kTileE, n_split);
   if (x_bf16)
     return launch_pdl(router_logits_kernel<__nv_bfloat16>, grid, dim3(kLogitThreads), 0, st,
