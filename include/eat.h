@@ -176,17 +176,22 @@ eat_status eat_route(eat_handle* h, const void* x, int32_t T, int32_t ppl_sign,
 eat_status eat_moe_forward(eat_handle* h, const void* x, int32_t T, int32_t ppl_sign, void* y,
                            int32_t* idx_opt, float* w_opt, int32_t* k_opt, void* stream);
 
-/* eat_moe_forward with HOST buffers: copies x_host [T, d] to the device, runs the layer, copies
- * y back into y_host [T, d] and synchronises the stream before returning.  Pinned host memory
- * gives asynchronous copies; pageable memory works but is staged by the driver.  The input copy
- * runs on a stream of the handle (created on the first host-buffer call) into one of two staging
- * buffers used in turn, so it overlaps the kernels of the handle's previous call; the layer's
- * kernels on `stream` wait for it. */
+/* eat_moe_forward with HOST buffers x_host [T, d] and y_host [T, d]: moves x to the device, runs
+ * the layer, moves y back and synchronises the stream before returning.
+ *  - Page-locked buffers (cudaHostAlloc / cudaHostRegister, 16-byte aligned) of a bf16 or fp8
+ *    layer: the router kernel reads x_host over the host link while it computes and writes the
+ *    device copy that the later kernels read, and the combine kernel writes y_host directly; no
+ *    copy-engine transfer.  (Except for a call whose shared experts run beside the routing: those
+ *    read x before the router has run, so such a call takes the copies below.)
+ *  - Otherwise the input is copied on a stream of the handle (created on the first host-buffer
+ *    call), and y is copied back on `stream`; pageable memory works but is staged by the driver.
+ * Either way x lands in one of two staging buffers of the handle used in turn, so a call's input
+ * never overwrites the input of the call before it while that call may still read it. */
 eat_status eat_moe_forward_host(eat_handle* h, const void* x_host, int32_t T, int32_t ppl_sign,
                                 void* y_host, void* stream);
 
-/* eat_moe_forward_host without the final synchronisation: enqueues the host-to-device copy of
- * x_host, the layer and the device-to-host copy of y_host on `stream`, and returns.  The caller
+/* eat_moe_forward_host without the final synchronisation: enqueues the layer and the movement of
+ * x_host and y_host (as eat_moe_forward_host) on `stream`, and returns.  The caller
  * keeps both host buffers alive, and x_host unchanged, until the stream has passed this call
  * (cudaStreamSynchronize or an event) and reads y_host only after that.  With page-locked host
  * buffers (cudaHostAlloc / cudaHostRegister) the copies are asynchronous and consecutive calls

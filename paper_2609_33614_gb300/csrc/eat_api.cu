@@ -199,9 +199,11 @@ eat_status check_call(eat_handle* h, const void* x, int32_t T, int32_t ppl_sign)
   return check_state(h);
 }
 
-// Router + selection into (idx, w, k, psel).
+// Router + selection into (idx, w, k, psel).  x_host (or null): the router kernel reads the
+// tokens there (a page-locked host buffer) and writes them to x, which later kernels read.
 eat_status run_route(eat_handle* h, const void* x, int T, int ppl_sign, int32_t* idx, float* w,
-                     int32_t* k, float* psel, bool write_tau, cudaStream_t st) {
+                     int32_t* k, float* psel, bool write_tau, cudaStream_t st,
+                     const void* x_host = nullptr) {
   RouteParams rp = route_params(h->prm, ppl_sign);
   rp.opd_scale = h->desc.opd_scale;
   rp.ppl_sign_dev = h->ppl_sign_src;
@@ -211,6 +213,9 @@ eat_status run_route(eat_handle* h, const void* x, int T, int ppl_sign, int32_t*
   }
   const int split = router_split(T, h->d, h->E);
   EAT_TRY(launch(h, kRoute, st, "router logits", [&] {
+    if (x_host)
+      return launch_router_logits(x_host, h->bf16, h->desc.w_router, T, h->d, h->E, split,
+                                  h->logit_part, st, const_cast<void*>(x));
     return launch_router_logits(x, h->bf16, h->desc.w_router, T, h->d, h->E, split,
                                 h->logit_part, st);
   }));
@@ -257,8 +262,11 @@ bool shared_on_side_stream(const eat_handle* h, int T, int tile_rows) {
   return units < h->tc.num_sms;
 }
 
+// x_host (or null): see run_route; the caller has checked that the router copies x for this call
+// and that no shared expert reads x before the router has run (side stream).
 eat_status run_forward(eat_handle* h, const void* x, int T, int ppl_sign, void* y,
-                       int32_t* idx_opt, float* w_opt, int32_t* k_opt, cudaStream_t st) {
+                       int32_t* idx_opt, float* w_opt, int32_t* k_opt, cudaStream_t st,
+                       const void* x_host = nullptr) {
   const int tile_rows = h->backend == 1 ? tc_tile_rows(h->tc, T) : kSimtTileRows;
   const int tile_rows_down = h->backend == 1 ? tc_tile_rows_down(h->tc, T) : kSimtTileRows;
   TcCall c;
@@ -289,7 +297,8 @@ eat_status run_forward(eat_handle* h, const void* x, int T, int ppl_sign, void* 
     e = cudaEventRecord(h->ev_join, h->side_st);
     if (e != cudaSuccess) return cuda_fail(h, e, "shared-expert stream join");
   }
-  EAT_TRY(run_route(h, x, T, ppl_sign, h->idx, h->w, h->k, h->psel, true, st));
+  if (x_host && side) return fail(h, EAT_ERR_UNSUPPORTED, "host-read input with side-stream experts");
+  EAT_TRY(run_route(h, x, T, ppl_sign, h->idx, h->w, h->k, h->psel, true, st, x_host));
   EAT_TRY(launch(h, kPermute, st, "permute", [&] {
     return launch_permute(h->idx, h->k, h->psel, T, h->K, h->E, tile_rows, tile_rows_down,
                           h->perm, h->chunk_cnt, st);
@@ -618,6 +627,17 @@ eat_status eat_moe_forward(eat_handle* h, const void* x, int32_t T, int32_t ppl_
   return run_forward(h, x, T, ppl_sign, y, idx_opt, w_opt, k_opt, (cudaStream_t)stream);
 }
 
+// The device address of a page-locked host buffer (cudaHostAlloc / cudaHostRegister), or null for
+// any other memory.
+static void* mapped_host(const void* p) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  return a.type == cudaMemoryTypeHost ? a.devicePointer : nullptr;
+}
+
 static eat_status forward_host(eat_handle* h, const void* x_host, int32_t T, int32_t ppl_sign,
                                void* y_host, void* stream, bool sync) {
   EAT_TRY(check_call(h, x_host, T, ppl_sign));
@@ -636,6 +656,26 @@ static eat_status forward_host(eat_handle* h, const void* x_host, int32_t T, int
   const int i = h->stage_i;
   h->stage_i ^= 1;
   void* xs = (char*)h->xstage + (size_t)i * h->elt * h->Tmax * h->d;
+  // Page-locked buffers on the tensor-core path: the router kernel reads x over the host link
+  // while it computes and leaves the device copy in the staging buffer, and the combine kernel
+  // writes y over the link, so no copy engine transfer and no extra launch sits on the call's
+  // path.  Not when shared experts run beside the routing (they read x before the router has
+  // run).
+  void* xd = h->backend == 1 ? mapped_host(x_host) : nullptr;
+  void* yd = xd ? mapped_host(y_host) : nullptr;
+  if (xd && yd && ((uintptr_t)xd & 15) == 0 && ((uintptr_t)yd & 15) == 0 &&
+      router_copies_x(xd, h->bf16, h->desc.w_router, T, h->d) &&
+      !shared_on_side_stream(h, T, tc_tile_rows(h->tc, T))) {
+    // a call on another stream may still read this staging buffer
+    e = cudaStreamWaitEvent(st, h->ev_done[i], 0);
+    if (e != cudaSuccess) return cuda_fail(h, e, "staging buffer wait");
+    EAT_TRY(run_forward(h, xs, T, ppl_sign, yd, nullptr, nullptr, nullptr, st, xd));
+    e = cudaEventRecord(h->ev_done[i], st);
+    if (e == cudaSuccess && sync) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return cuda_fail(h, e, "host-buffer call");
+    if (sync) return check_state(h);
+    return EAT_OK;
+  }
   // the copy waits for the call that last read this buffer (an event never recorded counts as
   // complete), and this call's kernels wait for the copy
   e = cudaStreamWaitEvent(h->copy_st, h->ev_done[i], 0);

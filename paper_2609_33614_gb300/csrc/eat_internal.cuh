@@ -93,8 +93,13 @@ struct RouteParams {
 
 // Partial router logits: part[s][t][e] = sum over the s-th slice of d of x[t,j] Wr[e,j], as an
 // unevaluated fp32 pair (hi, lo) whose exact sum carries the slice's score (see df_add).
+// xcopy (or null): the kernel also writes the x it reads there (16-byte aligned, [T, d]); x may
+// then be host memory the device can address (a page-locked host buffer).  Only calls for which
+// router_copies_x holds can copy.
 cudaError_t launch_router_logits(const void* x, int x_bf16, const float* w_router, int T, int d,
-                                 int E, int n_split, float2* part, cudaStream_t st);
+                                 int E, int n_split, float2* part, cudaStream_t st,
+                                 void* xcopy = nullptr);
+bool router_copies_x(const void* x, int x_bf16, const float* w_router, int T, int d);
 // Warp-per-token softmax + history score + threshold + selection + renormalisation; the router
 // scores are the sum over the n_split slices of part ([split][T][E] fp32 pairs).
 cudaError_t launch_route_select(const float2* part, int n_split, const float* b_router, int T,

@@ -109,27 +109,40 @@ router_logits_kernel(const TX* __restrict__ x, const float* __restrict__ wr, int
   }
 }
 
-// Router scores for small T (decode): block (t, s) computes part[s][t][e] for every expert over
-// the s-th slice of d; warp w takes experts w, w + 8, ...; lanes read float4 pieces of the weight
-// row and of x (coalesced), multiply in fp32, fold each 16 products into a compensated lane sum,
-// and the 32 lane sums are added compensated (a fixed tree).
+// Router scores for small T (decode): block (t, s, z) computes part[s][t][e] over the s-th slice
+// of d for the experts e = 8 z + w of its warps w; lanes read float4 pieces of the weight row and
+// of x (coalesced), multiply in fp32, fold each 16 products into a compensated lane sum, and the
+// 32 lane sums are added compensated (a fixed tree).
 constexpr int kSmallT = kSmallRouterT;
 constexpr int kSmallSlice = 512;
 
 
-__device__ __forceinline__ float4 load_x4(const float* p) { return *(const float4*)p; }
-__device__ __forceinline__ float4 load_x4(const __nv_bfloat16* p) {
-  const uint2 u = *(const uint2*)p;
-  const __nv_bfloat162 a = *(const __nv_bfloat162*)&u.x;
-  const __nv_bfloat162 b = *(const __nv_bfloat162*)&u.y;
-  const float2 fa = __bfloat1622float2(a), fb = __bfloat1622float2(b);
-  return make_float4(fa.x, fa.y, fb.x, fb.y);
-}
+// Four consecutive elements of x: their bits (copied as they are) and their fp32 values.
+struct X4f {
+  float4 bits;
+  __device__ __forceinline__ float4 val() const { return bits; }
+};
+struct X4b {
+  uint2 bits;
+  __device__ __forceinline__ float4 val() const {
+    const float2 fa = __bfloat1622float2(*(const __nv_bfloat162*)&bits.x);
+    const float2 fb = __bfloat1622float2(*(const __nv_bfloat162*)&bits.y);
+    return make_float4(fa.x, fa.y, fb.x, fb.y);
+  }
+};
+__device__ __forceinline__ X4f load_x4(const float* p) { return X4f{*(const float4*)p}; }
+__device__ __forceinline__ X4b load_x4(const __nv_bfloat16* p) { return X4b{*(const uint2*)p}; }
+__device__ __forceinline__ void store_x4(float* p, const X4f& v) { *(float4*)p = v.bits; }
+__device__ __forceinline__ void store_x4(__nv_bfloat16* p, const X4b& v) { *(uint2*)p = v.bits; }
 
+// xcopy (or null): x is read from memory the caller keeps on the host (a host-buffer call) and
+// warp 0 of the blocks of the first expert group also writes what it reads to xcopy, the device
+// copy every later kernel of the call reads.
 template <typename TX>
 __global__ void __launch_bounds__(kLogitThreads)
 router_logits_small_kernel(const TX* __restrict__ x, const float* __restrict__ wr, int T, int d,
-                           int E, int d_per_split, float2* __restrict__ part) {
+                           int E, int d_per_split, float2* __restrict__ part,
+                           TX* __restrict__ xcopy) {
   pdl_wait();
   pdl_launch_dependents();
   const int t = blockIdx.x, s = blockIdx.y;
@@ -137,6 +150,7 @@ router_logits_small_kernel(const TX* __restrict__ x, const float* __restrict__ w
   const int beg = s * d_per_split;
   const int end = min(d, beg + d_per_split);
   const TX* xr = x + (size_t)t * d;
+  TX* xc = xcopy && blockIdx.z == 0 && warp == 0 ? xcopy + (size_t)t * d : nullptr;
   // one expert per warp: blockIdx.z picks the group of kLogitThreads / 32 experts
   {
     const int e = blockIdx.z * (kLogitThreads / 32) + warp;
@@ -147,7 +161,9 @@ router_logits_small_kernel(const TX* __restrict__ x, const float* __restrict__ w
     int cnt = 0;
     for (int c = beg + lane * 4; c < end; c += 128) {
       const float4 wv = *(const float4*)(wrow + c);
-      const float4 xv = load_x4(xr + c);
+      const auto xb = load_x4(xr + c);
+      if (xc) store_x4(xc + c, xb);
+      const float4 xv = xb.val();
       acc = fmaf(xv.x, wv.x, acc);
       acc = fmaf(xv.y, wv.y, acc);
       acc = fmaf(xv.z, wv.z, acc);
@@ -226,7 +242,8 @@ struct SkCursor {
 template <int TM>
 __global__ void __launch_bounds__(SkCfg<TM>::kThreads, 2)
 router_logits_sk_kernel(const __nv_bfloat16* __restrict__ x, const float* __restrict__ wr, int T,
-                        int d, int E, int n_split, float2* __restrict__ part) {
+                        int d, int E, int n_split, float2* __restrict__ part,
+                        __nv_bfloat16* __restrict__ xcopy) {
   using C = SkCfg<TM>;
   extern __shared__ __align__(16) float sk_smem[];
   float* xs = sk_smem;                              // [stage][64 tokens][kSKS]
@@ -251,10 +268,15 @@ router_logits_sk_kernel(const __nv_bfloat16* __restrict__ x, const float* __rest
   // W_r: 64 rows x 32 floats in 16-byte pieces q = tid + kThreads r: row q / 8, columns (q % 8) * 4
   // x: 64 rows x 32 bf16 in 16-byte pieces q = tid + kThreads r: row q / 4, columns (q % 4) * 8
   uint4 xr[C::kXPieces];
+  int x_t0 = 0, x_k0 = 0;  // where the pieces in xr came from
+  bool x_keep = false;     // and whether they go to xcopy (units of the first expert tile)
   // the next unit's W_r pieces (cp.async) and x pieces (registers), then advance the cursor
   auto issue = [&](bool live, int stage) {
     if (live) {
       const int t0 = ld.tt * kSKT, e0 = ld.et * kSKE, k0 = ld.ch * kChunkK;
+      x_t0 = t0;
+      x_k0 = k0;
+      x_keep = xcopy != nullptr && ld.et == 0;
       float* wsb = ws + stage * kSKE * kSKS;
 #pragma unroll
       for (int r = 0; r < C::kWPieces; ++r) {
@@ -285,6 +307,7 @@ router_logits_sk_kernel(const __nv_bfloat16* __restrict__ x, const float* __rest
         bf16x8_to_f32(xr[r], v);
         *(float4*)&xsb[row * kSKS + c8] = make_float4(v[0], v[1], v[2], v[3]);
         *(float4*)&xsb[row * kSKS + c8 + 4] = make_float4(v[4], v[5], v[6], v[7]);
+        if (x_keep && x_t0 + row < T) *(uint4*)(xcopy + (size_t)(x_t0 + row) * d + x_k0 + c8) = xr[r];
       }
     }
   };
@@ -840,26 +863,34 @@ int router_split(int T, int d, int E) {
   return split;
 }
 
-cudaError_t launch_router_logits(const void* x, int x_bf16, const float* w_router, int T, int d,
-                                 int E, int n_split, float2* part, cudaStream_t st) {
+bool router_copies_x(const void* x, int x_bf16, const float* w_router, int T, int d) {
   const bool vec_ok = d % 4 == 0 && ((uintptr_t)x & 15) == 0 && ((uintptr_t)w_router & 15) == 0;
+  return vec_ok && (T <= kSmallT || (x_bf16 && sk_eligible(T, d)));
+}
+
+cudaError_t launch_router_logits(const void* x, int x_bf16, const float* w_router, int T, int d,
+                                 int E, int n_split, float2* part, cudaStream_t st, void* xcopy) {
+  const bool vec_ok = d % 4 == 0 && ((uintptr_t)x & 15) == 0 && ((uintptr_t)w_router & 15) == 0;
+  if (xcopy && (!router_copies_x(x, x_bf16, w_router, T, d) || ((uintptr_t)xcopy & 15) != 0))
+    return cudaErrorInvalidValue;
   if (T <= kSmallT && vec_ok) {
     int per = (d + n_split - 1) / n_split;
     per = (per + 127) / 128 * 128;
     dim3 grid(T, n_split, (E + kLogitThreads / 32 - 1) / (kLogitThreads / 32));
     if (x_bf16)
       return launch_pdl(router_logits_small_kernel<__nv_bfloat16>, grid, dim3(kLogitThreads), 0,
-                        st, (const __nv_bfloat16*)x, w_router, T, d, E, per, part);
+                        st, (const __nv_bfloat16*)x, w_router, T, d, E, per, part,
+                        (__nv_bfloat16*)xcopy);
     return launch_pdl(router_logits_small_kernel<float>, grid, dim3(kLogitThreads), 0, st,
-                      (const float*)x, w_router, T, d, E, per, part);
+                      (const float*)x, w_router, T, d, E, per, part, (float*)xcopy);
   }
   if (x_bf16 && sk_eligible(T, d) && vec_ok) {
     SkPlan pl;
     if (!sk_plan(T, d, E, n_split, pl)) return cudaErrorInvalidDevice;
     if (pl.n_split > n_split) return cudaErrorInvalidValue;
     return launch_pdl(router_logits_sk_kernel<kSKTM>, dim3(pl.grid), dim3(SkCfg<kSKTM>::kThreads),
-                      kSKSmem, st,
-                      (const __nv_bfloat16*)x, w_router, T, d, E, n_split, part);
+                      kSKSmem, st, (const __nv_bfloat16*)x, w_router, T, d, E, n_split, part,
+                      (__nv_bfloat16*)xcopy);
   }
   int per = (d + n_split - 1) / n_split;
   per = (per + kChunkK - 1) / kChunkK * kChunkK;

@@ -520,6 +520,52 @@ def test_max_tokens_bound_and_host_path():
     layer.close()
 
 
+@pytest.mark.parametrize("name,Ts", [("olmoe", [32, 300, 1100]), ("qwen", [16, 300, 1100])])
+def test_host_buffers_page_locked_and_pageable(name, Ts):
+    """eat_moe_forward_host with page-locked buffers (the router kernel reads x over the host link
+    and writes the device copy, the combine writes y to the host) and with pageable buffers (copy
+    engine), against eat_moe_forward on device buffers: outputs and accounts bit for bit, for
+    gathering decode tiles, single-SM tiles of 128 tokens and SM pairs; the Qwen-shaped layer's
+    small calls run their shared experts beside the routing and take the copies."""
+    sh = {"olmoe": OLMOE_S, "qwen": QWEN_S}[name]
+    lw = W.make_layer(sh)
+    layer = eat.EatLayer.from_workload(lw, max(Ts), gpu_params(sh))
+    for s in range(2):  # some history in the accounts
+        layer.forward(W.make_tokens(sh, 64, step=50 + s).cuda(), 0)
+    s = torch.cuda.current_stream()
+    for T in Ts:
+        x = W.make_tokens(sh, T, step=T).cuda()
+        acc = layer.accounts()
+        y_dev = layer.forward(x, 0).cpu()
+        acc_dev = [a.clone() for a in layer.accounts()]
+        for pinned in (True, False):
+            layer.set_accounts(*acc)
+            xh = x.cpu().pin_memory() if pinned else x.cpu().clone()
+            yh = torch.full_like(xh, float("nan"))
+            if pinned:
+                yh = yh.pin_memory()
+            eat.eat_moe_forward_host(layer.h, xh, T, 0, yh)
+            assert torch.equal(yh, y_dev), (name, T, pinned)
+            for u, v in zip(layer.accounts(), acc_dev):
+                assert torch.equal(u, v), (name, T, pinned)
+        # two enqueue-only calls back to back (the two staging buffers in turn), one
+        # synchronisation; the second routes with the accounts the first one updated
+        layer.set_accounts(*acc)
+        y2_dev = layer.forward(x, 0).cpu()
+        layer.set_accounts(*acc)
+        layer.forward(x, 0)
+        y3_dev = layer.forward(x, 0).cpu()
+        layer.set_accounts(*acc)
+        xh = x.cpu().pin_memory()
+        yh1 = torch.empty_like(xh).pin_memory()
+        yh2 = torch.empty_like(xh).pin_memory()
+        eat.eat_moe_forward_host_async(layer.h, xh, T, 0, yh1, s)
+        eat.eat_moe_forward_host_async(layer.h, xh, T, 0, yh2, s)
+        s.synchronize()
+        assert torch.equal(yh1, y2_dev) and torch.equal(yh2, y3_dev), (name, T)
+    layer.close()
+
+
 def test_deterministic_repeat():
     lw = W.make_layer(OLMOE_S)
     outs = []
