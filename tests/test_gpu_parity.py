@@ -199,6 +199,40 @@ def test_expert_counts_and_max_k(E, K, T):
     run_parity(sh, lw, [T, 1, T // 3])
 
 
+@pytest.mark.parametrize("E,d", [(64, 256), (100, 192), (256, 512)])
+def test_router_runs_split_between_blocks(E, d):
+    """Router scores of calls above 128 tokens: a persistent grid takes equal runs of
+    (64-token x 64-expert tile, 32-column chunk) units, so tiles are split between blocks at
+    chunk boundaries that depend on T, E and d, and the split slices are padded with zero pairs.
+    Selections and gates against the oracle (routing only, from seeded accounts) for token
+    counts around the tile size and the one-wave point, ragged expert tiles (E = 100) and
+    several expert tiles (E = 256); eat_route_noalloc, which may use fewer slices, on the same
+    inputs where its scratch holds the call."""
+    sh = W.scaled(W.OLMOE, f"rt{E}-{d}", d_model=d, n_experts=E, d_ff=64, max_k=8)
+    lw = W.make_layer(sh)
+    ref = oracle_layer(lw)
+    L = eat.EatLayer.from_workload(lw, 4099, gpu_params(sh))
+    L.forward(W.make_tokens(sh, 300, step=9).cuda(), 0)  # some history in the accounts
+    prm = orc.Params(max_k=sh.max_k, temperature=sh.temperature)
+    for T in (129, 191, 640, 2047, 4099):
+        x = W.make_tokens(sh, T, step=T).cuda()
+        idx, w, k = L.route(x, 0)
+        torch.cuda.synchronize()
+        N, P, C = (t.cpu().numpy() for t in L.accounts())
+        routing = orc.route(np64(x), ref, orc.Accounts(N, P, C), prm, 0)
+        par.check_routing(routing, par.gpu_selection(idx, k), w.cpu().numpy(), sh.max_k)
+        if T * E <= (1 << 20) // 8:
+            N, P, C = L.accounts()
+            idx2 = torch.empty_like(idx)
+            w2 = torch.empty_like(w)
+            k2 = torch.empty_like(k)
+            eat.eat_route_noalloc(x, T, d, E, eat.EAT_BF16, L._keep[0], L._keep[1], N, P, C,
+                                  L.params, 0, idx2, w2, k2)
+            torch.cuda.synchronize()
+            par.check_routing(routing, par.gpu_selection(idx2, k2), w2.cpu().numpy(), sh.max_k)
+    L.close()
+
+
 @pytest.mark.parametrize("E,K,T", [(256, 8, 1500), (64, 2, 1100)])
 def test_sm_pair_small_groups(E, K, T):
     """Calls of >= 1024 tokens run the SM-pair GEMMs; with many experts nearly every group is a
@@ -520,15 +554,18 @@ def test_max_tokens_bound_and_host_path():
     layer.close()
 
 
-@pytest.mark.parametrize("name,Ts", [("olmoe", [32, 300, 1100]), ("qwen", [16, 300, 1100])])
+@pytest.mark.parametrize("name,Ts", [("olmoe", [32, 300, 1100]), ("qwen", [16, 300, 1100]),
+                                     ("olmoe-fp8", [32, 300])])
 def test_host_buffers_page_locked_and_pageable(name, Ts):
     """eat_moe_forward_host with page-locked buffers (the router kernel reads x over the host link
     and writes the device copy, the combine writes y to the host) and with pageable buffers (copy
     engine), against eat_moe_forward on device buffers: outputs and accounts bit for bit, for
     gathering decode tiles, single-SM tiles of 128 tokens and SM pairs; the Qwen-shaped layer's
     small calls run their shared experts beside the routing and take the copies."""
-    sh = {"olmoe": OLMOE_S, "qwen": QWEN_S}[name]
+    sh = {"olmoe": OLMOE_S, "qwen": QWEN_S, "olmoe-fp8": OLMOE_S}[name]
     lw = W.make_layer(sh)
+    if name.endswith("fp8"):
+        lw = W.to_fp8(lw)
     layer = eat.EatLayer.from_workload(lw, max(Ts), gpu_params(sh))
     for s in range(2):  # some history in the accounts
         layer.forward(W.make_tokens(sh, 64, step=50 + s).cuda(), 0)
