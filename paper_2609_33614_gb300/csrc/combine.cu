@@ -97,8 +97,10 @@ __device__ __forceinline__ float warp_sum_many(float (&v)[N], int lane) {
 // outputs bf16 (s_bf16) or fp32.  Slots past k_t are -1 with gate 0.  All of a token's slot rows
 // are loaded before any use.  A token with no selected expert (k_t = 0, which only a NaN routing
 // probability produces) gets a NaN row.
+// (bf16 expert rows, the large calls: at most 64 registers, so four blocks share an SM and keep
+// more row loads in flight)
 template <typename TY, int KM, bool OB>
-__global__ void __launch_bounds__(kCombThreads)
+__global__ void __launch_bounds__(kCombThreads, OB ? 4 : 1)
 combine_kernel(const void* __restrict__ opart, int n_split, size_t split_stride,
                const int32_t* __restrict__ slot_of, const float* __restrict__ w,
                const void* __restrict__ sout, int s_bf16, int S, int T, int K, int d, int nseg,
