@@ -138,8 +138,10 @@ __device__ __forceinline__ void store_x4(__nv_bfloat16* p, const X4b& v) { *(uin
 // xcopy (or null): x is read from memory the caller keeps on the host (a host-buffer call) and
 // warp 0 of the blocks of the first expert group also writes what it reads to xcopy, the device
 // copy every later kernel of the call reads.
+// (bf16 x: at most 32 registers, so eight blocks share an SM and a 32-token decode call of a
+// 64-expert layer, 1024 blocks, runs in one wave)
 template <typename TX>
-__global__ void __launch_bounds__(kLogitThreads)
+__global__ void __launch_bounds__(kLogitThreads, sizeof(TX) == 2 ? 8 : 1)
 router_logits_small_kernel(const TX* __restrict__ x, const float* __restrict__ wr, int T, int d,
                            int E, int d_per_split, float2* __restrict__ part,
                            TX* __restrict__ xcopy) {
