@@ -256,6 +256,7 @@ struct TcArgs {
   int b_lo_rows;             // fp8: row offset of the B operand's lo plane in its tensor map
   int prefetch_a;            // the group layout was written two or more launches back: issue the
                              // first stages' weight loads before waiting for the previous kernel
+  int gate_first;            // 16-row interleaved gate/up A tile: the gate rows come first
   unsigned int* err;
 };
 
@@ -705,7 +706,7 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
 constexpr int kPairBN = 256;
 constexpr int kPairRows = kPairBN / 2;
 
-template <int MODE>
+template <int MODE, bool IL4 = false>
 struct PairCfg {
   static constexpr bool kIL = MODE == kModeGateUpIL;
   static constexpr int kABytes = kBM * kBK * 2;
@@ -721,8 +722,8 @@ struct PairCfg {
   static constexpr int kEpiWarps = 8;
   static constexpr int kThreads = 64 + 32 * kEpiWarps;
   // exchange buffers of the 4 (feature half, column half) warp pairs: 2 buffers x gate and up x
-  // 16 columns x 32 lanes
-  static constexpr int kXchgFloats = kIL ? 4 * 2 * 2 * 16 * 32 : 0;
+  // 16 columns x 32 lanes (not with the 16-row interleave, whose warps pair gate and up by shuffles)
+  static constexpr int kXchgFloats = (kIL && !IL4) ? 4 * 2 * 2 * 16 * 32 : 0;
   // the whole 227 KB a CTA may hold: 1 KB of alignment slack and 256 B of barriers besides the
   // stages (three, beside the gate/up exchange buffers too)
   static constexpr int kStagesRaw = (227 * 1024 - 1024 - 256 - kXchgFloats * 4) / kStageBytes;
@@ -756,6 +757,16 @@ __device__ __forceinline__ void tma_load_2d_pair(void* dst, const CUtensorMap* m
       "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
       " [%0], [%1, {%3, %4}], [%2];" ::"r"(smem_u32(dst)),
       "l"(map), "r"(bar_cluster), "r"(c0), "r"(c1)
+      : "memory");
+}
+// The same for a 4D tensor map (coordinates innermost first).
+__device__ __forceinline__ void tma_load_4d_pair(void* dst, const CUtensorMap* map,
+                                                 uint32_t bar_cluster, int c0, int c1, int c2,
+                                                 int c3) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4, %5, %6}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(map), "r"(bar_cluster), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
       : "memory");
 }
 __device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar_cluster) {
@@ -798,14 +809,20 @@ __device__ __forceinline__ int pair_n(int nrows) { return min(kPairBN, (nrows + 
 // With FOLD a launch carries two unit sets: the routed experts (args, mapA0/A1/B) and, after them,
 // the always-on shared experts of the same call (args_s, mapA0s/A1s/Bs), so a large call's
 // projection pays one ramp and one tail for both.  Without FOLD the second set is ignored.
-template <int MODE, bool FOLD>
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg<MODE>::kThreads, 1)
+//
+// IL4 (interleaved gate/up only): the A tile comes from one 4D view of the gate and up weights
+// that alternates 16 gate rows and 16 up rows (mapA0; see encode_gu4), so each TMEM lane quarter
+// holds the gate and up rows of the same 16 features and the epilogue pairs them with shuffles
+// instead of the shared-memory exchange.
+template <int MODE, bool FOLD, bool IL4>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(PairCfg<MODE, IL4>::kThreads, 1)
 tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__ CUtensorMap mapA1,
                const __grid_constant__ CUtensorMap mapB, const TcArgs args,
                const __grid_constant__ CUtensorMap mapA0s, const __grid_constant__ CUtensorMap mapA1s,
                const __grid_constant__ CUtensorMap mapBs, const TcArgs args_s) {
-  using C = PairCfg<MODE>;
+  using C = PairCfg<MODE, IL4>;
   constexpr bool IL = C::kIL;
+  static_assert(!IL4 || IL, "the 16-row interleave is a gate/up layout");
   constexpr int S = C::kStages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -905,7 +922,9 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
             if (j < nk) {
               uint8_t* sj = st + j * C::kSubBytes;
               const int kx = (kb + j) * kBK;
-              if (IL) {
+              if (IL4) {
+                tma_load_4d_pair(sj, mA0, fb, kx, 0, 0, a_row / 16);
+              } else if (IL) {
                 tma_load_2d_pair(sj, mA0, fb, kx, a_row);
                 tma_load_2d_pair(sj + C::kABytes / 2, mA1, fb, kx, a_row);
               } else {
@@ -978,6 +997,56 @@ tc_pair_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant_
       mma_commit_pair(mma_done);
     }
     if (lane == 0) mbar_wait(mma_done, 0u, abort_flag, args.err, 16u, false);
+  } else if (IL4) {
+    // ------------------------------ epilogue, gate/up interleaved in 16-row groups (warps 2..9)
+    // Warp w drains TMEM lane quarter q = w % 4 for the token columns [128 ch, 128 ch + 128),
+    // ch = (w - 2) / 4.  Lanes i and i + 16 hold the two rows (gate and up, in the order of the
+    // view) of feature 16 q + i.  Per 32 columns lanes 0-15 finish the first 16 and lanes 16-31
+    // the second 16; each takes the other row's value for its columns from its partner lane.
+    const int q = warp & 3;
+    const int ch = (warp - 2) >> 2;
+    const bool lo = lane < 16;
+    int local = 0;
+    for (int u = pair; u < units; u += n_pairs, ++local) {
+      Unit w;
+      const bool sh = unit_at(u, w);  // (scalars, as in the exchange epilogue below)
+      __nv_bfloat16* const out = (__nv_bfloat16*)(sh ? args_s.out : args.out);
+      const int M = sh ? args_s.M : args.M;
+      const bool gate_first = (sh ? args_s.gate_first : args.gate_first) != 0;
+      const bool mine_is_gate = lo == gate_first;
+      const int buf = local & 1;
+      const uint32_t tph = (uint32_t)((local >> 1) & 1);
+      if (!warp_wait(&tfull[buf], tph, abort_flag, args.err, 32u)) break;
+      tc_fence_after();
+      const uint32_t tbase =
+          tmem_base + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * C::kAccCols);
+      const int f = w.m0 + (int)rank * C::kFeat + 16 * q + (lane & 15);
+      const bool fok = f < M;
+      const int c_end = min(128 * ch + 128, w.nrows);
+      for (int c0 = 128 * ch; c0 < c_end; c0 += 32) {
+        uint32_t v0[16], v1[16];
+        tmem_ld16(tbase + c0, v0);
+        tmem_ld16(tbase + c0 + 16, v1);
+        tmem_wait_ld();
+        const int cb = c0 + (lo ? 0 : 16);
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          const float mine = __uint_as_float(lo ? v0[j] : v1[j]);
+          const float other =
+              __shfl_xor_sync(0xffffffffu, __uint_as_float(lo ? v1[j] : v0[j]), 16);
+          const float g = mine_is_gate ? mine : other;
+          const float up = mine_is_gate ? other : mine;
+          if (fok && cb + j < w.nrows)
+            out[(size_t)(w.slot0 + cb + j) * M + f] = __float2bfloat16_rn(silu_f(g) * up);
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) {
+        if (leader) mbar_arrive(&tempty[buf]);
+        else mbar_arrive_cluster(tempty0 + 8u * (uint32_t)buf);
+      }
+    }
   } else if (IL) {
     // ---------------------------------------- epilogue, interleaved gate/up (warps 2..9)
     // Warp w drains TMEM lane quarter w % 4 (gate rows in quarters 0-1, up rows in 2-3) for the
@@ -1183,9 +1252,40 @@ bool encode_2d_u8(CUtensorMap* m, const void* ptr, long long rows, long long col
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// The gate and up weights of one expert set ([rows, cols] bf16 each, rows a multiple of 16) as one
+// 4D view that alternates 16 rows of each: element (k, r, h, g) is row 16 g + r, column k of the
+// lower (h = 0) or higher (h = 1) of the two allocations, so the box {64, 16, 2, 4} holds 128 rows
+// [16 of one, 16 of the other, ...] of 64 columns, in the 128B-swizzled layout of a 2D box of 128
+// rows.  The two allocations need not be adjacent: the h stride is their distance.  false when
+// the view cannot be encoded (the caller then keeps the two 64-row boxes).
+bool encode_gu4(CUtensorMap* m, const void* gate, const void* up, long long rows, long long cols,
+                bool* gate_first) {
+  auto fn = encode_fn();
+  if (!fn || rows % 16 != 0 || gate == up) return false;
+  const bool gf = (uintptr_t)gate < (uintptr_t)up;
+  const char* lo = (const char*)(gf ? gate : up);
+  const char* hi = (const char*)(gf ? up : gate);
+  const unsigned long long dist = (unsigned long long)(hi - lo);
+  if (dist % 16 != 0 || dist >= (1ULL << 40)) return false;
+  cuuint64_t dims[4] = {(cuuint64_t)cols, 16, 2, (cuuint64_t)(rows / 16)};
+  cuuint64_t strides[3] = {(cuuint64_t)cols * 2, (cuuint64_t)dist, (cuuint64_t)cols * 2 * 16};
+  cuuint32_t box[4] = {(cuuint32_t)kBK, 16, 2, 4};
+  cuuint32_t estr[4] = {1, 1, 1, 1};
+  const bool ok = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<char*>(lo), dims, strides,
+                     box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+  *gate_first = gf;
+  return ok;
+}
+
 struct Maps {
   CUtensorMap wg, wu, wd, wsg, wsu, wsd;   // bf16 weights, or e4m3 weights of an fp8 layer
   CUtensorMap wg64, wu64, wsg64, wsu64;  // 64-row boxes for the interleaved gate/up A tile
+  // the 16-row interleave of gate and up (encode_gu4) for the SM-pair gate/up, when it encodes
+  CUtensorMap wgu4, wsgu4;
+  bool il4 = false, sil4 = false;                   // routed / shared view available
+  bool gate_first = true, sgate_first = true;       // gate rows first in the view
   CUtensorMap xperm[kNumBN], act[kNumBN], sact[kNumBN];
   // fp8 layers: the e4m3 hi/lo planes of the B operands (slot rows of x, token rows of x, the
   // routed and the shared activations)
@@ -1217,17 +1317,17 @@ cudaError_t launch_tc(const CUtensorMap& a0, const CUtensorMap& a1, const CUtens
 // SM-pair kernels: one 2-CTA cluster per pair of SMs, at most as many pairs as can be resident.
 // The routed set (a0, a1, b, args) and, when sargs is given, the shared set of the same call in
 // the same launch; units counts both.
-template <int MODE, bool FOLD>
+template <int MODE, bool FOLD, bool IL4>
 cudaError_t launch_pair_t(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& b,
                           const TcArgs& args, long long units, int num_sms, cudaStream_t st,
                           const CUtensorMap* sa0, const CUtensorMap* sa1, const CUtensorMap* sb,
                           const TcArgs* sargs) {
-  using C = PairCfg<MODE>;
+  using C = PairCfg<MODE, IL4>;
   static std::once_flag once;
   static cudaError_t attr_err = cudaSuccess;
   static int max_pairs = 0;
   std::call_once(once, [num_sms] {
-    attr_err = cudaFuncSetAttribute(tc_pair_kernel<MODE, FOLD>,
+    attr_err = cudaFuncSetAttribute(tc_pair_kernel<MODE, FOLD, IL4>,
                                     cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
     if (attr_err != cudaSuccess) return;
     cudaLaunchConfig_t cfg = {};
@@ -1242,7 +1342,8 @@ cudaError_t launch_pair_t(const CUtensorMap& a0, const CUtensorMap& a1, const CU
     cfg.attrs = at;
     cfg.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, tc_pair_kernel<MODE, FOLD>, &cfg) != cudaSuccess || n <= 0) {
+    if (cudaOccupancyMaxActiveClusters(&n, tc_pair_kernel<MODE, FOLD, IL4>, &cfg) != cudaSuccess ||
+        n <= 0) {
       cudaGetLastError();
       n = num_sms / 2;
     }
@@ -1253,19 +1354,20 @@ cudaError_t launch_pair_t(const CUtensorMap& a0, const CUtensorMap& a1, const CU
   if (pairs <= 0) return cudaSuccess;
   TcArgs none;
   std::memset(&none, 0, sizeof(none));
-  return launch_pdl(tc_pair_kernel<MODE, FOLD>, dim3((unsigned)(2 * pairs)), dim3(C::kThreads),
+  return launch_pdl(tc_pair_kernel<MODE, FOLD, IL4>, dim3((unsigned)(2 * pairs)), dim3(C::kThreads),
                     C::kSmemBytes, st, a0, a1, b, args, sa0 ? *sa0 : a0, sa1 ? *sa1 : a1,
                     sb ? *sb : b, sargs ? *sargs : none);
 }
-template <int MODE>
+template <int MODE, bool IL4 = false>
 cudaError_t launch_pair(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& b,
                         const TcArgs& args, long long units, int num_sms, cudaStream_t st,
                         const CUtensorMap* sa0 = nullptr, const CUtensorMap* sa1 = nullptr,
                         const CUtensorMap* sb = nullptr, const TcArgs* sargs = nullptr) {
   if (sargs)
-    return launch_pair_t<MODE, true>(a0, a1, b, args, units, num_sms, st, sa0, sa1, sb, sargs);
-  return launch_pair_t<MODE, false>(a0, a1, b, args, units, num_sms, st, nullptr, nullptr,
-                                    nullptr, nullptr);
+    return launch_pair_t<MODE, true, IL4>(a0, a1, b, args, units, num_sms, st, sa0, sa1, sb,
+                                          sargs);
+  return launch_pair_t<MODE, false, IL4>(a0, a1, b, args, units, num_sms, st, nullptr, nullptr,
+                                         nullptr, nullptr);
 }
 
 // Single-SM launches: token tiles of 16..128 rows (256-row tiles run on SM pairs); W8 for fp8
@@ -1412,12 +1514,19 @@ int tc_bind(TcLayer& L, const eat_layer_desc& D, void* xperm, void* act, void* s
          encode_2d(&m->wg64, D.w_gate, (long long)L.E * L.F, L.d, kBM / 2) &&
          encode_2d(&m->wu64, D.w_up, (long long)L.E * L.F, L.d, kBM / 2) &&
          encode_2d(&m->wd, D.w_down, (long long)L.E * L.d, L.F, kBM);
-    if (ok && L.S > 0)
+    if (ok)
+      m->il4 = L.F % 16 == 0 &&
+               encode_gu4(&m->wgu4, D.w_gate, D.w_up, (long long)L.E * L.F, L.d, &m->gate_first);
+    if (ok && L.S > 0) {
       ok = encode_2d(&m->wsg, D.ws_gate, (long long)L.S * L.Fs, L.d, kBM) &&
            encode_2d(&m->wsu, D.ws_up, (long long)L.S * L.Fs, L.d, kBM) &&
            encode_2d(&m->wsg64, D.ws_gate, (long long)L.S * L.Fs, L.d, kBM / 2) &&
            encode_2d(&m->wsu64, D.ws_up, (long long)L.S * L.Fs, L.d, kBM / 2) &&
            encode_2d(&m->wsd, D.ws_down, (long long)L.S * L.d, L.Fs, kBM);
+      if (ok)
+        m->sil4 = L.Fs % 16 == 0 && encode_gu4(&m->wsgu4, D.ws_gate, D.ws_up,
+                                                (long long)L.S * L.Fs, L.d, &m->sgate_first);
+    }
   }
   for (int i = 0; i < kNumBN && ok; ++i) {
     if (L.w8) {
@@ -1511,6 +1620,10 @@ cudaError_t tc_launch_up(const TcLayer& L, const TcCall& c, bool shared, cudaStr
     shared_args(a);
     max_tiles = (long long)L.S * ((c.T + bn - 1) / bn);
     const long long units = max_tiles * a.m_tiles;
+    if (pair && m->sil4) {
+      a.gate_first = m->sgate_first ? 1 : 0;
+      return launch_pair<kModeGateUpIL, true>(m->wsgu4, m->wsgu4, xm, a, units, L.num_sms, st);
+    }
     if (pair)
       return launch_pair<kModeGateUpIL>(m->wsg64, m->wsu64, xm, a, units, L.num_sms, st);
     const int grid = (int)std::min<long long>(L.num_sms, units);
@@ -1535,9 +1648,21 @@ cudaError_t tc_launch_up(const TcLayer& L, const TcCall& c, bool shared, cudaStr
     CUtensorMap xm;
     if (!encode_2d(&xm, c.x, c.T, L.d, kPairRows)) return cudaErrorInvalidValue;
     const long long s_units = (long long)L.S * ((c.T + bn - 1) / bn) * sa.m_tiles;
+    if (m->il4 && m->sil4) {
+      a.gate_first = m->gate_first ? 1 : 0;
+      sa.gate_first = m->sgate_first ? 1 : 0;
+      return launch_pair<kModeGateUpIL, true>(m->wgu4, m->wgu4, m->xperm[bn_index(kPairRows)], a,
+                                              units + s_units, L.num_sms, st, &m->wsgu4,
+                                              &m->wsgu4, &xm, &sa);
+    }
     return launch_pair<kModeGateUpIL>(m->wg64, m->wu64, m->xperm[bn_index(kPairRows)], a,
                                       units + s_units, L.num_sms, st, &m->wsg64, &m->wsu64, &xm,
                                       &sa);
+  }
+  if (pair && m->il4) {
+    a.gate_first = m->gate_first ? 1 : 0;
+    return launch_pair<kModeGateUpIL, true>(m->wgu4, m->wgu4, m->xperm[bn_index(kPairRows)], a,
+                                            units, L.num_sms, st);
   }
   if (pair)
     return launch_pair<kModeGateUpIL>(m->wg64, m->wu64, m->xperm[bn_index(kPairRows)], a, units,
