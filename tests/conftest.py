@@ -8,3 +8,13 @@ if ROOT not in sys.path:
 
 def pytest_configure(config):
     config.addinivalue_line("markers", "gpu: needs a CUDA GPU (GB300, sm_103a)")
+
+
+def pytest_terminal_summary(terminalreporter, exitstatus, config):
+    # the worst output error of every full-size parity step that ran (shown without -s)
+    mod = sys.modules.get("tests.parity")
+    lines = getattr(mod, "REPORT", None) if mod else None
+    if lines:
+        terminalreporter.section("full-size parity")
+        for line in lines:
+            terminalreporter.write_line(line)

@@ -19,6 +19,10 @@ import oracle.eat_oracle as orc
 
 from tests.helpers import np64
 
+# one line per full-size parity step (worst output error, near-tie tokens), printed at the end of
+# the session by tests/conftest.py
+REPORT: list = []
+
 
 def delta_of(tau):
     return 1e-5 * max(1.0, abs(tau))

@@ -111,8 +111,8 @@ def run_parity(shape, lw, Ts, signs=None, prm_kw=None, layer=None, L=None, sampl
         assert err.max() <= Y_TOL[shape.xdtype], \
             f"step {step}: output rel err {err.max():.3g} (token {toks[int(err.argmax())]})"
         if report is not None:
-            print(f"parity {shape.name} {report} step {step}: T={T} checked {len(toks)} rows, "
-                  f"max rel err {err.max():.3g}, near-tie tokens {len(amb)}")
+            par.REPORT.append(f"parity {shape.name} {report} step {step}: T={T} checked {len(toks)} "
+                              f"rows, max rel err {err.max():.3g}, near-tie tokens {len(amb)}")
         par.check_accounts(acc0, (N1, P1, C1), (n_e, s_p, s_n), routing, sel, norms_ref,
                            prm.alpha, C_TOL[shape.xdtype])
         outs.append(y)
