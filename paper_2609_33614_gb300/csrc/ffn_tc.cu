@@ -700,9 +700,10 @@ tc_ffn_kernel(const __grid_constant__ CUtensorMap mapA0, const __grid_constant__
 // CTAs load their halves with TMA completing on rank 0's full barrier (rank 0 expects the bytes
 // of both); each CTA drains its own TMEM rows, and rank 0 reuses an accumulator buffer once the
 // epilogues of both CTAs released it.  Modes: the down projection (256 output features per unit)
-// and the interleaved gate/up (each CTA 64 gate rows over the 64 up rows of its features, 128
-// features per unit).  The MMA width is the unit's token rows rounded up to 32 (each CTA loads
-// half of it), so a partial tile computes no padding beyond that.
+// and the interleaved gate/up (each CTA the gate and up rows of 64 features, 128 features per
+// unit: alternating in groups of 16 rows, or 64 gate rows over the 64 up rows; see IL4 below).
+// The MMA width is the unit's token rows rounded up to 32 (each CTA loads half of it), so a
+// partial tile computes no padding beyond that.
 constexpr int kPairBN = 256;
 constexpr int kPairRows = kPairBN / 2;
 
