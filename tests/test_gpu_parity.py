@@ -168,6 +168,29 @@ def test_shared_experts_in_the_routed_sm_pair_launches():
     run_parity(QWEN_S, lw, [1024, 2100, 40])
 
 
+@pytest.mark.parametrize("gate_first", [True, False])
+def test_gate_up_interleave_from_one_allocation(gate_first):
+    """The SM-pair gate/up tile interleaves 16 gate rows and 16 up rows through a 4D view whose
+    stride between the two weight tensors is their distance, with either tensor at the lower
+    address: here both are halves of one allocation, up first or gate first, for the routed and
+    the shared experts (1100 and 2100 tokens: SM pairs with a ragged last tile)."""
+    sh = QWEN_S
+    lw = W.make_layer(sh)
+    def pair_of(a, b):
+        buf = torch.empty((2,) + tuple(a.shape), dtype=a.dtype, device="cuda")
+        first, second = (buf[0], buf[1]) if gate_first else (buf[1], buf[0])
+        first.copy_(a)
+        second.copy_(b)
+        return first, second
+    wg, wu = pair_of(lw.w_gate, lw.w_up)
+    wsg, wsu = pair_of(lw.ws_gate, lw.ws_up)
+    assert (wg.data_ptr() < wu.data_ptr()) == gate_first
+    layer = eat.EatLayer(lw.w_router.cuda(), lw.b_router.cuda(), wg, wu, lw.w_down.cuda(), 2100,
+                         gpu_params(sh), wsg, wsu, lw.ws_down.cuda())
+    run_parity(sh, lw, [1100, 2100], layer=layer)
+    layer.close()
+
+
 def test_dsv2l_shaped_residual_chain():
     """Three layers, independent accounts, x_{l+1} = bf16(x_l + y_l) with the GPU's x_l."""
     T = 96
