@@ -503,11 +503,13 @@ def test_degenerate_fixed_topk_on_gpu():
 
 
 def test_all_tokens_one_expert():
-    """Router bias forces one expert for every token: a single group of n_e = T rows."""
+    """Router bias forces one expert for every token: a single group of n_e = T rows (2500: SM
+    pairs with a ragged last tile, and an account update over three 1024-slot chunks of one
+    expert, finished by the last of its blocks)."""
     lw = W.make_layer(OLMOE_S)
     lw.b_router = torch.full_like(lw.b_router, -30.0)
     lw.b_router[5] = 30.0
-    run_parity(OLMOE_S, lw, [257, 1])
+    run_parity(OLMOE_S, lw, [257, 2500, 1])
 
 
 def test_set_accounts_restore_and_route_is_pure():
