@@ -132,6 +132,13 @@ def test_toy_ppl_signs():
     run_parity(W.TOY, lw, [64] * 16, signs=W.ppl_signs(16))
 
 
+def test_toy_large_calls():
+    """fp32 layer, calls above 128 tokens: the fp32 router-score kernel over the slices the
+    stream-K plan sets for the call, and the CUDA-core expert kernels."""
+    lw = W.make_layer(W.TOY)
+    run_parity(W.TOY, lw, [300, 1100, 64])
+
+
 def test_toy_c_mode_raw_and_no_clamp():
     lw = W.make_layer(W.TOY)
     run_parity(W.TOY, lw, [64] * 6, prm_kw={"c_mode": eat.EAT_C_RAW})
