@@ -808,25 +808,28 @@ def test_expired_wait_leaves_accounts_and_fails_later_calls():
 
 
 # ------------------------------------------------------------------ CUDA graph capture
-@pytest.mark.parametrize("shape", ["mixtral", "qwen"])
-def test_forward_replays_as_cuda_graph(shape):
+@pytest.mark.parametrize("shape,T", [("mixtral", 64), ("qwen", 64), ("qwen", 1100),
+                                     ("olmoe", 1100)])
+def test_forward_replays_as_cuda_graph(shape, T):
     """A layer call has no host synchronisation and decides its expert schedule on the device, so
     it can be captured once and replayed: the replays must match direct calls bit for bit, accounts
     included (two handles on the same weights, same inputs).  The qwen-shaped layer's 64-token call
-    runs its shared experts on the handle's second stream, forked and joined inside the capture."""
-    sh = MIX_S if shape == "mixtral" else QWEN_S
+    runs its shared experts on the handle's second stream, forked and joined inside the capture;
+    the 1100-token calls capture the stream-K router, the chunked permute, the gather and the
+    SM-pair expert kernels (with the shared experts in the routed launches for qwen)."""
+    sh = {"mixtral": MIX_S, "qwen": QWEN_S, "olmoe": OLMOE_S}[shape]
     lw = W.make_layer(sh)
-    a = eat.EatLayer.from_workload(lw, 64, gpu_params(sh))
-    b = eat.EatLayer.from_workload(lw, 64, gpu_params(sh))
-    x = W.make_tokens(sh, 64).cuda()
+    a = eat.EatLayer.from_workload(lw, T, gpu_params(sh))
+    b = eat.EatLayer.from_workload(lw, T, gpu_params(sh))
+    x = W.make_tokens(sh, T).cuda()
     y_graph = torch.empty_like(x)
     stream = torch.cuda.Stream()
     g = torch.cuda.CUDAGraph()
     with torch.cuda.stream(stream):
-        eat.eat_moe_forward(a.h, x, 64, 0, y_graph, stream=stream.cuda_stream)  # warm-up call
+        eat.eat_moe_forward(a.h, x, T, 0, y_graph, stream=stream.cuda_stream)  # warm-up call
         torch.cuda.current_stream().synchronize()
         with torch.cuda.graph(g, stream=stream):
-            eat.eat_moe_forward(a.h, x, 64, 0, y_graph, stream=stream.cuda_stream)
+            eat.eat_moe_forward(a.h, x, T, 0, y_graph, stream=stream.cuda_stream)
     torch.cuda.synchronize()
     ys = [b.forward(x, 0)]  # matches the warm-up call of a
     for _ in range(4):
