@@ -372,28 +372,30 @@ def test_toy_free_running_first_divergence():
     layer.close()
 
 
-@pytest.mark.parametrize("shape", ["olmoe", "qwen"])
-def test_two_handles_on_two_streams_interleaved(shape):
+@pytest.mark.parametrize("shape,T", [("olmoe", 48), ("qwen", 48), ("olmoe", 1100),
+                                     ("qwen", 1100)])
+def test_two_handles_on_two_streams_interleaved(shape, T):
     """Two handles (one layer each) driven from two CUDA streams with their calls interleaved give
     the results of running each alone: a handle's workspace and accounts are its own (with shared
-    experts, so are the stream and events their small calls fork onto)."""
+    experts, so are the stream and events their small calls fork onto).  At 1100 tokens the two
+    handles' persistent SM-pair and stream-K router launches overlap on the GPU."""
     sh = OLMOE_S if shape == "olmoe" else QWEN_S
     lw = W.make_layer(sh)
-    xs = [W.make_tokens(sh, 48, step=s).cuda() for s in range(4)]
+    xs = [W.make_tokens(sh, T, step=s).cuda() for s in range(4)]
     ref = []
-    solo = eat.EatLayer.from_workload(lw, 48, gpu_params(sh))
+    solo = eat.EatLayer.from_workload(lw, T, gpu_params(sh))
     for x in xs:
         ref.append(solo.forward(x, 0).clone())
     solo.close()
-    a = eat.EatLayer.from_workload(lw, 48, gpu_params(sh))
-    b = eat.EatLayer.from_workload(lw, 48, gpu_params(sh))
+    a = eat.EatLayer.from_workload(lw, T, gpu_params(sh))
+    b = eat.EatLayer.from_workload(lw, T, gpu_params(sh))
     sa, sb = torch.cuda.Stream(), torch.cuda.Stream()
     ya = [torch.empty_like(x) for x in xs]
     yb = [torch.empty_like(x) for x in xs]
     torch.cuda.synchronize()
     for i, x in enumerate(xs):
-        eat.eat_moe_forward(a.h, x, 48, 0, ya[i], stream=sa)
-        eat.eat_moe_forward(b.h, x, 48, 0, yb[i], stream=sb)
+        eat.eat_moe_forward(a.h, x, T, 0, ya[i], stream=sa)
+        eat.eat_moe_forward(b.h, x, T, 0, yb[i], stream=sb)
     torch.cuda.synchronize()
     for i in range(4):
         assert torch.equal(ya[i], ref[i]) and torch.equal(yb[i], ref[i])
