@@ -552,7 +552,7 @@ route_select_kernel(const float2* __restrict__ part, int n_split, const float* _
     bv[i] = bias && valid[i] ? bias[e] : 0.f;
   }
   // the score partials in slice order, a chunk of slices' loads in flight before their sums
-  constexpr int kChunk = EPL <= 2 ? 4 : (EPL <= 4 ? 2 : 1);
+  constexpr int kChunk = EPL <= 1 ? 8 : (EPL <= 2 ? 4 : (EPL <= 4 ? 2 : 1));
   for (int sp0 = 0; sp0 < n_split; sp0 += kChunk) {
     float2 v[kChunk][EPL];
 #pragma unroll
